@@ -1,0 +1,202 @@
+/*
+ * cis.h -- C ABI of libcis, the GB300 (sm_103a) implementation of the
+ * training-side token pass of calibrated importance sampling (CIS),
+ * arxiv 2609.32444.
+ *
+ * The pass, per token t of a batch of T tokens over a vocabulary of V:
+ *   1. log-softmax of the training logits z_t and the gather of the sampled
+ *      token's log-probability  l_t = log softmax(z_t)_{y_t}     (Sec. 2.1);
+ *   2. the mismatch weight w_t from l_t (or l_old,t) and the inference-side
+ *      log-probability l_inf,t: CIS min{k, 1 + lambda*max(1-p, kappa)}
+ *      (Eq. 4, Algorithm 1), TIS min(k, C), the exact ratio clamped to
+ *      [lo, hi], or 1 (Table 8), with k = exp(l_w - l_inf), p = exp(l_w);
+ *   3. the weighted, PPO-clipped policy-gradient token loss (Eq. 1), with the
+ *      weight detached (stopgrad, Algorithm 1);
+ *   4. its gradient with respect to the logits,
+ *        dz_tj = c_t (softmax(z_t)_j - [j == y_t]),
+ *        c_t   = s_t m_t w_t A_t rho_t g_t,
+ *      s_t the normaliser, m_t the mask, A_t the advantage, rho_t the update
+ *      ratio and g_t = 0 where the PPO clip is active.
+ *
+ * Conventions shared by every entry point:
+ *   - Pointers marked "device" are CUDA device pointers (or managed memory);
+ *     they are owned by the caller and must stay valid until the work queued
+ *     on `stream` has finished.  The library never allocates device memory;
+ *     scratch space is the caller's `workspace`.
+ *   - `stream` is a cudaStream_t passed as void* (NULL = legacy default
+ *     stream).  Every call is asynchronous on that stream; the return value
+ *     covers host-side validation and launch errors only.  Errors that only
+ *     the device can see (an out-of-range token id, a bounded wait that ran
+ *     out) are OR-ed into a device status word that the caller reads after
+ *     synchronising (see cis_status_t).
+ *   - Logit rows are row-major with a row stride `ld` >= V elements.  Rows
+ *     already line up with their sampled token: the caller shifts the model
+ *     output by one position (the token at t is scored from the logits at
+ *     t - 1, App. C.4).
+ *   - Masked tokens (mask[t] == 0) are not read; they get dz = 0, w = 0,
+ *     trunc = 0, lp = 0 and contribute nothing to the loss.  mask == NULL
+ *     means every token is valid.  Any non-zero mask byte counts as 1.
+ *   - T == 0 is a valid no-op (loss 0).
+ *   - Non-finite logits: -inf is allowed anywhere except at the sampled
+ *     token; NaN propagates into that row's outputs.
+ */
+#ifndef CIS_H
+#define CIS_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    CIS_OK = 0,
+    CIS_ERR_INVALID_ARG = 1,   /* host validation failed; nothing was queued   */
+    CIS_ERR_UNSUPPORTED = 2,   /* valid, but not supported by this build/GPU    */
+    CIS_ERR_CUDA = 3,          /* a CUDA runtime call or launch failed          */
+    CIS_ERR_DEVICE_TIMEOUT = 4,/* device status bit: a bounded wait ran out     */
+    CIS_ERR_BAD_TOKEN_ID = 8   /* device status bit: some valid y_t not in [0,V)*/
+} cis_status_t;
+
+typedef enum { CIS_F32 = 0, CIS_BF16 = 1 } cis_dtype_t;
+
+/* Weight operators: CIS is Eq. 4 with the floor of Algorithm 1; the others are
+ * the token-level rows of Table 8. */
+typedef enum {
+    CIS_MODE_CIS = 0,   /* w = min{k, 1 + lambda*max(1-p, kappa)}            */
+    CIS_MODE_TIS = 1,   /* w = min(k, tis_cap)                               */
+    CIS_MODE_EXACT = 2, /* w = k clamped to [exact_lo, exact_hi]             */
+    CIS_MODE_NONE = 3   /* w = 1                                             */
+} cis_mode_t;
+
+/* Loss normaliser: Algorithm 1 averages over the n tokens of the batch; Eq. 1
+ * averages each response over its |y_i| tokens and the G responses. */
+typedef enum {
+    CIS_AGG_TOKEN_MEAN = 0,        /* s_t = 1/n, n = number of valid tokens      */
+    CIS_AGG_SEQ_MEAN_TOKEN_MEAN = 1/* s_t = 1/(G |y_i|) from cu_seqlens and mask */
+} cis_agg_t;
+
+/* Hyper-parameters.  Defaults (cis_default_params): the deployed CIS of
+ * App. C.1 / Table 8: lambda 2.3, kappa 5e-3, TIS cap 2, exact clamp
+ * [1e-6, 1e6], PPO clip (0.2, 0.28), token mean. */
+typedef struct {
+    int32_t mode;      /* cis_mode_t                                         */
+    int32_t agg;       /* cis_agg_t                                          */
+    double lambda;     /* >= 0: threshold on e^eps is 1 + lambda (Eq. 4)     */
+    double kappa;      /* in [0, 1]: floor on 1 - p (Algorithm 1)            */
+    double tis_cap;    /* >= 1: C of TIS (Eq. 5 assumes C >= 1)              */
+    double exact_lo;   /* > 0: clamp of the exact ratio                      */
+    double exact_hi;   /* >= exact_lo                                        */
+    double clip_low;   /* in [0, 1): rho clipped below at 1 - clip_low       */
+    double clip_high;  /* >= 0: rho clipped above at 1 + clip_high           */
+} cis_params_t;
+
+/* Reduction outputs of cis_loss_fwd_bwd, written on the device. */
+typedef struct {
+    double loss;          /* -sum_t s_t m_t w_t min(rho A, clip(rho) A)       */
+    double trunc_excess;  /* sum over truncated tokens of (k_t - w_t)         */
+    int64_t n_valid;      /* number of tokens with mask != 0                  */
+    int64_t n_truncated;  /* tokens whose weight was truncated or clamped     */
+    float max_abs_logk;   /* max over valid tokens of |log k_t|               */
+    int32_t status;       /* OR of device status bits (cis_status_t)          */
+} cis_stats_t;
+
+/* Fills *out with the defaults above.  Host only.  CIS_ERR_INVALID_ARG if out
+ * is NULL. */
+cis_status_t cis_default_params(cis_params_t *out);
+
+/* Human-readable name of a status value (static string, never NULL). */
+const char *cis_status_string(int32_t status);
+
+/*
+ * Sampled-token log-probabilities (Sec. 2.1): lp_out[t] = z_{t,y_t} -
+ * logsumexp_j z_tj, accumulated in fp32.  One read of the logits.
+ *   logits     device, [T, ld] of `dtype`, row-major; only j < V is read.
+ *   ids        device int32 [T], sampled token ids.
+ *   mask       device uint8 [T] or NULL.
+ *   lp_out     device float [T].
+ *   lse_out    device float [T] or NULL: logsumexp of each row.
+ *   dev_status device int32 [1] or NULL: device status bits are OR-ed in
+ *              (the caller zeroes it first).
+ * Errors: CIS_ERR_INVALID_ARG for NULL required pointers, T < 0, V <= 0,
+ * ld < V or an unknown dtype.
+ */
+cis_status_t cis_token_logprobs(const void *logits, int32_t dtype, int64_t T, int64_t V,
+                                int64_t ld, const int32_t *ids, const uint8_t *mask,
+                                float *lp_out, float *lse_out, int32_t *dev_status,
+                                void *stream);
+
+/*
+ * Elementwise weights (Algorithm 1, Eq. 4, Table 8) from fp32 log-probabilities.
+ *   lp_train  device float [T]: log p_t, the training-side log-probability
+ *             the weight is built from (l_old when updating off the snapshot).
+ *   lp_infer  device float [T]: log q_t, the raw value recorded at sampling.
+ *   mask      device uint8 [T] or NULL.
+ *   w_out     device float [T]: the weight (0 for masked tokens).
+ *   trunc_out device uint8 [T] or NULL: 1 where the weight differs from k
+ *             (CIS/TIS: k above the cap; EXACT: k outside the clamp).
+ *   eps_out   device float [T] or NULL: the log-odds displacement
+ *             eps = logit p - logit q (Lemma 3.1); +-inf or NaN where p or q
+ *             rounds to 1 (the weight itself stays finite).
+ * The truncation decision is taken as log k > log cap with log k = lp_train -
+ * lp_infer evaluated exactly; fp32 arithmetic is used where its error bound
+ * proves the answer and fp64 otherwise, so decisions equal those of an fp64
+ * evaluation.  Errors: CIS_ERR_INVALID_ARG for NULL required pointers, T < 0
+ * or parameters outside the ranges of cis_params_t.
+ */
+cis_status_t cis_weights(const float *lp_train, const float *lp_infer, const uint8_t *mask,
+                         int64_t T, const cis_params_t *params, float *w_out,
+                         uint8_t *trunc_out, float *eps_out, void *stream);
+
+/* Bytes of device workspace cis_loss_fwd_bwd needs for T tokens and
+ * vocabulary V.  Host only.  CIS_ERR_INVALID_ARG if bytes is NULL or T < 0. */
+cis_status_t cis_loss_workspace_size(int64_t T, int64_t V, size_t *bytes);
+
+/*
+ * The fused forward + backward token pass (Eq. 1 with the weight of
+ * Algorithm 1 / Table 8, the weight detached).
+ *   logits      device, [T, ld] of `dtype` (CIS_BF16 or CIS_F32).
+ *   ids         device int32 [T].
+ *   lp_infer    device float [T]: log q_t recorded by the inference engine.
+ *   lp_old      device float [T] or NULL: log p at the rollout snapshot.
+ *               NULL means the current parameters are the snapshot: the
+ *               weight is built from the current l_t (detached) and
+ *               rho = exp(l_t - stopgrad(l_t)) = 1 in value.
+ *   adv         device float [T]: advantage A_t.
+ *   mask        device uint8 [T] or NULL.
+ *   cu_seqlens  device int32 [B + 1] or NULL: response boundaries, needed for
+ *               CIS_AGG_SEQ_MEAN_TOKEN_MEAN (tokens outside every response
+ *               then get s_t = 0).  Must be non-decreasing with
+ *               cu_seqlens[B] <= T; not checked on the host.
+ *   params      host pointer.
+ *   dlogits     device, [T, ld_out] of `dlogits_dtype` (CIS_BF16 rounds to
+ *               nearest even, CIS_F32); every element j < V of every row is
+ *               written.  May not overlap the logits.
+ *   lp_out, w_out, trunc_out  device per-token outputs or NULL.
+ *   stats_out   device cis_stats_t* or NULL.
+ *   loss_out    device double [1] or NULL: the loss (also in stats_out).
+ *   workspace   device, >= cis_loss_workspace_size(T, V) bytes, 256-byte
+ *               aligned; its first int32 is the device status word, zeroed
+ *               by this call.
+ * Sums are deterministic: the same inputs give bit-identical outputs.
+ * Errors: CIS_ERR_INVALID_ARG for NULL required pointers, T < 0, V <= 0,
+ * ld < V, ld_out < V, bad parameters, a short or misaligned workspace, or
+ * CIS_AGG_SEQ_MEAN_TOKEN_MEAN without cu_seqlens; CIS_ERR_CUDA if a launch
+ * fails.
+ */
+cis_status_t cis_loss_fwd_bwd(const void *logits, int32_t dtype, int64_t T, int64_t V,
+                              int64_t ld, const int32_t *ids, const float *lp_infer,
+                              const float *lp_old, const float *adv, const uint8_t *mask,
+                              const int32_t *cu_seqlens, int64_t B,
+                              const cis_params_t *params, void *dlogits,
+                              int32_t dlogits_dtype, int64_t ld_out, float *lp_out,
+                              float *w_out, uint8_t *trunc_out, cis_stats_t *stats_out,
+                              double *loss_out, void *workspace, size_t workspace_bytes,
+                              void *stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* CIS_H */

@@ -1,0 +1,193 @@
+"""fp64 CPU oracle of the CIS token pass (arxiv 2609.32444).
+
+TEST INFRASTRUCTURE ONLY.  Only the test suite, ``__graft_entry__.smoke()`` and
+the CPU-baseline leg of ``bench.py`` may import this package.  The product
+library never imports it and shares no code with it.
+
+The arithmetic lives in ``cis_oracle.c`` (plain fp64 C, one row per host
+thread).  This module compiles it on first use with the host C compiler and
+marshals numpy arrays in and out.  Each function states the passage of the
+paper it follows.
+
+Pinned against the paper and mathematics (not against itself) by
+``tests/test_oracle_pins.py``: tiny-V brute force at 50 digits, shift
+invariance, normalisation, Lemma 3.1 (k = p + (1-p) e^eps from full inference
+logits), Lemma B.2, Corollary B.6, Eq. 5, the special cases lambda = 0 and
+lambda -> inf, the numbers the paper prints for lambda = 2.3, and central
+finite differences of the loss against its gradient.
+"""
+
+from __future__ import annotations
+
+import ctypes
+import os
+import subprocess
+import threading
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SRC = os.path.join(_HERE, "cis_oracle.c")
+_LIB_PATH = os.path.join(_HERE, "liboracle.so")
+_lock = threading.Lock()
+_lib = None
+
+MODE_CIS, MODE_TIS, MODE_EXACT, MODE_NONE = 0, 1, 2, 3
+AGG_TOKEN_MEAN, AGG_SEQ_MEAN = 0, 1
+F32, BF16 = 0, 1
+
+
+class OracleParams(ctypes.Structure):
+    _fields_ = [
+        ("mode", ctypes.c_int32),
+        ("agg", ctypes.c_int32),
+        ("lam", ctypes.c_double),
+        ("kappa", ctypes.c_double),
+        ("tis_cap", ctypes.c_double),
+        ("exact_lo", ctypes.c_double),
+        ("exact_hi", ctypes.c_double),
+        ("clip_low", ctypes.c_double),
+        ("clip_high", ctypes.c_double),
+    ]
+
+
+def params(mode=MODE_CIS, lam=2.3, kappa=5e-3, tis_cap=2.0, exact_lo=1e-6, exact_hi=1e6,
+           clip_low=0.2, clip_high=0.28, agg=AGG_TOKEN_MEAN) -> OracleParams:
+    """Hyper-parameters; defaults are the deployed values of App. C.1 / Table 8."""
+    return OracleParams(mode, agg, lam, kappa, tis_cap, exact_lo, exact_hi, clip_low, clip_high)
+
+
+def build(force: bool = False) -> str:
+    """Compile cis_oracle.c into liboracle.so (host C compiler, OpenMP)."""
+    with _lock:
+        if (not force and os.path.exists(_LIB_PATH)
+                and os.path.getmtime(_LIB_PATH) >= os.path.getmtime(_SRC)):
+            return _LIB_PATH
+        tmp = _LIB_PATH + f".tmp{os.getpid()}"
+        cmd = ["gcc", "-O2", "-std=c11", "-fPIC", "-shared", "-fopenmp", "-o", tmp, _SRC, "-lm"]
+        subprocess.run(cmd, check=True)
+        os.replace(tmp, _LIB_PATH)
+        return _LIB_PATH
+
+
+def _load():
+    global _lib
+    if _lib is None:
+        build()
+        lib = ctypes.CDLL(_LIB_PATH)
+        P = ctypes.c_void_p
+        i64, i32, dbl = ctypes.c_int64, ctypes.c_int32, ctypes.c_double
+        lib.oracle_token_logprobs.argtypes = [P, i32, i64, i64, i64, P, P, P, P, ctypes.c_int]
+        lib.oracle_token_logprobs.restype = ctypes.c_int
+        lib.oracle_weights.argtypes = [P, P, P, i64, ctypes.POINTER(OracleParams), P, P, P, P]
+        lib.oracle_weights.restype = None
+        lib.oracle_loss_scales.argtypes = [P, i64, P, i64, ctypes.c_int, P]
+        lib.oracle_loss_scales.restype = None
+        lib.oracle_loss_fwd_bwd.argtypes = [
+            P, i32, i64, i64, i64, P, P, P, P, P, P, i64, ctypes.POINTER(OracleParams), P,
+            P, i64, P, P, P, P, P, P, P, P, ctypes.c_int]
+        lib.oracle_loss_fwd_bwd.restype = ctypes.c_int
+        lib.oracle_max_threads.argtypes = []
+        lib.oracle_max_threads.restype = ctypes.c_int
+        _ = dbl
+        _lib = lib
+    return _lib
+
+
+def _ptr(a):
+    return None if a is None else a.ctypes.data_as(ctypes.c_void_p)
+
+
+def _logits_arg(logits):
+    """numpy float32 [T, ld] -> (array, F32); uint16 bf16 bit patterns -> (array, BF16)."""
+    a = np.ascontiguousarray(logits)
+    if a.dtype == np.float32:
+        return a, F32
+    if a.dtype == np.uint16:
+        return a, BF16
+    raise TypeError(f"oracle logits must be float32 or uint16 (bf16 bits), got {a.dtype}")
+
+
+def _opt(a, dtype):
+    return None if a is None else np.ascontiguousarray(a, dtype=dtype)
+
+
+def max_threads() -> int:
+    return int(_load().oracle_max_threads())
+
+
+def token_logprobs(logits, ids, V=None, mask=None, nthreads=0):
+    """log p_t = z_{t,y_t} - logsumexp(z_t) in fp64 (Sec. 2.1).  Returns (lp, lse, rc)."""
+    lib = _load()
+    a, dt = _logits_arg(logits)
+    T, ld = a.shape
+    V = ld if V is None else V
+    ids = np.ascontiguousarray(ids, dtype=np.int32)
+    mask = _opt(mask, np.uint8)
+    lp = np.zeros(T, np.float64)
+    lse = np.zeros(T, np.float64)
+    rc = lib.oracle_token_logprobs(_ptr(a), dt, T, V, ld, _ptr(ids), _ptr(mask), _ptr(lp),
+                                   _ptr(lse), nthreads)
+    return lp, lse, rc
+
+
+def weights(lp_w, lp_inf, P: OracleParams, mask=None):
+    """Algorithm 1 / Table 8 weights in fp64.  Returns (w, trunc, logk, eps)."""
+    lib = _load()
+    lp_w = np.ascontiguousarray(lp_w, dtype=np.float64)
+    lp_inf = np.ascontiguousarray(lp_inf, dtype=np.float64)
+    mask = _opt(mask, np.uint8)
+    T = lp_w.shape[0]
+    w = np.zeros(T, np.float64)
+    tr = np.zeros(T, np.uint8)
+    lk = np.zeros(T, np.float64)
+    eps = np.zeros(T, np.float64)
+    lib.oracle_weights(_ptr(lp_w), _ptr(lp_inf), _ptr(mask), T, ctypes.byref(P), _ptr(w),
+                       _ptr(tr), _ptr(lk), _ptr(eps))
+    return w, tr, lk, eps
+
+
+def loss_scales(T, mask=None, cu_seqlens=None, agg=AGG_TOKEN_MEAN):
+    """Per-token normaliser s_t (Algorithm 1's 1/n, or Eq. 1's 1/(G |y_i|))."""
+    lib = _load()
+    mask = _opt(mask, np.uint8)
+    cu = _opt(cu_seqlens, np.int32)
+    B = 0 if cu is None else cu.shape[0] - 1
+    s = np.zeros(T, np.float64)
+    lib.oracle_loss_scales(_ptr(mask), T, _ptr(cu), B, agg, _ptr(s))
+    return s
+
+
+def loss_fwd_bwd(logits, ids, lp_inf, adv, P: OracleParams, V=None, lp_old=None, mask=None,
+                 cu_seqlens=None, w_fixed=None, rows=None, want_dz=True, nthreads=0):
+    """Weighted PPO-clipped token loss (Eq. 1, Algorithm 1) and d loss / d logits, fp64.
+
+    ``rows``: indices of the rows whose dz is returned (None = all rows).
+    Returns a dict with loss, terms, lp, lse, w, trunc, c, dz ([len(rows), V] or
+    [T, V]) and rc (0, or -1 when a valid row has an out-of-range id).
+    """
+    lib = _load()
+    a, dt = _logits_arg(logits)
+    T, ld = a.shape
+    V = ld if V is None else V
+    ids = np.ascontiguousarray(ids, dtype=np.int32)
+    lp_inf = np.ascontiguousarray(lp_inf, dtype=np.float64)
+    adv = np.ascontiguousarray(adv, dtype=np.float64)
+    lp_old = _opt(lp_old, np.float64)
+    mask = _opt(mask, np.uint8)
+    cu = _opt(cu_seqlens, np.int32)
+    B = 0 if cu is None else cu.shape[0] - 1
+    w_fixed = _opt(w_fixed, np.float64)
+    rows_a = None if rows is None else np.ascontiguousarray(rows, dtype=np.int64)
+    nrows = T if rows_a is None else rows_a.shape[0]
+    dz = np.zeros((nrows, V), np.float64) if want_dz else None
+    out = {k: np.zeros(T, np.float64) for k in ("lp", "lse", "w", "terms", "c")}
+    trunc = np.zeros(T, np.uint8)
+    loss = ctypes.c_double(0.0)
+    rc = lib.oracle_loss_fwd_bwd(
+        _ptr(a), dt, T, V, ld, _ptr(ids), _ptr(lp_inf), _ptr(lp_old), _ptr(adv), _ptr(mask),
+        _ptr(cu), B, ctypes.byref(P), _ptr(w_fixed), _ptr(rows_a), nrows if rows_a is not None
+        else 0, _ptr(dz), _ptr(out["lp"]), _ptr(out["lse"]), _ptr(out["w"]), _ptr(trunc),
+        _ptr(out["terms"]), _ptr(out["c"]), ctypes.byref(loss), nthreads)
+    out.update(loss=loss.value, trunc=trunc, dz=dz, rc=rc)
+    return out

@@ -1,0 +1,411 @@
+/*
+ * cis_oracle.c -- fp64 CPU oracle for the calibrated-importance-sampling (CIS)
+ * token loss of arxiv 2609.32444.
+ *
+ * TEST INFRASTRUCTURE ONLY.  This file is the plain, slow, obviously correct
+ * statement of what the GPU path computes.  Only the test suite, the smoke
+ * check and the CPU-baseline leg of the benchmark may load it.  It shares no
+ * header, helper, table or constant generator with the CUDA library, and the
+ * CUDA library never calls it.
+ *
+ * Every quantity is computed in IEEE double precision with plain loops over
+ * the vocabulary: an exact maximum, then a plain sum of exp(z - max) -- no
+ * online rescaling, no blocking, no fusion.  Rows are independent, so rows
+ * are spread over host threads with OpenMP; each row is still computed by a
+ * single thread in index order, so results do not depend on the thread count.
+ *
+ * Passages followed (section / equation / algorithm of the paper):
+ *   - Sec. 2.1 and Sec. 3.1: p_t = softmax(z)_{y_t}, the probability the
+ *     training engine gives the sampled token; log p_t = z_y - logsumexp(z).
+ *   - Eq. 1: token-level GRPO surrogate with the PPO clip and the mismatch
+ *     weight k_t; normaliser (1/G) sum_i 1/|y_i|.
+ *   - Algorithm 1 (Sec. 3.3): p = exp(l_train), k = exp(l_train - l_infer),
+ *     phi = max(1 - p, kappa), f = min{k, 1 + lambda*phi}; the estimate is
+ *     (1/n) sum stopgrad(f_m) l'_m.
+ *   - Table 8 (App. C.1): the other weight operators (exact ratio clamped to
+ *     [1e-6, 1e6], TIS min(k, C), no correction) and their defaults.
+ *   - Lemma 3.1 / Lemma B.1: eps_t = logit p_t - logit q_t.
+ *
+ * Readings where the paper is silent (each also listed in the design notes):
+ *   - the truncation flag is "k > cap", decided in fp64 in the log domain:
+ *     log k = l_w - l_inf (exact in fp64 for fp32 inputs) against log(cap);
+ *   - 1 - p is evaluated as -expm1(log p);
+ *   - the loss is the negated objective, so d loss / d z = c (softmax - onehot);
+ *   - in min(rho*A, clip(rho)*A) a tie takes the unclipped branch, so the
+ *     gradient flows at rho = 1 +- c exactly.
+ */
+#include <math.h>
+#include <stdint.h>
+#include <stdlib.h>
+#include <string.h>
+#ifdef _OPENMP
+#include <omp.h>
+#endif
+
+/* Weight operators (Table 8 of the paper, plus CIS of Algorithm 1). */
+enum {
+    OR_MODE_CIS = 0,   /* min{k, 1 + lambda*max(1-p, kappa)}      Algorithm 1 */
+    OR_MODE_TIS = 1,   /* min(k, C)                                Table 8    */
+    OR_MODE_EXACT = 2, /* k clamped to [lo, hi]                    Table 8    */
+    OR_MODE_NONE = 3   /* 1                                        Table 8    */
+};
+
+enum { OR_AGG_TOKEN_MEAN = 0, OR_AGG_SEQ_MEAN = 1 };
+
+/* Hyper-parameters, all in double precision. */
+typedef struct {
+    int32_t mode;
+    int32_t agg;
+    double lambda;    /* CIS threshold on e^eps, Eq. 4                 */
+    double kappa;     /* floor on 1 - p, Algorithm 1                   */
+    double tis_cap;   /* C of TIS                                      */
+    double exact_lo;  /* clamp of the exact ratio                      */
+    double exact_hi;
+    double clip_low;  /* PPO clip range [1 - c_low, 1 + c_high], Eq. 1 */
+    double clip_high;
+} oracle_params_t;
+
+/* bf16 is the top half of an IEEE binary32; the upcast is exact. */
+static double bf16_to_double(uint16_t h)
+{
+    uint32_t u = ((uint32_t)h) << 16;
+    float f;
+    memcpy(&f, &u, sizeof f);
+    return (double)f;
+}
+
+static double logit_at(const void *logits, int dtype, int64_t ld, int64_t t, int64_t j)
+{
+    if (dtype == 0)
+        return (double)((const float *)logits)[t * ld + j];
+    return bf16_to_double(((const uint16_t *)logits)[t * ld + j]);
+}
+
+static int row_valid(const uint8_t *mask, int64_t t)
+{
+    return mask == NULL || mask[t] != 0;
+}
+
+/*
+ * logsumexp of one row, by its definition: M = max_j z_j, then
+ * lse = M + log(sum_j exp(z_j - M)).  Sec. 2.1 / 3.1 (softmax of the logits).
+ */
+static double row_lse(const void *logits, int dtype, int64_t ld, int64_t t, int64_t V)
+{
+    double M = -INFINITY;
+    int any_nan = 0;
+    for (int64_t j = 0; j < V; ++j) {
+        double z = logit_at(logits, dtype, ld, t, j);
+        if (isnan(z))
+            any_nan = 1;
+        if (z > M)
+            M = z;
+    }
+    if (any_nan)
+        return NAN;
+    if (M == -INFINITY)
+        return -INFINITY;
+    double S = 0.0;
+    for (int64_t j = 0; j < V; ++j)
+        S += exp(logit_at(logits, dtype, ld, t, j) - M);
+    return M + log(S);
+}
+
+static void set_threads(int nthreads)
+{
+#ifdef _OPENMP
+    if (nthreads > 0)
+        omp_set_num_threads(nthreads);
+#else
+    (void)nthreads;
+#endif
+}
+
+int oracle_max_threads(void)
+{
+#ifdef _OPENMP
+    return omp_get_max_threads();
+#else
+    return 1;
+#endif
+}
+
+/*
+ * Sampled-token log-probabilities: lp_t = z_{t,y_t} - lse_t, i.e. log p_t with
+ * p_t = softmax(z_t)_{y_t} (Sec. 2.1, Sec. 3.1).  Masked rows are not read and
+ * get lp = lse = 0.  Returns 0, or -1 if a valid row has an id outside [0, V)
+ * (that row then gets NaN).
+ */
+int oracle_token_logprobs(const void *logits, int dtype, int64_t T, int64_t V, int64_t ld,
+                          const int32_t *ids, const uint8_t *mask, double *lp_out,
+                          double *lse_out, int nthreads)
+{
+    int bad = 0;
+    set_threads(nthreads);
+#pragma omp parallel for schedule(dynamic, 4) reduction(| : bad)
+    for (int64_t t = 0; t < T; ++t) {
+        double lp = 0.0, lse = 0.0;
+        if (row_valid(mask, t)) {
+            int32_t y = ids[t];
+            if (y < 0 || (int64_t)y >= V) {
+                bad = 1;
+                lp = NAN;
+                lse = NAN;
+            } else {
+                lse = row_lse(logits, dtype, ld, t, V);
+                lp = logit_at(logits, dtype, ld, t, y) - lse;
+            }
+        }
+        lp_out[t] = lp;
+        if (lse_out)
+            lse_out[t] = lse;
+    }
+    return bad ? -1 : 0;
+}
+
+/*
+ * One token's weight, Algorithm 1 and Table 8.
+ *   lw   : log p used by the weight (training side), double
+ *   linf : log q (inference side, the raw sampling-step value), double
+ * Outputs the weight, the truncation flag, log k and eps.
+ */
+static void token_weight(double lw, double linf, const oracle_params_t *P, double *w,
+                         int *trunc, double *logk_out, double *eps_out)
+{
+    /* Algorithm 1: p <- exp(l_train), k <- exp(l_train - l_infer).
+     * 1 - p is evaluated as -expm1(l_train), the same number without the
+     * cancellation of 1 - exp(l) when p is close to 1. */
+    double logk = lw - linf;
+    double k = exp(logk);
+    double one_minus_p = -expm1(lw);
+    double wt = 1.0;
+    int tr = 0;
+    switch (P->mode) {
+    case OR_MODE_CIS: {
+        /* phi <- max(1 - p, kappa);  f <- min{k, 1 + lambda*phi}. */
+        double phi = one_minus_p > P->kappa ? one_minus_p : P->kappa;
+        double cap = 1.0 + P->lambda * phi;
+        wt = k < cap ? k : cap;
+        tr = logk > log1p(P->lambda * phi);
+        break;
+    }
+    case OR_MODE_TIS: {
+        /* Table 8: min(k, C). */
+        double cap = P->tis_cap;
+        wt = k < cap ? k : cap;
+        tr = logk > log(cap);
+        break;
+    }
+    case OR_MODE_EXACT: {
+        /* Table 8: k, clamped to [lo, hi]. */
+        wt = k;
+        if (wt > P->exact_hi)
+            wt = P->exact_hi;
+        if (wt < P->exact_lo)
+            wt = P->exact_lo;
+        tr = logk > log(P->exact_hi) || logk < log(P->exact_lo);
+        break;
+    }
+    default: /* OR_MODE_NONE: weight 1. */
+        wt = 1.0;
+        tr = 0;
+        break;
+    }
+    *w = wt;
+    *trunc = tr;
+    if (logk_out)
+        *logk_out = logk;
+    if (eps_out) {
+        /* Lemma 3.1: eps = logit p - logit q
+         *               = (log p - log(1-p)) - (log q - log(1-q)). */
+        double one_minus_q = -expm1(linf);
+        *eps_out = (lw - log(one_minus_p)) - (linf - log(one_minus_q));
+    }
+}
+
+/*
+ * Elementwise weights for T tokens (Algorithm 1 / Table 8).  Masked tokens get
+ * w = 0, trunc = 0, logk = eps = 0.
+ */
+void oracle_weights(const double *lp_w, const double *lp_inf, const uint8_t *mask, int64_t T,
+                    const oracle_params_t *P, double *w_out, uint8_t *trunc_out,
+                    double *logk_out, double *eps_out)
+{
+    for (int64_t t = 0; t < T; ++t) {
+        double w = 0.0, lk = 0.0, e = 0.0;
+        int tr = 0;
+        if (row_valid(mask, t))
+            token_weight(lp_w[t], lp_inf[t], P, &w, &tr, &lk, &e);
+        w_out[t] = w;
+        if (trunc_out)
+            trunc_out[t] = (uint8_t)tr;
+        if (logk_out)
+            logk_out[t] = lk;
+        if (eps_out)
+            eps_out[t] = e;
+    }
+}
+
+/*
+ * Per-token loss scale s_t.
+ *   token mean (Algorithm 1): s_t = m_t / n, n = number of valid tokens;
+ *   sequence mean (Eq. 1):    s_t = m_t / (G * |y_i|) for token t of response
+ *                             i, |y_i| = valid tokens of i, G = responses with
+ *                             at least one valid token.  Tokens outside every
+ *                             response get 0.
+ */
+void oracle_loss_scales(const uint8_t *mask, int64_t T, const int32_t *cu_seqlens, int64_t B,
+                        int agg, double *s_out)
+{
+    if (agg == OR_AGG_SEQ_MEAN && cu_seqlens != NULL) {
+        int64_t G = 0;
+        for (int64_t i = 0; i < B; ++i) {
+            int64_t n = 0;
+            for (int64_t t = cu_seqlens[i]; t < cu_seqlens[i + 1]; ++t)
+                n += row_valid(mask, t);
+            G += n > 0;
+        }
+        for (int64_t t = 0; t < T; ++t)
+            s_out[t] = 0.0;
+        for (int64_t i = 0; i < B; ++i) {
+            int64_t n = 0;
+            for (int64_t t = cu_seqlens[i]; t < cu_seqlens[i + 1]; ++t)
+                n += row_valid(mask, t);
+            for (int64_t t = cu_seqlens[i]; t < cu_seqlens[i + 1]; ++t)
+                s_out[t] = row_valid(mask, t) ? 1.0 / ((double)G * (double)n) : 0.0;
+        }
+        return;
+    }
+    int64_t n = 0;
+    for (int64_t t = 0; t < T; ++t)
+        n += row_valid(mask, t);
+    for (int64_t t = 0; t < T; ++t)
+        s_out[t] = (n > 0 && row_valid(mask, t)) ? 1.0 / (double)n : 0.0;
+}
+
+/*
+ * The weighted policy-gradient token loss and its gradient with respect to
+ * the logits.
+ *
+ *   rho_t = exp(l_t - l_old,t)        (update ratio, Eq. 1; = 1 in value when
+ *                                      no l_old is given, gradient still flows)
+ *   J_t   = w_t * min(rho_t A_t, clip(rho_t, 1-c_low, 1+c_high) A_t)   (Eq. 1)
+ *   loss  = -sum_t s_t J_t
+ *   w_t   = stopgrad weight of Algorithm 1 / Table 8, from l_old if given,
+ *           else from the current l_t (detached)
+ *   d loss / d z_tj = c_t (softmax_j - [j == y_t]),
+ *   c_t   = s_t w_t A_t rho_t g_t, g_t = 1 if the unclipped branch is taken.
+ *
+ * Inputs in double (the Python wrapper upcasts fp32 exactly).  lp_old, w_fixed
+ * may be NULL.  w_fixed replaces the computed weights (used to freeze them for
+ * finite differences).  dz is written for the rows listed in `rows` (nrows of
+ * them, dz_out is [nrows, V]); rows == NULL means every row (dz_out [T, V]).
+ * Per-token outputs (lp, lse, w, trunc, loss_terms, c) are for all T rows.
+ * Returns 0, or -1 if a valid row has an out-of-range id.
+ */
+int oracle_loss_fwd_bwd(const void *logits, int dtype, int64_t T, int64_t V, int64_t ld,
+                        const int32_t *ids, const double *lp_inf, const double *lp_old,
+                        const double *adv, const uint8_t *mask, const int32_t *cu_seqlens,
+                        int64_t B, const oracle_params_t *P, const double *w_fixed,
+                        const int64_t *rows, int64_t nrows, double *dz_out, double *lp_out,
+                        double *lse_out, double *w_out, uint8_t *trunc_out,
+                        double *loss_terms, double *c_out, double *loss_out, int nthreads)
+{
+    size_t nT = (size_t)(T > 0 ? T : 1);
+    double *s = (double *)malloc(sizeof(double) * nT);
+    double *lse = (double *)malloc(sizeof(double) * nT);
+    double *cc = (double *)malloc(sizeof(double) * nT);
+    double *terms = (double *)malloc(sizeof(double) * nT);
+    if (!s || !lse || !cc || !terms) {
+        free(s);
+        free(lse);
+        free(cc);
+        free(terms);
+        return -2;
+    }
+    oracle_loss_scales(mask, T, cu_seqlens, B, P->agg, s);
+    int bad = 0;
+    set_threads(nthreads);
+#pragma omp parallel for schedule(dynamic, 4) reduction(| : bad)
+    for (int64_t t = 0; t < T; ++t) {
+        double lp = 0.0, ls = 0.0, w = 0.0, term = 0.0, c = 0.0;
+        int tr = 0;
+        if (row_valid(mask, t)) {
+            int32_t y = ids[t];
+            if (y < 0 || (int64_t)y >= V) {
+                bad = 1;
+                lp = NAN;
+                ls = NAN;
+                term = NAN;
+            } else {
+                ls = row_lse(logits, dtype, ld, t, V);
+                lp = logit_at(logits, dtype, ld, t, y) - ls;
+                double lw = lp_old ? lp_old[t] : lp;
+                double lk;
+                token_weight(lw, lp_inf[t], P, &w, &tr, &lk, NULL);
+                if (w_fixed)
+                    w = w_fixed[t];
+                /* Eq. 1: rho = pi_theta / p_old, clipped to [1-c_low, 1+c_high]. */
+                double rho = lp_old ? exp(lp - lp_old[t]) : 1.0;
+                double A = adv[t];
+                double rho_c = rho;
+                if (rho_c < 1.0 - P->clip_low)
+                    rho_c = 1.0 - P->clip_low;
+                if (rho_c > 1.0 + P->clip_high)
+                    rho_c = 1.0 + P->clip_high;
+                double unclipped = rho * A;
+                double clipped = rho_c * A;
+                int g = unclipped <= clipped; /* the min takes the unclipped branch */
+                double obj = g ? unclipped : clipped;
+                term = -s[t] * w * obj;
+                c = s[t] * w * A * rho * (double)g;
+            }
+        }
+        lse[t] = ls;
+        cc[t] = c;
+        terms[t] = term;
+        lp_out[t] = lp;
+        if (w_out)
+            w_out[t] = w;
+        if (trunc_out)
+            trunc_out[t] = (uint8_t)tr;
+    }
+    /* loss = -sum_t s_t J_t, summed in index order. */
+    double loss = 0.0;
+    for (int64_t t = 0; t < T; ++t)
+        loss += terms[t];
+    if (loss_out)
+        *loss_out = loss;
+    if (loss_terms)
+        memcpy(loss_terms, terms, sizeof(double) * (size_t)T);
+    if (lse_out)
+        memcpy(lse_out, lse, sizeof(double) * (size_t)T);
+    if (c_out)
+        memcpy(c_out, cc, sizeof(double) * (size_t)T);
+
+    /* d loss / d z_tj = c_t (softmax_tj - [j == y_t]) for the requested rows. */
+    if (dz_out) {
+        int64_t nr = rows ? nrows : T;
+#pragma omp parallel for schedule(dynamic, 1)
+        for (int64_t r = 0; r < nr; ++r) {
+            int64_t t = rows ? rows[r] : r;
+            double *out = dz_out + r * V;
+            int valid = t >= 0 && t < T && row_valid(mask, t);
+            int32_t y = valid ? ids[t] : -1;
+            if (!valid || y < 0 || (int64_t)y >= V) {
+                for (int64_t j = 0; j < V; ++j)
+                    out[j] = 0.0;
+                continue;
+            }
+            for (int64_t j = 0; j < V; ++j) {
+                double sm = exp(logit_at(logits, dtype, ld, t, j) - lse[t]);
+                out[j] = cc[t] * (sm - (j == (int64_t)y ? 1.0 : 0.0));
+            }
+        }
+    }
+    free(s);
+    free(lse);
+    free(cc);
+    free(terms);
+    return bad ? -1 : 0;
+}

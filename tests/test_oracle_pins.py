@@ -1,0 +1,395 @@
+"""Pins of the fp64 oracle against what the paper and mathematics fix.
+
+None of these compares the oracle with itself: each check is a closed form, a
+special case that reduces to a textbook quantity, an identity the paper
+proves, a number the paper prints (tests/golden/paper_values.json), brute
+force at 50 digits, or central finite differences of the loss.
+"""
+import json
+import math
+import os
+
+import numpy as np
+import pytest
+
+import oracle
+
+mpmath = pytest.importorskip("mpmath")
+
+GOLDEN = json.load(open(os.path.join(os.path.dirname(__file__), "golden", "paper_values.json")))
+
+
+def _rng(seed):
+    return np.random.default_rng(seed)
+
+
+# ---------------------------------------------------------------- log-softmax
+@pytest.mark.parametrize("V", [1, 2, 5, 8])
+def test_logprob_tiny_v_matches_50_digit_brute_force(V):
+    """log p_y = log(e^{z_y} / sum_j e^{z_j}) (Sec. 2.1), evaluated at 50 digits."""
+    rng = _rng(V)
+    T = 16
+    z = (rng.standard_normal((T, V)) * 6).astype(np.float32)
+    ids = rng.integers(0, V, T).astype(np.int32)
+    lp, lse, rc = oracle.token_logprobs(z, ids)
+    assert rc == 0
+    mpmath.mp.dps = 50
+    for t in range(T):
+        num = mpmath.e ** mpmath.mpf(float(z[t, ids[t]]))
+        den = mpmath.fsum(mpmath.e ** mpmath.mpf(float(v)) for v in z[t])
+        ref = float(mpmath.log(num / den))
+        assert abs(lp[t] - ref) <= 1e-13 * max(1.0, abs(ref))
+        assert abs(lse[t] - float(mpmath.log(den))) <= 1e-13 * max(1.0, abs(float(mpmath.log(den))))
+
+
+def test_logprob_shift_invariance():
+    """softmax(z + c) = softmax(z): log p is unchanged by a constant shift."""
+    rng = _rng(1)
+    z = (rng.integers(-256, 256, (8, 300)) / 64.0).astype(np.float32)
+    ids = rng.integers(0, 300, 8).astype(np.int32)
+    lp0, _, _ = oracle.token_logprobs(z, ids)
+    lp1, _, _ = oracle.token_logprobs(z + np.float32(3.0), ids)  # exact in fp32
+    np.testing.assert_allclose(lp0, lp1, rtol=0, atol=1e-12)
+
+
+def test_logsumexp_normalises():
+    """sum_j exp(z_j - lse) = 1 for every row (the softmax is a distribution)."""
+    rng = _rng(2)
+    z = (rng.standard_normal((32, 1024)) * 4).astype(np.float32)
+    ids = np.zeros(32, np.int32)
+    _, lse, _ = oracle.token_logprobs(z, ids)
+    tot = np.exp(z.astype(np.float64) - lse[:, None]).sum(axis=1)
+    np.testing.assert_allclose(tot, 1.0, rtol=0, atol=1e-12)
+
+
+def test_bf16_decoding_matches_library_conversion():
+    """bf16 rows must give the same log p as the same values given as fp32."""
+    torch = pytest.importorskip("torch")
+    rng = _rng(3)
+    zf = torch.from_numpy((rng.standard_normal((16, 77)) * 5).astype(np.float32))
+    zb = zf.to(torch.bfloat16)
+    bits = zb.view(torch.int16).numpy().view(np.uint16)
+    ids = rng.integers(0, 77, 16).astype(np.int32)
+    lp_b, _, _ = oracle.token_logprobs(bits, ids)
+    lp_f, _, _ = oracle.token_logprobs(zb.float().numpy(), ids)
+    np.testing.assert_array_equal(lp_b, lp_f)
+
+
+def test_minus_inf_logits_and_masked_rows():
+    """-inf logits contribute e^-inf = 0; masked rows are skipped (lp = 0)."""
+    z = np.array([[0.0, -np.inf, math.log(3.0)], [1.0, 2.0, 3.0]], np.float32)
+    ids = np.array([0, 2], np.int32)
+    lp, _, rc = oracle.token_logprobs(z, ids, mask=np.array([1, 0], np.uint8))
+    assert rc == 0
+    ref = -math.log(1.0 + math.exp(float(z[0, 2])))  # e^0 / (e^0 + e^-inf + e^{z_2})
+    assert abs(lp[0] - ref) < 1e-15
+    assert lp[1] == 0.0
+
+
+def test_bad_token_id_is_reported():
+    z = np.zeros((2, 4), np.float32)
+    lp, _, rc = oracle.token_logprobs(z, np.array([0, 4], np.int32))
+    assert rc == -1 and math.isnan(lp[1]) and lp[0] == pytest.approx(-math.log(4))
+
+
+# ---------------------------------------------------------------- weights
+def _inference_pair(rng, V, n, scale=2.0, dscale=0.5):
+    """Training logits z, inference logits z + delta, and the sampled ids."""
+    z = rng.standard_normal((n, V)) * scale
+    delta = rng.standard_normal((n, V)) * dscale
+    ids = rng.integers(0, V, n)
+    return z, delta, ids
+
+
+def _log_softmax(x):
+    m = x.max(axis=1, keepdims=True)
+    return x - m - np.log(np.exp(x - m).sum(axis=1, keepdims=True))
+
+
+def test_lemma_3_1_ratio_displacement_identity():
+    """Lemma 3.1 / B.1: with eps := -delta_y + log sum_{j!=y} w_j e^{delta_j},
+    w_j = e^{z_j} / sum_{j'!=y} e^{z_j'}, one has k = p + (1-p) e^eps and
+    eps = logit p - logit q.  eps is computed here from the full logit
+    vectors by its definition; the oracle only sees log p and log q."""
+    rng = _rng(10)
+    n, V = 200, 50
+    z, delta, ids = _inference_pair(rng, V, n)
+    lp = _log_softmax(z)[np.arange(n), ids]
+    lq = _log_softmax(z + delta)[np.arange(n), ids]
+    _, _, logk, eps = oracle.weights(lp, lq, oracle.params(mode=oracle.MODE_EXACT, exact_lo=0,
+                                                           exact_hi=np.inf))
+    eps_def = np.empty(n)
+    for t in range(n):
+        y = ids[t]
+        others = np.arange(V) != y
+        wj = np.exp(z[t, others]) / np.exp(z[t, others]).sum()
+        eps_def[t] = -delta[t, y] + math.log(float((wj * np.exp(delta[t, others])).sum()))
+    np.testing.assert_allclose(eps, eps_def, rtol=1e-9, atol=1e-9)
+    p = np.exp(lp)
+    np.testing.assert_allclose(np.exp(logk), p + (1 - p) * np.exp(eps_def), rtol=1e-9)
+
+
+def test_ratio_is_one_without_perturbation_and_gauge_invariant():
+    """delta = 0, or delta = const (the gauge freedom of App. A.1), gives
+    q = p, k = 1, w = 1 in every mode and no truncation."""
+    rng = _rng(11)
+    n, V = 64, 40
+    z, _, ids = _inference_pair(rng, V, n)
+    lp = _log_softmax(z)[np.arange(n), ids]
+    lq = _log_softmax(z + 7.25)[np.arange(n), ids]
+    for mode in (oracle.MODE_CIS, oracle.MODE_TIS, oracle.MODE_EXACT, oracle.MODE_NONE):
+        w, tr, logk, _ = oracle.weights(lp, lq, oracle.params(mode=mode))
+        np.testing.assert_allclose(logk, 0.0, atol=1e-13)
+        np.testing.assert_allclose(w, 1.0, rtol=1e-12)
+        assert not tr.any()
+
+
+def _random_lw_linf(rng, n):
+    lw = -np.exp(rng.uniform(np.log(1e-7), np.log(12.0), n))  # log p over many decades
+    linf = lw + rng.standard_normal(n) * 1.5
+    linf = np.minimum(linf, -1e-9)
+    return lw, linf
+
+
+def test_lambda_zero_is_tis_with_cap_one():
+    """lambda = 0 gives f = min(k, 1), i.e. TIS with C = 1 (Sec. 4.3/4.4)."""
+    assert GOLDEN["lambda_zero_is_tis_c1"]["value"]
+    rng = _rng(12)
+    lw, linf = _random_lw_linf(rng, 2000)
+    w, tr, _, _ = oracle.weights(lw, linf, oracle.params(lam=0.0))
+    k = np.exp(lw - linf)
+    np.testing.assert_allclose(w, np.minimum(k, 1.0), rtol=1e-14)
+    np.testing.assert_array_equal(tr.astype(bool), lw - linf > 0)
+
+
+def test_lambda_to_infinity_is_exact_ratio():
+    """lambda -> inf recovers the exact ratio (Sec. 3.3, after Theorem 3.3)."""
+    assert GOLDEN["lambda_inf_is_exact"]["value"]
+    rng = _rng(13)
+    lw, linf = _random_lw_linf(rng, 2000)
+    w, tr, _, _ = oracle.weights(lw, linf, oracle.params(lam=1e300))
+    np.testing.assert_allclose(w, np.exp(lw - linf), rtol=1e-14)
+    assert not tr.any()
+
+
+def _cap(lw, lam=2.3, kappa=5e-3):
+    """The CIS cap as the weight of a token with an enormous ratio."""
+    lw = np.asarray(lw, np.float64)
+    w, tr, _, _ = oracle.weights(lw, lw - 800.0, oracle.params(lam=lam, kappa=kappa))
+    assert tr.all()
+    return w
+
+
+def test_cap_monotone_in_confidence_and_floor_value():
+    """cap(p) = 1 + lambda max(1-p, kappa) is non-increasing in p and equals
+    1 + lambda*kappa below the floor; the paper prints that value as ~1.01."""
+    p = np.linspace(1e-6, 1 - 1e-9, 20001)
+    caps = _cap(np.log(p))
+    assert np.all(np.diff(caps) <= 1e-15)
+    lam = GOLDEN["lambda_default"]["value"]
+    kap = GOLDEN["kappa_default"]["value"]
+    below = caps[(1 - p) < kap]
+    np.testing.assert_allclose(below, 1 + lam * kap, rtol=1e-15)
+    g = GOLDEN["cap_below_floor"]
+    assert round(float(below[0]), g["decimals"]) == g["value"]
+    # above the floor the cap follows 1 + lambda (1 - p) (Eq. 4)
+    above = (1 - p) > kap
+    np.testing.assert_allclose(caps[above], 1 + lam * (1 - p[above]), rtol=1e-12)
+
+
+def test_cis_cap_looser_than_tis2_below_printed_confidence():
+    """The CIS cap exceeds C = 2 exactly when p < 1 - 1/lambda; the paper
+    prints the crossing as p = 0.565 (Sec. 4.3)."""
+    g = GOLDEN["cis_looser_than_tis2_below_p"]
+    p = np.linspace(0.4, 0.7, 300001)
+    caps = _cap(np.log(p))
+    crossing = p[np.argmax(caps <= 2.0)]
+    assert round(float(crossing), g["decimals"]) == g["value"]
+    assert abs(crossing - (1 - 1 / 2.3)) < 2e-6
+
+
+def test_corollary_b6_floor_ordering():
+    """Corollary B.6: f_lambda <= f_{lambda,kappa} <= k and f_{lambda,kappa} <= 1 + lambda."""
+    rng = _rng(14)
+    lw, linf = _random_lw_linf(rng, 5000)
+    k = np.exp(lw - linf)
+    for lam in (0.0, 0.5, 2.3, 10.0):
+        for kap in (1e-3, 5e-3, 0.1, 1.0):
+            f0, _, _, _ = oracle.weights(lw, linf, oracle.params(lam=lam, kappa=0.0))
+            fk, _, _, _ = oracle.weights(lw, linf, oracle.params(lam=lam, kappa=kap))
+            assert np.all(f0 <= fk * (1 + 1e-15))
+            assert np.all(fk <= k * (1 + 1e-15))
+            assert np.all(fk <= (1 + lam) * (1 + 1e-15))
+
+
+def test_lemma_b2_truncated_excess_and_one_sidedness():
+    """Lemma B.2: k - f_lambda = (1-p)(e^eps - 1 - lambda)_+, and eps <= 0
+    implies p < k <= 1 (eps = logit p - logit q)."""
+    rng = _rng(15)
+    lw, linf = _random_lw_linf(rng, 5000)
+    p = np.exp(lw)
+    # logit p - logit q written out from the two probabilities
+    eps = (lw - np.log(-np.expm1(lw))) - (linf - np.log(-np.expm1(linf)))
+    k = np.exp(lw - linf)
+    for lam in (0.0, 1.0, 2.3):
+        f, _, _, _ = oracle.weights(lw, linf, oracle.params(lam=lam, kappa=0.0))
+        excess = (1 - p) * np.maximum(np.exp(eps) - 1 - lam, 0.0)
+        assert np.all(np.abs((k - f) - excess) <= 1e-8 * np.abs(excess) + 1e-12 * np.maximum(k, 1))
+    neg = eps <= 0
+    assert np.all(k[neg] <= 1 + 1e-15) and np.all(k[neg] > p[neg])
+
+
+def test_eq5_fixed_cap_in_displacement_coordinate():
+    """Eq. 5 / Lemma B.2: k <= C  <=>  e^eps <= 1 + (C-1)/(1-p)."""
+    rng = _rng(16)
+    lw, linf = _random_lw_linf(rng, 5000)
+    p = np.exp(lw)
+    eps = (lw - np.log(-np.expm1(lw))) - (linf - np.log(-np.expm1(linf)))
+    for C in (1.0, 1.13, 2.0, 5.0):
+        _, tr, _, _ = oracle.weights(lw, linf, oracle.params(mode=oracle.MODE_TIS, tis_cap=C))
+        rhs = np.exp(eps) <= 1 + (C - 1) / (1 - p)
+        lk = lw - linf
+        clear = np.abs(lk - math.log(C)) > 1e-9  # stay off exact ties
+        np.testing.assert_array_equal((tr == 0)[clear], rhs[clear])
+
+
+def test_exact_ratio_clamp_and_tis_defaults():
+    """Table 8: exact ratio clamped to [1e-6, 1e6]; TIS cap C = 2."""
+    lo, hi = GOLDEN["exact_clamp"]["value"]
+    lw = np.array([-1.0, -1.0, -1.0, -0.1])
+    linf = np.array([-30.0, -1.0 + 1e-3, 40.0, -0.1 - math.log(3.0)])
+    w, tr, _, _ = oracle.weights(lw, linf, oracle.params(mode=oracle.MODE_EXACT))
+    assert w[0] == hi and tr[0] == 1
+    assert w[1] == pytest.approx(math.exp(-1e-3)) and tr[1] == 0
+    assert w[2] == lo and tr[2] == 1
+    w, tr, _, _ = oracle.weights(lw, linf, oracle.params(mode=oracle.MODE_TIS))
+    assert w[3] == GOLDEN["tis_cap_default"]["value"] and tr[3] == 1
+
+
+def test_calibration_identity_by_brute_force():
+    """E_{y~q}[k_y] = sum_j q_j p_j / q_j = 1 per position (App. C.4), with
+    p_j from the oracle's log-softmax over every possible sampled token."""
+    rng = _rng(17)
+    V = 64
+    for _ in range(5):
+        z = (rng.standard_normal((1, V)) * 3).astype(np.float32)
+        delta = rng.standard_normal(V) * 0.7
+        zz = np.repeat(z, V, axis=0)
+        lp, _, _ = oracle.token_logprobs(zz, np.arange(V, dtype=np.int32))
+        lq = _log_softmax((z.astype(np.float64) + delta))[0]
+        _, _, logk, _ = oracle.weights(lp, lq, oracle.params(mode=oracle.MODE_NONE))
+        assert abs(float((np.exp(lq) * np.exp(logk)).sum()) - 1.0) < 1e-13
+
+
+# ---------------------------------------------------------------- normaliser
+def test_loss_scales_token_and_sequence_mean():
+    """Algorithm 1 averages over the n tokens; Eq. 1 averages each response
+    over its |y_i| tokens and then over the G responses."""
+    mask = np.array([1, 1, 1, 1, 1, 0, 1], np.uint8)
+    s = oracle.loss_scales(7, mask)
+    np.testing.assert_allclose(s, [1 / 6] * 5 + [0] + [1 / 6])
+    cu = np.array([0, 1, 6], np.int32)  # response 0: token 0; response 1: tokens 1..5
+    s = oracle.loss_scales(7, mask, cu, oracle.AGG_SEQ_MEAN)
+    np.testing.assert_allclose(s, [1 / 2, 1 / 8, 1 / 8, 1 / 8, 1 / 8, 0, 0])
+
+
+# ---------------------------------------------------------------- loss / gradient
+def test_loss_closed_forms():
+    """No correction, on-policy: loss = -(1/n) sum_t A_t.  A ratio of exactly 2
+    with A = 1 is clipped at 1 + c_high = 1.28 (Eq. 1)."""
+    rng = _rng(20)
+    T, V = 12, 9
+    z = (rng.integers(-64, 64, (T, V)) / 16).astype(np.float32)
+    ids = rng.integers(0, V, T).astype(np.int32)
+    adv = rng.standard_normal(T)
+    mask = np.ones(T, np.uint8)
+    mask[3] = 0
+    out = oracle.loss_fwd_bwd(z, ids, np.zeros(T), adv, oracle.params(mode=oracle.MODE_NONE),
+                              mask=mask, want_dz=False)
+    assert out["loss"] == pytest.approx(-adv[mask == 1].sum() / 11, rel=1e-14)
+    lp, _, _ = oracle.token_logprobs(z, ids)
+    out = oracle.loss_fwd_bwd(z, ids, lp, np.ones(T), oracle.params(mode=oracle.MODE_NONE),
+                              lp_old=lp - math.log(2.0), want_dz=True)
+    assert out["loss"] == pytest.approx(-1.28, rel=1e-13)
+    assert np.abs(out["dz"]).max() == 0.0  # the clip is active on every token
+    out = oracle.loss_fwd_bwd(z, ids, lp, -np.ones(T), oracle.params(mode=oracle.MODE_NONE),
+                              lp_old=lp - math.log(2.0), want_dz=False)
+    assert out["loss"] == pytest.approx(2.0, rel=1e-13)  # A < 0: min picks rho*A = -2
+
+
+def _fd_setup(seed, T, V):
+    rng = _rng(seed)
+    z = (rng.integers(-128, 128, (T, V)) / 32).astype(np.float32)  # exact fp32 +- 2^-16
+    ids = rng.integers(0, V, T).astype(np.int32)
+    adv = rng.standard_normal(T) * 1.5
+    lp_inf = _log_softmax(z.astype(np.float64) + rng.standard_normal((T, V)) * 0.4)[np.arange(T), ids]
+    return z, ids, adv, lp_inf
+
+
+@pytest.mark.parametrize("V", [2, 5, 8])
+@pytest.mark.parametrize("mode", [oracle.MODE_CIS, oracle.MODE_TIS, oracle.MODE_EXACT])
+def test_gradient_matches_central_finite_differences(V, mode):
+    """d loss / d z from the oracle equals central differences of its loss with
+    the weight frozen (stopgrad, Algorithm 1) and log p_old fixed.  Rows cover
+    the clip-inactive and clip-active branches for both signs of A, a masked
+    row, and the sequence-mean normaliser."""
+    T = 6
+    z, ids, adv, lp_inf = _fd_setup(100 + V + 10 * mode, T, V)
+    lp0, _, _ = oracle.token_logprobs(z, ids)
+    adv[:4] = [1.0, 1.0, -1.0, -1.0]
+    # rho = exp(l - l_old): 1.0 (inside), 1.6 (A>0 clipped), 1.6 (A<0 flows), 0.6 (A<0 clipped)
+    lp_old = lp0 - np.log([1.0, 1.6, 1.6, 0.6, 1.1, 0.9])
+    mask = np.ones(T, np.uint8)
+    mask[5] = 0
+    cu = np.array([0, 2, 6], np.int32)
+    for agg in (oracle.AGG_TOKEN_MEAN, oracle.AGG_SEQ_MEAN):
+        P = oracle.params(mode=mode, agg=agg)
+        base = oracle.loss_fwd_bwd(z, ids, lp_inf, adv, P, lp_old=lp_old, mask=mask,
+                                   cu_seqlens=cu)
+        w0 = base["w"]
+        h = np.float32(2.0 ** -16)
+        fd = np.zeros((T, V))
+        for t in range(T):
+            for j in range(V):
+                zp = z.copy()
+                zm = z.copy()
+                zp[t, j] += h
+                zm[t, j] -= h
+                Lp = oracle.loss_fwd_bwd(zp, ids, lp_inf, adv, P, lp_old=lp_old, mask=mask,
+                                         cu_seqlens=cu, w_fixed=w0, want_dz=False)["loss"]
+                Lm = oracle.loss_fwd_bwd(zm, ids, lp_inf, adv, P, lp_old=lp_old, mask=mask,
+                                         cu_seqlens=cu, w_fixed=w0, want_dz=False)["loss"]
+                fd[t, j] = (Lp - Lm) / (2 * float(h))
+        dz = base["dz"]
+        scale = np.abs(dz).max()
+        assert scale > 0
+        np.testing.assert_allclose(dz, fd, rtol=0, atol=1e-7 * scale)
+        assert np.all(dz[1] == 0) and np.all(dz[3] == 0) and np.all(dz[5] == 0)
+        assert np.abs(dz[2]).max() > 0 and np.abs(dz[0]).max() > 0
+
+
+def test_on_policy_gradient_equals_snapshot_gradient_at_rho_one():
+    """With no l_old the update ratio is exp(l - stopgrad l) = 1; its gradient
+    equals the one taken with l_old = l (rho = 1) and the weight built from l."""
+    z, ids, adv, lp_inf = _fd_setup(7, 8, 33)
+    lp0, _, _ = oracle.token_logprobs(z, ids)
+    P = oracle.params()
+    a = oracle.loss_fwd_bwd(z, ids, lp_inf, adv, P)
+    b = oracle.loss_fwd_bwd(z, ids, lp_inf, adv, P, lp_old=lp0)
+    np.testing.assert_allclose(a["dz"], b["dz"], rtol=1e-13, atol=1e-18)
+    assert a["loss"] == pytest.approx(b["loss"], rel=1e-13)
+
+
+def test_gradient_rows_sum_to_zero():
+    """sum_j dz_tj = c_t (sum_j softmax_j - 1) = 0."""
+    z, ids, adv, lp_inf = _fd_setup(8, 16, 500)
+    out = oracle.loss_fwd_bwd(z, ids, lp_inf, adv, oracle.params())
+    rs = out["dz"].sum(axis=1)
+    np.testing.assert_allclose(rs, 0.0, atol=1e-15 * np.abs(out["c"]).max() * 500)
+
+
+def test_row_subset_matches_full_gradient():
+    z, ids, adv, lp_inf = _fd_setup(9, 10, 40)
+    full = oracle.loss_fwd_bwd(z, ids, lp_inf, adv, oracle.params())
+    sub = oracle.loss_fwd_bwd(z, ids, lp_inf, adv, oracle.params(), rows=[7, 2])
+    np.testing.assert_array_equal(sub["dz"], full["dz"][[7, 2]])
