@@ -32,7 +32,9 @@
  *   - 1 - p is evaluated as -expm1(log p);
  *   - the loss is the negated objective, so d loss / d z = c (softmax - onehot);
  *   - in min(rho*A, clip(rho)*A) a tie takes the unclipped branch, so the
- *     gradient flows at rho = 1 +- c exactly.
+ *     gradient flows at rho = 1 +- c exactly;
+ *   - a NaN ratio gives a NaN weight (NaN propagates; min{NaN, cap} is not
+ *     read as cap).
  */
 #include <math.h>
 #include <stdint.h>
@@ -185,14 +187,14 @@ static void token_weight(double lw, double linf, const oracle_params_t *P, doubl
         /* phi <- max(1 - p, kappa);  f <- min{k, 1 + lambda*phi}. */
         double phi = one_minus_p > P->kappa ? one_minus_p : P->kappa;
         double cap = 1.0 + P->lambda * phi;
-        wt = k < cap ? k : cap;
+        wt = isnan(k) ? k : (k < cap ? k : cap);
         tr = logk > log1p(P->lambda * phi);
         break;
     }
     case OR_MODE_TIS: {
         /* Table 8: min(k, C). */
         double cap = P->tis_cap;
-        wt = k < cap ? k : cap;
+        wt = isnan(k) ? k : (k < cap ? k : cap);
         tr = logk > log(cap);
         break;
     }

@@ -393,3 +393,11 @@ def test_row_subset_matches_full_gradient():
     full = oracle.loss_fwd_bwd(z, ids, lp_inf, adv, oracle.params())
     sub = oracle.loss_fwd_bwd(z, ids, lp_inf, adv, oracle.params(), rows=[7, 2])
     np.testing.assert_array_equal(sub["dz"], full["dz"][[7, 2]])
+
+
+def test_nan_ratio_propagates():
+    """A NaN log-probability gives a NaN weight in every truncating mode."""
+    for mode in (oracle.MODE_CIS, oracle.MODE_TIS, oracle.MODE_EXACT):
+        w, tr, _, _ = oracle.weights(np.array([np.nan, -1.0]), np.array([-1.0, np.nan]),
+                                     oracle.params(mode=mode))
+        assert np.isnan(w).all() and not tr.any()
