@@ -1,0 +1,393 @@
+#!/usr/bin/env python3
+"""Benchmark of the fused CIS token pass (forward + backward) on one GB300.
+
+One step = one call of cis_loss_fwd_bwd over the whole batch: log-softmax of
+the [T, V] bf16 training logits, the sampled-token log-probability, the CIS
+weight (Algorithm 1), the PPO-clipped token loss (Eq. 1) and the bf16 gradient
+with respect to the logits.  Workload: T = 16384 tokens (64 responses of 256,
+groups of 8), V = 151936, temperatures spanning p in [1e-4, 0.9999]
+(paper_2609_32444_gb300.synth, workload 3).  The logits (4.98 GB) are far
+larger than the 129 MB L2, so no flush is needed between steps.
+
+    python bench.py [--steps K] [--warmup W] [--gpus N] [--impl ours|reference]
+
+Prints one JSON line (rank 0).  ``value`` is whole-job tokens/s with inputs
+already in HBM; ``e2e`` is the same metric through the same C ABI with the
+inputs in pinned host memory, copied in and the gradient copied out inside the
+timed region.  ``--impl reference`` times the fp64 CPU oracle on the host
+cores instead (a bounded sample of the same workload).
+"""
+import argparse
+import hashlib
+import json
+import os
+import re
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "CIS loss fwd+bwd tokens/s at V=151936 bf16; achieved % of HBM roofline"
+FALLBACK_HBM_GBS = 6800.0
+NOMINAL_HBM_GBS = 8000.0
+PROFILE_SUMMARY = os.path.join(ROOT, "profiles", "fused_pass_t16384_v151936_bf16.md")
+KERNEL_SOURCES = ["paper_2609_32444_gb300/csrc/cis_cluster.cu",
+                  "paper_2609_32444_gb300/csrc/cis_common.cuh"]
+
+
+def parse_args():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=400)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--mode", choices=["cis", "tis", "exact", "none"], default="cis")
+    ap.add_argument("--workload", type=int, default=3, choices=[2, 3, 4])
+    ap.add_argument("--dlogits", choices=["bf16", "f32"], default="bf16")
+    ap.add_argument("--e2e-steps", type=int, default=10)
+    ap.add_argument("--cpu-seconds", type=float, default=10.0)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    return ap.parse_args()
+
+
+def dist_setup():
+    import torch
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        import torch.distributed as dist
+        backend = "nccl" if torch.cuda.is_available() else "gloo"
+        dist.init_process_group(backend=backend)
+    return rank, world, local
+
+
+def barrier(world):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def max_over_ranks(x: float, world: int) -> float:
+    if world == 1:
+        return x
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64, device="cuda")
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def measured_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "MEASURED_PEAKS.json hbm_gbs (measured copy bandwidth)"
+    return FALLBACK_HBM_GBS, "fallback 6.8 TB/s (no MEASURED_PEAKS.json)"
+
+
+def kernel_source_hash() -> str:
+    h = hashlib.sha256()
+    for rel in KERNEL_SOURCES:
+        with open(os.path.join(ROOT, rel), "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()[:16]
+
+
+def profiled_traffic():
+    """DRAM bytes per launch of the main kernel from the committed ncu summary,
+    if it was taken on the current kernel source (else None)."""
+    if not os.path.exists(PROFILE_SUMMARY):
+        return None
+    txt = open(PROFILE_SUMMARY).read()
+    m = re.search(r"traffic_bytes_per_launch:\s*(\d+)", txt)
+    s = re.search(r"kernel_source_sha256_16:\s*([0-9a-f]+)", txt)
+    if not m or not s or s.group(1) != kernel_source_hash():
+        return None
+    return int(m.group(1))
+
+
+class ClockSampler:
+    """nvidia-smi samples of SM clock and throttle reasons during the timed region."""
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.samples = []
+        self.window = None
+        self.proc = None
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "100", "-i", str(gpu_index)],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except (OSError, ValueError):
+            return
+        self.thread = threading.Thread(target=self._read, daemon=True)
+        self.thread.start()
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.samples.append((time.time(), line.strip()))
+
+    def mark(self, t0, t1):
+        self.window = (t0, t1)
+
+    def summary(self):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+        rows = [s for t, s in self.samples
+                if self.window is None or self.window[0] <= t <= self.window[1] + 0.1]
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for r in rows:
+            parts = [p.strip() for p in r.split(",")]
+            if len(parts) < 8:
+                continue
+            try:
+                sm.append(float(parts[0]))
+                mx.append(float(parts[1]))
+            except ValueError:
+                continue
+            for nm, v in zip(names, parts[4:8]):
+                if v.lower() == "active":
+                    reasons.add(nm)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx),
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+def physical_gpu_index(local_rank: int) -> int:
+    vis = os.environ.get("CUDA_VISIBLE_DEVICES")
+    if vis:
+        ids = [v.strip() for v in vis.split(",") if v.strip()]
+        if local_rank < len(ids) and ids[local_rank].isdigit():
+            return int(ids[local_rank])
+    return local_rank
+
+
+def oracle_sample(batch_rows, mode, lam, seconds):
+    """Time the fp64 oracle on host cores over repeated chunks of real rows."""
+    import oracle
+    import numpy as np
+    logits, ids, lp, adv = batch_rows
+    P = oracle.params(mode={"cis": 0, "tis": 1, "exact": 2, "none": 3}[mode], lam=lam)
+    n = logits.shape[0]
+    done, t0 = 0, time.perf_counter()
+    while True:
+        oracle.loss_fwd_bwd(logits, ids, lp, adv, P, rows=np.arange(n))
+        done += n
+        el = time.perf_counter() - t0
+        if el >= seconds:
+            return done, el
+
+
+def host_rows(b, rows):
+    import numpy as np
+    import torch
+    idx = torch.as_tensor(rows, device=b.logits.device)
+    z = b.logits.index_select(0, idx).contiguous().cpu()
+    z = z.view(torch.int16).numpy().view(np.uint16) if z.dtype == torch.bfloat16 else z.numpy()
+    return (z, b.ids[idx].cpu().numpy(), b.lp_infer[idx].cpu().numpy(), b.adv[idx].cpu().numpy())
+
+
+def run_reference(args, rank, world):
+    """The reference arm: the fp64 oracle on the host cores, bounded samples."""
+    if rank != 0:
+        return
+    import numpy as np
+    import torch
+    import oracle
+    from paper_2609_32444_gb300 import synth
+    dev = "cuda" if torch.cuda.is_available() else "cpu"
+    T_gen = None if dev == "cuda" else 256
+    b = synth.make_batch(args.workload, device=dev, T=T_gen)
+    spec = synth.WORKLOADS[args.workload]
+    P = oracle.params(mode={"cis": 0, "tis": 1, "exact": 2, "none": 3}[args.mode], lam=b.lam)
+    rng = np.random.default_rng(0)
+    valid = np.nonzero(b.mask.cpu().numpy())[0]
+    # size one step to about 0.1 s of oracle work
+    probe = host_rows(b, rng.choice(valid, 16, replace=False))
+    t0 = time.perf_counter()
+    oracle.loss_fwd_bwd(*probe, P, rows=np.arange(16))
+    per_row = (time.perf_counter() - t0) / 16
+    nrows = int(max(8, min(len(valid), 0.1 / max(per_row, 1e-6))))
+    sample = host_rows(b, rng.choice(valid, nrows, replace=False))
+    for _ in range(args.warmup):
+        oracle.loss_fwd_bwd(*sample, P, rows=np.arange(nrows))
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        oracle.loss_fwd_bwd(*sample, P, rows=np.arange(nrows))
+    el = time.perf_counter() - t0
+    value = nrows * args.steps / el
+    cores = oracle.max_threads()
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": "tokens/s",
+        "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": el / args.steps * 1e3, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": spec["name"], "T": spec["T"], "V": spec["V"], "mode": args.mode,
+                   "lambda": b.lam, "kappa": 5e-3, "dlogits": "f64",
+                   "sample_rows_per_step": nrows},
+        "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": cores, "kind": "oracle",
+                         "sample": f"{nrows} valid rows of {spec['name']} per step, fp64 "
+                                   f"loss + weights + dlogits for every row"},
+        "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+def run_ours(args, rank, world, local):
+    import numpy as np
+    import torch
+    from paper_2609_32444_gb300 import binding, build, synth
+
+    build.build()
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    spec = synth.WORKLOADS[args.workload]
+    b = synth.make_batch(args.workload, device=dev, seed=1000 + args.workload + 7919 * rank)
+    T, V = b.T, b.V
+    dz_dt = torch.bfloat16 if args.dlogits == "bf16" else torch.float32
+    P = binding.cis_default_params(args.mode, lam=b.lam)
+    dz = torch.empty((T, V), dtype=dz_dt, device=dev)
+    ws = torch.empty(binding.cis_loss_workspace_size(T, V), dtype=torch.uint8, device=dev)
+
+    def step(logits=b.logits, ids=b.ids, lp=b.lp_infer, adv=b.adv, mask=b.mask):
+        return binding.cis_loss_fwd_bwd(logits, ids, lp, adv, P, mask=mask, dlogits=dz,
+                                        workspace=ws)
+
+    for _ in range(max(3, args.warmup)):
+        out = step()
+    torch.cuda.synchronize()
+    if binding.device_status(ws) != 0:
+        raise RuntimeError(f"device status {binding.device_status(ws)} after warm-up")
+    barrier(world)
+
+    stream = torch.cuda.current_stream()
+    kev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+           for _ in range(args.steps)]
+    clocks = ClockSampler(physical_gpu_index(local))
+    time.sleep(0.5)
+    start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize()
+    barrier(world)
+    h0 = time.time()
+    start.record(stream)
+    for i in range(args.steps):
+        binding.cis_profile_next_call(*kev[i])
+        out = step()
+    end.record(stream)
+    torch.cuda.synchronize()
+    h1 = time.time()
+    barrier(world)
+    clocks.mark(h0, h1)
+    elapsed_ms = start.elapsed_time(end)
+    kernel_ms = statistics.mean(a.elapsed_time(z) for a, z in kev)
+    elapsed_ms = max_over_ranks(elapsed_ms, world)
+    ms_per_step = elapsed_ms / args.steps
+    value = T * world / (ms_per_step / 1e3)
+    clk = clocks.summary()
+
+    # ---- end to end through the C ABI with pinned host buffers
+    e2e = None
+    if args.e2e_steps > 0:
+        hb = {k: v.cpu().pin_memory() for k, v in
+              dict(logits=b.logits, ids=b.ids, lp=b.lp_infer, adv=b.adv, mask=b.mask).items()}
+        dz_h = torch.empty((T, V), dtype=dz_dt).pin_memory()
+        loss_h = torch.empty(1, dtype=torch.float64).pin_memory()
+        dbufs = {k: torch.empty_like(v, device=dev) for k, v in hb.items()}
+        h2d = sum(v.numel() * v.element_size() for v in hb.values())
+        d2h = dz_h.numel() * dz_h.element_size() + 8
+        torch.cuda.synchronize()
+        barrier(world)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(args.e2e_steps):
+            for k in hb:
+                dbufs[k].copy_(hb[k], non_blocking=True)
+            o = step(dbufs["logits"], dbufs["ids"], dbufs["lp"], dbufs["adv"], dbufs["mask"])
+            dz_h.copy_(dz, non_blocking=True)
+            loss_h.copy_(o["loss"], non_blocking=True)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        e2e_ms = max_over_ranks(e0.elapsed_time(e1), world) / args.e2e_steps
+        e2e = {"value": T * world / (e2e_ms / 1e3), "unit": "tokens/s",
+               "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms}
+        del hb, dz_h, dbufs
+
+    # ---- roofline of the main kernel
+    isz = b.logits.element_size()
+    osz = dz.element_size()
+    side = 4 + 4 + 4 + 1 + 4 + 4 + 4 + 1 + 4 + 1 + 4 + 8  # per-token inputs/outputs, bytes
+    nvalid = int(b.mask.sum().item())
+    alg_bytes = nvalid * V * isz + T * V * osz + T * side
+    peak, peak_src = measured_peaks()
+    achieved = alg_bytes / (kernel_ms / 1e3) / 1e9
+    traffic = profiled_traffic()
+    roof = {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
+            "frac": achieved / peak, "traffic": traffic,
+            "kernel": "cluster_kernel<bf16,bf16> (fused fwd+bwd vocabulary pass)",
+            "kernel_ms": kernel_ms, "algorithmic_bytes_per_launch": alg_bytes,
+            "peak_source": peak_src, "frac_of_nominal_8000": achieved / NOMINAL_HBM_GBS,
+            "step_frac": alg_bytes / (ms_per_step / 1e3) / 1e9 / peak}
+
+    cpu = None
+    if rank == 0 and not args.no_cpu_baseline:
+        rng = np.random.default_rng(0)
+        valid = np.nonzero(b.mask.cpu().numpy())[0]
+        rows = rng.choice(valid, min(256, len(valid)), replace=False)
+        done, el = oracle_sample(host_rows(b, rows), args.mode, b.lam, args.cpu_seconds)
+        import oracle
+        cpu = {"value": done / el, "unit": "tokens/s", "cores": oracle.max_threads(),
+               "kind": "oracle",
+               "sample": f"{len(rows)} valid rows of {spec['name']} repeated for "
+                         f"{el:.1f} s ({done} rows), fp64 loss + weights + dlogits"}
+
+    st = binding.decode_stats(out["stats"])
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_per_step,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+            "data": "synthetic",
+            "config": {"workload": spec["name"], "T": T, "V": V, "mode": args.mode,
+                       "lambda": b.lam, "kappa": 5e-3, "io_dtype": "bf16" if isz == 2 else "f32",
+                       "dlogits": args.dlogits, "valid_tokens": nvalid,
+                       "l2": "no flush: the 4.98 GB of logits per step exceed the 129 MB L2",
+                       "parallelism": f"independent batch per GPU x{world}"},
+            "roofline": roof, "cpu_baseline": cpu, "e2e": e2e,
+            "gpu_launches": 3 * args.steps,
+            "clocks": clk,
+            "check": {"loss": st["loss"], "n_truncated": st["n_truncated"],
+                      "status": st["status"]},
+        }
+        print(json.dumps(line), flush=True)
+
+
+def main():
+    args = parse_args()
+    rank, world, local = dist_setup()
+    if args.impl == "reference":
+        run_reference(args, rank, world)
+    else:
+        run_ours(args, rank, world, local)
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -46,6 +46,12 @@
 #include <stddef.h>
 #include <stdint.h>
 
+#if defined(__GNUC__)
+#define CIS_API __attribute__((visibility("default")))
+#else
+#define CIS_API
+#endif
+
 #ifdef __cplusplus
 extern "C" {
 #endif
@@ -104,10 +110,10 @@ typedef struct {
 
 /* Fills *out with the defaults above.  Host only.  CIS_ERR_INVALID_ARG if out
  * is NULL. */
-cis_status_t cis_default_params(cis_params_t *out);
+CIS_API cis_status_t cis_default_params(cis_params_t *out);
 
 /* Human-readable name of a status value (static string, never NULL). */
-const char *cis_status_string(int32_t status);
+CIS_API const char *cis_status_string(int32_t status);
 
 /*
  * Sampled-token log-probabilities (Sec. 2.1): lp_out[t] = z_{t,y_t} -
@@ -122,7 +128,7 @@ const char *cis_status_string(int32_t status);
  * Errors: CIS_ERR_INVALID_ARG for NULL required pointers, T < 0, V <= 0,
  * ld < V or an unknown dtype.
  */
-cis_status_t cis_token_logprobs(const void *logits, int32_t dtype, int64_t T, int64_t V,
+CIS_API cis_status_t cis_token_logprobs(const void *logits, int32_t dtype, int64_t T, int64_t V,
                                 int64_t ld, const int32_t *ids, const uint8_t *mask,
                                 float *lp_out, float *lse_out, int32_t *dev_status,
                                 void *stream);
@@ -145,13 +151,13 @@ cis_status_t cis_token_logprobs(const void *logits, int32_t dtype, int64_t T, in
  * evaluation.  Errors: CIS_ERR_INVALID_ARG for NULL required pointers, T < 0
  * or parameters outside the ranges of cis_params_t.
  */
-cis_status_t cis_weights(const float *lp_train, const float *lp_infer, const uint8_t *mask,
+CIS_API cis_status_t cis_weights(const float *lp_train, const float *lp_infer, const uint8_t *mask,
                          int64_t T, const cis_params_t *params, float *w_out,
                          uint8_t *trunc_out, float *eps_out, void *stream);
 
 /* Bytes of device workspace cis_loss_fwd_bwd needs for T tokens and
  * vocabulary V.  Host only.  CIS_ERR_INVALID_ARG if bytes is NULL or T < 0. */
-cis_status_t cis_loss_workspace_size(int64_t T, int64_t V, size_t *bytes);
+CIS_API cis_status_t cis_loss_workspace_size(int64_t T, int64_t V, size_t *bytes);
 
 /*
  * The fused forward + backward token pass (Eq. 1 with the weight of
@@ -185,7 +191,7 @@ cis_status_t cis_loss_workspace_size(int64_t T, int64_t V, size_t *bytes);
  * CIS_AGG_SEQ_MEAN_TOKEN_MEAN without cu_seqlens; CIS_ERR_CUDA if a launch
  * fails.
  */
-cis_status_t cis_loss_fwd_bwd(const void *logits, int32_t dtype, int64_t T, int64_t V,
+CIS_API cis_status_t cis_loss_fwd_bwd(const void *logits, int32_t dtype, int64_t T, int64_t V,
                               int64_t ld, const int32_t *ids, const float *lp_infer,
                               const float *lp_old, const float *adv, const uint8_t *mask,
                               const int32_t *cu_seqlens, int64_t B,
@@ -194,6 +200,16 @@ cis_status_t cis_loss_fwd_bwd(const void *logits, int32_t dtype, int64_t T, int6
                               float *w_out, uint8_t *trunc_out, cis_stats_t *stats_out,
                               double *loss_out, void *workspace, size_t workspace_bytes,
                               void *stream);
+
+/*
+ * Profiling aid.  The next cis_loss_fwd_bwd call made from the calling host
+ * thread records `begin_event` on its stream just before its main kernel (the
+ * fused vocabulary pass) and `end_event` just after it, then forgets both.
+ * The events are cudaEvent_t handles passed as void*, owned by the caller.
+ * Passing NULL for both cancels a pending request.  Nothing else changes: the
+ * call does the same work.  CIS_ERR_INVALID_ARG if exactly one is NULL.
+ */
+CIS_API cis_status_t cis_profile_next_call(void *begin_event, void *end_event);
 
 #ifdef __cplusplus
 }

@@ -1,0 +1,252 @@
+"""Thin Python binding of libcis (include/cis.h), same names as the C ABI.
+
+Argument marshalling only: tensors are passed as raw device pointers with the
+current CUDA stream; every step of the token pass runs in libcis's kernels.
+There is no CPU path -- importing works without a GPU, but every call needs
+the compiled library and CUDA tensors, and raises otherwise.
+"""
+
+from __future__ import annotations
+
+import ctypes
+import os
+
+import torch
+
+from . import build as _build
+
+CIS_OK, CIS_ERR_INVALID_ARG, CIS_ERR_UNSUPPORTED, CIS_ERR_CUDA = 0, 1, 2, 3
+CIS_ERR_DEVICE_TIMEOUT, CIS_ERR_BAD_TOKEN_ID = 4, 8
+CIS_F32, CIS_BF16 = 0, 1
+CIS_MODE_CIS, CIS_MODE_TIS, CIS_MODE_EXACT, CIS_MODE_NONE = 0, 1, 2, 3
+CIS_AGG_TOKEN_MEAN, CIS_AGG_SEQ_MEAN_TOKEN_MEAN = 0, 1
+
+MODES = {"cis": CIS_MODE_CIS, "tis": CIS_MODE_TIS, "exact": CIS_MODE_EXACT,
+         "none": CIS_MODE_NONE}
+
+
+class cis_params_t(ctypes.Structure):
+    _fields_ = [
+        ("mode", ctypes.c_int32),
+        ("agg", ctypes.c_int32),
+        ("lam", ctypes.c_double),
+        ("kappa", ctypes.c_double),
+        ("tis_cap", ctypes.c_double),
+        ("exact_lo", ctypes.c_double),
+        ("exact_hi", ctypes.c_double),
+        ("clip_low", ctypes.c_double),
+        ("clip_high", ctypes.c_double),
+    ]
+
+
+class cis_stats_t(ctypes.Structure):
+    _fields_ = [
+        ("loss", ctypes.c_double),
+        ("trunc_excess", ctypes.c_double),
+        ("n_valid", ctypes.c_int64),
+        ("n_truncated", ctypes.c_int64),
+        ("max_abs_logk", ctypes.c_float),
+        ("status", ctypes.c_int32),
+    ]
+
+
+class CisError(RuntimeError):
+    pass
+
+
+_lib = None
+
+
+def library_path() -> str:
+    return _build.LIB_PATH
+
+
+def lib():
+    """The loaded libcis.so.  Raises if it has not been built."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    path = _build.LIB_PATH
+    if not os.path.exists(path):
+        raise ImportError(f"libcis.so is not built ({path}); run __graft_entry__.build()")
+    L = ctypes.CDLL(path)
+    P, i32, i64 = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64
+    L.cis_default_params.argtypes = [ctypes.POINTER(cis_params_t)]
+    L.cis_default_params.restype = ctypes.c_int
+    L.cis_status_string.argtypes = [i32]
+    L.cis_status_string.restype = ctypes.c_char_p
+    L.cis_token_logprobs.argtypes = [P, i32, i64, i64, i64, P, P, P, P, P, P]
+    L.cis_token_logprobs.restype = ctypes.c_int
+    L.cis_weights.argtypes = [P, P, P, i64, ctypes.POINTER(cis_params_t), P, P, P, P]
+    L.cis_weights.restype = ctypes.c_int
+    L.cis_loss_workspace_size.argtypes = [i64, i64, ctypes.POINTER(ctypes.c_size_t)]
+    L.cis_loss_workspace_size.restype = ctypes.c_int
+    L.cis_loss_fwd_bwd.argtypes = [P, i32, i64, i64, i64, P, P, P, P, P, P, i64,
+                                   ctypes.POINTER(cis_params_t), P, i32, i64, P, P, P, P, P, P,
+                                   ctypes.c_size_t, P]
+    L.cis_loss_fwd_bwd.restype = ctypes.c_int
+    L.cis_profile_next_call.argtypes = [P, P]
+    L.cis_profile_next_call.restype = ctypes.c_int
+    _lib = L
+    return L
+
+
+def status_string(code: int) -> str:
+    return lib().cis_status_string(int(code)).decode()
+
+
+def _check(rc: int, what: str):
+    if rc != CIS_OK:
+        raise CisError(f"{what}: {status_string(rc)}")
+
+
+def _ptr(t):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _stream():
+    return ctypes.c_void_p(torch.cuda.current_stream().cuda_stream)
+
+
+def _dtype_code(dt) -> int:
+    if dt == torch.bfloat16:
+        return CIS_BF16
+    if dt == torch.float32:
+        return CIS_F32
+    raise TypeError(f"unsupported dtype {dt}: libcis takes bfloat16 or float32")
+
+
+def _need_cuda(*ts):
+    for t in ts:
+        if t is not None and not t.is_cuda:
+            raise ValueError("libcis takes CUDA tensors")
+
+
+def _rows(x: torch.Tensor):
+    """(T, ld) of a 2-D tensor with unit column stride."""
+    if x.dim() != 2 or (x.shape[1] > 1 and x.stride(1) != 1):
+        raise ValueError("logits must be 2-D with contiguous rows")
+    return x.shape[0], (x.stride(0) if x.shape[0] > 1 else x.shape[1])
+
+
+def _vec(x, dtype, T, name):
+    if x is None:
+        return None
+    if x.dtype != dtype or x.dim() != 1 or x.shape[0] != T or not x.is_contiguous():
+        raise ValueError(f"{name} must be a contiguous [{T}] {dtype} tensor")
+    return x
+
+
+def cis_default_params(mode="cis", **kw) -> cis_params_t:
+    """Defaults of App. C.1 / Table 8, with keyword overrides (lam, kappa, tis_cap,
+    exact_lo, exact_hi, clip_low, clip_high, agg)."""
+    p = cis_params_t()
+    _check(lib().cis_default_params(ctypes.byref(p)), "cis_default_params")
+    p.mode = MODES[mode] if isinstance(mode, str) else int(mode)
+    for k, v in kw.items():
+        setattr(p, k, v)
+    return p
+
+
+def cis_token_logprobs(logits: torch.Tensor, ids: torch.Tensor, mask=None, V=None,
+                       want_lse=False, dev_status=None):
+    """log p of the sampled tokens (fp32) -- and the row logsumexp if asked."""
+    _need_cuda(logits, ids, mask)
+    T, ld = _rows(logits)
+    V = logits.shape[1] if V is None else V
+    _vec(ids, torch.int32, T, "ids")
+    _vec(mask, torch.uint8, T, "mask")
+    lp = torch.empty(T, dtype=torch.float32, device=logits.device)
+    lse = torch.empty(T, dtype=torch.float32, device=logits.device) if want_lse else None
+    rc = lib().cis_token_logprobs(_ptr(logits), _dtype_code(logits.dtype), T, V, ld, _ptr(ids),
+                                  _ptr(mask), _ptr(lp), _ptr(lse), _ptr(dev_status), _stream())
+    _check(rc, "cis_token_logprobs")
+    return (lp, lse) if want_lse else lp
+
+
+def cis_weights(lp_train: torch.Tensor, lp_infer: torch.Tensor, params: cis_params_t,
+                mask=None, want_trunc=True, want_eps=False):
+    """Weights of Algorithm 1 / Table 8.  Returns (w, trunc or None, eps or None)."""
+    _need_cuda(lp_train, lp_infer, mask)
+    T = lp_train.shape[0]
+    _vec(lp_train, torch.float32, T, "lp_train")
+    _vec(lp_infer, torch.float32, T, "lp_infer")
+    _vec(mask, torch.uint8, T, "mask")
+    dev = lp_train.device
+    w = torch.empty(T, dtype=torch.float32, device=dev)
+    tr = torch.empty(T, dtype=torch.uint8, device=dev) if want_trunc else None
+    eps = torch.empty(T, dtype=torch.float32, device=dev) if want_eps else None
+    rc = lib().cis_weights(_ptr(lp_train), _ptr(lp_infer), _ptr(mask), T, ctypes.byref(params),
+                           _ptr(w), _ptr(tr), _ptr(eps), _stream())
+    _check(rc, "cis_weights")
+    return w, tr, eps
+
+
+def cis_loss_workspace_size(T: int, V: int) -> int:
+    n = ctypes.c_size_t(0)
+    _check(lib().cis_loss_workspace_size(T, V, ctypes.byref(n)), "cis_loss_workspace_size")
+    return n.value
+
+
+def cis_loss_fwd_bwd(logits: torch.Tensor, ids: torch.Tensor, lp_infer: torch.Tensor,
+                     adv: torch.Tensor, params: cis_params_t, lp_old=None, mask=None,
+                     cu_seqlens=None, dlogits=None, dlogits_dtype=None, V=None,
+                     want_lp=True, want_w=True, want_trunc=True, workspace=None):
+    """Fused forward + backward token pass.  Returns a dict with dlogits, lp, w,
+    trunc, loss (device fp64 [1]), stats (device bytes of cis_stats_t) and the
+    workspace (its first int32 is the device status word)."""
+    _need_cuda(logits, ids, lp_infer, adv, lp_old, mask, cu_seqlens, dlogits)
+    T, ld = _rows(logits)
+    V = logits.shape[1] if V is None else V
+    dev = logits.device
+    for x, dt, nm in ((ids, torch.int32, "ids"), (lp_infer, torch.float32, "lp_infer"),
+                      (adv, torch.float32, "adv"), (lp_old, torch.float32, "lp_old"),
+                      (mask, torch.uint8, "mask")):
+        _vec(x, dt, T, nm)
+    B = 0
+    if cu_seqlens is not None:
+        if cu_seqlens.dtype != torch.int32 or cu_seqlens.dim() != 1:
+            raise ValueError("cu_seqlens must be int32 [B + 1]")
+        B = cu_seqlens.shape[0] - 1
+    if dlogits is None:
+        dt = logits.dtype if dlogits_dtype is None else dlogits_dtype
+        dlogits = torch.empty((T, V), dtype=dt, device=dev)
+    To, ld_out = _rows(dlogits)
+    if To != T or dlogits.shape[1] < V:
+        raise ValueError("dlogits must be [T, >= V]")
+    lp = torch.empty(T, dtype=torch.float32, device=dev) if want_lp else None
+    w = torch.empty(T, dtype=torch.float32, device=dev) if want_w else None
+    tr = torch.empty(T, dtype=torch.uint8, device=dev) if want_trunc else None
+    stats = torch.empty(ctypes.sizeof(cis_stats_t), dtype=torch.uint8, device=dev)
+    loss = torch.empty(1, dtype=torch.float64, device=dev)
+    nws = cis_loss_workspace_size(T, V)
+    if workspace is None or workspace.numel() < nws:
+        workspace = torch.empty(nws, dtype=torch.uint8, device=dev)
+    rc = lib().cis_loss_fwd_bwd(
+        _ptr(logits), _dtype_code(logits.dtype), T, V, ld, _ptr(ids), _ptr(lp_infer),
+        _ptr(lp_old), _ptr(adv), _ptr(mask), _ptr(cu_seqlens), B, ctypes.byref(params),
+        _ptr(dlogits), _dtype_code(dlogits.dtype), ld_out, _ptr(lp), _ptr(w), _ptr(tr),
+        _ptr(stats), _ptr(loss), _ptr(workspace), workspace.numel(), _stream())
+    _check(rc, "cis_loss_fwd_bwd")
+    return {"dlogits": dlogits, "lp": lp, "w": w, "trunc": tr, "loss": loss, "stats": stats,
+            "workspace": workspace}
+
+
+def cis_profile_next_call(begin: "torch.cuda.Event | None", end: "torch.cuda.Event | None"):
+    """Have the next cis_loss_fwd_bwd on this thread record these events around
+    its main kernel (timing aid; the call does the same work)."""
+    b = None if begin is None else ctypes.c_void_p(begin.cuda_event)
+    e = None if end is None else ctypes.c_void_p(end.cuda_event)
+    _check(lib().cis_profile_next_call(b, e), "cis_profile_next_call")
+
+
+def decode_stats(stats: torch.Tensor) -> dict:
+    """Read a cis_stats_t written on the device (synchronises)."""
+    raw = bytes(stats.cpu().numpy().tobytes())
+    s = cis_stats_t.from_buffer_copy(raw)
+    return {f: getattr(s, f) for f, _ in cis_stats_t._fields_}
+
+
+def device_status(workspace: torch.Tensor) -> int:
+    """The device status word of the last call that used this workspace."""
+    return int(workspace[:4].view(torch.int32).item())

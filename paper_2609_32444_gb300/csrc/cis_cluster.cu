@@ -1,0 +1,382 @@
+// cis_cluster.cu -- fused forward + backward token pass, fast path (sm_103a).
+//
+// A bf16 row of the 151,936-entry vocabulary is 303,872 bytes, more than one
+// CTA's shared memory.  A cluster of CS CTAs (CS = 1, 2, 4 or 8) therefore
+// splits each row into CS contiguous slices.  Per row:
+//   1. each CTA copies its slice from HBM into shared memory with one bulk
+//      asynchronous copy (cp.async.bulk, completion counted on an mbarrier;
+//      no multicast);
+//   2. pass 1 over shared memory: per thread the exact maximum of its entries
+//      (j != y), then the sum of e^{z - max}; a block reduction gives the CTA's
+//      pair (m_c, s_c);
+//   3. every CTA writes its pair into slot [rank] of every CTA of the cluster
+//      (distributed shared memory), then a cluster barrier; each CTA combines
+//      the CS pairs in rank order, so all CTAs hold bit-identical row scalars;
+//   4. thread 0 forms log p (log-odds form, cis_common.cuh), the weight
+//      (Algorithm 1 / Table 8) and the token loss (Eq. 1);
+//   5. pass 2 over shared memory writes dz = c (softmax - onehot) with 16-byte
+//      streaming stores.
+// HBM traffic is one read of the logits and one write of dz.  Rows are
+// independent; several clusters share an SM, so one cluster's copy overlaps
+// another's arithmetic.
+#include <cooperative_groups.h>
+#include <stdlib.h>
+
+#include "cis_kernels.h"
+
+namespace cg = cooperative_groups;
+
+namespace cis {
+namespace {
+
+constexpr int kThreads = 256;
+constexpr int kMaxCluster = 8;
+
+__device__ __forceinline__ float max_nan(float a, float b)
+{
+    float r;
+    asm("max.NaN.f32 %0, %1, %2;" : "=f"(r) : "f"(a), "f"(b));
+    return r;
+}
+
+__device__ __forceinline__ uint32_t smem_u32(const void *p)
+{
+    return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count)
+{
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+}
+
+__device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes)
+{
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes)
+                 : "memory");
+}
+
+__device__ __forceinline__ void bulk_g2s(uint32_t dst, const void *src, uint32_t bytes,
+                                         uint32_t bar)
+{
+    asm volatile(
+        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
+        ::"r"(dst), "l"(src), "r"(bytes), "r"(bar)
+        : "memory");
+}
+
+// Bounded wait on phase `parity` of an mbarrier; false if it never completed.
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity)
+{
+    for (uint32_t i = 0; i < kMaxPolls; ++i) {
+        uint32_t done;
+        asm volatile(
+            "{\n\t.reg .pred p;\n\t"
+            "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
+            "selp.u32 %0, 1, 0, p;\n\t}"
+            : "=r"(done)
+            : "r"(bar), "r"(parity), "r"(kPollSuspendNs)
+            : "memory");
+        if (done)
+            return true;
+    }
+    return false;
+}
+
+__device__ __forceinline__ void cluster_arrive_relaxed()
+{
+    asm volatile("barrier.cluster.arrive.relaxed.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void cluster_wait()
+{
+    asm volatile("barrier.cluster.wait.aligned;" ::: "memory");
+}
+
+// 8 consecutive entries from shared memory as floats.
+template <typename InT> __device__ __forceinline__ void load8(const uint8_t *sm, int64_t g,
+                                                              float (&z)[8]);
+template <>
+__device__ __forceinline__ void load8<__nv_bfloat16>(const uint8_t *sm, int64_t g, float (&z)[8])
+{
+    const uint4 q = reinterpret_cast<const uint4 *>(sm)[g];
+    z[0] = bf16_lo(q.x); z[1] = bf16_hi(q.x);
+    z[2] = bf16_lo(q.y); z[3] = bf16_hi(q.y);
+    z[4] = bf16_lo(q.z); z[5] = bf16_hi(q.z);
+    z[6] = bf16_lo(q.w); z[7] = bf16_hi(q.w);
+}
+template <>
+__device__ __forceinline__ void load8<float>(const uint8_t *sm, int64_t g, float (&z)[8])
+{
+    const uint4 q0 = reinterpret_cast<const uint4 *>(sm)[2 * g];
+    const uint4 q1 = reinterpret_cast<const uint4 *>(sm)[2 * g + 1];
+    z[0] = __uint_as_float(q0.x); z[1] = __uint_as_float(q0.y);
+    z[2] = __uint_as_float(q0.z); z[3] = __uint_as_float(q0.w);
+    z[4] = __uint_as_float(q1.x); z[5] = __uint_as_float(q1.y);
+    z[6] = __uint_as_float(q1.z); z[7] = __uint_as_float(q1.w);
+}
+
+// 8 results to global memory with streaming (evict-first) 16-byte stores.
+template <typename OutT> __device__ __forceinline__ void store8(OutT *dst, const float (&v)[8]);
+template <>
+__device__ __forceinline__ void store8<__nv_bfloat16>(__nv_bfloat16 *dst, const float (&v)[8])
+{
+    uint4 q;
+    __nv_bfloat162 h;
+    h = __floats2bfloat162_rn(v[0], v[1]); q.x = *reinterpret_cast<uint32_t *>(&h);
+    h = __floats2bfloat162_rn(v[2], v[3]); q.y = *reinterpret_cast<uint32_t *>(&h);
+    h = __floats2bfloat162_rn(v[4], v[5]); q.z = *reinterpret_cast<uint32_t *>(&h);
+    h = __floats2bfloat162_rn(v[6], v[7]); q.w = *reinterpret_cast<uint32_t *>(&h);
+    __stcs(reinterpret_cast<uint4 *>(dst), q);
+}
+template <>
+__device__ __forceinline__ void store8<float>(float *dst, const float (&v)[8])
+{
+    __stcs(reinterpret_cast<float4 *>(dst), make_float4(v[0], v[1], v[2], v[3]));
+    __stcs(reinterpret_cast<float4 *>(dst) + 1, make_float4(v[4], v[5], v[6], v[7]));
+}
+
+struct ClusterShared {
+    alignas(8) uint64_t bar;
+    float2 part[kMaxCluster];
+    MaxSum red[kThreads / 32];
+    float c, m, bias, lp;
+};
+
+template <typename InT, typename OutT>
+__global__ void __launch_bounds__(kThreads) cluster_kernel(const PassArgs a, int64_t slice)
+{
+    extern __shared__ __align__(128) uint8_t dyn_smem[];
+    __shared__ ClusterShared sh;
+    // the bulk copy needs a 16-byte aligned destination; 128 bytes of slack
+    // are allocated so the slab can start on a 128-byte boundary
+    uint8_t *slab = dyn_smem + ((128 - (smem_u32(dyn_smem) & 127)) & 127);
+    cg::cluster_group cluster = cg::this_cluster();
+    const unsigned rank = cluster.block_rank();
+    const unsigned cs = cluster.num_blocks();
+    const int64_t t = blockIdx.x / cs;
+    const int64_t v0 = (int64_t)rank * slice;
+    const int64_t n = v0 < a.V ? (a.V - v0 < slice ? a.V - v0 : slice) : 0;  // multiple of 8
+    const int64_t ng = n / 8;
+    OutT *orow = reinterpret_cast<OutT *>(a.dz) + t * a.ld_out + v0;
+
+    const bool valid = a.mask == nullptr || a.mask[t] != 0;
+    const int64_t y = a.ids[t];
+    const bool id_ok = y >= 0 && y < a.V;
+    if (!valid || !id_ok) {  // same branch in every CTA of the cluster
+        const float zero[8] = {0, 0, 0, 0, 0, 0, 0, 0};
+        for (int64_t g = threadIdx.x; g < ng; g += kThreads)
+            store8<OutT>(orow + 8 * g, zero);
+        if (rank == 0 && threadIdx.x == 0) {
+            const float lp = valid ? NAN : 0.0f;
+            if (valid)
+                set_status(a.status, kStatusBadId);
+            if (a.lp_out) a.lp_out[t] = lp;
+            if (a.w_out) a.w_out[t] = 0.0f;
+            if (a.trunc_out) a.trunc_out[t] = 0;
+            a.ws_w[t] = 0.0f;
+            a.ws_trunc[t] = 0;
+            a.ws_logk[t] = 0.0f;
+            a.ws_terms[t] = valid ? (double)NAN : 0.0;
+        }
+        return;
+    }
+
+    const uint32_t bar = smem_u32(&sh.bar);
+    if (threadIdx.x == 0) {
+        mbar_init(bar, 1);
+        if (n > 0) {
+            const uint32_t bytes = (uint32_t)(n * sizeof(InT));
+            mbar_expect_tx(bar, bytes);
+            const uint8_t *src = reinterpret_cast<const uint8_t *>(a.logits) +
+                                 (t * a.ld + v0) * (int64_t)sizeof(InT);
+            bulk_g2s(smem_u32(slab), src, bytes, bar);
+        }
+    }
+    // Arrive now, wait before the first remote store: every CTA of the
+    // cluster has started by then.
+    cluster_arrive_relaxed();
+
+    // Per-token inputs, fetched while the copy is in flight.
+    float zy = 0.0f, linf = 0.0f, lold = 0.0f, adv = 0.0f, sc = 0.0f;
+    if (threadIdx.x == 0) {
+        zy = to_f32(reinterpret_cast<const InT *>(a.logits)[t * a.ld + y]);
+        linf = a.lp_inf[t];
+        lold = a.lp_old ? a.lp_old[t] : 0.0f;
+        adv = a.adv[t];
+        sc = a.scale[t];
+    }
+    __syncthreads();  // barrier initialised before anyone polls it
+    if (n > 0 && !mbar_wait(bar, 0)) {
+        if (threadIdx.x == 0)
+            set_status(a.status, kStatusTimeout);
+        mbar_wait(bar, 0);  // give the copy one more bounded chance to land
+    }
+
+    // Pass 1: exact max of this thread's entries (j != y), then the sum.
+    const int64_t yl = y - v0;
+    const int64_t gy = (yl >= 0 && yl < n) ? yl / 8 : -1;
+    const int iy = (int)(yl & 7);
+    float m = -INFINITY;
+    for (int64_t g = threadIdx.x; g < ng; g += kThreads) {
+        float z[8];
+        load8<InT>(slab, g, z);
+        const int skip = g == gy ? iy : -1;
+#pragma unroll
+        for (int i = 0; i < 8; ++i)
+            m = max_nan(m, i == skip ? -INFINITY : z[i]);
+    }
+    float s = 0.0f;
+    if (m != -INFINITY) {
+        for (int64_t g = threadIdx.x; g < ng; g += kThreads) {
+            float z[8];
+            load8<InT>(slab, g, z);
+            s += sum8_exp(z, m, g == gy ? iy : -1);
+        }
+    }
+    const MaxSum mine = block_ms<kThreads>(MaxSum{m, s}, sh.red);
+
+    // Exchange the CTA pairs through distributed shared memory.
+    cluster_wait();
+    if (threadIdx.x == 0) {
+        for (unsigned r = 0; r < cs; ++r) {
+            float2 *dst = cluster.map_shared_rank(&sh.part[rank], r);
+            *dst = make_float2(mine.m, mine.s);
+        }
+    }
+    cluster.sync();
+    MaxSum o{sh.part[0].x, sh.part[0].y};
+    for (unsigned r = 1; r < cs; ++r)
+        o = ms_combine(o, MaxSum{sh.part[r].x, sh.part[r].y});
+
+    if (threadIdx.x == 0) {
+        const RowScalars rs = row_scalars(o, zy);
+        const bool has_old = a.lp_old != nullptr;
+        const TokenWeight tw = token_weight(has_old ? lold : rs.lp, linf, a.P);
+        const TokenLoss tl = token_loss(rs.lp, has_old, lold, adv, sc, tw.w, a.P);
+        if (rank == 0) {
+            if (a.lp_out) a.lp_out[t] = rs.lp;
+            if (a.w_out) a.w_out[t] = tw.w;
+            if (a.trunc_out) a.trunc_out[t] = tw.trunc;
+            a.ws_w[t] = tw.w;
+            a.ws_trunc[t] = tw.trunc;
+            a.ws_logk[t] = tw.logk;
+            a.ws_terms[t] = tl.term;
+        }
+        sh.c = tl.c;
+        sh.m = rs.m;
+        sh.bias = rs.bias_log2;
+        sh.lp = rs.lp;
+    }
+    __syncthreads();
+
+    // Pass 2: dz = c (softmax - onehot) from the slice in shared memory.
+    const float c = sh.c, mo = sh.m, bias = sh.bias;
+    const float dzy = c * expm1f(sh.lp);  // c (p - 1)
+    for (int64_t g = threadIdx.x; g < ng; g += kThreads) {
+        float z[8], v[8];
+        load8<InT>(slab, g, z);
+        const int skip = g == gy ? iy : -1;
+#pragma unroll
+        for (int i = 0; i < 8; ++i)
+            v[i] = i == skip ? dzy : c * ex2_full(fmaf(z[i] - mo, kLog2e, -bias));
+        store8<OutT>(orow + 8 * g, v);
+    }
+}
+
+// Cluster size and slice (entries, a multiple of 8) for a row of V entries.
+struct Plan {
+    int cs;
+    int64_t slice;
+    size_t smem;
+};
+
+int64_t slice_target_bytes()
+{
+    static int64_t v = [] {
+        const char *e = getenv("CIS_SLICE_KB");
+        long kb = e ? atol(e) : 80;
+        if (kb < 8) kb = 8;
+        if (kb > 200) kb = 200;
+        return (int64_t)kb * 1024;
+    }();
+    return v;
+}
+
+bool make_plan(int64_t V, int in_bytes, Plan *p)
+{
+    const int64_t target = slice_target_bytes();
+    for (int cs = 1; cs <= kMaxCluster; cs *= 2) {
+        const int64_t per = (V + cs - 1) / cs;
+        const int64_t slice = (per + 7) / 8 * 8;
+        if (slice * in_bytes <= target || cs == kMaxCluster) {
+            if (slice * in_bytes > 200 * 1024)
+                return false;
+            p->cs = cs;
+            p->slice = slice;
+            p->smem = (size_t)(slice * in_bytes) + 128;
+            return true;
+        }
+    }
+    return false;
+}
+
+template <typename InT, typename OutT>
+cudaError_t launch_cluster_t(const PassArgs &a, const Plan &p, cudaStream_t s)
+{
+    auto kern = cluster_kernel<InT, OutT>;
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)p.smem);
+    if (e != cudaSuccess)
+        return e;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)(a.T * p.cs), 1, 1);
+    cfg.blockDim = dim3(kThreads, 1, 1);
+    cfg.dynamicSmemBytes = p.smem;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = (unsigned)p.cs;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kern, a, p.slice);
+}
+
+}  // namespace
+
+bool cluster_path_applies(const PassArgs &a, int dtype, int out_dtype)
+{
+    const int ib = dtype == CIS_BF16 ? 2 : 4;
+    const int ob = out_dtype == CIS_BF16 ? 2 : 4;
+    if (a.V % 8 != 0)
+        return false;
+    if ((reinterpret_cast<uintptr_t>(a.logits) & 15) || (a.ld * ib) % 16)
+        return false;
+    if ((reinterpret_cast<uintptr_t>(a.dz) & 15) || (a.ld_out * ob) % 16)
+        return false;
+    if (a.T * 8 > 0x7fffffffLL)
+        return false;
+    Plan p;
+    return make_plan(a.V, ib, &p);
+}
+
+cudaError_t launch_cluster_fwd_bwd(const PassArgs &a, int dtype, int out_dtype, cudaStream_t s)
+{
+    if (!cluster_path_applies(a, dtype, out_dtype))
+        return cudaErrorNotSupported;
+    if (a.T == 0)
+        return cudaSuccess;
+    Plan p;
+    make_plan(a.V, dtype == CIS_BF16 ? 2 : 4, &p);
+    if (dtype == CIS_BF16) {
+        if (out_dtype == CIS_BF16)
+            return launch_cluster_t<__nv_bfloat16, __nv_bfloat16>(a, p, s);
+        return launch_cluster_t<__nv_bfloat16, float>(a, p, s);
+    }
+    if (out_dtype == CIS_BF16)
+        return launch_cluster_t<float, __nv_bfloat16>(a, p, s);
+    return launch_cluster_t<float, float>(a, p, s);
+}
+
+}  // namespace cis

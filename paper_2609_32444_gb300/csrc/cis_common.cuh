@@ -1,0 +1,281 @@
+// cis_common.cuh -- device helpers shared by the libcis kernels (sm_103a).
+//
+// Per-token arithmetic of the CIS token pass (arxiv 2609.32444):
+//   * the mismatch weight of Algorithm 1 / Eq. 4 (CIS) and Table 8 (TIS,
+//     exact ratio, no correction),
+//   * the PPO-clipped token objective of Eq. 1 and the scalar c_t that
+//     multiplies (softmax - onehot) in the logit gradient,
+//   * the row statistics (max / sum of exponentials) the log-softmax needs.
+//
+// Decisions (truncated or not, PPO clip active or not) are defined in fp64:
+// "log k > log cap" with log k = l_w - l_inf evaluated exactly.  The kernels
+// evaluate them in fp32 and keep that answer only when it is certain: the
+// fp32 operands carry relative errors of a few ulp (expm1f/log1pf/logf are
+// accurate to 1-2 ulp, the subtraction to 0.5 ulp), so a gap larger than
+// 4e-6 relative cannot change sign in exact arithmetic.  Inside that band the
+// comparison is redone in fp64.  The result equals the fp64 decision.
+#pragma once
+
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <math.h>
+#include <stdint.h>
+
+#include "cis.h"
+
+namespace cis {
+
+constexpr float kLog2e = 1.4426950408889634f;
+
+// Hyper-parameters as the kernels use them: fp32 copies for the fast path and
+// fp64 values (with logs taken on the host) for the certified fallback.
+struct DevParams {
+    int32_t mode;
+    int32_t agg;
+    float lam_f, kappa_f;
+    float tis_cap_f, exact_lo_f, exact_hi_f;
+    float rho_lo_f, rho_hi_f;  // 1 - c_low, 1 + c_high
+    float log_tis_cap_f, log_exact_lo_f, log_exact_hi_f, log_rho_lo_f, log_rho_hi_f;
+    double lam, kappa;
+    double log_tis_cap, log_exact_lo, log_exact_hi, log_rho_lo, log_rho_hi;
+};
+
+// Device status bits (cis_status_t values that can only be seen on the GPU).
+constexpr int32_t kStatusTimeout = CIS_ERR_DEVICE_TIMEOUT;
+constexpr int32_t kStatusBadId = CIS_ERR_BAD_TOKEN_ID;
+
+// Bounded waits: each mbarrier poll suspends for at most kPollSuspendNs, and a
+// wait gives up after kMaxPolls polls (about 2 s) and reports a timeout.
+constexpr uint32_t kPollSuspendNs = 1000;
+constexpr uint32_t kMaxPolls = 1u << 21;
+
+__device__ __forceinline__ void set_status(int32_t *status, int32_t bits)
+{
+    if (status)
+        atomicOr(status, bits);
+}
+
+// bf16 -> fp32 is exact: the bf16 bits are the top half of the binary32.
+__device__ __forceinline__ float bf16_lo(uint32_t w) { return __uint_as_float(w << 16); }
+__device__ __forceinline__ float bf16_hi(uint32_t w) { return __uint_as_float(w & 0xffff0000u); }
+
+template <typename T> __device__ __forceinline__ float to_f32(T v);
+template <> __device__ __forceinline__ float to_f32<float>(float v) { return v; }
+template <> __device__ __forceinline__ float to_f32<__nv_bfloat16>(__nv_bfloat16 v)
+{
+    return __bfloat162float(v);
+}
+
+// 2^x.  Pass 1 only sums these, so denormal results may flush (.ftz); pass 2
+// writes them out, so it keeps subnormal results.
+__device__ __forceinline__ float ex2_ftz(float x)
+{
+    float y;
+    asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
+__device__ __forceinline__ float ex2_full(float x)
+{
+    float y;
+    asm("ex2.approx.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
+
+// +1: a > b for certain; -1: a < b for certain (a <= b in the fp64 sense);
+// 0: too close to call from fp32 values with relative errors below ~1e-6.
+__device__ __forceinline__ int certain_cmp(float a, float b)
+{
+    float d = a - b;
+    float tol = 4e-6f * (fabsf(a) + fabsf(b)) + 1e-35f;
+    if (d > tol)
+        return 1;
+    if (d < -tol)
+        return -1;
+    return 0;
+}
+
+struct TokenWeight {
+    float w;
+    float logk;
+    uint8_t trunc;
+};
+
+// Mismatch weight from log p (lw, training side) and log q (linf, inference
+// side).  Algorithm 1: p = exp(lw), k = exp(lw - linf), phi = max(1-p, kappa),
+// w = min{k, 1 + lambda*phi}; Table 8 for the other modes.
+__device__ __forceinline__ TokenWeight token_weight(float lw, float linf, const DevParams &P)
+{
+    TokenWeight r;
+    const float logk = lw - linf;
+    r.logk = logk;
+    r.trunc = 0;
+    r.w = 1.0f;
+    switch (P.mode) {
+    case CIS_MODE_CIS: {
+        const float lam_phi = P.lam_f * fmaxf(-expm1f(lw), P.kappa_f);
+        const float lcap = log1pf(lam_phi);
+        const int s = certain_cmp(logk, lcap);
+        bool tr;
+        if (s != 0) {
+            tr = s > 0;
+        } else {
+            const double phi = fmax(-expm1((double)lw), P.kappa);
+            tr = ((double)lw - (double)linf) > log1p(P.lam * phi);
+        }
+        r.trunc = tr;
+        r.w = tr ? 1.0f + lam_phi : expf(logk);
+        break;
+    }
+    case CIS_MODE_TIS: {
+        const int s = certain_cmp(logk, P.log_tis_cap_f);
+        const bool tr = s != 0 ? s > 0 : ((double)lw - (double)linf) > P.log_tis_cap;
+        r.trunc = tr;
+        r.w = tr ? P.tis_cap_f : expf(logk);
+        break;
+    }
+    case CIS_MODE_EXACT: {
+        const int sh = certain_cmp(logk, P.log_exact_hi_f);
+        const bool hi = sh != 0 ? sh > 0 : ((double)lw - (double)linf) > P.log_exact_hi;
+        const int sl = certain_cmp(P.log_exact_lo_f, logk);
+        const bool lo = sl != 0 ? sl > 0 : ((double)lw - (double)linf) < P.log_exact_lo;
+        r.trunc = hi || lo;
+        r.w = hi ? P.exact_hi_f : (lo ? P.exact_lo_f : expf(logk));
+        break;
+    }
+    default:
+        break;
+    }
+    return r;
+}
+
+// eps = logit p - logit q (Lemma 3.1), from the two log-probabilities.
+__device__ __forceinline__ float token_eps(float lw, float linf)
+{
+    return (lw - linf) - logf(-expm1f(lw)) + logf(-expm1f(linf));
+}
+
+struct TokenLoss {
+    float c;      // s w A rho g: multiplies (softmax - onehot) in d loss / d z
+    double term;  // -s w min(rho A, clip(rho) A)
+};
+
+// Eq. 1 for one token: rho = exp(lp - lp_old) (1 in value without lp_old),
+// objective w min(rho A, clip(rho) A); the min takes the unclipped branch on
+// ties, so g = 0 only where the clip is strictly active.
+__device__ __forceinline__ TokenLoss token_loss(float lp, bool has_old, float lp_old, float A,
+                                                float s, float w, const DevParams &P)
+{
+    float rho = 1.0f;
+    bool g = true;
+    if (has_old) {
+        const float lr = lp - lp_old;
+        rho = expf(lr);
+        if (A > 0.0f) {
+            const int c = certain_cmp(lr, P.log_rho_hi_f);
+            g = c != 0 ? c < 0 : !(((double)lp - (double)lp_old) > P.log_rho_hi);
+        } else if (A < 0.0f) {
+            const int c = certain_cmp(lr, P.log_rho_lo_f);
+            g = c != 0 ? c > 0 : !(((double)lp - (double)lp_old) < P.log_rho_lo);
+        }
+    }
+    const float rho_c = fminf(fmaxf(rho, P.rho_lo_f), P.rho_hi_f);
+    const float obj = g ? rho * A : rho_c * A;
+    TokenLoss r;
+    r.term = -(double)s * (double)w * (double)obj;
+    r.c = g ? s * w * A * rho : 0.0f;
+    return r;
+}
+
+// log p of the sampled token from its log-odds d = z_y - log sum_{j != y} e^{z_j}:
+// log p = -softplus(-d), accurate for p near 0 and near 1.
+__device__ __forceinline__ float logprob_from_logodds(float d)
+{
+    return d > 0.0f ? -log1pf(expf(-d)) : d - log1pf(expf(d));
+}
+
+// ---------------------------------------------------------------------------
+// Row statistics over the entries j != y: (m, s) with s = sum e^{z_j - m}.
+struct MaxSum {
+    float m;
+    float s;
+};
+
+__device__ __forceinline__ MaxSum ms_combine(MaxSum a, MaxSum b)
+{
+    const float m = fmaxf(a.m, b.m);
+    if (m == -INFINITY)
+        return {m, a.s + b.s};  // both empty (their sums are 0 or NaN)
+    const float sa = a.m == -INFINITY ? a.s * 0.0f : a.s * ex2_ftz((a.m - m) * kLog2e);
+    const float sb = b.m == -INFINITY ? b.s * 0.0f : b.s * ex2_ftz((b.m - m) * kLog2e);
+    return {m, sa + sb};
+}
+
+__device__ __forceinline__ MaxSum warp_ms(MaxSum v)
+{
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        MaxSum u;
+        u.m = __shfl_xor_sync(0xffffffffu, v.m, o);
+        u.s = __shfl_xor_sync(0xffffffffu, v.s, o);
+        v = ms_combine(v, u);
+    }
+    return v;
+}
+
+// Block-wide (m, s); every thread gets the result.  `sh` needs NT/32 slots.
+template <int NT>
+__device__ __forceinline__ MaxSum block_ms(MaxSum v, MaxSum *sh)
+{
+    v = warp_ms(v);
+    const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+    if (lane == 0)
+        sh[wid] = v;
+    __syncthreads();
+    MaxSum r = sh[0];
+#pragma unroll
+    for (int i = 1; i < NT / 32; ++i)
+        r = ms_combine(r, sh[i]);
+    __syncthreads();
+    return r;
+}
+
+// Per-row scalars that pass 2 needs, from (m', s') over j != y and z_y.
+struct RowScalars {
+    float lp;         // log p of the sampled token
+    float lse;        // logsumexp of the row
+    float m;          // offset used for the exponent (m' or 0)
+    float bias_log2;  // (lse - m) * log2(e), +inf when no other entry is finite
+};
+
+__device__ __forceinline__ RowScalars row_scalars(MaxSum o, float zy)
+{
+    RowScalars r;
+    if (o.m == -INFINITY && o.s == 0.0f) {
+        // every other entry is -inf: p = 1
+        r.lp = zy != zy ? zy : 0.0f;
+        r.lse = zy;
+        r.m = 0.0f;
+        r.bias_log2 = INFINITY;
+        return r;
+    }
+    const float a = o.m + logf(o.s);  // log sum_{j != y} e^{z_j}
+    const float d = zy - a;           // logit p
+    r.lp = logprob_from_logodds(d);
+    r.lse = zy - r.lp;
+    r.m = o.m;
+    r.bias_log2 = ((zy - o.m) - r.lp) * kLog2e;
+    return r;
+}
+
+// Sum of e^{z - m} over 8 values, excluding lane index `skip` (-1 = none),
+// added pairwise to keep the rounding error independent of the row length.
+__device__ __forceinline__ float sum8_exp(const float (&z)[8], float m, int skip)
+{
+    float e[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i)
+        e[i] = (i == skip) ? 0.0f : ex2_ftz((z[i] - m) * kLog2e);
+    return ((e[0] + e[1]) + (e[2] + e[3])) + ((e[4] + e[5]) + (e[6] + e[7]));
+}
+
+}  // namespace cis

@@ -1,0 +1,69 @@
+// cis_kernels.h -- launch interface between the C ABI (cis_api.cu) and the
+// kernels.  Internal to libcis.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "cis_common.cuh"
+
+namespace cis {
+
+// Everything one fused token-pass launch needs.  Pointers are device pointers.
+struct PassArgs {
+    const void *logits;
+    int64_t T, V, ld;
+    const int32_t *ids;
+    const float *lp_inf;   // may be null for the forward-only kernel
+    const float *lp_old;   // null: on-policy (rho = 1 in value)
+    const float *adv;
+    const uint8_t *mask;   // null: every token valid
+    const float *scale;    // s_t [T]
+    void *dz;              // [T, ld_out] of the output dtype
+    int64_t ld_out;
+    float *lp_out;         // optional user outputs
+    float *lse_out;
+    float *w_out;
+    uint8_t *trunc_out;
+    float *ws_w;           // workspace copies used by the reduction
+    uint8_t *ws_trunc;
+    float *ws_logk;
+    double *ws_terms;
+    int32_t *status;
+    DevParams P;
+};
+
+// Workspace layout (offsets in bytes from the 256-byte aligned base).
+struct WsLayout {
+    size_t status, scale, terms, logk, w, trunc, total;
+};
+WsLayout ws_layout(int64_t T);
+
+// Forward-only: lp (and lse) of the sampled token, one CTA per row.
+cudaError_t launch_token_logprobs(const PassArgs &a, int dtype, cudaStream_t s);
+
+// Fused forward + backward, any layout: one CTA per row, second read from L2.
+cudaError_t launch_rowwise_fwd_bwd(const PassArgs &a, int dtype, int out_dtype,
+                                   cudaStream_t s);
+
+// Fused forward + backward, 16-byte aligned rows: a cluster of CTAs splits
+// each row, each CTA keeps its slice in shared memory (one HBM read).
+// Returns cudaErrorNotSupported when the shape does not fit the kernel.
+cudaError_t launch_cluster_fwd_bwd(const PassArgs &a, int dtype, int out_dtype,
+                                   cudaStream_t s);
+bool cluster_path_applies(const PassArgs &a, int dtype, int out_dtype);
+
+// Loss scales s_t (and clears the status word).
+cudaError_t launch_scales(const uint8_t *mask, int64_t T, const int32_t *cu_seqlens, int64_t B,
+                          int agg, float *scale, int32_t *status, cudaStream_t s);
+
+// Elementwise weights (cis_weights).
+cudaError_t launch_weights(const float *lp_w, const float *lp_inf, const uint8_t *mask,
+                           int64_t T, const DevParams &P, float *w_out, uint8_t *trunc_out,
+                           float *eps_out, cudaStream_t s);
+
+// Deterministic reduction of the per-token terms into the loss and stats.
+cudaError_t launch_reduce(const PassArgs &a, cis_stats_t *stats, double *loss,
+                          cudaStream_t s);
+
+}  // namespace cis

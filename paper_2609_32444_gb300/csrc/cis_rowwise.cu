@@ -1,0 +1,210 @@
+// cis_rowwise.cu -- row-streaming kernels of libcis (any row layout).
+//
+// One CTA per token row.  Pass 1 streams the row once and keeps a running
+// (max, sum of exponentials) over the entries j != y_t; the sampled entry is
+// left out so that its log-probability comes from the log-odds
+//   d = z_y - log sum_{j != y} e^{z_j},   log p = -softplus(-d),
+// which stays accurate when p is within an ulp of 1 (Sec. 3.3 notes that the
+// logits of p and q stop being finite there; the log-odds form avoids the
+// cancellation in 1 - p).  The forward kernel stops there.  The fused kernel
+// then forms the weight and the token loss (cis_common.cuh) and streams the
+// row a second time -- from L2 when it is still resident -- to write
+//   dz_j = c (softmax_j - [j == y]).
+// These kernels accept any alignment and row stride; the cluster kernel in
+// cis_cluster.cu is the fast path for 16-byte aligned rows.
+#include "cis_kernels.h"
+
+namespace cis {
+namespace {
+
+constexpr int kRowThreads = 256;
+
+__device__ __forceinline__ float max_nan(float a, float b)
+{
+    float r;
+    asm("max.NaN.f32 %0, %1, %2;" : "=f"(r) : "f"(a), "f"(b));
+    return r;
+}
+
+template <typename T> __device__ __forceinline__ T from_f32(float v);
+template <> __device__ __forceinline__ float from_f32<float>(float v) { return v; }
+template <> __device__ __forceinline__ __nv_bfloat16 from_f32<__nv_bfloat16>(float v)
+{
+    return __float2bfloat16_rn(v);
+}
+
+// Add EV values to a running (m, s), leaving out position `skip` (-1: none).
+template <int EV>
+__device__ __forceinline__ void ms_update(MaxSum &acc, const float (&z)[EV], int skip)
+{
+    float lm = -INFINITY;
+#pragma unroll
+    for (int i = 0; i < EV; ++i)
+        lm = max_nan(lm, i == skip ? -INFINITY : z[i]);
+    if (lm > acc.m || lm != lm) {
+        acc.s = acc.s * ex2_ftz((acc.m - lm) * kLog2e);
+        acc.m = lm;
+    }
+    if (acc.m != -INFINITY) {
+        float e[EV];
+#pragma unroll
+        for (int i = 0; i < EV; ++i)
+            e[i] = i == skip ? 0.0f : ex2_ftz((z[i] - acc.m) * kLog2e);
+#pragma unroll
+        for (int w = 1; w < EV; w <<= 1)
+#pragma unroll
+            for (int i = 0; i + w < EV; i += 2 * w)
+                e[i] += e[i + w];
+        acc.s += e[0];
+    }
+}
+
+template <typename InT, bool kStream>
+__device__ __forceinline__ uint4 load16(const uint4 *p)
+{
+    return kStream ? __ldcs(p) : __ldg(p);
+}
+
+// Unpack one 16-byte vector into floats.
+__device__ __forceinline__ void unpack(uint4 q, float (&z)[8])
+{
+    z[0] = bf16_lo(q.x); z[1] = bf16_hi(q.x);
+    z[2] = bf16_lo(q.y); z[3] = bf16_hi(q.y);
+    z[4] = bf16_lo(q.z); z[5] = bf16_hi(q.z);
+    z[6] = bf16_lo(q.w); z[7] = bf16_hi(q.w);
+}
+__device__ __forceinline__ void unpack(uint4 q, float (&z)[4])
+{
+    z[0] = __uint_as_float(q.x); z[1] = __uint_as_float(q.y);
+    z[2] = __uint_as_float(q.z); z[3] = __uint_as_float(q.w);
+}
+
+// This thread's (m, s) over entries j != y of one row.
+template <typename InT, bool kStream>
+__device__ MaxSum row_stats(const InT *row, int64_t V, int64_t y)
+{
+    constexpr int EV = 16 / sizeof(InT);
+    MaxSum acc{-INFINITY, 0.0f};
+    int64_t j0 = 0;
+    if ((reinterpret_cast<uintptr_t>(row) & 15) == 0) {
+        const int64_t nvec = V / EV;
+        const uint4 *rv = reinterpret_cast<const uint4 *>(row);
+        for (int64_t v = threadIdx.x; v < nvec; v += kRowThreads) {
+            float z[EV];
+            unpack(load16<InT, kStream>(rv + v), z);
+            const int64_t rel = y - v * EV;
+            ms_update<EV>(acc, z, (rel >= 0 && rel < EV) ? (int)rel : -1);
+        }
+        j0 = nvec * EV;
+    }
+    for (int64_t j = j0 + threadIdx.x; j < V; j += kRowThreads) {
+        float z[1] = {to_f32(row[j])};
+        ms_update<1>(acc, z, j == y ? 0 : -1);
+    }
+    return acc;
+}
+
+struct RowShared {
+    MaxSum red[kRowThreads / 32];
+    float c, m, bias, lp;
+};
+
+template <typename InT, typename OutT, bool kBwd>
+__global__ void __launch_bounds__(kRowThreads) row_kernel(const PassArgs a)
+{
+    __shared__ RowShared sh;
+    const int64_t t = blockIdx.x;
+    const bool valid = a.mask == nullptr || a.mask[t] != 0;
+    const int64_t y = a.ids[t];
+    const bool id_ok = y >= 0 && y < a.V;
+    if (!valid || !id_ok) {
+        if (kBwd) {
+            OutT *orow = reinterpret_cast<OutT *>(a.dz) + t * a.ld_out;
+            for (int64_t j = threadIdx.x; j < a.V; j += kRowThreads)
+                orow[j] = from_f32<OutT>(0.0f);
+        }
+        if (threadIdx.x == 0) {
+            const float lp = valid ? NAN : 0.0f;
+            if (valid)
+                set_status(a.status, kStatusBadId);
+            if (a.lp_out) a.lp_out[t] = lp;
+            if (a.lse_out) a.lse_out[t] = lp;
+            if (kBwd) {
+                if (a.w_out) a.w_out[t] = 0.0f;
+                if (a.trunc_out) a.trunc_out[t] = 0;
+                a.ws_w[t] = 0.0f;
+                a.ws_trunc[t] = 0;
+                a.ws_logk[t] = 0.0f;
+                a.ws_terms[t] = valid ? (double)NAN : 0.0;
+            }
+        }
+        return;
+    }
+    const InT *row = reinterpret_cast<const InT *>(a.logits) + t * a.ld;
+    const MaxSum o = block_ms<kRowThreads>(row_stats<InT, !kBwd>(row, a.V, y), sh.red);
+    if (threadIdx.x == 0) {
+        const RowScalars rs = row_scalars(o, to_f32(row[y]));
+        if (a.lp_out) a.lp_out[t] = rs.lp;
+        if (a.lse_out) a.lse_out[t] = rs.lse;
+        if (kBwd) {
+            const bool has_old = a.lp_old != nullptr;
+            const float lw = has_old ? a.lp_old[t] : rs.lp;
+            const TokenWeight tw = token_weight(lw, a.lp_inf[t], a.P);
+            const TokenLoss tl = token_loss(rs.lp, has_old, has_old ? a.lp_old[t] : 0.0f,
+                                            a.adv[t], a.scale[t], tw.w, a.P);
+            if (a.w_out) a.w_out[t] = tw.w;
+            if (a.trunc_out) a.trunc_out[t] = tw.trunc;
+            a.ws_w[t] = tw.w;
+            a.ws_trunc[t] = tw.trunc;
+            a.ws_logk[t] = tw.logk;
+            a.ws_terms[t] = tl.term;
+            sh.c = tl.c;
+            sh.m = rs.m;
+            sh.bias = rs.bias_log2;
+            sh.lp = rs.lp;
+        }
+    }
+    if (!kBwd)
+        return;
+    __syncthreads();
+    const float c = sh.c, m = sh.m, bias = sh.bias;
+    const float dzy = c * expm1f(sh.lp);  // c (p - 1)
+    OutT *orow = reinterpret_cast<OutT *>(a.dz) + t * a.ld_out;
+    for (int64_t j = threadIdx.x; j < a.V; j += kRowThreads) {
+        const float z = to_f32(row[j]);
+        const float v = j == y ? dzy : c * ex2_full(fmaf(z - m, kLog2e, -bias));
+        orow[j] = from_f32<OutT>(v);
+    }
+}
+
+template <typename InT, typename OutT, bool kBwd>
+cudaError_t launch_row(const PassArgs &a, cudaStream_t s)
+{
+    if (a.T == 0)
+        return cudaSuccess;
+    row_kernel<InT, OutT, kBwd><<<(unsigned)a.T, kRowThreads, 0, s>>>(a);
+    return cudaGetLastError();
+}
+
+}  // namespace
+
+cudaError_t launch_token_logprobs(const PassArgs &a, int dtype, cudaStream_t s)
+{
+    if (dtype == CIS_BF16)
+        return launch_row<__nv_bfloat16, float, false>(a, s);
+    return launch_row<float, float, false>(a, s);
+}
+
+cudaError_t launch_rowwise_fwd_bwd(const PassArgs &a, int dtype, int out_dtype, cudaStream_t s)
+{
+    if (dtype == CIS_BF16) {
+        if (out_dtype == CIS_BF16)
+            return launch_row<__nv_bfloat16, __nv_bfloat16, true>(a, s);
+        return launch_row<__nv_bfloat16, float, true>(a, s);
+    }
+    if (out_dtype == CIS_BF16)
+        return launch_row<float, __nv_bfloat16, true>(a, s);
+    return launch_row<float, float, true>(a, s);
+}
+
+}  // namespace cis

@@ -1,0 +1,204 @@
+// cis_small.cu -- the [T]-sized kernels of libcis.
+//
+//   scales_kernel   the loss normaliser s_t: 1/n over the n valid tokens
+//                   (Algorithm 1) or 1/(G |y_i|) per response (Eq. 1); it
+//                   also clears the device status word of the call.
+//   weights_kernel  cis_weights: Algorithm 1 / Table 8, one thread per token.
+//   reduce_kernel   deterministic sums of the per-token loss terms and the
+//                   statistics the paper logs (App. D.1: share of tokens acted
+//                   on, largest |log k|; App. D.5: the truncated excess).
+#include "cis_kernels.h"
+
+namespace cis {
+namespace {
+
+constexpr int kSmallThreads = 1024;
+constexpr int kMaxSeqInShared = 12000;
+
+__device__ __forceinline__ bool is_valid(const uint8_t *mask, int64_t t)
+{
+    return mask == nullptr || mask[t] != 0;
+}
+
+template <typename T>
+__device__ __forceinline__ T warp_sum(T v)
+{
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1)
+        v += __shfl_xor_sync(0xffffffffu, v, o);
+    return v;
+}
+
+__global__ void __launch_bounds__(kSmallThreads)
+    scales_kernel(const uint8_t *mask, int64_t T, const int32_t *cu, int64_t B, int agg,
+                  float *scale, int32_t *status)
+{
+    __shared__ long long part[kSmallThreads / 32];
+    __shared__ int cnt[kMaxSeqInShared];
+    const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+    if (threadIdx.x == 0 && status)
+        *status = 0;
+    if (agg == CIS_AGG_SEQ_MEAN_TOKEN_MEAN && cu != nullptr) {
+        // valid tokens of each response (one warp per response)
+        for (int64_t i = wid; i < B; i += kSmallThreads / 32) {
+            int64_t lo = cu[i], hi = cu[i + 1];
+            lo = lo < 0 ? 0 : (lo > T ? T : lo);
+            hi = hi < lo ? lo : (hi > T ? T : hi);
+            int c = 0;
+            for (int64_t t = lo + lane; t < hi; t += 32)
+                c += is_valid(mask, t);
+            c = warp_sum(c);
+            if (lane == 0)
+                cnt[i] = c;
+        }
+        __syncthreads();
+        long long g = 0;
+        for (int64_t i = threadIdx.x; i < B; i += kSmallThreads)
+            g += cnt[i] > 0;
+        g = warp_sum(g);
+        if (lane == 0)
+            part[wid] = g;
+        for (int64_t t = threadIdx.x; t < T; t += kSmallThreads)
+            scale[t] = 0.0f;
+        __syncthreads();
+        long long G = 0;
+        for (int i = 0; i < kSmallThreads / 32; ++i)
+            G += part[i];
+        for (int64_t i = wid; i < B; i += kSmallThreads / 32) {
+            int64_t lo = cu[i], hi = cu[i + 1];
+            lo = lo < 0 ? 0 : (lo > T ? T : lo);
+            hi = hi < lo ? lo : (hi > T ? T : hi);
+            const int n = cnt[i];
+            const float s = n > 0 ? (float)(1.0 / ((double)G * (double)n)) : 0.0f;
+            for (int64_t t = lo + lane; t < hi; t += 32)
+                scale[t] = is_valid(mask, t) ? s : 0.0f;
+        }
+        return;
+    }
+    long long n = 0;
+    for (int64_t t = threadIdx.x; t < T; t += kSmallThreads)
+        n += is_valid(mask, t);
+    n = warp_sum(n);
+    if (lane == 0)
+        part[wid] = n;
+    __syncthreads();
+    long long N = 0;
+    for (int i = 0; i < kSmallThreads / 32; ++i)
+        N += part[i];
+    const float s = N > 0 ? (float)(1.0 / (double)N) : 0.0f;
+    for (int64_t t = threadIdx.x; t < T; t += kSmallThreads)
+        scale[t] = is_valid(mask, t) ? s : 0.0f;
+}
+
+__global__ void weights_kernel(const float *lp_w, const float *lp_inf, const uint8_t *mask,
+                               int64_t T, const DevParams P, float *w_out, uint8_t *trunc_out,
+                               float *eps_out)
+{
+    for (int64_t t = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; t < T;
+         t += (int64_t)gridDim.x * blockDim.x) {
+        float w = 0.0f, e = 0.0f;
+        uint8_t tr = 0;
+        if (is_valid(mask, t)) {
+            const float lw = lp_w[t], li = lp_inf[t];
+            const TokenWeight tw = token_weight(lw, li, P);
+            w = tw.w;
+            tr = tw.trunc;
+            if (eps_out)
+                e = token_eps(lw, li);
+        }
+        w_out[t] = w;
+        if (trunc_out)
+            trunc_out[t] = tr;
+        if (eps_out)
+            eps_out[t] = e;
+    }
+}
+
+struct RedPart {
+    double loss, excess;
+    long long nvalid, ntrunc;
+    float maxlk;
+};
+
+// One CTA: thread i sums tokens i, i + 1024, ... in order, then a fixed tree.
+__global__ void __launch_bounds__(kSmallThreads)
+    reduce_kernel(const uint8_t *mask, int64_t T, const double *terms, const float *logk,
+                  const float *w, const uint8_t *trunc, const int32_t *status,
+                  cis_stats_t *stats, double *loss_out)
+{
+    __shared__ RedPart sh[kSmallThreads];
+    RedPart p{0.0, 0.0, 0, 0, 0.0f};
+    for (int64_t t = threadIdx.x; t < T; t += kSmallThreads) {
+        p.loss += terms[t];
+        if (!is_valid(mask, t))
+            continue;
+        p.nvalid += 1;
+        const float lk = logk[t];
+        p.maxlk = fmaxf(p.maxlk, fabsf(lk));
+        if (trunc[t]) {
+            p.ntrunc += 1;
+            p.excess += exp((double)lk) - (double)w[t];
+        }
+    }
+    sh[threadIdx.x] = p;
+    __syncthreads();
+    for (int stride = kSmallThreads / 2; stride > 0; stride >>= 1) {
+        if (threadIdx.x < stride) {
+            RedPart &a = sh[threadIdx.x];
+            const RedPart &b = sh[threadIdx.x + stride];
+            a.loss += b.loss;
+            a.excess += b.excess;
+            a.nvalid += b.nvalid;
+            a.ntrunc += b.ntrunc;
+            a.maxlk = fmaxf(a.maxlk, b.maxlk);
+        }
+        __syncthreads();
+    }
+    if (threadIdx.x == 0) {
+        const RedPart &r = sh[0];
+        if (loss_out)
+            *loss_out = r.loss;
+        if (stats) {
+            stats->loss = r.loss;
+            stats->trunc_excess = r.excess;
+            stats->n_valid = r.nvalid;
+            stats->n_truncated = r.ntrunc;
+            stats->max_abs_logk = r.maxlk;
+            stats->status = status ? *status : 0;
+        }
+    }
+}
+
+}  // namespace
+
+cudaError_t launch_scales(const uint8_t *mask, int64_t T, const int32_t *cu_seqlens, int64_t B,
+                          int agg, float *scale, int32_t *status, cudaStream_t s)
+{
+    if (agg == CIS_AGG_SEQ_MEAN_TOKEN_MEAN && B > kMaxSeqInShared)
+        return cudaErrorNotSupported;
+    scales_kernel<<<1, kSmallThreads, 0, s>>>(mask, T, cu_seqlens, B, agg, scale, status);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_weights(const float *lp_w, const float *lp_inf, const uint8_t *mask,
+                           int64_t T, const DevParams &P, float *w_out, uint8_t *trunc_out,
+                           float *eps_out, cudaStream_t s)
+{
+    if (T == 0)
+        return cudaSuccess;
+    int64_t blocks = (T + 255) / 256;
+    if (blocks > 4096)
+        blocks = 4096;
+    weights_kernel<<<(unsigned)blocks, 256, 0, s>>>(lp_w, lp_inf, mask, T, P, w_out, trunc_out,
+                                                    eps_out);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_reduce(const PassArgs &a, cis_stats_t *stats, double *loss, cudaStream_t s)
+{
+    reduce_kernel<<<1, kSmallThreads, 0, s>>>(a.mask, a.T, a.ws_terms, a.ws_logk, a.ws_w,
+                                               a.ws_trunc, a.status, stats, loss);
+    return cudaGetLastError();
+}
+
+}  // namespace cis

@@ -1,0 +1,122 @@
+"""Host-side tests of the C ABI: the library builds, loads, exports exactly the
+functions include/*.h declares, and rejects bad arguments before touching the
+GPU.  No compute call is made, so these run without a GPU."""
+import ctypes
+import glob
+import os
+import re
+import shutil
+import subprocess
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+pytestmark = pytest.mark.skipif(shutil.which("nvcc") is None and
+                                not os.path.exists("/usr/local/cuda/bin/nvcc"),
+                                reason="needs nvcc to build libcis")
+
+
+@pytest.fixture(scope="module")
+def binding():
+    from paper_2609_32444_gb300 import build, binding as b
+    build.build()
+    b.lib()
+    return b
+
+
+def _declared():
+    names = set()
+    for h in glob.glob(os.path.join(ROOT, "include", "*.h")):
+        src = open(h).read()
+        names |= set(re.findall(r"CIS_API\s+[\w\s\*]+?\b(cis_\w+)\s*\(", src))
+    return names
+
+
+def test_exports_match_header(binding):
+    declared = _declared()
+    assert {"cis_loss_fwd_bwd", "cis_weights", "cis_token_logprobs"} <= declared
+    out = subprocess.run(["nm", "-D", "--defined-only", binding.library_path()],
+                         capture_output=True, text=True, check=True).stdout
+    exported = {ln.split()[-1] for ln in out.splitlines() if " T " in ln}
+    exported = {n for n in exported if n.startswith("cis_")}
+    assert exported == declared
+    lib = binding.lib()
+    for n in declared:
+        assert hasattr(lib, n)
+
+
+def test_default_params_are_the_papers(binding):
+    p = binding.cis_default_params()
+    assert (p.mode, p.agg) == (0, 0)
+    assert (p.lam, p.kappa, p.tis_cap) == (2.3, 5e-3, 2.0)
+    assert (p.exact_lo, p.exact_hi, p.clip_low, p.clip_high) == (1e-6, 1e6, 0.2, 0.28)
+
+
+def test_status_strings(binding):
+    for code in (0, 1, 2, 3, 4, 8):
+        assert binding.status_string(code).startswith("CIS_")
+    assert binding.status_string(12345) == "unknown cis status"
+
+
+def test_workspace_size_grows_with_tokens(binding):
+    a = binding.cis_loss_workspace_size(0, 10)
+    b = binding.cis_loss_workspace_size(1000, 10)
+    assert a >= 4 and b >= a + 1000 * (4 + 8 + 4 + 4 + 1)
+    assert binding.lib().cis_loss_workspace_size(-1, 10, ctypes.byref(ctypes.c_size_t())) == 1
+
+
+def _fwd_bwd_rc(binding, **over):
+    """Call cis_loss_fwd_bwd with fake non-null pointers; validation must fail
+    before any pointer is dereferenced or any kernel launched."""
+    L = binding.lib()
+    fake = ctypes.c_void_p(0x10000)
+    ws = ctypes.c_void_p(0x20000)
+    p = binding.cis_default_params()
+    for k, v in over.pop("params", {}).items():
+        setattr(p, k, v)
+    args = dict(logits=fake, dtype=1, T=4, V=8, ld=8, ids=fake, lp_inf=fake, lp_old=None,
+                adv=fake, mask=None, cu=None, B=0, dz=ctypes.c_void_p(0x40000), dz_dt=1,
+                ld_out=8, ws=ws, ws_bytes=1 << 20)
+    args.update(over)
+    return L.cis_loss_fwd_bwd(args["logits"], args["dtype"], args["T"], args["V"], args["ld"],
+                              args["ids"], args["lp_inf"], args["lp_old"], args["adv"],
+                              args["mask"], args["cu"], args["B"], ctypes.byref(p), args["dz"],
+                              args["dz_dt"], args["ld_out"], None, None, None, None, None,
+                              args["ws"], args["ws_bytes"], None)
+
+
+@pytest.mark.parametrize("over", [
+    dict(T=-1), dict(V=0), dict(ld=7), dict(ld_out=7), dict(dtype=5), dict(dz_dt=2),
+    dict(logits=None), dict(ids=None), dict(lp_inf=None), dict(adv=None), dict(dz=None),
+    dict(ws=None), dict(ws=ctypes.c_void_p(0x20010)), dict(ws_bytes=16),
+    dict(params=dict(lam=-1.0)), dict(params=dict(kappa=1.5)), dict(params=dict(tis_cap=0.5)),
+    dict(params=dict(exact_lo=0.0)), dict(params=dict(clip_low=1.0)),
+    dict(params=dict(mode=9)), dict(params=dict(agg=1)),  # seq mean without cu_seqlens
+    dict(params=dict(lam=float("nan"))),
+    dict(dz=ctypes.c_void_p(0x10000 + 16)),  # dlogits overlaps the logits
+])
+def test_fwd_bwd_rejects_bad_arguments(binding, over):
+    assert _fwd_bwd_rc(binding, **over) == 1
+
+
+def test_other_entry_points_reject_bad_arguments(binding):
+    L = binding.lib()
+    fake = ctypes.c_void_p(0x10000)
+    p = binding.cis_default_params()
+    assert L.cis_token_logprobs(fake, 1, 4, 8, 7, fake, None, fake, None, None, None) == 1
+    assert L.cis_token_logprobs(None, 1, 4, 8, 8, fake, None, fake, None, None, None) == 1
+    assert L.cis_token_logprobs(fake, 1, 0, 8, 8, None, None, None, None, None, None) == 0
+    p.kappa = 2.0
+    assert L.cis_weights(fake, fake, None, 4, ctypes.byref(p), fake, None, None, None) == 1
+    p.kappa = 5e-3
+    assert L.cis_weights(None, fake, None, 4, ctypes.byref(p), fake, None, None, None) == 1
+    assert L.cis_weights(None, None, None, 0, ctypes.byref(p), None, None, None, None) == 0
+    assert L.cis_default_params(None) == 1
+
+
+def test_binding_refuses_cpu_tensors(binding):
+    import torch
+    x = torch.zeros(2, 8)
+    with pytest.raises(ValueError):
+        binding.cis_token_logprobs(x, torch.zeros(2, dtype=torch.int32))
