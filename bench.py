@@ -51,6 +51,8 @@ def parse_args():
     ap.add_argument("--e2e-steps", type=int, default=10)
     ap.add_argument("--cpu-seconds", type=float, default=10.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--tokens", type=int, default=None,
+                    help="smaller T with the same recipe (for profiler captures only)")
     return ap.parse_args()
 
 
@@ -258,7 +260,8 @@ def run_ours(args, rank, world, local):
     torch.cuda.set_device(local)
     dev = torch.device("cuda", local)
     spec = synth.WORKLOADS[args.workload]
-    b = synth.make_batch(args.workload, device=dev, seed=1000 + args.workload + 7919 * rank)
+    b = synth.make_batch(args.workload, device=dev, seed=1000 + args.workload + 7919 * rank,
+                         T=args.tokens)
     T, V = b.T, b.V
     dz_dt = torch.bfloat16 if args.dlogits == "bf16" else torch.float32
     P = binding.cis_default_params(args.mode, lam=b.lam)
@@ -279,6 +282,9 @@ def run_ours(args, rank, world, local):
     stream = torch.cuda.current_stream()
     kev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
            for _ in range(args.steps)]
+    for a_, z_ in kev:  # torch creates the CUDA event on first record
+        a_.record(stream)
+        z_.record(stream)
     clocks = ClockSampler(physical_gpu_index(local))
     time.sleep(0.5)
     start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
@@ -363,7 +369,8 @@ def run_ours(args, rank, world, local):
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_per_step,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
             "data": "synthetic",
-            "config": {"workload": spec["name"], "T": T, "V": V, "mode": args.mode,
+            "config": {"workload": spec["name"] if args.tokens is None else
+                       f"{spec['name']} (T reduced to {T})", "T": T, "V": V, "mode": args.mode,
                        "lambda": b.lam, "kappa": 5e-3, "io_dtype": "bf16" if isz == 2 else "f32",
                        "dlogits": args.dlogits, "valid_tokens": nvalid,
                        "l2": "no flush: the 4.98 GB of logits per step exceed the 129 MB L2",

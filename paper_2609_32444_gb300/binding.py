@@ -237,6 +237,8 @@ def cis_profile_next_call(begin: "torch.cuda.Event | None", end: "torch.cuda.Eve
     its main kernel (timing aid; the call does the same work)."""
     b = None if begin is None else ctypes.c_void_p(begin.cuda_event)
     e = None if end is None else ctypes.c_void_p(end.cuda_event)
+    if (begin is not None and not b.value) or (end is not None and not e.value):
+        raise ValueError("record the events once first: torch creates them lazily")
     _check(lib().cis_profile_next_call(b, e), "cis_profile_next_call")
 
 

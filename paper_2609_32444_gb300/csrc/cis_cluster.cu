@@ -251,8 +251,8 @@ __global__ void __launch_bounds__(kThreads) cluster_kernel(const PassArgs a, int
     if (threadIdx.x == 0) {
         const RowScalars rs = row_scalars(o, zy);
         const bool has_old = a.lp_old != nullptr;
-        const TokenWeight tw = token_weight(has_old ? lold : rs.lp, linf, a.P);
-        const TokenLoss tl = token_loss(rs.lp, has_old, lold, adv, sc, tw.w, a.P);
+        const TokenWeight tw = token_weight(has_old ? (double)lold : rs.lp64, linf, a.P);
+        const TokenLoss tl = token_loss(rs.lp64, has_old, lold, adv, sc, tw.w, a.P);
         if (rank == 0) {
             if (a.lp_out) a.lp_out[t] = rs.lp;
             if (a.w_out) a.w_out[t] = tw.w;

@@ -100,27 +100,30 @@ struct TokenWeight {
     uint8_t trunc;
 };
 
-// Mismatch weight from log p (lw, training side) and log q (linf, inference
-// side).  Algorithm 1: p = exp(lw), k = exp(lw - linf), phi = max(1-p, kappa),
+// Mismatch weight from log p (lw, training side, fp64 so that a log p carried
+// to better than fp32 keeps its accuracy) and log q (linf, inference side).
+// Algorithm 1: p = exp(lw), k = exp(lw - linf), phi = max(1-p, kappa),
 // w = min{k, 1 + lambda*phi}; Table 8 for the other modes.
-__device__ __forceinline__ TokenWeight token_weight(float lw, float linf, const DevParams &P)
+__device__ __forceinline__ TokenWeight token_weight(double lw, float linf, const DevParams &P)
 {
     TokenWeight r;
-    const float logk = lw - linf;
+    const double logk64 = lw - (double)linf;  // exact when lw is an fp32 value
+    const float logk = (float)logk64;
+    const float lwf = (float)lw;
     r.logk = logk;
     r.trunc = 0;
     r.w = 1.0f;
     switch (P.mode) {
     case CIS_MODE_CIS: {
-        const float lam_phi = P.lam_f * fmaxf(-expm1f(lw), P.kappa_f);
+        const float lam_phi = P.lam_f * fmaxf(-expm1f(lwf), P.kappa_f);
         const float lcap = log1pf(lam_phi);
         const int s = certain_cmp(logk, lcap);
         bool tr;
         if (s != 0) {
             tr = s > 0;
         } else {
-            const double phi = fmax(-expm1((double)lw), P.kappa);
-            tr = ((double)lw - (double)linf) > log1p(P.lam * phi);
+            const double phi = fmax(-expm1(lw), P.kappa);
+            tr = logk64 > log1p(P.lam * phi);
         }
         r.trunc = tr;
         r.w = tr ? 1.0f + lam_phi : expf(logk);
@@ -128,16 +131,16 @@ __device__ __forceinline__ TokenWeight token_weight(float lw, float linf, const 
     }
     case CIS_MODE_TIS: {
         const int s = certain_cmp(logk, P.log_tis_cap_f);
-        const bool tr = s != 0 ? s > 0 : ((double)lw - (double)linf) > P.log_tis_cap;
+        const bool tr = s != 0 ? s > 0 : logk64 > P.log_tis_cap;
         r.trunc = tr;
         r.w = tr ? P.tis_cap_f : expf(logk);
         break;
     }
     case CIS_MODE_EXACT: {
         const int sh = certain_cmp(logk, P.log_exact_hi_f);
-        const bool hi = sh != 0 ? sh > 0 : ((double)lw - (double)linf) > P.log_exact_hi;
+        const bool hi = sh != 0 ? sh > 0 : logk64 > P.log_exact_hi;
         const int sl = certain_cmp(P.log_exact_lo_f, logk);
-        const bool lo = sl != 0 ? sl > 0 : ((double)lw - (double)linf) < P.log_exact_lo;
+        const bool lo = sl != 0 ? sl > 0 : logk64 < P.log_exact_lo;
         r.trunc = hi || lo;
         r.w = hi ? P.exact_hi_f : (lo ? P.exact_lo_f : expf(logk));
         break;
@@ -161,21 +164,23 @@ struct TokenLoss {
 
 // Eq. 1 for one token: rho = exp(lp - lp_old) (1 in value without lp_old),
 // objective w min(rho A, clip(rho) A); the min takes the unclipped branch on
-// ties, so g = 0 only where the clip is strictly active.
-__device__ __forceinline__ TokenLoss token_loss(float lp, bool has_old, float lp_old, float A,
+// ties, so g = 0 only where the clip is strictly active.  lp in fp64 (see
+// token_weight).
+__device__ __forceinline__ TokenLoss token_loss(double lp, bool has_old, float lp_old, float A,
                                                 float s, float w, const DevParams &P)
 {
     float rho = 1.0f;
     bool g = true;
     if (has_old) {
-        const float lr = lp - lp_old;
+        const double lr64 = lp - (double)lp_old;
+        const float lr = (float)lr64;
         rho = expf(lr);
         if (A > 0.0f) {
             const int c = certain_cmp(lr, P.log_rho_hi_f);
-            g = c != 0 ? c < 0 : !(((double)lp - (double)lp_old) > P.log_rho_hi);
+            g = c != 0 ? c < 0 : !(lr64 > P.log_rho_hi);
         } else if (A < 0.0f) {
             const int c = certain_cmp(lr, P.log_rho_lo_f);
-            g = c != 0 ? c > 0 : !(((double)lp - (double)lp_old) < P.log_rho_lo);
+            g = c != 0 ? c > 0 : !(lr64 < P.log_rho_lo);
         }
     }
     const float rho_c = fminf(fmaxf(rho, P.rho_lo_f), P.rho_hi_f);
@@ -184,13 +189,6 @@ __device__ __forceinline__ TokenLoss token_loss(float lp, bool has_old, float lp
     r.term = -(double)s * (double)w * (double)obj;
     r.c = g ? s * w * A * rho : 0.0f;
     return r;
-}
-
-// log p of the sampled token from its log-odds d = z_y - log sum_{j != y} e^{z_j}:
-// log p = -softplus(-d), accurate for p near 0 and near 1.
-__device__ __forceinline__ float logprob_from_logodds(float d)
-{
-    return d > 0.0f ? -log1pf(expf(-d)) : d - log1pf(expf(d));
 }
 
 // ---------------------------------------------------------------------------
@@ -239,9 +237,16 @@ __device__ __forceinline__ MaxSum block_ms(MaxSum v, MaxSum *sh)
     return r;
 }
 
-// Per-row scalars that pass 2 needs, from (m', s') over j != y and z_y.
+// Per-row scalars from (m', s') over j != y and z_y.  With the log-odds
+//   d = z_y - log sum_{j != y} e^{z_j} = (z_y - m') - log s',
+// log p = -softplus(-d) is accurate for p near 0 and near 1 (Sec. 3.3 notes
+// that logit p stops being finite when p rounds to 1; d itself stays finite).
+// For d <= 0, log p = d - log1p(e^d) can be large in magnitude, so it is also
+// kept in fp64 (lp64, ~1e-6 absolute) for the weight; lse - m' is formed
+// without cancellation for pass 2.
 struct RowScalars {
-    float lp;         // log p of the sampled token
+    float lp;         // log p of the sampled token (fp32 output)
+    double lp64;      // the same, carried in fp64
     float lse;        // logsumexp of the row
     float m;          // offset used for the exponent (m' or 0)
     float bias_log2;  // (lse - m) * log2(e), +inf when no other entry is finite
@@ -253,17 +258,30 @@ __device__ __forceinline__ RowScalars row_scalars(MaxSum o, float zy)
     if (o.m == -INFINITY && o.s == 0.0f) {
         // every other entry is -inf: p = 1
         r.lp = zy != zy ? zy : 0.0f;
+        r.lp64 = r.lp;
         r.lse = zy;
         r.m = 0.0f;
         r.bias_log2 = INFINITY;
         return r;
     }
-    const float a = o.m + logf(o.s);  // log sum_{j != y} e^{z_j}
-    const float d = zy - a;           // logit p
-    r.lp = logprob_from_logodds(d);
-    r.lse = zy - r.lp;
+    const double dz64 = (double)zy - (double)o.m;  // exact
+    const float ls = logf(o.s);
+    const float d = (float)(dz64 - (double)ls);      // logit p
+    float lse_m;                                     // lse - m'
+    if (d > 0.0f) {
+        const float t = log1pf(expf(-d));            // softplus(-d) = -log p
+        r.lp = -t;
+        r.lp64 = -(double)t;
+        lse_m = (float)(dz64 + (double)t);
+    } else {
+        const float t = log1pf(expf(d));             // softplus(d)
+        r.lp64 = (dz64 - (double)ls) - (double)t;
+        r.lp = (float)r.lp64;
+        lse_m = ls + t;
+    }
+    r.lse = o.m + lse_m;
     r.m = o.m;
-    r.bias_log2 = ((zy - o.m) - r.lp) * kLog2e;
+    r.bias_log2 = lse_m * kLog2e;
     return r;
 }
 

@@ -148,9 +148,9 @@ __global__ void __launch_bounds__(kRowThreads) row_kernel(const PassArgs a)
         if (a.lse_out) a.lse_out[t] = rs.lse;
         if (kBwd) {
             const bool has_old = a.lp_old != nullptr;
-            const float lw = has_old ? a.lp_old[t] : rs.lp;
+            const double lw = has_old ? (double)a.lp_old[t] : rs.lp64;
             const TokenWeight tw = token_weight(lw, a.lp_inf[t], a.P);
-            const TokenLoss tl = token_loss(rs.lp, has_old, has_old ? a.lp_old[t] : 0.0f,
+            const TokenLoss tl = token_loss(rs.lp64, has_old, has_old ? a.lp_old[t] : 0.0f,
                                             a.adv[t], a.scale[t], tw.w, a.P);
             if (a.w_out) a.w_out[t] = tw.w;
             if (a.trunc_out) a.trunc_out[t] = tw.trunc;

@@ -100,7 +100,7 @@ __global__ void weights_kernel(const float *lp_w, const float *lp_inf, const uin
         uint8_t tr = 0;
         if (is_valid(mask, t)) {
             const float lw = lp_w[t], li = lp_inf[t];
-            const TokenWeight tw = token_weight(lw, li, P);
+            const TokenWeight tw = token_weight((double)lw, li, P);
             w = tw.w;
             tr = tw.trunc;
             if (eps_out)

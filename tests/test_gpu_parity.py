@@ -2,7 +2,10 @@
 
 Tolerances (fixed by the requirements of the token pass; readings where they
 need one):
-  - log p of the sampled token: 2e-5 absolute;
+  - log p of the sampled token: 2e-5 absolute, plus 4 fp32 ulps of |log p|
+    (the output is fp32: the workloads' logits reach |z| ~ 650, so log p reaches
+    ~ -1200, where one fp32 step is 1.2e-4; internally the weight uses log p
+    carried in fp64, so the weight tolerance below is not widened);
   - weights: 1e-5 relative;
   - truncation decisions: bit-exact when both sides get the same fp32 log-probs
     (cis_weights); end to end, bit-exact except for tokens whose fp64 log k lies
@@ -65,6 +68,11 @@ def run_oracle(b, mode, lam, rows=None, lp_old=None, agg=0, use_mask=True, want_
         cu_seqlens=b.cu_seqlens.cpu().numpy() if agg else None, rows=rows, want_dz=want_dz)
 
 
+def lp_tol(ref_lp):
+    """2e-5 absolute plus 4 fp32 ulps of the value (2^-21 |lp| >= 4 ulp)."""
+    return TOL_LP + 2.0 ** -21 * np.abs(ref_lp)
+
+
 def decision_band(ref, lp_inf, mode, lam, kappa=5e-3, lp_old=None):
     """Tokens whose fp64 log k is within BAND of a truncation boundary."""
     lw = ref["lp"] if lp_old is None else lp_old.astype(np.float64)
@@ -89,7 +97,7 @@ def check_token_outputs(out, ref, b, mode, lam, lp_old=None, use_mask=True):
     nan_rows = np.isnan(ref["lp"])
     assert np.array_equal(np.isnan(lp), nan_rows)
     ok = ~nan_rows
-    assert np.abs(lp[ok] - ref["lp"][ok]).max(initial=0) <= TOL_LP
+    assert np.all(np.abs(lp[ok] - ref["lp"][ok]) <= lp_tol(ref["lp"][ok]))
     wr = ref["w"][ok]
     assert np.all(np.abs(w[ok] - wr) <= TOL_W * np.abs(wr) + 1e-30)
     band = decision_band(ref, b.lp_infer.cpu().numpy(), mode, lam,
@@ -143,8 +151,8 @@ def test_token_logprobs_match_oracle(cfg, T, V):
     assert rc == 0
     torch.cuda.synchronize()
     m = b.mask.cpu().numpy().astype(bool)
-    assert np.abs(lp.cpu().numpy() - ref_lp)[m].max() <= TOL_LP
-    assert np.abs(lse.cpu().numpy() - ref_lse)[m].max() <= TOL_LP * max(1.0, np.abs(ref_lse).max())
+    assert np.all(np.abs(lp.cpu().numpy() - ref_lp)[m] <= lp_tol(ref_lp[m]))
+    assert np.all(np.abs(lse.cpu().numpy() - ref_lse)[m] <= lp_tol(ref_lse[m]))
     assert np.all(lp.cpu().numpy()[~m] == 0)
 
 
