@@ -7,8 +7,8 @@
 //      asynchronous copy (cp.async.bulk, completion counted on an mbarrier;
 //      no multicast);
 //   2. pass 1 over shared memory: per thread the exact maximum of its entries
-//      (j != y), then the sum of e^{z - max}; a block reduction gives the CTA's
-//      pair (m_c, s_c);
+//      (j != y; bf16 pairs compared packed), then the sum of e^{z - max}; a
+//      block reduction gives the CTA's pair (m_c, s_c);
 //   3. every CTA writes its pair into slot [rank] of every CTA of the cluster
 //      (distributed shared memory), then a cluster barrier; each CTA combines
 //      the CS pairs in rank order, so all CTAs hold bit-identical row scalars;
@@ -29,7 +29,6 @@ namespace cg = cooperative_groups;
 namespace cis {
 namespace {
 
-constexpr int kThreads = 256;
 constexpr int kMaxCluster = 8;
 
 __device__ __forceinline__ float max_nan(float a, float b)
@@ -93,10 +92,10 @@ __device__ __forceinline__ void cluster_wait()
 }
 
 // 8 consecutive entries from shared memory as floats.
-template <typename InT> __device__ __forceinline__ void load8(const uint8_t *sm, int64_t g,
+template <typename InT> __device__ __forceinline__ void load8(const uint8_t *sm, int g,
                                                               float (&z)[8]);
 template <>
-__device__ __forceinline__ void load8<__nv_bfloat16>(const uint8_t *sm, int64_t g, float (&z)[8])
+__device__ __forceinline__ void load8<__nv_bfloat16>(const uint8_t *sm, int g, float (&z)[8])
 {
     const uint4 q = reinterpret_cast<const uint4 *>(sm)[g];
     z[0] = bf16_lo(q.x); z[1] = bf16_hi(q.x);
@@ -105,7 +104,7 @@ __device__ __forceinline__ void load8<__nv_bfloat16>(const uint8_t *sm, int64_t 
     z[6] = bf16_lo(q.w); z[7] = bf16_hi(q.w);
 }
 template <>
-__device__ __forceinline__ void load8<float>(const uint8_t *sm, int64_t g, float (&z)[8])
+__device__ __forceinline__ void load8<float>(const uint8_t *sm, int g, float (&z)[8])
 {
     const uint4 q0 = reinterpret_cast<const uint4 *>(sm)[2 * g];
     const uint4 q1 = reinterpret_cast<const uint4 *>(sm)[2 * g + 1];
@@ -114,6 +113,51 @@ __device__ __forceinline__ void load8<float>(const uint8_t *sm, int64_t g, float
     z[4] = __uint_as_float(q1.x); z[5] = __uint_as_float(q1.y);
     z[6] = __uint_as_float(q1.z); z[7] = __uint_as_float(q1.w);
 }
+
+// Overwrite entry j of the slab with -inf.
+template <typename InT> __device__ __forceinline__ void poke_neg_inf(uint8_t *sm, int j);
+template <> __device__ __forceinline__ void poke_neg_inf<__nv_bfloat16>(uint8_t *sm, int j)
+{
+    reinterpret_cast<uint16_t *>(sm)[j] = 0xff80u;  // bf16 -inf
+}
+template <> __device__ __forceinline__ void poke_neg_inf<float>(uint8_t *sm, int j)
+{
+    reinterpret_cast<float *>(sm)[j] = -INFINITY;
+}
+
+// Maximum over this thread's groups (NaN propagates).  bf16 rows are compared
+// two entries at a time without unpacking.
+template <typename InT, int NT> struct ThreadMax;
+template <int NT> struct ThreadMax<__nv_bfloat16, NT> {
+static __device__ __forceinline__ float run(const uint8_t *sm, int ng)
+{
+    const uint32_t ninf2 = 0xff80ff80u;
+    __nv_bfloat162 a0 = *reinterpret_cast<const __nv_bfloat162 *>(&ninf2), a1 = a0;
+    for (int g = threadIdx.x; g < ng; g += NT) {
+        const uint4 q = reinterpret_cast<const uint4 *>(sm)[g];
+        a0 = __hmax2_nan(a0, *reinterpret_cast<const __nv_bfloat162 *>(&q.x));
+        a1 = __hmax2_nan(a1, *reinterpret_cast<const __nv_bfloat162 *>(&q.y));
+        a0 = __hmax2_nan(a0, *reinterpret_cast<const __nv_bfloat162 *>(&q.z));
+        a1 = __hmax2_nan(a1, *reinterpret_cast<const __nv_bfloat162 *>(&q.w));
+    }
+    a0 = __hmax2_nan(a0, a1);
+    return max_nan(__low2float(a0), __high2float(a0));
+}
+};
+template <int NT> struct ThreadMax<float, NT> {
+static __device__ __forceinline__ float run(const uint8_t *sm, int ng)
+{
+    float m = -INFINITY;
+    for (int g = threadIdx.x; g < ng; g += NT) {
+        float z[8];
+        load8<float>(sm, g, z);
+#pragma unroll
+        for (int i = 0; i < 8; ++i)
+            m = max_nan(m, z[i]);
+    }
+    return m;
+}
+};
 
 // 8 results to global memory with streaming (evict-first) 16-byte stores.
 template <typename OutT> __device__ __forceinline__ void store8(OutT *dst, const float (&v)[8]);
@@ -138,11 +182,11 @@ __device__ __forceinline__ void store8<float>(float *dst, const float (&v)[8])
 struct ClusterShared {
     alignas(8) uint64_t bar;
     float2 part[kMaxCluster];
-    MaxSum red[kThreads / 32];
+    MaxSum red[512 / 32];
     float c, m, bias, lp;
 };
 
-template <typename InT, typename OutT>
+template <typename InT, typename OutT, int kThreads>
 __global__ void __launch_bounds__(kThreads) cluster_kernel(const PassArgs a, int64_t slice)
 {
     extern __shared__ __align__(128) uint8_t dyn_smem[];
@@ -212,25 +256,25 @@ __global__ void __launch_bounds__(kThreads) cluster_kernel(const PassArgs a, int
         mbar_wait(bar, 0);  // give the copy one more bounded chance to land
     }
 
-    // Pass 1: exact max of this thread's entries (j != y), then the sum.
+    // The sampled entry takes no part in the sums over j != y: the thread that
+    // owns its 8-entry group (the only thread that reads that group in either
+    // pass) overwrites it with -inf in shared memory once the copy has landed.
     const int64_t yl = y - v0;
-    const int64_t gy = (yl >= 0 && yl < n) ? yl / 8 : -1;
+    const int gy = (yl >= 0 && yl < n) ? (int)(yl >> 3) : -1;
     const int iy = (int)(yl & 7);
-    float m = -INFINITY;
-    for (int64_t g = threadIdx.x; g < ng; g += kThreads) {
-        float z[8];
-        load8<InT>(slab, g, z);
-        const int skip = g == gy ? iy : -1;
-#pragma unroll
-        for (int i = 0; i < 8; ++i)
-            m = max_nan(m, i == skip ? -INFINITY : z[i]);
-    }
+    if (gy >= 0 && gy % kThreads == (int)threadIdx.x)
+        poke_neg_inf<InT>(slab, 8 * gy + iy);
+    const int ngi = (int)ng;
+
+    // Pass 1: exact maximum of this thread's entries, then the sum of
+    // e^{z - max} (no rescaling; 8 exponentials added pairwise per group).
+    const float m = ThreadMax<InT, kThreads>::run(slab, ngi);
     float s = 0.0f;
     if (m != -INFINITY) {
-        for (int64_t g = threadIdx.x; g < ng; g += kThreads) {
+        for (int g = threadIdx.x; g < ngi; g += kThreads) {
             float z[8];
             load8<InT>(slab, g, z);
-            s += sum8_exp(z, m, g == gy ? iy : -1);
+            s += sum8_exp(z, m);
         }
     }
     const MaxSum mine = block_ms<kThreads>(MaxSum{m, s}, sh.red);
@@ -272,13 +316,17 @@ __global__ void __launch_bounds__(kThreads) cluster_kernel(const PassArgs a, int
     // Pass 2: dz = c (softmax - onehot) from the slice in shared memory.
     const float c = sh.c, mo = sh.m, bias = sh.bias;
     const float dzy = c * expm1f(sh.lp);  // c (p - 1)
-    for (int64_t g = threadIdx.x; g < ng; g += kThreads) {
+    for (int g = threadIdx.x; g < ngi; g += kThreads) {
         float z[8], v[8];
         load8<InT>(slab, g, z);
-        const int skip = g == gy ? iy : -1;
 #pragma unroll
         for (int i = 0; i < 8; ++i)
-            v[i] = i == skip ? dzy : c * ex2_full(fmaf(z[i] - mo, kLog2e, -bias));
+            v[i] = c * ex2_full(fmaf(z[i] - mo, kLog2e, -bias));
+        if (g == gy) {  // the sampled entry: c (p - 1)
+#pragma unroll
+            for (int i = 0; i < 8; ++i)
+                v[i] = i == iy ? dzy : v[i];
+        }
         store8<OutT>(orow + 8 * g, v);
     }
 }
@@ -320,17 +368,26 @@ bool make_plan(int64_t V, int in_bytes, Plan *p)
     return false;
 }
 
-template <typename InT, typename OutT>
-cudaError_t launch_cluster_t(const PassArgs &a, const Plan &p, cudaStream_t s)
+int cluster_threads()
 {
-    auto kern = cluster_kernel<InT, OutT>;
+    static int v = [] {
+        const char *e = getenv("CIS_CLUSTER_THREADS");
+        return (e && atoi(e) == 512) ? 512 : 256;
+    }();
+    return v;
+}
+
+template <typename InT, typename OutT, int NT>
+cudaError_t launch_cluster_nt(const PassArgs &a, const Plan &p, cudaStream_t s)
+{
+    auto kern = cluster_kernel<InT, OutT, NT>;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          (int)p.smem);
     if (e != cudaSuccess)
         return e;
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3((unsigned)(a.T * p.cs), 1, 1);
-    cfg.blockDim = dim3(kThreads, 1, 1);
+    cfg.blockDim = dim3(NT, 1, 1);
     cfg.dynamicSmemBytes = p.smem;
     cfg.stream = s;
     cudaLaunchAttribute attr[1];
@@ -341,6 +398,14 @@ cudaError_t launch_cluster_t(const PassArgs &a, const Plan &p, cudaStream_t s)
     cfg.attrs = attr;
     cfg.numAttrs = 1;
     return cudaLaunchKernelEx(&cfg, kern, a, p.slice);
+}
+
+template <typename InT, typename OutT>
+cudaError_t launch_cluster_t(const PassArgs &a, const Plan &p, cudaStream_t s)
+{
+    if (cluster_threads() == 512)
+        return launch_cluster_nt<InT, OutT, 512>(a, p, s);
+    return launch_cluster_nt<InT, OutT, 256>(a, p, s);
 }
 
 }  // namespace

@@ -285,14 +285,14 @@ __device__ __forceinline__ RowScalars row_scalars(MaxSum o, float zy)
     return r;
 }
 
-// Sum of e^{z - m} over 8 values, excluding lane index `skip` (-1 = none),
-// added pairwise to keep the rounding error independent of the row length.
-__device__ __forceinline__ float sum8_exp(const float (&z)[8], float m, int skip)
+// Sum of e^{z - m} over 8 values, added pairwise so that the rounding error
+// does not grow with the row length.
+__device__ __forceinline__ float sum8_exp(const float (&z)[8], float m)
 {
     float e[8];
 #pragma unroll
     for (int i = 0; i < 8; ++i)
-        e[i] = (i == skip) ? 0.0f : ex2_ftz((z[i] - m) * kLog2e);
+        e[i] = ex2_ftz((z[i] - m) * kLog2e);
     return ((e[0] + e[1]) + (e[2] + e[3])) + ((e[4] + e[5]) + (e[6] + e[7]));
 }
 
