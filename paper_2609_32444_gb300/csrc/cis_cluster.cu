@@ -3,15 +3,17 @@
 // A bf16 row of the 151,936-entry vocabulary is 303,872 bytes, more than one
 // CTA's shared memory.  A cluster of CS CTAs (CS = 1, 2, 4 or 8) therefore
 // splits each row into CS contiguous slices.  Per row:
-//   1. each CTA copies its slice from HBM into shared memory with one bulk
-//      asynchronous copy (cp.async.bulk, completion counted on an mbarrier;
-//      no multicast);
+//   1. each CTA copies its slice from HBM into shared memory with bulk
+//      asynchronous copies (cp.async.bulk, four chunks, each completing on its
+//      own mbarrier so that pass 1 starts on the first chunk; no multicast);
 //   2. pass 1 over shared memory: per thread the exact maximum of its entries
 //      (j != y; bf16 pairs compared packed), then the sum of e^{z - max}; a
 //      block reduction gives the CTA's pair (m_c, s_c);
-//   3. every CTA writes its pair into slot [rank] of every CTA of the cluster
-//      (distributed shared memory), then a cluster barrier; each CTA combines
-//      the CS pairs in rank order, so all CTAs hold bit-identical row scalars;
+//   3. every CTA stores its pair into slot [rank] of every CTA of the cluster
+//      (st.async into distributed shared memory, counted on the receiver's
+//      mbarrier, so a CTA waits for the data only, not for a cluster barrier);
+//      each CTA combines the CS pairs in rank order, so all CTAs hold
+//      bit-identical row scalars;
 //   4. thread 0 forms log p (log-odds form, cis_common.cuh), the weight
 //      (Algorithm 1 / Table 8) and the token loss (Eq. 1);
 //   5. pass 2 over shared memory writes dz = c (softmax - onehot) with 16-byte
@@ -125,38 +127,45 @@ template <> __device__ __forceinline__ void poke_neg_inf<float>(uint8_t *sm, int
     reinterpret_cast<float *>(sm)[j] = -INFINITY;
 }
 
-// Maximum over this thread's groups (NaN propagates).  bf16 rows are compared
-// two entries at a time without unpacking.
-template <typename InT, int NT> struct ThreadMax;
-template <int NT> struct ThreadMax<__nv_bfloat16, NT> {
-static __device__ __forceinline__ float run(const uint8_t *sm, int ng)
-{
-    const uint32_t ninf2 = 0xff80ff80u;
-    __nv_bfloat162 a0 = *reinterpret_cast<const __nv_bfloat162 *>(&ninf2), a1 = a0;
-    for (int g = threadIdx.x; g < ng; g += NT) {
-        const uint4 q = reinterpret_cast<const uint4 *>(sm)[g];
-        a0 = __hmax2_nan(a0, *reinterpret_cast<const __nv_bfloat162 *>(&q.x));
-        a1 = __hmax2_nan(a1, *reinterpret_cast<const __nv_bfloat162 *>(&q.y));
-        a0 = __hmax2_nan(a0, *reinterpret_cast<const __nv_bfloat162 *>(&q.z));
-        a1 = __hmax2_nan(a1, *reinterpret_cast<const __nv_bfloat162 *>(&q.w));
+// Running maximum over this thread's groups (NaN propagates), fed chunk by
+// chunk.  bf16 rows are compared two entries at a time without unpacking.
+template <typename InT> struct MaxAcc;
+template <> struct MaxAcc<__nv_bfloat16> {
+    __nv_bfloat162 a0, a1;
+    __device__ __forceinline__ MaxAcc()
+    {
+        const uint32_t ninf2 = 0xff80ff80u;
+        a0 = a1 = *reinterpret_cast<const __nv_bfloat162 *>(&ninf2);
     }
-    a0 = __hmax2_nan(a0, a1);
-    return max_nan(__low2float(a0), __high2float(a0));
-}
+    __device__ __forceinline__ void consume(const uint8_t *sm, int g0, int g1, int step)
+    {
+        for (int g = g0; g < g1; g += step) {
+            const uint4 q = reinterpret_cast<const uint4 *>(sm)[g];
+            a0 = __hmax2_nan(a0, *reinterpret_cast<const __nv_bfloat162 *>(&q.x));
+            a1 = __hmax2_nan(a1, *reinterpret_cast<const __nv_bfloat162 *>(&q.y));
+            a0 = __hmax2_nan(a0, *reinterpret_cast<const __nv_bfloat162 *>(&q.z));
+            a1 = __hmax2_nan(a1, *reinterpret_cast<const __nv_bfloat162 *>(&q.w));
+        }
+    }
+    __device__ __forceinline__ float result() const
+    {
+        const __nv_bfloat162 a = __hmax2_nan(a0, a1);
+        return max_nan(__low2float(a), __high2float(a));
+    }
 };
-template <int NT> struct ThreadMax<float, NT> {
-static __device__ __forceinline__ float run(const uint8_t *sm, int ng)
-{
+template <> struct MaxAcc<float> {
     float m = -INFINITY;
-    for (int g = threadIdx.x; g < ng; g += NT) {
-        float z[8];
-        load8<float>(sm, g, z);
+    __device__ __forceinline__ void consume(const uint8_t *sm, int g0, int g1, int step)
+    {
+        for (int g = g0; g < g1; g += step) {
+            float z[8];
+            load8<float>(sm, g, z);
 #pragma unroll
-        for (int i = 0; i < 8; ++i)
-            m = max_nan(m, z[i]);
+            for (int i = 0; i < 8; ++i)
+                m = max_nan(m, z[i]);
+        }
     }
-    return m;
-}
+    __device__ __forceinline__ float result() const { return m; }
 };
 
 // 8 results to global memory with streaming (evict-first) 16-byte stores.
@@ -179,12 +188,62 @@ __device__ __forceinline__ void store8<float>(float *dst, const float (&v)[8])
     __stcs(reinterpret_cast<float4 *>(dst) + 1, make_float4(v[4], v[5], v[6], v[7]));
 }
 
+constexpr int kChunks = 4;  // the slice is copied in this many pieces
+
 struct ClusterShared {
-    alignas(8) uint64_t bar;
+    alignas(8) uint64_t bar[kChunks];  // completion of each copy chunk
+    alignas(8) uint64_t xbar;          // arrival of the cluster's (m, s) pairs
     float2 part[kMaxCluster];
     MaxSum red[512 / 32];
     float c, m, bias, lp;
 };
+
+__device__ __forceinline__ uint32_t map_rank(uint32_t addr, uint32_t rank)
+{
+    uint32_t r;
+    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(addr), "r"(rank));
+    return r;
+}
+
+// Store (m, s) into another CTA's shared memory; its mbarrier counts the bytes.
+__device__ __forceinline__ void st_async_pair(uint32_t dst, float m, float s, uint32_t bar)
+{
+    asm volatile(
+        "st.async.shared::cluster.mbarrier::complete_tx::bytes.v2.f32 [%0], {%1, %2}, [%3];"
+        ::"r"(dst), "f"(m), "f"(s), "r"(bar)
+        : "memory");
+}
+
+// Bounded wait for data written by other CTAs of the cluster.
+__device__ __forceinline__ bool mbar_wait_cluster(uint32_t bar, uint32_t parity)
+{
+    for (uint32_t i = 0; i < kMaxPolls; ++i) {
+        uint32_t done;
+        asm volatile(
+            "{\n\t.reg .pred p;\n\t"
+            "mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2, %3;\n\t"
+            "selp.u32 %0, 1, 0, p;\n\t}"
+            : "=r"(done)
+            : "r"(bar), "r"(parity), "r"(kPollSuspendNs)
+            : "memory");
+        if (done)
+            return true;
+    }
+    return false;
+}
+
+__device__ __forceinline__ void wait_or_flag(uint32_t bar, bool cluster_scope, int32_t *status)
+{
+    const bool ok = cluster_scope ? mbar_wait_cluster(bar, 0) : mbar_wait(bar, 0);
+    if (!ok) {
+        if (threadIdx.x == 0)
+            set_status(status, kStatusTimeout);
+        if (cluster_scope)  // one more bounded chance before the data is used
+            mbar_wait_cluster(bar, 0);
+        else
+            mbar_wait(bar, 0);
+    }
+}
 
 template <typename InT, typename OutT, int kThreads>
 __global__ void __launch_bounds__(kThreads) cluster_kernel(const PassArgs a, int64_t slice)
@@ -200,7 +259,8 @@ __global__ void __launch_bounds__(kThreads) cluster_kernel(const PassArgs a, int
     const int64_t t = blockIdx.x / cs;
     const int64_t v0 = (int64_t)rank * slice;
     const int64_t n = v0 < a.V ? (a.V - v0 < slice ? a.V - v0 : slice) : 0;  // multiple of 8
-    const int64_t ng = n / 8;
+    const int ng = (int)(n / 8);
+    constexpr int kGroupBytes = 8 * sizeof(InT);
     OutT *orow = reinterpret_cast<OutT *>(a.dz) + t * a.ld_out + v0;
 
     const bool valid = a.mask == nullptr || a.mask[t] != 0;
@@ -208,7 +268,7 @@ __global__ void __launch_bounds__(kThreads) cluster_kernel(const PassArgs a, int
     const bool id_ok = y >= 0 && y < a.V;
     if (!valid || !id_ok) {  // same branch in every CTA of the cluster
         const float zero[8] = {0, 0, 0, 0, 0, 0, 0, 0};
-        for (int64_t g = threadIdx.x; g < ng; g += kThreads)
+        for (int g = threadIdx.x; g < ng; g += kThreads)
             store8<OutT>(orow + 8 * g, zero);
         if (rank == 0 && threadIdx.x == 0) {
             const float lp = valid ? NAN : 0.0f;
@@ -225,19 +285,30 @@ __global__ void __launch_bounds__(kThreads) cluster_kernel(const PassArgs a, int
         return;
     }
 
-    const uint32_t bar = smem_u32(&sh.bar);
+    // Copy the slice in kChunks pieces, each completing on its own mbarrier.
+    const int qg = (ng + kChunks - 1) / kChunks;  // groups per chunk
+    const uint32_t xbar = smem_u32(&sh.xbar);
     if (threadIdx.x == 0) {
-        mbar_init(bar, 1);
-        if (n > 0) {
-            const uint32_t bytes = (uint32_t)(n * sizeof(InT));
-            mbar_expect_tx(bar, bytes);
-            const uint8_t *src = reinterpret_cast<const uint8_t *>(a.logits) +
-                                 (t * a.ld + v0) * (int64_t)sizeof(InT);
-            bulk_g2s(smem_u32(slab), src, bytes, bar);
+        for (int c = 0; c < kChunks; ++c)
+            mbar_init(smem_u32(&sh.bar[c]), 1);
+        mbar_init(xbar, 1);
+        // the one local arrival on xbar; the peers' stores bring the bytes
+        mbar_expect_tx(xbar, (uint32_t)(cs * sizeof(float2)));
+        const uint8_t *src = reinterpret_cast<const uint8_t *>(a.logits) +
+                             (t * a.ld + v0) * (int64_t)sizeof(InT);
+        for (int c = 0; c < kChunks; ++c) {
+            const int g0 = c * qg, g1 = min(ng, g0 + qg);
+            if (g0 >= g1)
+                break;
+            const uint32_t bytes = (uint32_t)((g1 - g0) * kGroupBytes);
+            const uint32_t b = smem_u32(&sh.bar[c]);
+            mbar_expect_tx(b, bytes);
+            bulk_g2s(smem_u32(slab) + g0 * kGroupBytes, src + (int64_t)g0 * kGroupBytes, bytes,
+                     b);
         }
     }
     // Arrive now, wait before the first remote store: every CTA of the
-    // cluster has started by then.
+    // cluster has started and initialised its barriers by then.
     cluster_arrive_relaxed();
 
     // Per-token inputs, fetched while the copy is in flight.
@@ -249,45 +320,53 @@ __global__ void __launch_bounds__(kThreads) cluster_kernel(const PassArgs a, int
         adv = a.adv[t];
         sc = a.scale[t];
     }
-    __syncthreads();  // barrier initialised before anyone polls it
-    if (n > 0 && !mbar_wait(bar, 0)) {
-        if (threadIdx.x == 0)
-            set_status(a.status, kStatusTimeout);
-        mbar_wait(bar, 0);  // give the copy one more bounded chance to land
-    }
+    __syncthreads();  // barriers initialised before anyone polls them
 
     // The sampled entry takes no part in the sums over j != y: the thread that
     // owns its 8-entry group (the only thread that reads that group in either
-    // pass) overwrites it with -inf in shared memory once the copy has landed.
+    // pass) overwrites it with -inf in shared memory once its chunk has landed.
     const int64_t yl = y - v0;
     const int gy = (yl >= 0 && yl < n) ? (int)(yl >> 3) : -1;
     const int iy = (int)(yl & 7);
-    if (gy >= 0 && gy % kThreads == (int)threadIdx.x)
-        poke_neg_inf<InT>(slab, 8 * gy + iy);
-    const int ngi = (int)ng;
 
-    // Pass 1: exact maximum of this thread's entries, then the sum of
-    // e^{z - max} (no rescaling; 8 exponentials added pairwise per group).
-    const float m = ThreadMax<InT, kThreads>::run(slab, ngi);
+    // Pass 1a: exact maximum of this thread's entries, chunk by chunk as the
+    // copy lands.
+    MaxAcc<InT> macc;
+    for (int c = 0; c < kChunks; ++c) {
+        const int g0 = c * qg, g1 = min(ng, g0 + qg);
+        if (g0 >= g1)
+            break;
+        wait_or_flag(smem_u32(&sh.bar[c]), false, a.status);
+        if (gy >= g0 && gy < g1 && gy % kThreads == (int)threadIdx.x)
+            poke_neg_inf<InT>(slab, 8 * gy + iy);
+        const int first = g0 + (int)(((unsigned)threadIdx.x + kThreads - (unsigned)(g0 % kThreads)) %
+                                     kThreads);
+        macc.consume(slab, first, g1, kThreads);
+    }
+    const float m = macc.result();
+
+    // Pass 1b: sum of e^{z - max} (8 exponentials added pairwise per group).
     float s = 0.0f;
     if (m != -INFINITY) {
-        for (int g = threadIdx.x; g < ngi; g += kThreads) {
+        for (int g = threadIdx.x; g < ng; g += kThreads) {
             float z[8];
             load8<InT>(slab, g, z);
             s += sum8_exp(z, m);
         }
     }
-    const MaxSum mine = block_ms<kThreads>(MaxSum{m, s}, sh.red);
+    const MaxSum mine = block_ms<kThreads, false>(MaxSum{m, s}, sh.red);
 
-    // Exchange the CTA pairs through distributed shared memory.
+    // Exchange the CTA pairs: lane r of warp 0 stores this CTA's pair into
+    // slot [rank] of CTA r, counted on CTA r's xbar.
     cluster_wait();
-    if (threadIdx.x == 0) {
-        for (unsigned r = 0; r < cs; ++r) {
-            float2 *dst = cluster.map_shared_rank(&sh.part[rank], r);
-            *dst = make_float2(mine.m, mine.s);
-        }
-    }
-    cluster.sync();
+    if (threadIdx.x < cs)
+        st_async_pair(map_rank(smem_u32(&sh.part[rank]), threadIdx.x), mine.m, mine.s,
+                      map_rank(xbar, threadIdx.x));
+    wait_or_flag(xbar, true, a.status);
+    // Everything addressed to this CTA has landed; tell the cluster, and wait
+    // for the others' word only at exit (so no CTA leaves while stores into
+    // its shared memory may be in flight).
+    cluster_arrive_relaxed();
     MaxSum o{sh.part[0].x, sh.part[0].y};
     for (unsigned r = 1; r < cs; ++r)
         o = ms_combine(o, MaxSum{sh.part[r].x, sh.part[r].y});
@@ -316,7 +395,7 @@ __global__ void __launch_bounds__(kThreads) cluster_kernel(const PassArgs a, int
     // Pass 2: dz = c (softmax - onehot) from the slice in shared memory.
     const float c = sh.c, mo = sh.m, bias = sh.bias;
     const float dzy = c * expm1f(sh.lp);  // c (p - 1)
-    for (int g = threadIdx.x; g < ngi; g += kThreads) {
+    for (int g = threadIdx.x; g < ng; g += kThreads) {
         float z[8], v[8];
         load8<InT>(slab, g, z);
 #pragma unroll
@@ -329,6 +408,7 @@ __global__ void __launch_bounds__(kThreads) cluster_kernel(const PassArgs a, int
         }
         store8<OutT>(orow + 8 * g, v);
     }
+    cluster_wait();
 }
 
 // Cluster size and slice (entries, a multiple of 8) for a row of V entries.

@@ -221,7 +221,8 @@ __device__ __forceinline__ MaxSum warp_ms(MaxSum v)
 }
 
 // Block-wide (m, s); every thread gets the result.  `sh` needs NT/32 slots.
-template <int NT>
+// kReuse: the slots are used again later, so wait until all have read them.
+template <int NT, bool kReuse = true>
 __device__ __forceinline__ MaxSum block_ms(MaxSum v, MaxSum *sh)
 {
     v = warp_ms(v);
@@ -233,7 +234,8 @@ __device__ __forceinline__ MaxSum block_ms(MaxSum v, MaxSum *sh)
 #pragma unroll
     for (int i = 1; i < NT / 32; ++i)
         r = ms_combine(r, sh[i]);
-    __syncthreads();
+    if (kReuse)
+        __syncthreads();
     return r;
 }
 
