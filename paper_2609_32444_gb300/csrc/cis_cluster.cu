@@ -348,6 +348,7 @@ __global__ void __launch_bounds__(kThreads) cluster_kernel(const PassArgs a, int
     // Pass 1b: sum of e^{z - max} (8 exponentials added pairwise per group).
     float s = 0.0f;
     if (m != -INFINITY) {
+#pragma unroll 2
         for (int g = threadIdx.x; g < ng; g += kThreads) {
             float z[8];
             load8<InT>(slab, g, z);
@@ -393,14 +394,24 @@ __global__ void __launch_bounds__(kThreads) cluster_kernel(const PassArgs a, int
     __syncthreads();
 
     // Pass 2: dz = c (softmax - onehot) from the slice in shared memory.
-    const float c = sh.c, mo = sh.m, bias = sh.bias;
+    // c softmax_j is formed as (c 2^-K) 2^(x_j + K) with the flushing
+    // exponential.  With K = clamp(ilogb(c) + 25, 0, 127): wherever
+    // 2^(x_j + K) would be subnormal, |c softmax_j| < 2^-150 rounds to zero in
+    // fp32 and bf16 anyway; c 2^-K stays normal and 2^(x_j + K) finite.  The
+    // final multiply keeps subnormal products.
+    const float c = sh.c, mo = sh.m;
+    const int kexp = (int)((__float_as_uint(c) >> 23) & 0xff) - 127 + 25;
+    const int K = kexp < 0 ? 0 : (kexp > 127 ? 127 : kexp);
+    const float cs2 = ldexpf(c, -K);
+    const float bias = sh.bias - (float)K;
     const float dzy = c * expm1f(sh.lp);  // c (p - 1)
+#pragma unroll 2
     for (int g = threadIdx.x; g < ng; g += kThreads) {
         float z[8], v[8];
         load8<InT>(slab, g, z);
 #pragma unroll
         for (int i = 0; i < 8; ++i)
-            v[i] = c * ex2_full(fmaf(z[i] - mo, kLog2e, -bias));
+            v[i] = cs2 * ex2_ftz(fmaf(z[i] - mo, kLog2e, -bias));
         if (g == gy) {  // the sampled entry: c (p - 1)
 #pragma unroll
             for (int i = 0; i < 8; ++i)
