@@ -1,7 +1,7 @@
 // cis_cluster.cu -- fused forward + backward token pass, fast path (sm_103a).
 //
 // A bf16 row of the 151,936-entry vocabulary is 303,872 bytes, more than one
-// CTA's shared memory.  A cluster of CS CTAs (CS = 1, 2, 4 or 8) therefore
+// CTA's shared memory.  A cluster of CS CTAs (1 <= CS <= 8) therefore
 // splits each row into CS contiguous slices.  Per row:
 //   1. each CTA copies its slice from HBM into shared memory with bulk
 //      asynchronous copies (cp.async.bulk, four chunks, each completing on its
@@ -441,13 +441,26 @@ int64_t slice_target_bytes()
     return v;
 }
 
+// Cluster size forced for tuning sweeps (0: chosen from the slice target).
+int forced_cluster()
+{
+    static int v = [] {
+        const char *e = getenv("CIS_CLUSTER");
+        const int c = e ? atoi(e) : 0;
+        return (c >= 1 && c <= kMaxCluster) ? c : 0;
+    }();
+    return v;
+}
+
+// Smallest cluster size whose slices fit the target (any size 1..8).
 bool make_plan(int64_t V, int in_bytes, Plan *p)
 {
     const int64_t target = slice_target_bytes();
-    for (int cs = 1; cs <= kMaxCluster; cs *= 2) {
+    const int forced = forced_cluster();
+    for (int cs = forced ? forced : 1; cs <= kMaxCluster; ++cs) {
         const int64_t per = (V + cs - 1) / cs;
         const int64_t slice = (per + 7) / 8 * 8;
-        if (slice * in_bytes <= target || cs == kMaxCluster) {
+        if (forced || slice * in_bytes <= target || cs == kMaxCluster) {
             if (slice * in_bytes > 200 * 1024)
                 return false;
             p->cs = cs;
@@ -459,11 +472,13 @@ bool make_plan(int64_t V, int in_bytes, Plan *p)
     return false;
 }
 
+// CTA width forced for tuning sweeps (default 256 threads).
 int cluster_threads()
 {
     static int v = [] {
         const char *e = getenv("CIS_CLUSTER_THREADS");
-        return (e && atoi(e) == 512) ? 512 : 256;
+        const int n = e ? atoi(e) : 256;
+        return (n == 512 || n == 384 || n == 128) ? n : 256;
     }();
     return v;
 }
@@ -494,9 +509,12 @@ cudaError_t launch_cluster_nt(const PassArgs &a, const Plan &p, cudaStream_t s)
 template <typename InT, typename OutT>
 cudaError_t launch_cluster_t(const PassArgs &a, const Plan &p, cudaStream_t s)
 {
-    if (cluster_threads() == 512)
-        return launch_cluster_nt<InT, OutT, 512>(a, p, s);
-    return launch_cluster_nt<InT, OutT, 256>(a, p, s);
+    switch (cluster_threads()) {
+    case 512: return launch_cluster_nt<InT, OutT, 512>(a, p, s);
+    case 384: return launch_cluster_nt<InT, OutT, 384>(a, p, s);
+    case 128: return launch_cluster_nt<InT, OutT, 128>(a, p, s);
+    default: return launch_cluster_nt<InT, OutT, 256>(a, p, s);
+    }
 }
 
 }  // namespace
