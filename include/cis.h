@@ -202,6 +202,43 @@ CIS_API cis_status_t cis_loss_fwd_bwd(const void *logits, int32_t dtype, int64_t
                               void *stream);
 
 /*
+ * Largest T that cis_loss_fwd_bwd_noalloc accepts.
+ */
+#define CIS_NOALLOC_MAX_TOKENS 65536
+
+/*
+ * cis_loss_fwd_bwd without the workspace arguments, for callers that cannot
+ * allocate device memory: extensions running inside a host framework that owns
+ * all device memory and gives them no allocator (serving engines, training
+ * runtimes), and C callers with no device allocator of their own.  The paper
+ * has no counterpart; this is an interface convenience around the same pass.
+ *   - All other arguments, outputs and errors are those of cis_loss_fwd_bwd.
+ *   - The scratch is an array of about 1.3 MiB in the library's static device
+ *     memory, sized for CIS_NOALLOC_MAX_TOKENS tokens; every GPU that loads the
+ *     library keeps one until the process exits.  T > CIS_NOALLOC_MAX_TOKENS
+ *     returns CIS_ERR_UNSUPPORTED before any GPU work.
+ *   - The first call on a device looks the array's device address up
+ *     (cudaGetSymbolAddress) with that device current; make that first call
+ *     before any stream capture on that device.
+ *   - No allocating routine is called.
+ *   - All calls share the array.  Each call resets the status word and
+ *     overwrites everything else it reads, so sequential calls are
+ *     independent; calls whose GPU work overlaps (different streams or host
+ *     threads) race and give wrong results.
+ *   - Device status bits are reported in stats_out->status.
+ */
+CIS_API cis_status_t cis_loss_fwd_bwd_noalloc(const void *logits, int32_t dtype, int64_t T,
+                                              int64_t V, int64_t ld, const int32_t *ids,
+                                              const float *lp_infer, const float *lp_old,
+                                              const float *adv, const uint8_t *mask,
+                                              const int32_t *cu_seqlens, int64_t B,
+                                              const cis_params_t *params, void *dlogits,
+                                              int32_t dlogits_dtype, int64_t ld_out,
+                                              float *lp_out, float *w_out, uint8_t *trunc_out,
+                                              cis_stats_t *stats_out, double *loss_out,
+                                              void *stream);
+
+/*
  * Profiling aid.  The next cis_loss_fwd_bwd call made from the calling host
  * thread records `begin_event` on its stream just before its main kernel (the
  * fused vocabulary pass) and `end_event` just after it, then forgets both.
