@@ -346,7 +346,7 @@ def run_ours(args, rank, world, local):
     traffic = profiled_traffic()
     roof = {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
             "frac": achieved / peak, "traffic": traffic,
-            "kernel": "cluster_kernel<bf16,bf16> (fused fwd+bwd vocabulary pass)",
+            "kernel": "cis_fused_cluster_kernel<bf16,bf16,256> (fused fwd+bwd vocabulary pass)",
             "kernel_ms": kernel_ms, "algorithmic_bytes_per_launch": alg_bytes,
             "peak_source": peak_src, "frac_of_nominal_8000": achieved / NOMINAL_HBM_GBS,
             "step_frac": alg_bytes / (ms_per_step / 1e3) / 1e9 / peak}

@@ -246,7 +246,7 @@ __device__ __forceinline__ void wait_or_flag(uint32_t bar, bool cluster_scope, i
 }
 
 template <typename InT, typename OutT, int kThreads>
-__global__ void __launch_bounds__(kThreads) cluster_kernel(const PassArgs a, int64_t slice)
+__global__ void __launch_bounds__(kThreads) cis_fused_cluster_kernel(const PassArgs a, int64_t slice)
 {
     extern __shared__ __align__(128) uint8_t dyn_smem[];
     __shared__ ClusterShared sh;
@@ -486,7 +486,7 @@ int cluster_threads()
 template <typename InT, typename OutT, int NT>
 cudaError_t launch_cluster_nt(const PassArgs &a, const Plan &p, cudaStream_t s)
 {
-    auto kern = cluster_kernel<InT, OutT, NT>;
+    auto kern = cis_fused_cluster_kernel<InT, OutT, NT>;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          (int)p.smem);
     if (e != cudaSuccess)

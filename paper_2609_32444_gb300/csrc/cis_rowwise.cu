@@ -110,7 +110,7 @@ struct RowShared {
 };
 
 template <typename InT, typename OutT, bool kBwd>
-__global__ void __launch_bounds__(kRowThreads) row_kernel(const PassArgs a)
+__global__ void __launch_bounds__(kRowThreads) cis_fused_row_kernel(const PassArgs a)
 {
     __shared__ RowShared sh;
     const int64_t t = blockIdx.x;
@@ -182,7 +182,7 @@ cudaError_t launch_row(const PassArgs &a, cudaStream_t s)
 {
     if (a.T == 0)
         return cudaSuccess;
-    row_kernel<InT, OutT, kBwd><<<(unsigned)a.T, kRowThreads, 0, s>>>(a);
+    cis_fused_row_kernel<InT, OutT, kBwd><<<(unsigned)a.T, kRowThreads, 0, s>>>(a);
     return cudaGetLastError();
 }
 

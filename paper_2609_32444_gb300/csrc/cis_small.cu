@@ -1,10 +1,10 @@
 // cis_small.cu -- the [T]-sized kernels of libcis.
 //
-//   scales_kernel   the loss normaliser s_t: 1/n over the n valid tokens
+//   cis_scales_kernel   the loss normaliser s_t: 1/n over the n valid tokens
 //                   (Algorithm 1) or 1/(G |y_i|) per response (Eq. 1); it
 //                   also clears the device status word of the call.
-//   weights_kernel  cis_weights: Algorithm 1 / Table 8, one thread per token.
-//   reduce_kernel   deterministic sums of the per-token loss terms and the
+//   cis_weights_kernel  cis_weights: Algorithm 1 / Table 8, one thread per token.
+//   cis_reduce_kernel   deterministic sums of the per-token loss terms and the
 //                   statistics the paper logs (App. D.1: share of tokens acted
 //                   on, largest |log k|; App. D.5: the truncated excess).
 #include "cis_kernels.h"
@@ -30,7 +30,7 @@ __device__ __forceinline__ T warp_sum(T v)
 }
 
 __global__ void __launch_bounds__(kSmallThreads)
-    scales_kernel(const uint8_t *mask, int64_t T, const int32_t *cu, int64_t B, int agg,
+    cis_scales_kernel(const uint8_t *mask, int64_t T, const int32_t *cu, int64_t B, int agg,
                   float *scale, int32_t *status)
 {
     __shared__ long long part[kSmallThreads / 32];
@@ -90,7 +90,7 @@ __global__ void __launch_bounds__(kSmallThreads)
         scale[t] = is_valid(mask, t) ? s : 0.0f;
 }
 
-__global__ void weights_kernel(const float *lp_w, const float *lp_inf, const uint8_t *mask,
+__global__ void cis_weights_kernel(const float *lp_w, const float *lp_inf, const uint8_t *mask,
                                int64_t T, const DevParams P, float *w_out, uint8_t *trunc_out,
                                float *eps_out)
 {
@@ -122,7 +122,7 @@ struct RedPart {
 
 // One CTA: thread i sums tokens i, i + 1024, ... in order, then a fixed tree.
 __global__ void __launch_bounds__(kSmallThreads)
-    reduce_kernel(const uint8_t *mask, int64_t T, const double *terms, const float *logk,
+    cis_reduce_kernel(const uint8_t *mask, int64_t T, const double *terms, const float *logk,
                   const float *w, const uint8_t *trunc, const int32_t *status,
                   cis_stats_t *stats, double *loss_out)
 {
@@ -176,7 +176,7 @@ cudaError_t launch_scales(const uint8_t *mask, int64_t T, const int32_t *cu_seql
 {
     if (agg == CIS_AGG_SEQ_MEAN_TOKEN_MEAN && B > kMaxSeqInShared)
         return cudaErrorNotSupported;
-    scales_kernel<<<1, kSmallThreads, 0, s>>>(mask, T, cu_seqlens, B, agg, scale, status);
+    cis_scales_kernel<<<1, kSmallThreads, 0, s>>>(mask, T, cu_seqlens, B, agg, scale, status);
     return cudaGetLastError();
 }
 
@@ -189,14 +189,14 @@ cudaError_t launch_weights(const float *lp_w, const float *lp_inf, const uint8_t
     int64_t blocks = (T + 255) / 256;
     if (blocks > 4096)
         blocks = 4096;
-    weights_kernel<<<(unsigned)blocks, 256, 0, s>>>(lp_w, lp_inf, mask, T, P, w_out, trunc_out,
+    cis_weights_kernel<<<(unsigned)blocks, 256, 0, s>>>(lp_w, lp_inf, mask, T, P, w_out, trunc_out,
                                                     eps_out);
     return cudaGetLastError();
 }
 
 cudaError_t launch_reduce(const PassArgs &a, cis_stats_t *stats, double *loss, cudaStream_t s)
 {
-    reduce_kernel<<<1, kSmallThreads, 0, s>>>(a.mask, a.T, a.ws_terms, a.ws_logk, a.ws_w,
+    cis_reduce_kernel<<<1, kSmallThreads, 0, s>>>(a.mask, a.T, a.ws_terms, a.ws_logk, a.ws_w,
                                                a.ws_trunc, a.status, stats, loss);
     return cudaGetLastError();
 }
