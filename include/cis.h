@@ -202,6 +202,44 @@ CIS_API cis_status_t cis_loss_fwd_bwd(const void *logits, int32_t dtype, int64_t
                               void *stream);
 
 /*
+ * Bytes of device workspace cis_lmhead_fused needs.  Host only.
+ * CIS_ERR_INVALID_ARG if bytes is NULL, T < 0, V <= 0 or H <= 0.
+ */
+CIS_API cis_status_t cis_lmhead_workspace_size(int64_t T, int64_t V, int64_t H, size_t *bytes);
+
+/*
+ * The token pass fused with the LM head: logits z = hidden W^T are computed
+ * in tiles on the tensor cores and never written to memory; the weight, the
+ * loss and the gradients are those of cis_loss_fwd_bwd (Eq. 1, Algorithm 1,
+ * Table 8), taken through the LM head:
+ *   dhidden = dz W,   dweight = dz^T hidden,   dz = c (softmax - onehot).
+ *   hidden      device bf16 [T, H], contiguous rows, 16-byte aligned.
+ *   weight      device bf16 [V, H], contiguous rows, 16-byte aligned.
+ *   H           hidden size; a multiple of 256 (else CIS_ERR_UNSUPPORTED).
+ *   ids, lp_infer, lp_old, adv, mask, cu_seqlens, B, params: as for
+ *               cis_loss_fwd_bwd.
+ *   dhidden     device [T, H] of grad_dtype (CIS_F32 or CIS_BF16), written.
+ *   dweight     device [V, H] of grad_dtype, written (rows of tokens that are
+ *               masked contribute nothing).
+ *   lp_out, w_out, trunc_out, stats_out, loss_out: as for cis_loss_fwd_bwd.
+ *   workspace   device, >= cis_lmhead_workspace_size(T, V, H) bytes,
+ *               1024-byte aligned; its first int32 is the device status word.
+ * dz enters the two gradient products in bf16 (the tensor-core operand type);
+ * the products accumulate in fp32.  Errors: as for cis_loss_fwd_bwd, plus
+ * CIS_ERR_UNSUPPORTED if the tensor-map encoder is unavailable.
+ */
+CIS_API cis_status_t cis_lmhead_fused(const void *hidden, const void *weight, int64_t T,
+                                      int64_t H, int64_t V, const int32_t *ids,
+                                      const float *lp_infer, const float *lp_old,
+                                      const float *adv, const uint8_t *mask,
+                                      const int32_t *cu_seqlens, int64_t B,
+                                      const cis_params_t *params, void *dhidden, void *dweight,
+                                      int32_t grad_dtype, float *lp_out, float *w_out,
+                                      uint8_t *trunc_out, cis_stats_t *stats_out,
+                                      double *loss_out, void *workspace, size_t workspace_bytes,
+                                      void *stream);
+
+/*
  * Largest T that cis_loss_fwd_bwd_noalloc accepts.
  */
 #define CIS_NOALLOC_MAX_TOKENS 65536

@@ -98,14 +98,25 @@ def _ptr(a):
     return None if a is None else a.ctypes.data_as(ctypes.c_void_p)
 
 
+F64 = 2
+
+
 def _logits_arg(logits):
-    """numpy float32 [T, ld] -> (array, F32); uint16 bf16 bit patterns -> (array, BF16)."""
+    """float32 [T, ld] -> F32; uint16 bf16 bit patterns -> BF16; float64 -> F64."""
     a = np.ascontiguousarray(logits)
     if a.dtype == np.float32:
         return a, F32
     if a.dtype == np.uint16:
         return a, BF16
-    raise TypeError(f"oracle logits must be float32 or uint16 (bf16 bits), got {a.dtype}")
+    if a.dtype == np.float64:
+        return a, F64
+    raise TypeError(f"oracle logits must be float32, float64 or uint16 (bf16 bits), got {a.dtype}")
+
+
+def bf16_bits_to_f64(bits) -> np.ndarray:
+    """Exact upcast of bf16 bit patterns (uint16) to float64."""
+    b = np.ascontiguousarray(bits, dtype=np.uint16)
+    return (b.astype(np.uint32) << 16).view(np.float32).astype(np.float64)
 
 
 def _opt(a, dtype):
@@ -190,4 +201,45 @@ def loss_fwd_bwd(logits, ids, lp_inf, adv, P: OracleParams, V=None, lp_old=None,
         else 0, _ptr(dz), _ptr(out["lp"]), _ptr(out["lse"]), _ptr(out["w"]), _ptr(trunc),
         _ptr(out["terms"]), _ptr(out["c"]), ctypes.byref(loss), nthreads)
     out.update(loss=loss.value, trunc=trunc, dz=dz, rc=rc)
+    return out
+
+
+def lmhead_fwd_bwd(hidden, weight, ids, lp_inf, adv, P: OracleParams, lp_old=None, mask=None,
+                   rows=None, n_valid_total=None, w_fixed=None, want_dw=True):
+    """The token pass through the LM head, in fp64.
+
+    Logits z = H W^T (Sec. 2.1; the softmax is over these logits) are formed
+    with an fp64 matrix product; the token pass itself is loss_fwd_bwd on those
+    logits (Eq. 1, Algorithm 1, Table 8); the chain rule through z = H W^T gives
+    dH = dz W and dW = dz^T H.
+
+    ``hidden`` [T, H] and ``weight`` [V, H] as bf16 bit patterns (uint16) or
+    float arrays.  ``rows``: evaluate only these tokens (their dH rows; dW then
+    needs every valid token, so it is returned only when rows is None).  With a
+    row subset and the token-mean normaliser, ``n_valid_total`` gives the number
+    of valid tokens of the whole batch.
+    """
+    Hf = bf16_bits_to_f64(hidden) if np.asarray(hidden).dtype == np.uint16 else \
+        np.asarray(hidden, np.float64)
+    Wf = bf16_bits_to_f64(weight) if np.asarray(weight).dtype == np.uint16 else \
+        np.asarray(weight, np.float64)
+    idx = np.arange(Hf.shape[0]) if rows is None else np.asarray(rows, np.int64)
+    sel = lambda a: None if a is None else np.asarray(a)[idx]  # noqa: E731
+    Z = Hf[idx] @ Wf.T
+    out = loss_fwd_bwd(Z, sel(ids), sel(lp_inf), sel(adv), P, lp_old=sel(lp_old),
+                       mask=sel(mask), w_fixed=sel(w_fixed))
+    if rows is not None and n_valid_total is not None:
+        if P.agg != AGG_TOKEN_MEAN:
+            raise ValueError("row subsets need the token-mean normaliser")
+        m = np.ones(len(idx), bool) if mask is None else np.asarray(mask)[idx].astype(bool)
+        f = m.sum() / float(n_valid_total)
+        for k in ("c", "terms", "dz"):
+            out[k] = out[k] * f
+        out["loss"] = float(out["terms"].sum())
+    out["dhidden"] = out["dz"] @ Wf
+    out["dhidden_abs"] = np.abs(out["dz"]) @ np.abs(Wf)
+    if want_dw and rows is None:
+        out["dweight"] = out["dz"].T @ Hf
+        out["dweight_abs"] = np.abs(out["dz"]).T @ np.abs(Hf)
+    out["logits"] = Z
     return out

@@ -76,10 +76,13 @@ static double bf16_to_double(uint16_t h)
     return (double)f;
 }
 
+/* Logit (t, j): dtype 0 = float32, 1 = bf16 bit patterns, 2 = float64. */
 static double logit_at(const void *logits, int dtype, int64_t ld, int64_t t, int64_t j)
 {
     if (dtype == 0)
         return (double)((const float *)logits)[t * ld + j];
+    if (dtype == 2)
+        return ((const double *)logits)[t * ld + j];
     return bf16_to_double(((const uint16_t *)logits)[t * ld + j]);
 }
 

@@ -85,6 +85,12 @@ def lib():
                                    ctypes.POINTER(cis_params_t), P, i32, i64, P, P, P, P, P, P,
                                    ctypes.c_size_t, P]
     L.cis_loss_fwd_bwd.restype = ctypes.c_int
+    L.cis_lmhead_workspace_size.argtypes = [i64, i64, i64, ctypes.POINTER(ctypes.c_size_t)]
+    L.cis_lmhead_workspace_size.restype = ctypes.c_int
+    L.cis_lmhead_fused.argtypes = [P, P, i64, i64, i64, P, P, P, P, P, P, i64,
+                                   ctypes.POINTER(cis_params_t), P, P, i32, P, P, P, P, P, P,
+                                   ctypes.c_size_t, P]
+    L.cis_lmhead_fused.restype = ctypes.c_int
     L.cis_profile_next_call.argtypes = [P, P]
     L.cis_profile_next_call.restype = ctypes.c_int
     _lib = L
@@ -230,6 +236,56 @@ def cis_loss_fwd_bwd(logits: torch.Tensor, ids: torch.Tensor, lp_infer: torch.Te
     _check(rc, "cis_loss_fwd_bwd")
     return {"dlogits": dlogits, "lp": lp, "w": w, "trunc": tr, "loss": loss, "stats": stats,
             "workspace": workspace}
+
+
+def cis_lmhead_workspace_size(T: int, V: int, H: int) -> int:
+    n = ctypes.c_size_t(0)
+    _check(lib().cis_lmhead_workspace_size(T, V, H, ctypes.byref(n)),
+           "cis_lmhead_workspace_size")
+    return n.value
+
+
+def cis_lmhead_fused(hidden: torch.Tensor, weight: torch.Tensor, ids: torch.Tensor,
+                     lp_infer: torch.Tensor, adv: torch.Tensor, params: cis_params_t,
+                     lp_old=None, mask=None, cu_seqlens=None, grad_dtype=torch.float32,
+                     workspace=None):
+    """Token pass through the LM head (logits never stored).  Returns a dict with
+    dhidden, dweight, lp, w, trunc, loss, stats and the workspace."""
+    _need_cuda(hidden, weight, ids, lp_infer, adv, lp_old, mask, cu_seqlens)
+    if hidden.dtype != torch.bfloat16 or weight.dtype != torch.bfloat16:
+        raise TypeError("hidden and weight must be bfloat16")
+    if not (hidden.is_contiguous() and weight.is_contiguous()):
+        raise ValueError("hidden and weight must be contiguous")
+    T, H = hidden.shape
+    V = weight.shape[0]
+    if weight.shape[1] != H:
+        raise ValueError("weight must be [V, H]")
+    dev = hidden.device
+    for x, dt, nm in ((ids, torch.int32, "ids"), (lp_infer, torch.float32, "lp_infer"),
+                      (adv, torch.float32, "adv"), (lp_old, torch.float32, "lp_old"),
+                      (mask, torch.uint8, "mask")):
+        _vec(x, dt, T, nm)
+    B = 0 if cu_seqlens is None else cu_seqlens.shape[0] - 1
+    dh = torch.empty((T, H), dtype=grad_dtype, device=dev)
+    dw = torch.empty((V, H), dtype=grad_dtype, device=dev)
+    lp = torch.empty(T, dtype=torch.float32, device=dev)
+    w = torch.empty(T, dtype=torch.float32, device=dev)
+    tr = torch.empty(T, dtype=torch.uint8, device=dev)
+    stats = torch.empty(ctypes.sizeof(cis_stats_t), dtype=torch.uint8, device=dev)
+    loss = torch.empty(1, dtype=torch.float64, device=dev)
+    nws = cis_lmhead_workspace_size(T, V, H) + 1024
+    if workspace is None or workspace.numel() < nws:
+        workspace = torch.empty(nws, dtype=torch.uint8, device=dev)
+    off = (-workspace.data_ptr()) % 1024  # 1024-byte aligned start
+    ws = workspace[off:]
+    rc = lib().cis_lmhead_fused(
+        _ptr(hidden), _ptr(weight), T, H, V, _ptr(ids), _ptr(lp_infer), _ptr(lp_old),
+        _ptr(adv), _ptr(mask), _ptr(cu_seqlens), B, ctypes.byref(params), _ptr(dh), _ptr(dw),
+        _dtype_code(grad_dtype), _ptr(lp), _ptr(w), _ptr(tr), _ptr(stats), _ptr(loss),
+        _ptr(ws), ws.numel(), _stream())
+    _check(rc, "cis_lmhead_fused")
+    return {"dhidden": dh, "dweight": dw, "lp": lp, "w": w, "trunc": tr, "loss": loss,
+            "stats": stats, "workspace": ws}
 
 
 def cis_profile_next_call(begin: "torch.cuda.Event | None", end: "torch.cuda.Event | None"):

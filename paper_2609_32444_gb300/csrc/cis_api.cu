@@ -35,7 +35,7 @@ WsLayout ws_layout(int64_t T)
 
 static bool finite_or_inf_nonneg(double x) { return x == x && x >= 0.0; }
 
-static bool params_ok(const cis_params_t *p)
+bool params_ok(const cis_params_t *p)
 {
     if (p == nullptr)
         return false;
@@ -58,7 +58,7 @@ static bool params_ok(const cis_params_t *p)
     return true;
 }
 
-static DevParams make_dev_params(const cis_params_t &p)
+DevParams make_dev_params(const cis_params_t &p)
 {
     DevParams d;
     d.mode = p.mode;

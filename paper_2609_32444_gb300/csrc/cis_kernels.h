@@ -33,6 +33,10 @@ struct PassArgs {
     DevParams P;
 };
 
+// Host-side parameter checks and the kernels' copy of the parameters.
+bool params_ok(const cis_params_t *p);
+DevParams make_dev_params(const cis_params_t &p);
+
 // Workspace layout (offsets in bytes from the 256-byte aligned base).
 struct WsLayout {
     size_t status, scale, terms, logk, w, trunc, total;

@@ -146,7 +146,7 @@ def _tempered_rows(n: int, V: int, pstar: torch.Tensor, g: torch.Generator, devi
 
 
 def make_batch(cfg: int, device="cpu", seed: int | None = None, T: int | None = None,
-               V: int | None = None, chunk_rows: int = 1024) -> Batch:
+               V: int | None = None, chunk_rows: int = 1024, H: int | None = None) -> Batch:
     """Draw the synthetic batch of workload ``cfg`` (see module docstring)."""
     spec = WORKLOADS[cfg]
     T = spec["T"] if T is None else T
@@ -209,7 +209,7 @@ def make_batch(cfg: int, device="cpu", seed: int | None = None, T: int | None = 
         cu, mask, adv = _pack(lengths, T, _group_advantages(rewards, 8), device)
 
         if cfg == 5:
-            H = spec["H"]
+            H = spec["H"] if H is None else H
             hidden = torch.randn((T, H), generator=g, device=device).to(torch.bfloat16)
             weight = (torch.randn((V, H), generator=g, device=device) * 0.02).to(torch.bfloat16)
             ids = torch.empty(T, dtype=torch.int64, device=device)

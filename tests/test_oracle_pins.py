@@ -401,3 +401,42 @@ def test_nan_ratio_propagates():
         w, tr, _, _ = oracle.weights(np.array([np.nan, -1.0]), np.array([-1.0, np.nan]),
                                      oracle.params(mode=mode))
         assert np.isnan(w).all() and not tr.any()
+
+
+def test_lmhead_chain_rule_matches_finite_differences():
+    """Through the LM head z = H W^T: dH = dz W and dW = dz^T H equal central
+    differences of the loss in H and W (weights frozen, l_old fixed)."""
+    rng = _rng(30)
+    T, Hd, V = 4, 6, 7
+    Hm = rng.integers(-16, 16, (T, Hd)) / 16.0
+    Wm = rng.integers(-16, 16, (V, Hd)) / 16.0
+    ids = rng.integers(0, V, T)
+    adv = np.array([1.0, -0.7, 0.4, -1.3])
+    z0 = Hm @ Wm.T
+    lp0 = _log_softmax(z0)[np.arange(T), ids]
+    lp_old = lp0 - np.log([1.0, 1.1, 0.95, 1.5])   # last token: A<0, rho>1 -> flows
+    lp_inf = lp0 + rng.standard_normal(T) * 0.5
+    P = oracle.params()
+    base = oracle.lmhead_fwd_bwd(Hm, Wm, ids, lp_inf, adv, P, lp_old=lp_old)
+    w0 = base["w"]
+    h = 2.0 ** -20
+    def loss(Hx, Wx):
+        return oracle.lmhead_fwd_bwd(Hx, Wx, ids, lp_inf, adv, P, lp_old=lp_old, w_fixed=w0,
+                                     want_dw=False)["loss"]
+    fdH = np.zeros_like(Hm)
+    for t in range(T):
+        for k in range(Hd):
+            a, b = Hm.copy(), Hm.copy()
+            a[t, k] += h
+            b[t, k] -= h
+            fdH[t, k] = (loss(a, Wm) - loss(b, Wm)) / (2 * h)
+    fdW = np.zeros_like(Wm)
+    for v in range(V):
+        for k in range(Hd):
+            a, b = Wm.copy(), Wm.copy()
+            a[v, k] += h
+            b[v, k] -= h
+            fdW[v, k] = (loss(Hm, a) - loss(Hm, b)) / (2 * h)
+    scale = max(np.abs(base["dhidden"]).max(), np.abs(base["dweight"]).max())
+    np.testing.assert_allclose(base["dhidden"], fdH, rtol=0, atol=1e-8 * scale)
+    np.testing.assert_allclose(base["dweight"], fdW, rtol=0, atol=1e-8 * scale)
