@@ -53,6 +53,7 @@ def parse_args():
     ap.add_argument("--workload", type=int, default=3, choices=[2, 3, 4, 5])
     ap.add_argument("--dlogits", choices=["bf16", "f32"], default="bf16")
     ap.add_argument("--e2e-steps", type=int, default=10)
+    ap.add_argument("--e2e-chunk", type=int, default=2048)
     ap.add_argument("--cpu-seconds", type=float, default=10.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--tokens", type=int, default=None,
@@ -313,32 +314,40 @@ def run_ours(args, rank, world, local):
     value = T * world / (ms_per_step / 1e3)
     clk = clocks.summary()
 
-    # ---- end to end through the C ABI with pinned host buffers
+    # ---- end to end through the C ABI with the batch in (pinned) host memory:
+    # cis_loss_fwd_bwd_host streams the rows through the GPU in chunks
     e2e = None
     if args.e2e_steps > 0:
-        hb = {k: v.cpu().pin_memory() for k, v in
+        hb = {k: v.cpu().contiguous().pin_memory() for k, v in
               dict(logits=b.logits, ids=b.ids, lp=b.lp_infer, adv=b.adv, mask=b.mask).items()}
         dz_h = torch.empty((T, V), dtype=dz_dt).pin_memory()
-        loss_h = torch.empty(1, dtype=torch.float64).pin_memory()
-        dbufs = {k: torch.empty_like(v, device=dev) for k, v in hb.items()}
-        h2d = sum(v.numel() * v.element_size() for v in hb.values())
-        d2h = dz_h.numel() * dz_h.element_size() + 8
+        hout = {}
+        hws = torch.empty(binding.cis_loss_host_workspace_size(T, V, b.logits.dtype, dz_dt,
+                                                               args.e2e_chunk),
+                          dtype=torch.uint8, device=dev)
+
+        def host_step():
+            return binding.cis_loss_fwd_bwd_host(hb["logits"], hb["ids"], hb["lp"], hb["adv"], P,
+                                                 dz_h, mask=hb["mask"],
+                                                 chunk_tokens=args.e2e_chunk, workspace=hws,
+                                                 outputs=hout)
+        host_step()
         torch.cuda.synchronize()
+        h2d = sum(v.numel() * v.element_size() for v in hb.values())
+        d2h = dz_h.numel() * dz_h.element_size() + T * (4 + 4 + 1) + 8 + 48
         barrier(world)
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         e0.record(stream)
         for _ in range(args.e2e_steps):
-            for k in hb:
-                dbufs[k].copy_(hb[k], non_blocking=True)
-            o = step(dbufs["logits"], dbufs["ids"], dbufs["lp"], dbufs["adv"], dbufs["mask"])
-            dz_h.copy_(dz, non_blocking=True)
-            loss_h.copy_(o["loss"], non_blocking=True)
+            host_step()
         e1.record(stream)
         torch.cuda.synchronize()
         e2e_ms = max_over_ranks(e0.elapsed_time(e1), world) / args.e2e_steps
         e2e = {"value": T * world / (e2e_ms / 1e3), "unit": "tokens/s",
-               "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms}
-        del hb, dz_h, dbufs
+               "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms,
+               "api": f"cis_loss_fwd_bwd_host, chunks of {args.e2e_chunk} tokens",
+               "link_GBps": (h2d + d2h) / (e2e_ms / 1e3) / 1e9}
+        del hb, dz_h, hws
 
     # ---- roofline of the main kernel
     isz = b.logits.element_size()

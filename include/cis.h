@@ -202,6 +202,41 @@ CIS_API cis_status_t cis_loss_fwd_bwd(const void *logits, int32_t dtype, int64_t
                               void *stream);
 
 /*
+ * Bytes of device workspace cis_loss_fwd_bwd_host needs for T tokens of V
+ * entries, the two element types, chunks of chunk_tokens rows and B responses
+ * (B = 0 without cu_seqlens).  Host only.  CIS_ERR_INVALID_ARG on bad values.
+ */
+CIS_API cis_status_t cis_loss_host_workspace_size(int64_t T, int64_t V, int32_t dtype,
+                                                  int32_t dlogits_dtype, int64_t chunk_tokens,
+                                                  int64_t B, size_t *bytes);
+
+/*
+ * cis_loss_fwd_bwd for callers whose buffers are in host memory.
+ *   Every tensor argument is a HOST pointer: logits [T, V] and dlogits [T, V]
+ *   (contiguous rows), ids, lp_infer, lp_old, adv, mask, cu_seqlens, and the
+ *   outputs lp_out, w_out, trunc_out, stats_out, loss_out.  Page-locked
+ *   (pinned) memory lets the copies overlap; pageable memory works but the
+ *   copies then serialise.
+ *   workspace is DEVICE memory of cis_loss_host_workspace_size(...) bytes,
+ *   256-byte aligned: the per-token arrays, the loss workspace and three
+ *   staging buffers of chunk_tokens rows in each direction.
+ * The rows stream through the GPU in chunks of chunk_tokens: while the fused
+ * kernel runs on chunk k (on `stream`), the next chunks are copied in and the
+ * previous ones copied out on copy streams the library creates once per
+ * device (one per staging buffer and direction).  The
+ * normaliser and the loss cover the whole batch, so every output equals that
+ * of cis_loss_fwd_bwd.  Asynchronous on `stream`: the host outputs are valid
+ * once `stream` has completed the call's work.  Errors: as cis_loss_fwd_bwd.
+ */
+CIS_API cis_status_t cis_loss_fwd_bwd_host(
+    const void *logits, int32_t dtype, int64_t T, int64_t V, const int32_t *ids,
+    const float *lp_infer, const float *lp_old, const float *adv, const uint8_t *mask,
+    const int32_t *cu_seqlens, int64_t B, const cis_params_t *params, void *dlogits,
+    int32_t dlogits_dtype, float *lp_out, float *w_out, uint8_t *trunc_out,
+    cis_stats_t *stats_out, double *loss_out, int64_t chunk_tokens, void *workspace,
+    size_t workspace_bytes, void *stream);
+
+/*
  * Bytes of device workspace cis_lmhead_fused needs.  Host only.
  * CIS_ERR_INVALID_ARG if bytes is NULL, T < 0, V <= 0 or H <= 0.
  */

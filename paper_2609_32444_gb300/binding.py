@@ -91,6 +91,13 @@ def lib():
                                    ctypes.POINTER(cis_params_t), P, P, i32, P, P, P, P, P, P,
                                    ctypes.c_size_t, P]
     L.cis_lmhead_fused.restype = ctypes.c_int
+    L.cis_loss_host_workspace_size.argtypes = [i64, i64, i32, i32, i64, i64,
+                                               ctypes.POINTER(ctypes.c_size_t)]
+    L.cis_loss_host_workspace_size.restype = ctypes.c_int
+    L.cis_loss_fwd_bwd_host.argtypes = [P, i32, i64, i64, P, P, P, P, P, P, i64,
+                                        ctypes.POINTER(cis_params_t), P, i32, P, P, P, P, P,
+                                        i64, P, ctypes.c_size_t, P]
+    L.cis_loss_fwd_bwd_host.restype = ctypes.c_int
     L.cis_profile_next_call.argtypes = [P, P]
     L.cis_profile_next_call.restype = ctypes.c_int
     _lib = L
@@ -236,6 +243,49 @@ def cis_loss_fwd_bwd(logits: torch.Tensor, ids: torch.Tensor, lp_infer: torch.Te
     _check(rc, "cis_loss_fwd_bwd")
     return {"dlogits": dlogits, "lp": lp, "w": w, "trunc": tr, "loss": loss, "stats": stats,
             "workspace": workspace}
+
+
+def cis_loss_host_workspace_size(T, V, dtype, dlogits_dtype, chunk_tokens, B=0) -> int:
+    n = ctypes.c_size_t(0)
+    _check(lib().cis_loss_host_workspace_size(T, V, _dtype_code(dtype), _dtype_code(dlogits_dtype),
+                                              chunk_tokens, B, ctypes.byref(n)),
+           "cis_loss_host_workspace_size")
+    return n.value
+
+
+def cis_loss_fwd_bwd_host(logits: torch.Tensor, ids: torch.Tensor, lp_infer: torch.Tensor,
+                          adv: torch.Tensor, params: cis_params_t, dlogits: torch.Tensor,
+                          lp_old=None, mask=None, cu_seqlens=None, chunk_tokens=2048,
+                          workspace=None, outputs=None):
+    """The fused pass with every tensor in HOST memory (pinned for overlap);
+    rows stream through the GPU in chunks.  ``outputs``: optional dict of host
+    tensors lp, w, trunc, stats, loss to fill.  Returns that dict; it is valid
+    after the current stream completes."""
+    for x in (logits, ids, lp_infer, adv, dlogits, lp_old, mask, cu_seqlens):
+        if x is not None and x.is_cuda:
+            raise ValueError("cis_loss_fwd_bwd_host takes host tensors")
+    if not (logits.is_contiguous() and dlogits.is_contiguous()):
+        raise ValueError("logits and dlogits must be contiguous")
+    T, V = logits.shape
+    B = 0 if cu_seqlens is None else cu_seqlens.shape[0] - 1
+    out = outputs or {}
+    out.setdefault("lp", torch.empty(T, dtype=torch.float32).pin_memory())
+    out.setdefault("w", torch.empty(T, dtype=torch.float32).pin_memory())
+    out.setdefault("trunc", torch.empty(T, dtype=torch.uint8).pin_memory())
+    out.setdefault("stats", torch.empty(ctypes.sizeof(cis_stats_t), dtype=torch.uint8).pin_memory())
+    out.setdefault("loss", torch.empty(1, dtype=torch.float64).pin_memory())
+    nws = cis_loss_host_workspace_size(T, V, logits.dtype, dlogits.dtype, chunk_tokens, B)
+    if workspace is None or workspace.numel() < nws:
+        workspace = torch.empty(nws, dtype=torch.uint8, device="cuda")
+    rc = lib().cis_loss_fwd_bwd_host(
+        _ptr(logits), _dtype_code(logits.dtype), T, V, _ptr(ids), _ptr(lp_infer), _ptr(lp_old),
+        _ptr(adv), _ptr(mask), _ptr(cu_seqlens), B, ctypes.byref(params), _ptr(dlogits),
+        _dtype_code(dlogits.dtype), _ptr(out["lp"]), _ptr(out["w"]), _ptr(out["trunc"]),
+        _ptr(out["stats"]), _ptr(out["loss"]), chunk_tokens, _ptr(workspace), workspace.numel(),
+        _stream())
+    _check(rc, "cis_loss_fwd_bwd_host")
+    out["workspace"] = workspace
+    return out
 
 
 def cis_lmhead_workspace_size(T: int, V: int, H: int) -> int:
