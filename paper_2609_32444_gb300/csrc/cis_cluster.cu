@@ -168,6 +168,16 @@ template <> struct MaxAcc<float> {
     __device__ __forceinline__ float result() const { return m; }
 };
 
+// Sum of 2^{z_i log2e - off} over 8 values, added pairwise.
+__device__ __forceinline__ float sum8_exp2_off(const float (&z)[8], float off)
+{
+    float e[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i)
+        e[i] = ex2_ftz(fmaf(z[i], kLog2e, -off));
+    return ((e[0] + e[1]) + (e[2] + e[3])) + ((e[4] + e[5]) + (e[6] + e[7]));
+}
+
 // 8 results to global memory with streaming (evict-first) 16-byte stores.
 template <typename OutT> __device__ __forceinline__ void store8(OutT *dst, const float (&v)[8]);
 template <>
@@ -195,7 +205,7 @@ struct ClusterShared {
     alignas(8) uint64_t xbar;          // arrival of the cluster's (m, s) pairs
     float2 part[kMaxCluster];
     MaxSum red[512 / 32];
-    float c, m, bias, lp;
+    float c, cs, B, lp;
 };
 
 __device__ __forceinline__ uint32_t map_rank(uint32_t addr, uint32_t rank)
@@ -346,14 +356,20 @@ __global__ void __launch_bounds__(kThreads) cis_fused_cluster_kernel(const PassA
     const float m = macc.result();
 
     // Pass 1b: sum of e^{z - max} (8 exponentials added pairwise per group).
+    // 2^{(z - m) log2e} is formed with one FMA as 2^{z log2e - cm}, cm = fl(m log2e);
+    // the rounding residual of cm is exact (an FMA) and is taken out once at
+    // the end, so the sum equals the one over (z - m) log2e.
     float s = 0.0f;
     if (m != -INFINITY) {
+        const float cm = m * kLog2e;
+        const float cm_err = fmaf(m, kLog2e, -cm);  // m log2e - cm, exactly
 #pragma unroll 2
         for (int g = threadIdx.x; g < ng; g += kThreads) {
             float z[8];
             load8<InT>(slab, g, z);
-            s += sum8_exp(z, m);
+            s += sum8_exp2_off(z, cm);
         }
+        s *= ex2_ftz(-cm_err);
     }
     const MaxSum mine = block_ms<kThreads, false>(MaxSum{m, s}, sh.red);
 
@@ -386,9 +402,22 @@ __global__ void __launch_bounds__(kThreads) cis_fused_cluster_kernel(const PassA
             a.ws_logk[t] = tw.logk;
             a.ws_terms[t] = tl.term;
         }
-        sh.c = tl.c;
-        sh.m = rs.m;
-        sh.bias = rs.bias_log2;
+        // Pass 2 forms c softmax_j as cs 2^{z_j log2e - B}: with the power-of-two
+        // scale K = clamp(ilogb(c) + 25, 0, 127) (below), B = fl(m log2e + bias
+        // - K), and the rounding residual of B folded into cs.
+        const float c = tl.c;
+        const int kexp = (int)((__float_as_uint(c) >> 23) & 0xff) - 127 + 25;
+        const int K = kexp < 0 ? 0 : (kexp > 127 ? 127 : kexp);
+        float cs = ldexpf(c, -K);
+        float B = INFINITY;
+        if (rs.bias_log2 != INFINITY) {
+            const double Bd = (double)rs.m * (double)kLog2e + ((double)rs.bias_log2 - K);
+            B = (float)Bd;
+            cs *= ex2_ftz((float)((double)B - Bd));
+        }
+        sh.c = c;
+        sh.cs = cs;
+        sh.B = B;
         sh.lp = rs.lp;
     }
     __syncthreads();
@@ -399,11 +428,7 @@ __global__ void __launch_bounds__(kThreads) cis_fused_cluster_kernel(const PassA
     // 2^(x_j + K) would be subnormal, |c softmax_j| < 2^-150 rounds to zero in
     // fp32 and bf16 anyway; c 2^-K stays normal and 2^(x_j + K) finite.  The
     // final multiply keeps subnormal products.
-    const float c = sh.c, mo = sh.m;
-    const int kexp = (int)((__float_as_uint(c) >> 23) & 0xff) - 127 + 25;
-    const int K = kexp < 0 ? 0 : (kexp > 127 ? 127 : kexp);
-    const float cs2 = ldexpf(c, -K);
-    const float bias = sh.bias - (float)K;
+    const float c = sh.c, cs2 = sh.cs, B = sh.B;
     const float dzy = c * expm1f(sh.lp);  // c (p - 1)
 #pragma unroll 2
     for (int g = threadIdx.x; g < ng; g += kThreads) {
@@ -411,7 +436,7 @@ __global__ void __launch_bounds__(kThreads) cis_fused_cluster_kernel(const PassA
         load8<InT>(slab, g, z);
 #pragma unroll
         for (int i = 0; i < 8; ++i)
-            v[i] = cs2 * ex2_ftz(fmaf(z[i] - mo, kLog2e, -bias));
+            v[i] = cs2 * ex2_ftz(fmaf(z[i], kLog2e, -B));
         if (g == gy) {  // the sampled entry: c (p - 1)
 #pragma unroll
             for (int i = 0; i < 8; ++i)

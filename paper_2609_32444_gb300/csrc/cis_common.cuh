@@ -287,15 +287,4 @@ __device__ __forceinline__ RowScalars row_scalars(MaxSum o, float zy)
     return r;
 }
 
-// Sum of e^{z - m} over 8 values, added pairwise so that the rounding error
-// does not grow with the row length.
-__device__ __forceinline__ float sum8_exp(const float (&z)[8], float m)
-{
-    float e[8];
-#pragma unroll
-    for (int i = 0; i < 8; ++i)
-        e[i] = ex2_ftz((z[i] - m) * kLog2e);
-    return ((e[0] + e[1]) + (e[2] + e[3])) + ((e[4] + e[5]) + (e[6] + e[7]));
-}
-
 }  // namespace cis
