@@ -23,10 +23,15 @@
 // carries on to its end so that TMEM is always released.
 #include <cuda.h>
 #include <cudaTypedefs.h>
+#include <stdlib.h>
 #include <mutex>
+
+#include <cooperative_groups.h>
 
 #include "cis_kernels.h"
 #include "cis_tc.cuh"
+
+namespace cg = cooperative_groups;
 
 namespace cis {
 namespace lm {
@@ -427,6 +432,395 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
 }
 
+// ---------------------------------------------------------------------------
+// Gradient passes shared by a cluster: R = Hd / 256 CTAs, CTA r accumulating
+// block r (256 columns) of dH (or dW).  Step j of the sweep is vocabulary tile
+// j (dW: token tile j).  Its logit tile is computed once, by the CTA that owns
+// the step (j mod R), which forms the bf16 dz tile in its own shared memory
+// and bulk-copies it into the same mailbox slot (j mod 2) of every other CTA
+// of the cluster; each copy is counted on the receiver's mbarrier.  Every CTA
+// consumes every step: block r += dz_j x (W^T or H^T)[block r, tile j].  After
+// consuming step j a CTA's MMA commit is multicast to the slot-free mbarrier
+// of the owner of step j + 2, which reuses the slot.  A CTA computes the logit
+// tile of its k-th owned step t_k = r + kR spread over the R steps of the
+// period two before it (4 K blocks per step), so no commit waits on a whole
+// tile, and the tile is ready R + 1 steps before it is consumed.
+//
+// Phases.  Copies into slot s of a CTA arrive in step order, each only after
+// the CTA has consumed the previous step of that slot, so neither the mailbox
+// nor the per-slot slot-free barrier can run a phase ahead of its waiter.
+// Teardown.  Each copy is first recorded in the receiver (a remote max of the
+// step index), so after a cluster barrier that ends all copying a CTA knows
+// whether a copy into it may still be in flight and waits for it (bounded)
+// before the second cluster barrier; only then may a CTA leave.
+constexpr int kSlotBytes = 32768;
+
+struct CBarriers {
+    uint64_t full[kStages], empty[kStages];
+    uint64_t zfull[2], zempty[2];
+    uint64_t dzfull[2];     // the dz tile of the step in slot s has landed
+    uint64_t slot_free[2];  // every CTA has consumed the step that last used slot s
+    uint64_t accfull;
+};
+
+template <int MODE>
+__global__ void __launch_bounds__(kThreads, 1)
+    cis_lmhead_grad_kernel(const __grid_constant__ CUtensorMap tmA,
+                           const __grid_constant__ CUtensorMap tmB,
+                           const __grid_constant__ CUtensorMap tmB2, const Params p)
+{
+    extern __shared__ __align__(1024) uint8_t dsm[];
+    uint8_t *base = dsm + ((1024 - (tc::smem_addr(dsm) & 1023)) & 1023);
+    uint8_t *ring = base;                            // kStages x 32 KB
+    uint8_t *slots = base + kStages * kStageBytes;   // 2 x 32 KB dz mailboxes
+    __shared__ __align__(8) CBarriers bars;
+    __shared__ uint32_t tmem_base;
+    __shared__ int aborted;
+    __shared__ int last_copied[2];  // latest step copied into slot s by its owner
+    __shared__ float col_lse[kBN], col_c[kBN];
+    __shared__ int col_y[kBN];
+
+    cg::cluster_group cluster = cg::this_cluster();
+    const int R = (int)cluster.num_blocks();
+    const int rank = (int)cluster.block_rank();
+    const int a_tile = blockIdx.x / R;
+    const int nB = MODE == kDh ? p.nVt : p.nTt;
+    const int Q = p.nK / R;  // K blocks of a logit tile issued per step
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+    if (threadIdx.x == 0) {
+        aborted = 0;
+        last_copied[0] = last_copied[1] = -1;
+        for (int s = 0; s < kStages; ++s) {
+            tc::bar_init(&bars.full[s], 1);
+            tc::bar_init(&bars.empty[s], 1);
+        }
+        for (int b = 0; b < 2; ++b) {
+            tc::bar_init(&bars.zfull[b], 1);
+            tc::bar_init(&bars.zempty[b], 128);
+            tc::bar_init(&bars.dzfull[b], 1);
+            tc::bar_init(&bars.slot_free[b], R);
+        }
+        tc::bar_init(&bars.accfull, 1);
+        tc::bar_init_fence();
+    }
+    if (warp == 1)
+        tc::tmem_alloc(&tmem_base, 512);
+    tc::fence_before_sync();
+    __syncthreads();
+    tc::fence_after_sync();
+    // every CTA of the cluster has initialised its barriers before any remote use
+    tc::cluster_arrive();
+    tc::cluster_wait();
+    const uint32_t tmem = tmem_base;
+    const uint32_t tmem_acc = tmem + 256;
+    const Abort ab{&aborted, p.status};
+    int consumed = 0;  // MMA thread: steps 0 .. consumed-1 are fully issued
+    int expected = -1; // MMA thread: latest step whose copy it announced
+
+    // The ring items in the order both the producer and the MMA issuer take
+    // them: fn_z(k, kb) for K block kb of owned tile t_k, fn_step(j) before
+    // the two B2 items fn_b2(j, 0), fn_b2(j, 1) of step j.
+    auto walk = [&](auto &&fn_z, auto &&fn_step, auto &&fn_b2) {
+        if (rank < nB)
+            for (int kb = 0; kb < p.nK; ++kb)
+                fn_z(0, kb);
+        if (rank + R < nB)
+            for (int kb = 0; kb < (R - rank) * Q; ++kb)
+                fn_z(1, kb);
+        for (int j = 0; j < nB && !ab.on(); ++j) {
+            int k, pi;
+            if (j < rank) {
+                k = 1;
+                pi = j - rank + R;
+            } else {
+                k = (j - rank) / R + 2;
+                pi = (j - rank) % R;
+            }
+            if (rank + k * R < nB)
+                for (int kb = pi * Q; kb < (pi + 1) * Q; ++kb)
+                    fn_z(k, kb);
+            fn_step(j);
+            fn_b2(j, 0);
+            fn_b2(j, 1);
+        }
+    };
+
+    if (warp == 0) {
+        if (lane == 0) {
+            int stage = 0;
+            uint32_t phase = 0;
+            uint32_t used = 0, last_phase = 0;  // per stage: loaded, parity of its last load
+            auto next = [&]() -> bool {
+                if (ab.on())
+                    return false;
+                ab.wait(&bars.empty[stage], phase ^ 1, p.status);
+                if (ab.on())
+                    return false;
+                tc::bar_expect_tx(&bars.full[stage], kStageBytes);
+                used |= 1u << stage;
+                last_phase = (last_phase & ~(1u << stage)) | (phase << stage);
+                return true;
+            };
+            auto adv = [&]() {
+                if (++stage == kStages) {
+                    stage = 0;
+                    phase ^= 1;
+                }
+            };
+            walk(
+                [&](int k, int kb) {
+                    if (!next())
+                        return;
+                    uint8_t *st = ring + stage * kStageBytes;
+                    tc::tma_load_2d(st, &tmA, kb * kBK, a_tile * kBM, &bars.full[stage]);
+                    tc::tma_load_2d(st + kStageBytes / 2, &tmB, kb * kBK, (rank + k * R) * kBN,
+                                    &bars.full[stage]);
+                    adv();
+                },
+                [&](int) {},
+                [&](int j, int kb2) {
+                    if (!next())
+                        return;
+                    tc::tma_load_2d(ring + stage * kStageBytes, &tmB2, j * kBN + kb2 * kBK,
+                                    rank * kN2, &bars.full[stage]);
+                    adv();
+                });
+            // no load may still be landing when the CTA leaves
+            for (int s = 0; s < kStages; ++s)
+                if (used & (1u << s))
+                    tc::bar_wait(&bars.full[s], (last_phase >> s) & 1);
+        }
+    } else if (warp == 1) {
+        if (lane == 0) {
+            constexpr uint32_t kIdZ = tc::idesc_bf16(kBM, kBN);
+            constexpr uint32_t kId2 = tc::idesc_bf16(kBM, kN2);
+            int stage = 0;
+            uint32_t phase = 0;
+            auto adv = [&]() {
+                if (++stage == kStages) {
+                    stage = 0;
+                    phase ^= 1;
+                }
+            };
+            walk(
+                [&](int k, int kb) {
+                    if (ab.on())
+                        return;
+                    const int zb = k & 1;
+                    if (kb == 0)  // the buffer's previous tile has been read
+                        ab.wait(&bars.zempty[zb], ((k >> 1) & 1) ^ 1, p.status);
+                    ab.wait(&bars.full[stage], phase, p.status);
+                    if (ab.on())
+                        return;
+                    tc::fence_after_sync();
+                    const uint32_t sa = tc::smem_addr(ring + stage * kStageBytes);
+                    const uint32_t sb = sa + kStageBytes / 2;
+#pragma unroll
+                    for (int kk = 0; kk < kBK / 16; ++kk)
+                        tc::mma_bf16(tmem + zb * kBN, tc::desc_sw128(sa + kk * 32),
+                                     tc::desc_sw128(sb + kk * 32), kIdZ, (kb | kk) != 0);
+                    tc::mma_commit(&bars.empty[stage]);
+                    adv();
+                    if (kb == p.nK - 1)
+                        tc::mma_commit(&bars.zfull[zb]);
+                },
+                [&](int j) {
+                    if (ab.on())
+                        return;
+                    const int s = j & 1;
+                    if (j % R != rank) {  // the owner's copy brings the bytes
+                        tc::bar_expect_tx(&bars.dzfull[s], kSlotBytes);
+                        expected = j;
+                    }
+                    if (!tc::bar_wait_cluster(&bars.dzfull[s], (j >> 1) & 1)) {
+                        aborted = 1;
+                        set_status(p.status, kStatusTimeout);
+                    }
+                },
+                [&](int j, int kb2) {
+                    if (ab.on())
+                        return;
+                    ab.wait(&bars.full[stage], phase, p.status);
+                    if (ab.on())
+                        return;
+                    tc::fence_after_sync();
+                    const uint32_t sdz = tc::smem_addr(slots + (j & 1) * kSlotBytes);
+                    const uint32_t sb2 = tc::smem_addr(ring + stage * kStageBytes);
+#pragma unroll
+                    for (int kk = 0; kk < kBK / 16; ++kk)
+                        tc::mma_bf16(tmem_acc, tc::desc_sw128(sdz + kb2 * 16384 + kk * 32),
+                                     tc::desc_sw128(sb2 + kk * 32), kId2,
+                                     j > 0 || kb2 > 0 || kk > 0);
+                    tc::mma_commit(&bars.empty[stage]);
+                    adv();
+                    if (kb2 == 1) {
+                        if (j + 2 < nB)  // slot j & 1 is free here for step j + 2
+                            tc::mma_commit_multicast(&bars.slot_free[j & 1],
+                                                     (uint16_t)(1u << ((j + 2) % R)));
+                        consumed = j + 1;
+                    }
+                });
+            // every MMA of this CTA (and the arrivals committed with them) is
+            // done before the epilogue reads the block or the CTA leaves
+            tc::mma_commit(&bars.accfull);
+            tc::bar_wait(&bars.accfull, 0);
+        }
+    } else {
+        const int lg = warp & 3;
+        const int r = lg * 32 + lane;
+        const uint32_t lane_off = (uint32_t)(lg * 32) << 16;
+        const int e = threadIdx.x - 64;
+        const int row = a_tile * kBM + r;  // token (DH) or vocabulary entry (DW)
+        int y_r = -1;
+        float lse_r = 0.0f, c_r = 0.0f;
+        if (MODE == kDh && row < p.T) {
+            y_r = p.ids[row];
+            lse_r = p.lse[row];
+            c_r = p.cvec[row];
+        }
+        uint32_t nfree = 0;  // per slot (bit s): parity of its next slot-free phase
+        for (int k = 0; rank + k * R < nB; ++k) {
+            const int t = rank + k * R;  // the owned step
+            const int zb = k & 1, s = t & 1;
+            if (__syncthreads_or_epi(ab.on()))
+                break;
+            if (MODE == kDw) {
+                const int tt = t * kBN + e;
+                const bool ok = tt < p.T;
+                col_lse[e] = ok ? p.lse[tt] : 0.0f;
+                col_c[e] = ok ? p.cvec[tt] : 0.0f;
+                col_y[e] = ok ? p.ids[tt] : -1;
+            }
+            ab.wait(&bars.zfull[zb], (k >> 1) & 1, p.status);
+            tc::fence_after_sync();
+            if (t >= 2) {  // slot s still holds step t - 2 somewhere in the cluster
+                if (!ab.on() && !tc::bar_wait_cluster(&bars.slot_free[s], (nfree >> s) & 1)) {
+                    aborted = 1;
+                    set_status(p.status, kStatusTimeout);
+                }
+                nfree ^= 1u << s;
+            }
+            asm volatile("bar.sync 1, 128;" ::: "memory");  // column scalars visible
+            uint8_t *slot = slots + s * kSlotBytes;
+            const int col0 = t * kBN;
+            for (int c0 = 0; c0 < kBN; c0 += 32) {
+                float v[32];
+                tc::tmem_ld32(tmem + lane_off + zb * kBN + c0, v);
+#pragma unroll
+                for (int i = 0; i < 32; ++i) {
+                    const int col = c0 + i;
+                    float d;
+                    // tokens with c = 0 (masked, clipped, past T) give 0 without
+                    // touching the exponential (their lse is a placeholder)
+                    if (MODE == kDh) {
+                        const int gcol = col0 + col;
+                        d = (gcol < p.V && c_r != 0.0f)
+                                ? c_r * ex2_ftz((v[i] - lse_r) * kLog2e) -
+                                      (gcol == y_r ? c_r : 0.0f)
+                                : 0.0f;
+                    } else {
+                        const float lt = col_lse[col], ct = col_c[col];
+                        d = (row < p.V && ct != 0.0f)
+                                ? ct * ex2_ftz((v[i] - lt) * kLog2e) -
+                                      (col_y[col] == row ? ct : 0.0f)
+                                : 0.0f;
+                    }
+                    v[i] = d;
+                }
+                uint8_t *blk = slot + (c0 >> 6) * 16384;
+#pragma unroll
+                for (int q = 0; q < 4; ++q) {
+                    uint4 w;
+                    __nv_bfloat162 h;
+                    h = __floats2bfloat162_rn(v[8 * q + 0], v[8 * q + 1]);
+                    w.x = *reinterpret_cast<uint32_t *>(&h);
+                    h = __floats2bfloat162_rn(v[8 * q + 2], v[8 * q + 3]);
+                    w.y = *reinterpret_cast<uint32_t *>(&h);
+                    h = __floats2bfloat162_rn(v[8 * q + 4], v[8 * q + 5]);
+                    w.z = *reinterpret_cast<uint32_t *>(&h);
+                    h = __floats2bfloat162_rn(v[8 * q + 6], v[8 * q + 7]);
+                    w.w = *reinterpret_cast<uint32_t *>(&h);
+                    *reinterpret_cast<uint4 *>(blk + tc::sw128_offset(r, ((c0 & 63) >> 3) + q)) = w;
+                }
+            }
+            tc::fence_before_sync();
+            tc::bar_arrive(&bars.zempty[zb]);
+            tc::fence_proxy_async_smem();
+            asm volatile("bar.sync 1, 128;" ::: "memory");  // the whole tile is written
+            if (e == 0 && !ab.on()) {
+                const uint32_t src = tc::smem_addr(slot);
+                const uint32_t bar = tc::smem_addr(&bars.dzfull[s]);
+                const uint32_t rec = tc::smem_addr(&last_copied[s]);
+                for (int q = 0; q < R; ++q)
+                    if (q != rank) {
+                        tc::red_max_cluster(tc::map_rank(rec, q), t);
+                        tc::bulk_s2s(tc::map_rank(src, q), src, kSlotBytes, tc::map_rank(bar, q));
+                    }
+                tc::bar_arrive(&bars.dzfull[s]);
+            }
+        }
+        // the accumulated block: 128 rows x 256 columns
+        ab.wait(&bars.accfull, 0, p.status);
+        tc::fence_after_sync();
+        const int nrows = MODE == kDh ? p.T : p.V;
+        for (int c0 = 0; c0 < kN2; c0 += 32) {
+            float v[32];
+            tc::tmem_ld32(tmem_acc + lane_off + c0, v);
+            if (row < nrows) {
+                const int64_t o = (int64_t)row * p.ld_out + (int64_t)rank * kN2 + c0;
+                if (p.out_bf16) {
+                    __nv_bfloat16 *dst = reinterpret_cast<__nv_bfloat16 *>(p.out) + o;
+#pragma unroll
+                    for (int q = 0; q < 4; ++q) {
+                        uint4 w;
+                        __nv_bfloat162 h;
+                        h = __floats2bfloat162_rn(v[8 * q + 0], v[8 * q + 1]);
+                        w.x = *reinterpret_cast<uint32_t *>(&h);
+                        h = __floats2bfloat162_rn(v[8 * q + 2], v[8 * q + 3]);
+                        w.y = *reinterpret_cast<uint32_t *>(&h);
+                        h = __floats2bfloat162_rn(v[8 * q + 4], v[8 * q + 5]);
+                        w.z = *reinterpret_cast<uint32_t *>(&h);
+                        h = __floats2bfloat162_rn(v[8 * q + 6], v[8 * q + 7]);
+                        w.w = *reinterpret_cast<uint32_t *>(&h);
+                        reinterpret_cast<uint4 *>(dst)[q] = w;
+                    }
+                } else {
+                    float4 *dst =
+                        reinterpret_cast<float4 *>(reinterpret_cast<float *>(p.out) + o);
+#pragma unroll
+                    for (int q = 0; q < 8; ++q)
+                        dst[q] = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+                }
+            }
+        }
+    }
+    // Teardown: after the first cluster barrier no CTA issues another copy;
+    // each CTA then waits for any copy recorded into it that it has not seen
+    // land, and no CTA leaves before all have done so.
+    __syncwarp();
+    tc::fence_before_sync();
+    tc::cluster_arrive();
+    tc::cluster_wait();
+    if (warp == 1 && lane == 0) {
+        for (int s = 0; s < 2; ++s) {
+            const int L = *reinterpret_cast<volatile int *>(&last_copied[s]);
+            if (L >= consumed) {  // recorded but not consumed: it may be landing
+                if (L != expected)
+                    tc::bar_expect_tx(&bars.dzfull[s], kSlotBytes);
+                tc::bar_wait_cluster(&bars.dzfull[s], (L >> 1) & 1);
+            }
+        }
+    }
+    __syncwarp();
+    tc::cluster_arrive();
+    tc::cluster_wait();
+    if (warp == 1) {
+        tc::fence_after_sync();
+        tc::tmem_dealloc(tmem, 512);
+    }
+}
+
 // Per token: combine the FWD pairs, then log p, weight, loss, c_t (one warp).
 __global__ void cis_lmhead_token_kernel(const PassArgs a, const float2 *part, const float *zy,
                                         int nVt, float *lse_out, float *c_out)
@@ -545,6 +939,43 @@ cudaError_t launch_mode(const CUtensorMap &a, const CUtensorMap &b, const CUtens
         return e;
     k<<<grid, kThreads, kSmemBytes, s>>>(a, b, b2, p);
     return cudaGetLastError();
+}
+
+constexpr size_t kGradSmemBytes = kStages * kStageBytes + 2 * kSlotBytes + 1024;
+
+template <int MODE>
+cudaError_t launch_grad(const CUtensorMap &a, const CUtensorMap &b, const CUtensorMap &b2,
+                        const Params &p, int clusters, int R, cudaStream_t s)
+{
+    auto k = cis_lmhead_grad_kernel<MODE>;
+    cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)kGradSmemBytes);
+    if (e != cudaSuccess)
+        return e;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)(clusters * R), 1, 1);
+    cfg.blockDim = dim3(kThreads, 1, 1);
+    cfg.dynamicSmemBytes = kGradSmemBytes;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = (unsigned)R;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, k, a, b, b2, p);
+}
+
+// Use the cluster gradient kernels?  Needs a portable cluster (Hd <= 2048);
+// CIS_LMHEAD_RECOMPUTE=1 selects the recompute kernels instead (for comparison).
+bool use_cluster_grad(int64_t H)
+{
+    static int force_recompute = [] {
+        const char *e = getenv("CIS_LMHEAD_RECOMPUTE");
+        return e ? atoi(e) : 0;
+    }();
+    return !force_recompute && H / kN2 <= 8;
 }
 
 }  // namespace lm
@@ -705,12 +1136,16 @@ CIS_API cis_status_t cis_lmhead_fused(const void *hidden, const void *weight, in
         p.out = dhidden;
         p.out_bf16 = grad_dtype == CIS_BF16;
         p.ld_out = H;
-        e = lm::launch_mode<lm::kDh>(mH, mW, mWt, p, nTt * (int)(H / lm::kN2), s);
+        const int R = (int)(H / lm::kN2);
+        const bool clustered = lm::use_cluster_grad(H);
+        e = clustered ? lm::launch_grad<lm::kDh>(mH, mW, mWt, p, nTt, R, s)
+                      : lm::launch_mode<lm::kDh>(mH, mW, mWt, p, nTt * R, s);
         if (e != cudaSuccess)
             return CIS_ERR_CUDA;
         // dW: A = W (vocab tiles), B = H (token tiles), B2 = H^T
         p.out = dweight;
-        e = lm::launch_mode<lm::kDw>(mW, mH, mHt, p, nVt * (int)(H / lm::kN2), s);
+        e = clustered ? lm::launch_grad<lm::kDw>(mW, mH, mHt, p, nVt, R, s)
+                      : lm::launch_mode<lm::kDw>(mW, mH, mHt, p, nVt * R, s);
         if (e != cudaSuccess)
             return CIS_ERR_CUDA;
     }

@@ -154,6 +154,70 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32])
         v[i] = __uint_as_float(r[i]);
 }
 
+// ------------------------------------------------------------------ cluster
+__device__ __forceinline__ uint32_t map_rank(uint32_t saddr, uint32_t rank)
+{
+    uint32_t r;
+    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(saddr), "r"(rank));
+    return r;
+}
+__device__ __forceinline__ void cluster_arrive()
+{
+    asm volatile("barrier.cluster.arrive.release.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void cluster_wait()
+{
+    asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+// Bounded wait for a phase completed by another CTA of the cluster (its bulk
+// copies or its tensor cores).
+__device__ __forceinline__ bool bar_wait_cluster(uint64_t *bar, uint32_t parity)
+{
+    const uint32_t a = smem_addr(bar);
+    for (uint32_t i = 0; i < kMaxPolls; ++i) {
+        uint32_t done;
+        asm volatile(
+            "{\n\t.reg .pred p;\n\t"
+            "mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2, %3;\n\t"
+            "selp.u32 %0, 1, 0, p;\n\t}"
+            : "=r"(done)
+            : "r"(a), "r"(parity), "r"(kPollSuspendNs)
+            : "memory");
+        if (done)
+            return true;
+    }
+    return false;
+}
+// Copy `bytes` of this CTA's shared memory to another CTA's shared memory
+// (addresses from map_rank); the receiver's mbarrier counts the bytes.
+__device__ __forceinline__ void bulk_s2s(uint32_t dst_cluster, uint32_t src_cta, uint32_t bytes,
+                                         uint32_t bar_cluster)
+{
+    asm volatile(
+        "cp.async.bulk.shared::cluster.shared::cta.mbarrier::complete_tx::bytes"
+        " [%0], [%1], %2, [%3];" ::"r"(dst_cluster),
+        "r"(src_cta), "r"(bytes), "r"(bar_cluster)
+        : "memory");
+}
+// Once every MMA issued so far by this thread is done, arrive on the mbarrier
+// at the same shared-memory offset in each CTA of `cta_mask`.
+__device__ __forceinline__ void mma_commit_multicast(uint64_t *bar, uint16_t cta_mask)
+{
+    asm volatile(
+        "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64"
+        " [%0], %1;" ::"r"(smem_addr(bar)),
+        "h"(cta_mask)
+        : "memory");
+}
+
+// max(*addr, v) on a 32-bit word of a CTA of the cluster (address from map_rank).
+__device__ __forceinline__ void red_max_cluster(uint32_t addr_cluster, int v)
+{
+    asm volatile("red.relaxed.cluster.shared::cluster.max.s32 [%0], %1;" ::"r"(addr_cluster),
+                 "r"(v)
+                 : "memory");
+}
+
 // Byte offset of 16-byte chunk q (0..7) of row r inside a 128-byte-swizzled
 // K-major block (the layout TMA SWIZZLE_128B produces).
 __device__ __forceinline__ uint32_t sw128_offset(int r, int q)
