@@ -237,10 +237,21 @@ CIS_API cis_status_t cis_loss_fwd_bwd_host(
     size_t workspace_bytes, void *stream);
 
 /*
- * Bytes of device workspace cis_lmhead_fused needs.  Host only.
+ * Bytes of device workspace cis_lmhead_fused needs with its default
+ * vocabulary chunk (dz and dz^T of one chunk within about 1 GiB).  Host only.
  * CIS_ERR_INVALID_ARG if bytes is NULL, T < 0, V <= 0 or H <= 0.
  */
 CIS_API cis_status_t cis_lmhead_workspace_size(int64_t T, int64_t V, int64_t H, size_t *bytes);
+
+/*
+ * Bytes of device workspace for vocabulary chunks of `chunk` columns (a
+ * positive multiple of 256; wider than V rounded up to 256 counts as that).
+ * The workspace grows by 4 * ceil(T / 128) * 128 bytes per chunk column.
+ * Host only.  CIS_ERR_INVALID_ARG for a NULL bytes, T < 0, V <= 0, H <= 0 or
+ * a chunk that is not a positive multiple of 256.
+ */
+CIS_API cis_status_t cis_lmhead_workspace_size_chunk(int64_t T, int64_t V, int64_t H,
+                                                     int64_t chunk, size_t *bytes);
 
 /*
  * The token pass fused with the LM head: logits z = hidden W^T are computed
@@ -248,6 +259,9 @@ CIS_API cis_status_t cis_lmhead_workspace_size(int64_t T, int64_t V, int64_t H, 
  * loss and the gradients are those of cis_loss_fwd_bwd (Eq. 1, Algorithm 1,
  * Table 8), taken through the LM head:
  *   dhidden = dz W,   dweight = dz^T hidden,   dz = c (softmax - onehot).
+ * The forward sweep keeps per-token softmax statistics only; the gradient
+ * sweep recomputes z one vocabulary chunk at a time and holds that chunk's dz
+ * (bf16, twice: [T, chunk] and [chunk, T]) in the workspace.
  *   hidden      device bf16 [T, H], contiguous rows, 16-byte aligned.
  *   weight      device bf16 [V, H], contiguous rows, 16-byte aligned.
  *   H           hidden size; a multiple of 256 (else CIS_ERR_UNSUPPORTED).
@@ -257,11 +271,14 @@ CIS_API cis_status_t cis_lmhead_workspace_size(int64_t T, int64_t V, int64_t H, 
  *   dweight     device [V, H] of grad_dtype, written (rows of tokens that are
  *               masked contribute nothing).
  *   lp_out, w_out, trunc_out, stats_out, loss_out: as for cis_loss_fwd_bwd.
- *   workspace   device, >= cis_lmhead_workspace_size(T, V, H) bytes,
- *               1024-byte aligned; its first int32 is the device status word.
+ *   workspace   device, 1024-byte aligned; its first int32 is the device
+ *               status word.  workspace_bytes picks the chunk: the widest
+ *               multiple of 256 columns whose cis_lmhead_workspace_size_chunk
+ *               fits; CIS_ERR_INVALID_ARG if not even 256 columns fit.
  * dz enters the two gradient products in bf16 (the tensor-core operand type);
- * the products accumulate in fp32.  Errors: as for cis_loss_fwd_bwd, plus
- * CIS_ERR_UNSUPPORTED if the tensor-map encoder is unavailable.
+ * the products accumulate in fp32 (dhidden across chunks too).  Errors: as
+ * for cis_loss_fwd_bwd, plus CIS_ERR_UNSUPPORTED if the tensor-map encoder is
+ * unavailable.
  */
 CIS_API cis_status_t cis_lmhead_fused(const void *hidden, const void *weight, int64_t T,
                                       int64_t H, int64_t V, const int32_t *ids,

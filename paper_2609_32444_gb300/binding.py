@@ -87,6 +87,9 @@ def lib():
     L.cis_loss_fwd_bwd.restype = ctypes.c_int
     L.cis_lmhead_workspace_size.argtypes = [i64, i64, i64, ctypes.POINTER(ctypes.c_size_t)]
     L.cis_lmhead_workspace_size.restype = ctypes.c_int
+    L.cis_lmhead_workspace_size_chunk.argtypes = [i64, i64, i64, i64,
+                                                  ctypes.POINTER(ctypes.c_size_t)]
+    L.cis_lmhead_workspace_size_chunk.restype = ctypes.c_int
     L.cis_lmhead_fused.argtypes = [P, P, i64, i64, i64, P, P, P, P, P, P, i64,
                                    ctypes.POINTER(cis_params_t), P, P, i32, P, P, P, P, P, P,
                                    ctypes.c_size_t, P]
@@ -295,12 +298,21 @@ def cis_lmhead_workspace_size(T: int, V: int, H: int) -> int:
     return n.value
 
 
+def cis_lmhead_workspace_size_chunk(T: int, V: int, H: int, chunk: int) -> int:
+    n = ctypes.c_size_t()
+    _check(lib().cis_lmhead_workspace_size_chunk(T, V, H, chunk, ctypes.byref(n)),
+           "cis_lmhead_workspace_size_chunk")
+    return n.value
+
+
 def cis_lmhead_fused(hidden: torch.Tensor, weight: torch.Tensor, ids: torch.Tensor,
                      lp_infer: torch.Tensor, adv: torch.Tensor, params: cis_params_t,
                      lp_old=None, mask=None, cu_seqlens=None, grad_dtype=torch.float32,
-                     workspace=None):
-    """Token pass through the LM head (logits never stored).  Returns a dict with
-    dhidden, dweight, lp, w, trunc, loss, stats and the workspace."""
+                     workspace=None, chunk=None):
+    """Token pass through the LM head (logits never stored).  `chunk` (a
+    multiple of 256) sizes the workspace for vocabulary chunks of that many
+    columns; by default the library's choice.  Returns a dict with dhidden,
+    dweight, lp, w, trunc, loss, stats and the workspace."""
     _need_cuda(hidden, weight, ids, lp_infer, adv, lp_old, mask, cu_seqlens)
     if hidden.dtype != torch.bfloat16 or weight.dtype != torch.bfloat16:
         raise TypeError("hidden and weight must be bfloat16")
@@ -323,11 +335,14 @@ def cis_lmhead_fused(hidden: torch.Tensor, weight: torch.Tensor, ids: torch.Tens
     tr = torch.empty(T, dtype=torch.uint8, device=dev)
     stats = torch.empty(ctypes.sizeof(cis_stats_t), dtype=torch.uint8, device=dev)
     loss = torch.empty(1, dtype=torch.float64, device=dev)
-    nws = cis_lmhead_workspace_size(T, V, H) + 1024
-    if workspace is None or workspace.numel() < nws:
-        workspace = torch.empty(nws, dtype=torch.uint8, device=dev)
-    off = (-workspace.data_ptr()) % 1024  # 1024-byte aligned start
-    ws = workspace[off:]
+    if workspace is None:  # else the caller's, as given (the library checks its size)
+        need = (cis_lmhead_workspace_size(T, V, H) if chunk is None
+                else cis_lmhead_workspace_size_chunk(T, V, H, chunk))
+        workspace = torch.empty(need + 1024, dtype=torch.uint8, device=dev)
+        off = (-workspace.data_ptr()) % 1024  # 1024-byte aligned start
+        ws = workspace[off:off + need]
+    else:
+        ws = workspace
     rc = lib().cis_lmhead_fused(
         _ptr(hidden), _ptr(weight), T, H, V, _ptr(ids), _ptr(lp_infer), _ptr(lp_old),
         _ptr(adv), _ptr(mask), _ptr(cu_seqlens), B, ctypes.byref(params), _ptr(dh), _ptr(dw),

@@ -2,50 +2,58 @@
 //
 // Logits z = H W^T (H: [T, Hd] hidden states, W: [V, Hd] unembedding, bf16)
 // are computed tile by tile on the tensor cores (tcgen05.mma, fp32 in TMEM)
-// and never written to global memory.  Three passes:
+// and never written to global memory.  One persistent GEMM kernel, its tile
+// epilogue chosen at compile time, serves every pass:
 //
-//   FWD  z tiles -> for every token, (max, sum of e^{z - max}) over the tile's
-//        entries j != y, and z_y; one pair per (vocab tile, token).
+//   FWD  z tiles [128 tokens x 256 vocab] -> per token, (max, sum e^{z - max})
+//        over the tile's entries j != y, and z_y.
 //   TOK  per token: combine the pairs, then log p, the weight (Algorithm 1 /
 //        Table 8) and the token loss (Eq. 1) with the same device code as the
 //        logits entry points; gives lse_t and c_t.
-//   DH   per (token tile, 256-column block of Hd): recompute each z tile,
-//        form dz = c (softmax - onehot) in bf16 straight into shared memory in
-//        the MMA operand layout, and accumulate dH += dz W in TMEM.
-//   DW   per (vocab tile, 256-column block of Hd): recompute the transposed
-//        z tile W_j H_i^T, form dz^T the same way, accumulate dW += dz^T H.
+//   then for each vocabulary chunk [v0, v0 + w):
+//   DZ   recompute the chunk's z tiles, form dz = c (softmax - onehot) in bf16
+//        and write it twice, as dz [T, w] and as dz^T [w, T];
+//   DH   dH (+)= dz W[v0 : v0 + w]   (K = w, fp32 accumulator);
+//   DW   dW[v0 : v0 + w] = dz^T H    (K = T).
 //
-// Every operand is K-major: dH and dW take W^T and H^T, which the call first
-// writes into its workspace.  Warp roles per CTA: warp 0 issues TMA loads into
-// a 4-stage ring, warp 1 issues tcgen05.mma (one thread) and owns TMEM, warps
-// 2..5 are the epilogue (one TMEM lane = one tile row per thread).  All waits
-// are bounded; a wait that runs out sets CIS_ERR_DEVICE_TIMEOUT and the CTA
-// carries on to its end so that TMEM is always released.
+// dz exists one chunk at a time (the chunk width follows the workspace the
+// caller gives); z never exists outside TMEM.  Every MMA operand is K-major:
+// DH reads W^T and DW reads H^T, which the call writes into its workspace.
+//
+// The GEMM kernel: 128 x 256 tiles, K blocks of 64 (one 128-byte swizzled row
+// of bf16), a 4-stage ring of 48 KB (A 16 KB + B 32 KB), two 256-column fp32
+// accumulators in TMEM so that the epilogue of one tile overlaps the main loop
+// of the next; persistent CTAs take tiles i, i + grid, i + 2 grid, ...  Warp
+// roles: warp 0 issues TMA loads, warp 1 issues tcgen05.mma (one thread) and
+// owns TMEM, warps 2..5 are the epilogue (one TMEM lane = one tile row per
+// thread).  All waits are bounded: a wait that runs out sets
+// CIS_ERR_DEVICE_TIMEOUT, and the CTA drains its own loads and MMAs and runs
+// to its end, so that TMEM is always released.
 #include <cuda.h>
 #include <cudaTypedefs.h>
-#include <stdlib.h>
 #include <mutex>
-
-#include <cooperative_groups.h>
 
 #include "cis_kernels.h"
 #include "cis_tc.cuh"
 
-namespace cg = cooperative_groups;
-
 namespace cis {
 namespace lm {
 
-constexpr int kBM = 128;     // tile rows (M)
-constexpr int kBN = 128;     // tile columns of z (N)
-constexpr int kBK = 64;      // K block: one 128-byte swizzled row of bf16
-constexpr int kN2 = 256;     // Hd columns of dH / dW per CTA
+constexpr int kBM = 128;                // tile rows (M)
+constexpr int kBN = 256;                // tile columns (N)
+constexpr int kBK = 64;                 // K block: one 128-byte swizzled row of bf16
 constexpr int kStages = 4;
-constexpr int kStageBytes = 32768;
+constexpr int kStageA = kBM * kBK * 2;  // 16 KB
+constexpr int kStageB = kBN * kBK * 2;  // 32 KB
+constexpr int kStageBytes = kStageA + kStageB;
 constexpr int kThreads = 192;
-constexpr int kFwdGroup = 16;  // vocab tiles per FWD CTA
+constexpr uint32_t kTmemCols = 2 * kBN;  // two accumulators
+constexpr size_t kSmemBytes = (size_t)kStages * kStageBytes + 1024;
+// dz + dz^T of one chunk take 4 Tp bytes per vocabulary column; the default
+// chunk keeps them within this many bytes.
+constexpr int64_t kDefaultChunkBytes = 1ll << 30;
 
-enum Mode { kFwd = 0, kDh = 1, kDw = 2 };
+enum Epi { kStats = 0, kDz = 1, kStore = 2, kAccum = 3 };
 
 // OR of `pred` over the 128 epilogue threads (named barrier 1), so that the
 // four epilogue warps leave their loop together.
@@ -61,84 +69,85 @@ __device__ __forceinline__ int __syncthreads_or_epi(int pred)
     return r;
 }
 
-struct Params {
-    int T, V, Hd;
-    int nTt, nVt, nK;
+__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi)
+{
+    __nv_bfloat162 h = __floats2bfloat162_rn(lo, hi);
+    return *reinterpret_cast<uint32_t *>(&h);
+}
+
+// One launch of the GEMM kernel: C[M, N] = A[M, K] B[N, K]^T over tiles
+// (m, n) of 128 x 256, with TMA coordinates offset by (a_k0, a_row0) and
+// (b_k0, b_row0).
+struct GemmArgs {
+    int nMt, nNt, nK;
+    int raster_n;  // 1: tile i -> (m = i % nMt, n = i / nMt); 0: (m = i / nNt, n = i % nNt)
+    int a_row0, a_k0, b_row0, b_k0;
+    // kStats, kDz: rows are tokens, columns vocabulary entries col0 + n 256 + c
+    int T, V, col0;
     const int32_t *ids;
-    const uint8_t *mask;
-    const float *lse;    // DH / DW: per token
-    const float *cvec;   // DH / DW: per token, 0 where the token has no gradient
-    float2 *part;        // FWD: [nVt, T] (max, sum) over j != y
-    float *zy;           // FWD: z at the sampled token
-    void *out;           // DH: dH [T, ld_out]; DW: dW [V, ld_out]
-    int out_bf16;
+    const float *lse, *cvec;
+    float2 *part;     // kStats: [nNt, T] (max, sum) over j != y
+    float *zy;        // kStats: z at the sampled token
+    uint16_t *dz;     // kDz: bf16 [Tp, ld_dz], column = chunk-local vocabulary index
+    uint16_t *dzt;    // kDz: bf16 [chunk, ld_dzt], column = token
+    int64_t ld_dz, ld_dzt;
+    // kStore, kAccum: rows m 128 + r < rows_valid of out [., ld_out]
+    void *out;
+    int out_bf16, rows_valid;
     int64_t ld_out;
     int32_t *status;
 };
 
 struct Barriers {
     uint64_t full[kStages], empty[kStages];
-    uint64_t zfull[2], zempty[2];
-    uint64_t dzfull, dzempty, accfull;
+    uint64_t accfull[2], accempty[2];
+    uint64_t done;
 };
 
-// A wait that runs out marks the CTA (and, through the status word, every
-// later CTA) as aborted: the roles then stop waiting and run to the end, so a
-// broken pipeline costs one bounded wait per role instead of one per tile.
+// A wait that runs out marks the CTA (shared flag) and the grid (status word)
+// as aborted: the roles then stop waiting and run to the end, so a broken
+// pipeline costs one bounded wait per role instead of one per tile.  on()
+// reads the shared flag only; the status word (global memory, one L2 round
+// trip) is consulted inside waits that are already taking long.
 struct Abort {
     volatile int *local;
-    const volatile int32_t *status;
-    __device__ __forceinline__ bool on() const
-    {
-        return *local != 0 || (*status & kStatusTimeout) != 0;
-    }
-    __device__ __forceinline__ void wait(uint64_t *bar, uint32_t parity, int32_t *st) const
+    int32_t *status;
+    __device__ __forceinline__ bool on() const { return *local != 0; }
+    __device__ __forceinline__ void wait(uint64_t *bar, uint32_t parity) const
     {
         if (*local)
             return;
-        if (!tc::bar_wait(bar, parity)) {
+        if (!tc::bar_wait(bar, parity, status)) {
             *local = 1;
-            set_status(st, kStatusTimeout);
+            set_status(status, kStatusTimeout);
         }
     }
 };
 
-template <int MODE>
+__device__ __forceinline__ void tile_mn(const GemmArgs &g, int i, int &m, int &n)
+{
+    if (g.raster_n) {
+        n = i / g.nMt;
+        m = i - n * g.nMt;
+    } else {
+        m = i / g.nNt;
+        n = i - m * g.nNt;
+    }
+}
+
+template <int EPI>
 __global__ void __launch_bounds__(kThreads, 1)
-    cis_lmhead_kernel(const __grid_constant__ CUtensorMap tmA,
-                      const __grid_constant__ CUtensorMap tmB,
-                      const __grid_constant__ CUtensorMap tmB2, const Params p)
+    cis_lmhead_gemm_kernel(const __grid_constant__ CUtensorMap tmA,
+                           const __grid_constant__ CUtensorMap tmB, const GemmArgs g)
 {
     extern __shared__ __align__(1024) uint8_t dsm[];
-    uint8_t *base = dsm + ((1024 - (tc::smem_addr(dsm) & 1023)) & 1023);
-    uint8_t *ring = base;                          // kStages x 32 KB
-    uint8_t *dzbuf = base + kStages * kStageBytes; // 32 KB: dz tile, 2 K blocks
+    uint8_t *ring = dsm + ((1024 - (tc::smem_addr(dsm) & 1023)) & 1023);
     __shared__ __align__(8) Barriers bars;
     __shared__ uint32_t tmem_base;
     __shared__ int aborted;
-    __shared__ float col_lse[2][kBN], col_c[2][kBN];
-    __shared__ int col_y[2][kBN];
 
-    constexpr uint32_t kTmemCols = MODE == kFwd ? 256 : 512;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-
-    // tile assignment
-    int a_tile, nB, b_first, hblk = 0;
-    if (MODE == kFwd) {
-        a_tile = blockIdx.x % p.nTt;
-        b_first = (blockIdx.x / p.nTt) * kFwdGroup;
-        nB = min(kFwdGroup, p.nVt - b_first);
-    } else if (MODE == kDh) {
-        a_tile = blockIdx.x % p.nTt;
-        hblk = blockIdx.x / p.nTt;
-        b_first = 0;
-        nB = p.nVt;
-    } else {
-        a_tile = blockIdx.x % p.nVt;
-        hblk = blockIdx.x / p.nVt;
-        b_first = 0;
-        nB = p.nTt;
-    }
+    const int nTiles = g.nMt * g.nNt;
 
     if (threadIdx.x == 0) {
         aborted = 0;
@@ -147,12 +156,10 @@ __global__ void __launch_bounds__(kThreads, 1)
             tc::bar_init(&bars.empty[s], 1);
         }
         for (int b = 0; b < 2; ++b) {
-            tc::bar_init(&bars.zfull[b], 1);
-            tc::bar_init(&bars.zempty[b], 128);
+            tc::bar_init(&bars.accfull[b], 1);
+            tc::bar_init(&bars.accempty[b], 128);
         }
-        tc::bar_init(&bars.dzfull, 128);
-        tc::bar_init(&bars.dzempty, 1);
-        tc::bar_init(&bars.accfull, 1);
+        tc::bar_init(&bars.done, 1);
         tc::bar_init_fence();
     }
     if (warp == 1)
@@ -161,269 +168,209 @@ __global__ void __launch_bounds__(kThreads, 1)
     __syncthreads();
     tc::fence_after_sync();
     const uint32_t tmem = tmem_base;
-    const uint32_t tmem_acc = tmem + 256;  // DH / DW accumulator, 256 columns
-    const Abort ab{&aborted, p.status};
+    const Abort ab{&aborted, g.status};
 
     if (warp == 0) {
         // ---------------------------------------------------------- producer
         if (lane == 0) {
             int stage = 0;
-            uint32_t phase = 0;
-            auto next = [&]() {
-                ab.wait(&bars.empty[stage], phase ^ 1, p.status);
-                tc::bar_expect_tx(&bars.full[stage], kStageBytes);
-            };
-            auto advance = [&]() {
-                if (++stage == kStages) {
-                    stage = 0;
-                    phase ^= 1;
-                }
-            };
-            auto load_b2 = [&](int jb) {
-                for (int kb = 0; kb < 2; ++kb) {
-                    next();
-                    tc::tma_load_2d(ring + stage * kStageBytes, &tmB2,
-                                    (b_first + jb) * kBN + kb * kBK, hblk * kN2,
-                                    &bars.full[stage]);
-                    advance();
-                }
-            };
-            for (int jb = 0; jb < nB && !ab.on(); ++jb) {
-                for (int k = 0; k < p.nK; ++k) {
-                    next();
+            uint32_t phase = 0, used = 0, last = 0;  // per stage: loaded, parity of its last load
+            for (int t = blockIdx.x; t < nTiles && !ab.on(); t += gridDim.x) {
+                int m, n;
+                tile_mn(g, t, m, n);
+                for (int kb = 0; kb < g.nK; ++kb) {
+                    ab.wait(&bars.empty[stage], phase ^ 1);
+                    if (ab.on())
+                        break;
+                    tc::bar_expect_tx(&bars.full[stage], kStageBytes);
+                    used |= 1u << stage;
+                    last = (last & ~(1u << stage)) | (phase << stage);
                     uint8_t *st = ring + stage * kStageBytes;
-                    tc::tma_load_2d(st, &tmA, k * kBK, a_tile * kBM, &bars.full[stage]);
-                    tc::tma_load_2d(st + kStageBytes / 2, &tmB, k * kBK, (b_first + jb) * kBN,
+                    tc::tma_load_2d(st, &tmA, g.a_k0 + kb * kBK, g.a_row0 + m * kBM,
                                     &bars.full[stage]);
-                    advance();
+                    tc::tma_load_2d(st + kStageA, &tmB, g.b_k0 + kb * kBK, g.b_row0 + n * kBN,
+                                    &bars.full[stage]);
+                    if (++stage == kStages) {
+                        stage = 0;
+                        phase ^= 1;
+                    }
                 }
-                if (MODE != kFwd && jb >= 1)
-                    load_b2(jb - 1);
             }
-            if (MODE != kFwd && nB >= 1 && !ab.on())
-                load_b2(nB - 1);
+            // no load may still be landing when the CTA leaves
+            for (int s = 0; s < kStages; ++s)
+                if (used & (1u << s))
+                    tc::bar_wait(&bars.full[s], (last >> s) & 1);
         }
     } else if (warp == 1) {
         // ---------------------------------------------------------- MMA issue
         if (lane == 0) {
-            constexpr uint32_t kIdZ = tc::idesc_bf16(kBM, kBN);
-            constexpr uint32_t kId2 = tc::idesc_bf16(kBM, kN2);
+            constexpr uint32_t kId = tc::idesc_bf16(kBM, kBN);
             int stage = 0;
             uint32_t phase = 0;
-            auto advance = [&]() {
-                if (++stage == kStages) {
-                    stage = 0;
-                    phase ^= 1;
-                }
-            };
-            for (int jb = 0; jb <= nB && !ab.on(); ++jb) {
-                if (jb < nB) {
-                    const int zb = jb & 1;
-                    ab.wait(&bars.zempty[zb], ((jb >> 1) & 1) ^ 1, p.status);
+            int i = 0;
+            for (int t = blockIdx.x; t < nTiles && !ab.on(); t += gridDim.x, ++i) {
+                const int acc = i & 1;
+                ab.wait(&bars.accempty[acc], ((i >> 1) & 1) ^ 1);
+                tc::fence_after_sync();
+                const uint32_t d = tmem + acc * kBN;
+                for (int kb = 0; kb < g.nK; ++kb) {
+                    ab.wait(&bars.full[stage], phase);
+                    if (ab.on())
+                        break;
                     tc::fence_after_sync();
-                    const uint32_t dz = tmem + zb * kBN;
-                    for (int k = 0; k < p.nK; ++k) {
-                        ab.wait(&bars.full[stage], phase, p.status);
-                        tc::fence_after_sync();
-                        const uint32_t sa = tc::smem_addr(ring + stage * kStageBytes);
-                        const uint32_t sb = sa + kStageBytes / 2;
+                    const uint32_t sa = tc::smem_addr(ring + stage * kStageBytes);
+                    const uint32_t sb = sa + kStageA;
 #pragma unroll
-                        for (int kk = 0; kk < kBK / 16; ++kk)
-                            tc::mma_bf16(dz, tc::desc_sw128(sa + kk * 32),
-                                         tc::desc_sw128(sb + kk * 32), kIdZ, (k | kk) != 0);
-                        tc::mma_commit(&bars.empty[stage]);
-                        advance();
+                    for (int kk = 0; kk < kBK / 16; ++kk)
+                        tc::mma_bf16(d, tc::desc_sw128(sa + kk * 32), tc::desc_sw128(sb + kk * 32),
+                                     kId, (kb | kk) != 0);
+                    tc::mma_commit(&bars.empty[stage]);
+                    if (++stage == kStages) {
+                        stage = 0;
+                        phase ^= 1;
                     }
-                    tc::mma_commit(&bars.zfull[zb]);
                 }
-                if (MODE != kFwd && jb >= 1) {
-                    // dH (or dW) += dz (tile jb-1, in shared memory) x B2 chunk
-                    ab.wait(&bars.dzfull, (jb - 1) & 1, p.status);
-                    tc::fence_after_sync();
-                    const uint32_t sdz = tc::smem_addr(dzbuf);
-                    for (int kb = 0; kb < 2; ++kb) {
-                        ab.wait(&bars.full[stage], phase, p.status);
-                        tc::fence_after_sync();
-                        const uint32_t sb2 = tc::smem_addr(ring + stage * kStageBytes);
-#pragma unroll
-                        for (int kk = 0; kk < kBK / 16; ++kk)
-                            tc::mma_bf16(tmem_acc, tc::desc_sw128(sdz + kb * 16384 + kk * 32),
-                                         tc::desc_sw128(sb2 + kk * 32), kId2,
-                                         (jb - 1) > 0 || kb > 0 || kk > 0);
-                        tc::mma_commit(&bars.empty[stage]);
-                        advance();
-                    }
-                    tc::mma_commit(&bars.dzempty);
-                }
+                tc::mma_commit(&bars.accfull[acc]);
             }
-            if (MODE != kFwd)
-                tc::mma_commit(&bars.accfull);
+            // every MMA of this CTA is done before TMEM is released
+            tc::mma_commit(&bars.done);
+            tc::bar_wait(&bars.done, 0);
         }
     } else {
         // ---------------------------------------------------------- epilogue
-        const int lg = warp & 3;           // TMEM lane group of this warp
-        const int r = lg * 32 + lane;      // tile row of this thread
+        const int lg = warp & 3;  // TMEM lane quadrant of this warp
+        const int r = lg * 32 + lane;
         const uint32_t lane_off = (uint32_t)(lg * 32) << 16;
-        const int e = threadIdx.x - 64;    // 0..127
-        const int row = (MODE == kDw ? a_tile * kBM : a_tile * kBM) + r;
-
-        // per-row scalars
-        int y_r = -1;
-        float lse_r = 0.0f, c_r = 0.0f;
-        if (MODE != kDw && row < p.T) {
-            y_r = p.ids[row];
-            if (MODE == kDh) {
-                lse_r = p.lse[row];
-                c_r = p.cvec[row];
-            }
-        }
-        for (int jb = 0; jb < nB; ++jb) {
-            const int zb = jb & 1;
-            const int col0 = (b_first + jb) * kBN;
-            // every epilogue warp takes the same path (named barrier below)
-            const int stop = ab.on();
-            if (__syncthreads_or_epi(stop))
+        int i = 0;
+        for (int t = blockIdx.x; t < nTiles; t += gridDim.x, ++i) {
+            if (__syncthreads_or_epi(ab.on()))
                 break;
-            if (MODE == kDw) {
-                // scalars of this token tile's 128 columns
-                const int t = col0 + e;
-                const bool ok = t < p.T;
-                col_lse[zb][e] = ok ? p.lse[t] : 0.0f;
-                col_c[zb][e] = ok ? p.cvec[t] : 0.0f;
-                col_y[zb][e] = ok ? p.ids[t] : -1;
-                asm volatile("bar.sync 1, 128;" ::: "memory");
-            }
-            ab.wait(&bars.zfull[zb], (jb >> 1) & 1, p.status);
+            int m, n;
+            tile_mn(g, t, m, n);
+            const int acc = i & 1;
+            ab.wait(&bars.accfull[acc], (i >> 1) & 1);
             tc::fence_after_sync();
-            const uint32_t zaddr = tmem + lane_off + zb * kBN;
-            if (MODE == kFwd) {
-                float m = -INFINITY, s = 0.0f, zyv = 0.0f;
+            const uint32_t taddr = tmem + lane_off + acc * kBN;
+            if (EPI == kStats) {
+                const int row = m * kBM + r;  // token
+                const int y_r = row < g.T ? g.ids[row] : -1;
+                float mx = -INFINITY, s = 0.0f, zyv = 0.0f;
                 bool got_y = false;
                 for (int c0 = 0; c0 < kBN; c0 += 32) {
                     float v[32];
-                    tc::tmem_ld32(zaddr + c0, v);
-                    const int cbase = col0 + c0;
-                    if (y_r >= cbase && y_r < cbase + 32) {
+                    tc::tmem_ld32(taddr + c0, v);
+                    const int base = g.col0 + n * kBN + c0;
+                    if (y_r >= base && y_r < base + 32) {
 #pragma unroll
-                        for (int i = 0; i < 32; ++i)
-                            if (cbase + i == y_r)
-                                zyv = v[i];
+                        for (int q = 0; q < 32; ++q)
+                            if (base + q == y_r)
+                                zyv = v[q];
                         got_y = true;
                     }
                     float cm = -INFINITY;
 #pragma unroll
-                    for (int i = 0; i < 32; ++i) {
-                        const int col = cbase + i;
-                        v[i] = (col == y_r || col >= p.V) ? -INFINITY : v[i];
-                        cm = fmaxf(cm, v[i]);
+                    for (int q = 0; q < 32; ++q) {
+                        const int col = base + q;
+                        v[q] = (col == y_r || col >= g.V) ? -INFINITY : v[q];
+                        cm = fmaxf(cm, v[q]);
                     }
-                    if (cm > m) {
-                        s = m == -INFINITY ? 0.0f : s * ex2_ftz((m - cm) * kLog2e);
-                        m = cm;
+                    if (cm > mx) {
+                        s = mx == -INFINITY ? 0.0f : s * ex2_ftz((mx - cm) * kLog2e);
+                        mx = cm;
                     }
-                    if (m != -INFINITY) {
-                        float acc = 0.0f;
+                    if (mx != -INFINITY) {
+                        float a = 0.0f;
 #pragma unroll
-                        for (int i = 0; i < 32; ++i)
-                            acc += ex2_ftz((v[i] - m) * kLog2e);
-                        s += acc;
+                        for (int q = 0; q < 32; ++q)
+                            a += ex2_ftz((v[q] - mx) * kLog2e);
+                        s += a;
                     }
                 }
-                tc::fence_before_sync();
-                tc::bar_arrive(&bars.zempty[zb]);
-                if (row < p.T) {
-                    p.part[(int64_t)(b_first + jb) * p.T + row] = make_float2(m, s);
+                if (row < g.T) {
+                    g.part[(int64_t)n * g.T + row] = make_float2(mx, s);
                     if (got_y)
-                        p.zy[row] = zyv;
+                        g.zy[row] = zyv;
                 }
-            } else {
-                // dz tile (bf16) into shared memory, operand layout; wait until the
-                // previous tile's dz has been consumed by its MMA
-                ab.wait(&bars.dzempty, (jb & 1) ^ 1, p.status);
+            } else if (EPI == kDz) {
+                const int row = m * kBM + r;  // token; rows up to Tp are allocated
+                const bool live = row < g.T;
+                // tokens with c = 0 (masked, clipped, past T) give 0 without
+                // touching the exponential (their lse is a placeholder)
+                const float c_r = live ? g.cvec[row] : 0.0f;
+                const float lse_r = live ? g.lse[row] : 0.0f;
+                const int y_r = live ? g.ids[row] : -1;
+                const int cl0 = n * kBN;  // chunk-local column of the tile
                 for (int c0 = 0; c0 < kBN; c0 += 32) {
                     float v[32];
-                    tc::tmem_ld32(zaddr + c0, v);
+                    tc::tmem_ld32(taddr + c0, v);
+                    const int gc0 = g.col0 + cl0 + c0;  // vocabulary index of v[0]
+                    uint32_t w[16];
 #pragma unroll
-                    for (int i = 0; i < 32; ++i) {
-                        const int col = c0 + i;  // column within the tile
-                        float d;
-                        // tokens with c = 0 (masked, clipped, past T) give 0 without
-                        // touching the exponential (their lse is a placeholder)
-                        if (MODE == kDh) {
-                            const int gcol = col0 + col;  // vocab index
-                            d = (gcol < p.V && c_r != 0.0f)
-                                    ? c_r * ex2_ftz((v[i] - lse_r) * kLog2e) -
-                                          (gcol == y_r ? c_r : 0.0f)
-                                    : 0.0f;
-                        } else {
-                            const float lt = col_lse[zb][col], ct = col_c[zb][col];
-                            d = (row < p.V && ct != 0.0f)
-                                    ? ct * ex2_ftz((v[i] - lt) * kLog2e) -
-                                          (col_y[zb][col] == row ? ct : 0.0f)
-                                    : 0.0f;
+                    for (int q = 0; q < 32; q += 2) {
+                        float d[2];
+#pragma unroll
+                        for (int h = 0; h < 2; ++h) {
+                            const int gc = gc0 + q + h;
+                            d[h] = (gc < g.V && c_r != 0.0f)
+                                       ? c_r * ex2_ftz((v[q + h] - lse_r) * kLog2e) -
+                                             (gc == y_r ? c_r : 0.0f)
+                                       : 0.0f;
                         }
-                        v[i] = d;
+                        w[q >> 1] = pack_bf16x2(d[0], d[1]);
                     }
-                    // 32 values = 4 chunks of 8 bf16 in K block c0 / 64
-                    uint8_t *blk = dzbuf + (c0 >> 6) * 16384;
+                    uint4 *drow = reinterpret_cast<uint4 *>(g.dz + (int64_t)row * g.ld_dz + cl0 + c0);
 #pragma unroll
-                    for (int q = 0; q < 4; ++q) {
-                        uint4 w;
-                        __nv_bfloat162 h;
-                        h = __floats2bfloat162_rn(v[8 * q + 0], v[8 * q + 1]);
-                        w.x = *reinterpret_cast<uint32_t *>(&h);
-                        h = __floats2bfloat162_rn(v[8 * q + 2], v[8 * q + 3]);
-                        w.y = *reinterpret_cast<uint32_t *>(&h);
-                        h = __floats2bfloat162_rn(v[8 * q + 4], v[8 * q + 5]);
-                        w.z = *reinterpret_cast<uint32_t *>(&h);
-                        h = __floats2bfloat162_rn(v[8 * q + 6], v[8 * q + 7]);
-                        w.w = *reinterpret_cast<uint32_t *>(&h);
-                        const int chunk = ((c0 & 63) >> 3) + q;
-                        *reinterpret_cast<uint4 *>(blk + tc::sw128_offset(r, chunk)) = w;
-                    }
+                    for (int q = 0; q < 4; ++q)
+                        drow[q] = make_uint4(w[4 * q], w[4 * q + 1], w[4 * q + 2], w[4 * q + 3]);
+                    // dz^T: the warp's 32 consecutive tokens make one 64-byte run per column
+                    uint16_t *dcol = g.dzt + (int64_t)(cl0 + c0) * g.ld_dzt + row;
+#pragma unroll
+                    for (int q = 0; q < 32; ++q)
+                        dcol[(int64_t)q * g.ld_dzt] =
+                            (uint16_t)((q & 1) ? (w[q >> 1] >> 16) : (w[q >> 1] & 0xFFFFu));
                 }
-                tc::fence_before_sync();
-                tc::bar_arrive(&bars.zempty[zb]);
-                tc::fence_proxy_async_smem();
-                tc::bar_arrive(&bars.dzfull);
-            }
-        }
-        if (MODE != kFwd) {
-            // the accumulated dH / dW block: 128 rows x 256 columns
-            ab.wait(&bars.accfull, 0, p.status);
-            tc::fence_after_sync();
-            const int nrows = MODE == kDh ? p.T : p.V;
-            for (int c0 = 0; c0 < kN2; c0 += 32) {
-                float v[32];
-                tc::tmem_ld32(tmem_acc + lane_off + c0, v);
-                if (row < nrows) {
-                    const int64_t o = (int64_t)row * p.ld_out + (int64_t)hblk * kN2 + c0;
-                    if (p.out_bf16) {
-                        __nv_bfloat16 *dst = reinterpret_cast<__nv_bfloat16 *>(p.out) + o;
+            } else {
+                const int lr = m * kBM + r;  // row of the output block
+                const bool live = lr < g.rows_valid;
+                const int64_t o = (int64_t)lr * g.ld_out + (int64_t)n * kBN;
+                for (int c0 = 0; c0 < kBN; c0 += 32) {
+                    float v[32];
+                    tc::tmem_ld32(taddr + c0, v);
+                    if (!live)
+                        continue;
+                    if (g.out_bf16) {
+                        uint4 *dst = reinterpret_cast<uint4 *>(
+                            reinterpret_cast<uint16_t *>(g.out) + o + c0);
 #pragma unroll
-                        for (int q = 0; q < 4; ++q) {
-                            uint4 w;
-                            __nv_bfloat162 h;
-                            h = __floats2bfloat162_rn(v[8 * q + 0], v[8 * q + 1]);
-                            w.x = *reinterpret_cast<uint32_t *>(&h);
-                            h = __floats2bfloat162_rn(v[8 * q + 2], v[8 * q + 3]);
-                            w.y = *reinterpret_cast<uint32_t *>(&h);
-                            h = __floats2bfloat162_rn(v[8 * q + 4], v[8 * q + 5]);
-                            w.z = *reinterpret_cast<uint32_t *>(&h);
-                            h = __floats2bfloat162_rn(v[8 * q + 6], v[8 * q + 7]);
-                            w.w = *reinterpret_cast<uint32_t *>(&h);
-                            reinterpret_cast<uint4 *>(dst)[q] = w;
-                        }
+                        for (int q = 0; q < 4; ++q)
+                            dst[q] = make_uint4(pack_bf16x2(v[8 * q + 0], v[8 * q + 1]),
+                                                pack_bf16x2(v[8 * q + 2], v[8 * q + 3]),
+                                                pack_bf16x2(v[8 * q + 4], v[8 * q + 5]),
+                                                pack_bf16x2(v[8 * q + 6], v[8 * q + 7]));
                     } else {
-                        float4 *dst = reinterpret_cast<float4 *>(reinterpret_cast<float *>(p.out) + o);
+                        float4 *dst = reinterpret_cast<float4 *>(
+                            reinterpret_cast<float *>(g.out) + o + c0);
 #pragma unroll
-                        for (int q = 0; q < 8; ++q)
-                            dst[q] = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+                        for (int q = 0; q < 8; ++q) {
+                            float4 x = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2],
+                                                   v[4 * q + 3]);
+                            if (EPI == kAccum) {
+                                const float4 old = dst[q];
+                                x.x += old.x;
+                                x.y += old.y;
+                                x.z += old.z;
+                                x.w += old.w;
+                            }
+                            dst[q] = x;
+                        }
                     }
                 }
             }
+            tc::fence_before_sync();
+            tc::bar_arrive(&bars.accempty[acc]);
         }
     }
+    __syncwarp();
     tc::fence_before_sync();
     __syncthreads();
     if (warp == 1) {
@@ -432,393 +379,12 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
 }
 
-// ---------------------------------------------------------------------------
-// Gradient passes shared by a cluster: R = Hd / 256 CTAs, CTA r accumulating
-// block r (256 columns) of dH (or dW).  Step j of the sweep is vocabulary tile
-// j (dW: token tile j).  Its logit tile is computed once, by the CTA that owns
-// the step (j mod R), which forms the bf16 dz tile in its own shared memory
-// and bulk-copies it into the same mailbox slot (j mod 2) of every other CTA
-// of the cluster; each copy is counted on the receiver's mbarrier.  Every CTA
-// consumes every step: block r += dz_j x (W^T or H^T)[block r, tile j].  After
-// consuming step j a CTA's MMA commit is multicast to the slot-free mbarrier
-// of the owner of step j + 2, which reuses the slot.  A CTA computes the logit
-// tile of its k-th owned step t_k = r + kR spread over the R steps of the
-// period two before it (4 K blocks per step), so no commit waits on a whole
-// tile, and the tile is ready R + 1 steps before it is consumed.
-//
-// Phases.  Copies into slot s of a CTA arrive in step order, each only after
-// the CTA has consumed the previous step of that slot, so neither the mailbox
-// nor the per-slot slot-free barrier can run a phase ahead of its waiter.
-// Teardown.  Each copy is first recorded in the receiver (a remote max of the
-// step index), so after a cluster barrier that ends all copying a CTA knows
-// whether a copy into it may still be in flight and waits for it (bounded)
-// before the second cluster barrier; only then may a CTA leave.
-constexpr int kSlotBytes = 32768;
-
-struct CBarriers {
-    uint64_t full[kStages], empty[kStages];
-    uint64_t zfull[2], zempty[2];
-    uint64_t dzfull[2];     // the dz tile of the step in slot s has landed
-    uint64_t slot_free[2];  // every CTA has consumed the step that last used slot s
-    uint64_t accfull;
-};
-
-template <int MODE>
-__global__ void __launch_bounds__(kThreads, 1)
-    cis_lmhead_grad_kernel(const __grid_constant__ CUtensorMap tmA,
-                           const __grid_constant__ CUtensorMap tmB,
-                           const __grid_constant__ CUtensorMap tmB2, const Params p)
+// dst[i] = bf16(src[i]) (round to nearest even)
+__global__ void cis_lmhead_to_bf16_kernel(const float *src, uint16_t *dst, int64_t n)
 {
-    extern __shared__ __align__(1024) uint8_t dsm[];
-    uint8_t *base = dsm + ((1024 - (tc::smem_addr(dsm) & 1023)) & 1023);
-    uint8_t *ring = base;                            // kStages x 32 KB
-    uint8_t *slots = base + kStages * kStageBytes;   // 2 x 32 KB dz mailboxes
-    __shared__ __align__(8) CBarriers bars;
-    __shared__ uint32_t tmem_base;
-    __shared__ int aborted;
-    __shared__ int last_copied[2];  // latest step copied into slot s by its owner
-    __shared__ float col_lse[kBN], col_c[kBN];
-    __shared__ int col_y[kBN];
-
-    cg::cluster_group cluster = cg::this_cluster();
-    const int R = (int)cluster.num_blocks();
-    const int rank = (int)cluster.block_rank();
-    const int a_tile = blockIdx.x / R;
-    const int nB = MODE == kDh ? p.nVt : p.nTt;
-    const int Q = p.nK / R;  // K blocks of a logit tile issued per step
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-
-    if (threadIdx.x == 0) {
-        aborted = 0;
-        last_copied[0] = last_copied[1] = -1;
-        for (int s = 0; s < kStages; ++s) {
-            tc::bar_init(&bars.full[s], 1);
-            tc::bar_init(&bars.empty[s], 1);
-        }
-        for (int b = 0; b < 2; ++b) {
-            tc::bar_init(&bars.zfull[b], 1);
-            tc::bar_init(&bars.zempty[b], 128);
-            tc::bar_init(&bars.dzfull[b], 1);
-            tc::bar_init(&bars.slot_free[b], R);
-        }
-        tc::bar_init(&bars.accfull, 1);
-        tc::bar_init_fence();
-    }
-    if (warp == 1)
-        tc::tmem_alloc(&tmem_base, 512);
-    tc::fence_before_sync();
-    __syncthreads();
-    tc::fence_after_sync();
-    // every CTA of the cluster has initialised its barriers before any remote use
-    tc::cluster_arrive();
-    tc::cluster_wait();
-    const uint32_t tmem = tmem_base;
-    const uint32_t tmem_acc = tmem + 256;
-    const Abort ab{&aborted, p.status};
-    int consumed = 0;  // MMA thread: steps 0 .. consumed-1 are fully issued
-    int expected = -1; // MMA thread: latest step whose copy it announced
-
-    // The ring items in the order both the producer and the MMA issuer take
-    // them: fn_z(k, kb) for K block kb of owned tile t_k, fn_step(j) before
-    // the two B2 items fn_b2(j, 0), fn_b2(j, 1) of step j.
-    auto walk = [&](auto &&fn_z, auto &&fn_step, auto &&fn_b2) {
-        if (rank < nB)
-            for (int kb = 0; kb < p.nK; ++kb)
-                fn_z(0, kb);
-        if (rank + R < nB)
-            for (int kb = 0; kb < (R - rank) * Q; ++kb)
-                fn_z(1, kb);
-        for (int j = 0; j < nB && !ab.on(); ++j) {
-            int k, pi;
-            if (j < rank) {
-                k = 1;
-                pi = j - rank + R;
-            } else {
-                k = (j - rank) / R + 2;
-                pi = (j - rank) % R;
-            }
-            if (rank + k * R < nB)
-                for (int kb = pi * Q; kb < (pi + 1) * Q; ++kb)
-                    fn_z(k, kb);
-            fn_step(j);
-            fn_b2(j, 0);
-            fn_b2(j, 1);
-        }
-    };
-
-    if (warp == 0) {
-        if (lane == 0) {
-            int stage = 0;
-            uint32_t phase = 0;
-            uint32_t used = 0, last_phase = 0;  // per stage: loaded, parity of its last load
-            auto next = [&]() -> bool {
-                if (ab.on())
-                    return false;
-                ab.wait(&bars.empty[stage], phase ^ 1, p.status);
-                if (ab.on())
-                    return false;
-                tc::bar_expect_tx(&bars.full[stage], kStageBytes);
-                used |= 1u << stage;
-                last_phase = (last_phase & ~(1u << stage)) | (phase << stage);
-                return true;
-            };
-            auto adv = [&]() {
-                if (++stage == kStages) {
-                    stage = 0;
-                    phase ^= 1;
-                }
-            };
-            walk(
-                [&](int k, int kb) {
-                    if (!next())
-                        return;
-                    uint8_t *st = ring + stage * kStageBytes;
-                    tc::tma_load_2d(st, &tmA, kb * kBK, a_tile * kBM, &bars.full[stage]);
-                    tc::tma_load_2d(st + kStageBytes / 2, &tmB, kb * kBK, (rank + k * R) * kBN,
-                                    &bars.full[stage]);
-                    adv();
-                },
-                [&](int) {},
-                [&](int j, int kb2) {
-                    if (!next())
-                        return;
-                    tc::tma_load_2d(ring + stage * kStageBytes, &tmB2, j * kBN + kb2 * kBK,
-                                    rank * kN2, &bars.full[stage]);
-                    adv();
-                });
-            // no load may still be landing when the CTA leaves
-            for (int s = 0; s < kStages; ++s)
-                if (used & (1u << s))
-                    tc::bar_wait(&bars.full[s], (last_phase >> s) & 1);
-        }
-    } else if (warp == 1) {
-        if (lane == 0) {
-            constexpr uint32_t kIdZ = tc::idesc_bf16(kBM, kBN);
-            constexpr uint32_t kId2 = tc::idesc_bf16(kBM, kN2);
-            int stage = 0;
-            uint32_t phase = 0;
-            auto adv = [&]() {
-                if (++stage == kStages) {
-                    stage = 0;
-                    phase ^= 1;
-                }
-            };
-            walk(
-                [&](int k, int kb) {
-                    if (ab.on())
-                        return;
-                    const int zb = k & 1;
-                    if (kb == 0)  // the buffer's previous tile has been read
-                        ab.wait(&bars.zempty[zb], ((k >> 1) & 1) ^ 1, p.status);
-                    ab.wait(&bars.full[stage], phase, p.status);
-                    if (ab.on())
-                        return;
-                    tc::fence_after_sync();
-                    const uint32_t sa = tc::smem_addr(ring + stage * kStageBytes);
-                    const uint32_t sb = sa + kStageBytes / 2;
-#pragma unroll
-                    for (int kk = 0; kk < kBK / 16; ++kk)
-                        tc::mma_bf16(tmem + zb * kBN, tc::desc_sw128(sa + kk * 32),
-                                     tc::desc_sw128(sb + kk * 32), kIdZ, (kb | kk) != 0);
-                    tc::mma_commit(&bars.empty[stage]);
-                    adv();
-                    if (kb == p.nK - 1)
-                        tc::mma_commit(&bars.zfull[zb]);
-                },
-                [&](int j) {
-                    if (ab.on())
-                        return;
-                    const int s = j & 1;
-                    if (j % R != rank) {  // the owner's copy brings the bytes
-                        tc::bar_expect_tx(&bars.dzfull[s], kSlotBytes);
-                        expected = j;
-                    }
-                    if (!tc::bar_wait_cluster(&bars.dzfull[s], (j >> 1) & 1)) {
-                        aborted = 1;
-                        set_status(p.status, kStatusTimeout);
-                    }
-                },
-                [&](int j, int kb2) {
-                    if (ab.on())
-                        return;
-                    ab.wait(&bars.full[stage], phase, p.status);
-                    if (ab.on())
-                        return;
-                    tc::fence_after_sync();
-                    const uint32_t sdz = tc::smem_addr(slots + (j & 1) * kSlotBytes);
-                    const uint32_t sb2 = tc::smem_addr(ring + stage * kStageBytes);
-#pragma unroll
-                    for (int kk = 0; kk < kBK / 16; ++kk)
-                        tc::mma_bf16(tmem_acc, tc::desc_sw128(sdz + kb2 * 16384 + kk * 32),
-                                     tc::desc_sw128(sb2 + kk * 32), kId2,
-                                     j > 0 || kb2 > 0 || kk > 0);
-                    tc::mma_commit(&bars.empty[stage]);
-                    adv();
-                    if (kb2 == 1) {
-                        if (j + 2 < nB)  // slot j & 1 is free here for step j + 2
-                            tc::mma_commit_multicast(&bars.slot_free[j & 1],
-                                                     (uint16_t)(1u << ((j + 2) % R)));
-                        consumed = j + 1;
-                    }
-                });
-            // every MMA of this CTA (and the arrivals committed with them) is
-            // done before the epilogue reads the block or the CTA leaves
-            tc::mma_commit(&bars.accfull);
-            tc::bar_wait(&bars.accfull, 0);
-        }
-    } else {
-        const int lg = warp & 3;
-        const int r = lg * 32 + lane;
-        const uint32_t lane_off = (uint32_t)(lg * 32) << 16;
-        const int e = threadIdx.x - 64;
-        const int row = a_tile * kBM + r;  // token (DH) or vocabulary entry (DW)
-        int y_r = -1;
-        float lse_r = 0.0f, c_r = 0.0f;
-        if (MODE == kDh && row < p.T) {
-            y_r = p.ids[row];
-            lse_r = p.lse[row];
-            c_r = p.cvec[row];
-        }
-        uint32_t nfree = 0;  // per slot (bit s): parity of its next slot-free phase
-        for (int k = 0; rank + k * R < nB; ++k) {
-            const int t = rank + k * R;  // the owned step
-            const int zb = k & 1, s = t & 1;
-            if (__syncthreads_or_epi(ab.on()))
-                break;
-            if (MODE == kDw) {
-                const int tt = t * kBN + e;
-                const bool ok = tt < p.T;
-                col_lse[e] = ok ? p.lse[tt] : 0.0f;
-                col_c[e] = ok ? p.cvec[tt] : 0.0f;
-                col_y[e] = ok ? p.ids[tt] : -1;
-            }
-            ab.wait(&bars.zfull[zb], (k >> 1) & 1, p.status);
-            tc::fence_after_sync();
-            if (t >= 2) {  // slot s still holds step t - 2 somewhere in the cluster
-                if (!ab.on() && !tc::bar_wait_cluster(&bars.slot_free[s], (nfree >> s) & 1)) {
-                    aborted = 1;
-                    set_status(p.status, kStatusTimeout);
-                }
-                nfree ^= 1u << s;
-            }
-            asm volatile("bar.sync 1, 128;" ::: "memory");  // column scalars visible
-            uint8_t *slot = slots + s * kSlotBytes;
-            const int col0 = t * kBN;
-            for (int c0 = 0; c0 < kBN; c0 += 32) {
-                float v[32];
-                tc::tmem_ld32(tmem + lane_off + zb * kBN + c0, v);
-#pragma unroll
-                for (int i = 0; i < 32; ++i) {
-                    const int col = c0 + i;
-                    float d;
-                    // tokens with c = 0 (masked, clipped, past T) give 0 without
-                    // touching the exponential (their lse is a placeholder)
-                    if (MODE == kDh) {
-                        const int gcol = col0 + col;
-                        d = (gcol < p.V && c_r != 0.0f)
-                                ? c_r * ex2_ftz((v[i] - lse_r) * kLog2e) -
-                                      (gcol == y_r ? c_r : 0.0f)
-                                : 0.0f;
-                    } else {
-                        const float lt = col_lse[col], ct = col_c[col];
-                        d = (row < p.V && ct != 0.0f)
-                                ? ct * ex2_ftz((v[i] - lt) * kLog2e) -
-                                      (col_y[col] == row ? ct : 0.0f)
-                                : 0.0f;
-                    }
-                    v[i] = d;
-                }
-                uint8_t *blk = slot + (c0 >> 6) * 16384;
-#pragma unroll
-                for (int q = 0; q < 4; ++q) {
-                    uint4 w;
-                    __nv_bfloat162 h;
-                    h = __floats2bfloat162_rn(v[8 * q + 0], v[8 * q + 1]);
-                    w.x = *reinterpret_cast<uint32_t *>(&h);
-                    h = __floats2bfloat162_rn(v[8 * q + 2], v[8 * q + 3]);
-                    w.y = *reinterpret_cast<uint32_t *>(&h);
-                    h = __floats2bfloat162_rn(v[8 * q + 4], v[8 * q + 5]);
-                    w.z = *reinterpret_cast<uint32_t *>(&h);
-                    h = __floats2bfloat162_rn(v[8 * q + 6], v[8 * q + 7]);
-                    w.w = *reinterpret_cast<uint32_t *>(&h);
-                    *reinterpret_cast<uint4 *>(blk + tc::sw128_offset(r, ((c0 & 63) >> 3) + q)) = w;
-                }
-            }
-            tc::fence_before_sync();
-            tc::bar_arrive(&bars.zempty[zb]);
-            tc::fence_proxy_async_smem();
-            asm volatile("bar.sync 1, 128;" ::: "memory");  // the whole tile is written
-            if (e == 0 && !ab.on()) {
-                const uint32_t src = tc::smem_addr(slot);
-                const uint32_t bar = tc::smem_addr(&bars.dzfull[s]);
-                const uint32_t rec = tc::smem_addr(&last_copied[s]);
-                for (int q = 0; q < R; ++q)
-                    if (q != rank) {
-                        tc::red_max_cluster(tc::map_rank(rec, q), t);
-                        tc::bulk_s2s(tc::map_rank(src, q), src, kSlotBytes, tc::map_rank(bar, q));
-                    }
-                tc::bar_arrive(&bars.dzfull[s]);
-            }
-        }
-        // the accumulated block: 128 rows x 256 columns
-        ab.wait(&bars.accfull, 0, p.status);
-        tc::fence_after_sync();
-        const int nrows = MODE == kDh ? p.T : p.V;
-        for (int c0 = 0; c0 < kN2; c0 += 32) {
-            float v[32];
-            tc::tmem_ld32(tmem_acc + lane_off + c0, v);
-            if (row < nrows) {
-                const int64_t o = (int64_t)row * p.ld_out + (int64_t)rank * kN2 + c0;
-                if (p.out_bf16) {
-                    __nv_bfloat16 *dst = reinterpret_cast<__nv_bfloat16 *>(p.out) + o;
-#pragma unroll
-                    for (int q = 0; q < 4; ++q) {
-                        uint4 w;
-                        __nv_bfloat162 h;
-                        h = __floats2bfloat162_rn(v[8 * q + 0], v[8 * q + 1]);
-                        w.x = *reinterpret_cast<uint32_t *>(&h);
-                        h = __floats2bfloat162_rn(v[8 * q + 2], v[8 * q + 3]);
-                        w.y = *reinterpret_cast<uint32_t *>(&h);
-                        h = __floats2bfloat162_rn(v[8 * q + 4], v[8 * q + 5]);
-                        w.z = *reinterpret_cast<uint32_t *>(&h);
-                        h = __floats2bfloat162_rn(v[8 * q + 6], v[8 * q + 7]);
-                        w.w = *reinterpret_cast<uint32_t *>(&h);
-                        reinterpret_cast<uint4 *>(dst)[q] = w;
-                    }
-                } else {
-                    float4 *dst =
-                        reinterpret_cast<float4 *>(reinterpret_cast<float *>(p.out) + o);
-#pragma unroll
-                    for (int q = 0; q < 8; ++q)
-                        dst[q] = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
-                }
-            }
-        }
-    }
-    // Teardown: after the first cluster barrier no CTA issues another copy;
-    // each CTA then waits for any copy recorded into it that it has not seen
-    // land, and no CTA leaves before all have done so.
-    __syncwarp();
-    tc::fence_before_sync();
-    tc::cluster_arrive();
-    tc::cluster_wait();
-    if (warp == 1 && lane == 0) {
-        for (int s = 0; s < 2; ++s) {
-            const int L = *reinterpret_cast<volatile int *>(&last_copied[s]);
-            if (L >= consumed) {  // recorded but not consumed: it may be landing
-                if (L != expected)
-                    tc::bar_expect_tx(&bars.dzfull[s], kSlotBytes);
-                tc::bar_wait_cluster(&bars.dzfull[s], (L >> 1) & 1);
-            }
-        }
-    }
-    __syncwarp();
-    tc::cluster_arrive();
-    tc::cluster_wait();
-    if (warp == 1) {
-        tc::fence_after_sync();
-        tc::tmem_dealloc(tmem, 512);
-    }
+    for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n;
+         i += (int64_t)gridDim.x * blockDim.x)
+        dst[i] = __bfloat16_as_ushort(__float2bfloat16_rn(src[i]));
 }
 
 // Per token: combine the FWD pairs, then log p, weight, loss, c_t (one warp).
@@ -926,75 +492,49 @@ bool make_map(CUtensorMap *m, const void *ptr, int64_t inner, int64_t outer, int
                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-constexpr size_t kSmemBytes = kStages * kStageBytes + 32768 + 1024;
-
-template <int MODE>
-cudaError_t launch_mode(const CUtensorMap &a, const CUtensorMap &b, const CUtensorMap &b2,
-                        const Params &p, int grid, cudaStream_t s)
+template <int EPI>
+cudaError_t launch_gemm(const CUtensorMap &a, const CUtensorMap &b, const GemmArgs &g,
+                        cudaStream_t s)
 {
-    auto k = cis_lmhead_kernel<MODE>;
+    const int tiles = g.nMt * g.nNt;
+    if (tiles <= 0 || g.nK <= 0)
+        return cudaSuccess;
+    auto k = cis_lmhead_gemm_kernel<EPI>;
     cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          (int)kSmemBytes);
     if (e != cudaSuccess)
         return e;
-    k<<<grid, kThreads, kSmemBytes, s>>>(a, b, b2, p);
-    return cudaGetLastError();
-}
-
-constexpr size_t kGradSmemBytes = kStages * kStageBytes + 2 * kSlotBytes + 1024;
-
-template <int MODE>
-cudaError_t launch_grad(const CUtensorMap &a, const CUtensorMap &b, const CUtensorMap &b2,
-                        const Params &p, int clusters, int R, cudaStream_t s)
-{
-    auto k = cis_lmhead_grad_kernel<MODE>;
-    cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         (int)kGradSmemBytes);
-    if (e != cudaSuccess)
+    int dev = 0, sms = 0;
+    if ((e = cudaGetDevice(&dev)) != cudaSuccess ||
+        (e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess)
         return e;
-    cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3((unsigned)(clusters * R), 1, 1);
-    cfg.blockDim = dim3(kThreads, 1, 1);
-    cfg.dynamicSmemBytes = kGradSmemBytes;
-    cfg.stream = s;
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeClusterDimension;
-    attr[0].val.clusterDim.x = (unsigned)R;
-    attr[0].val.clusterDim.y = 1;
-    attr[0].val.clusterDim.z = 1;
-    cfg.attrs = attr;
-    cfg.numAttrs = 1;
-    return cudaLaunchKernelEx(&cfg, k, a, b, b2, p);
-}
-
-// Use the cluster gradient kernels?  Needs a portable cluster (Hd <= 2048);
-// CIS_LMHEAD_RECOMPUTE=1 selects the recompute kernels instead (for comparison).
-bool use_cluster_grad(int64_t H)
-{
-    static int force_recompute = [] {
-        const char *e = getenv("CIS_LMHEAD_RECOMPUTE");
-        return e ? atoi(e) : 0;
-    }();
-    return !force_recompute && H / kN2 <= 8;
+    const int grid = tiles < sms ? tiles : sms;
+    k<<<grid, kThreads, kSmemBytes, s>>>(a, b, g);
+    return cudaGetLastError();
 }
 
 }  // namespace lm
 
-// Workspace of cis_lmhead_fused, after the token-pass layout of ws_layout(T).
+// Workspace of cis_lmhead_fused, after the token-pass layout of ws_layout(T),
+// for vocabulary chunks of Vc columns (a multiple of 256).
 struct LmLayout {
     WsLayout base;
-    size_t lse, c, zy, part, wt, ht, total;
-    int64_t vp, tp;
+    size_t lse, c, zy, part, wt, ht, dh, dz, dzt, total;
+    int64_t vp, tp, Tp, Vc;
 };
 
-LmLayout lm_layout(int64_t T, int64_t V, int64_t Hd)
+static int64_t round_up(int64_t x, int64_t m) { return (x + m - 1) / m * m; }
+
+LmLayout lm_layout(int64_t T, int64_t V, int64_t Hd, int64_t Vc)
 {
     auto up = [](size_t x) { return (x + 1023) / 1024 * 1024; };
     LmLayout L;
     L.base = ws_layout(T);
     const int64_t nVt = (V + lm::kBN - 1) / lm::kBN;
-    L.vp = (V + 7) / 8 * 8;
-    L.tp = (T + 7) / 8 * 8;
+    L.vp = round_up(V, 8);
+    L.tp = round_up(T, 8);
+    L.Tp = round_up(T, lm::kBM);
+    L.Vc = Vc;
     size_t o = up(L.base.total);
     L.lse = o;
     o = up(o + 4 * (size_t)T);
@@ -1008,8 +548,42 @@ LmLayout lm_layout(int64_t T, int64_t V, int64_t Hd)
     o = up(o + 2 * (size_t)Hd * (size_t)L.vp);
     L.ht = o;
     o = up(o + 2 * (size_t)Hd * (size_t)L.tp);
+    L.dh = o;
+    o = up(o + 4 * (size_t)T * (size_t)Hd);
+    L.dz = o;
+    o = up(o + 2 * (size_t)L.Tp * (size_t)Vc);
+    L.dzt = o;
+    o = up(o + 2 * (size_t)Vc * (size_t)L.Tp);
     L.total = o;
     return L;
+}
+
+// The widest chunk: every vocabulary column at once.
+static int64_t max_chunk(int64_t V) { return round_up(V, lm::kBN); }
+
+// The default chunk: dz and dz^T within kDefaultChunkBytes.
+static int64_t default_chunk(int64_t T, int64_t V)
+{
+    const int64_t Tp = round_up(T, lm::kBM);
+    int64_t c = Tp > 0 ? lm::kDefaultChunkBytes / (4 * Tp) / lm::kBN * lm::kBN : max_chunk(V);
+    if (c < lm::kBN)
+        c = lm::kBN;
+    return c < max_chunk(V) ? c : max_chunk(V);
+}
+
+// The widest chunk whose layout fits in `bytes`; 0 if not even 256 columns do.
+static int64_t chunk_for_bytes(int64_t T, int64_t V, int64_t Hd, size_t bytes)
+{
+    const size_t fixed = lm_layout(T, V, Hd, 0).total;
+    if (bytes < fixed)
+        return 0;
+    const size_t per = 4 * (size_t)round_up(T, lm::kBM);
+    int64_t c = per > 0 ? (int64_t)((bytes - fixed) / per) / lm::kBN * lm::kBN : max_chunk(V);
+    if (c > max_chunk(V))
+        c = max_chunk(V);
+    while (c >= lm::kBN && lm_layout(T, V, Hd, c).total > bytes)
+        c -= lm::kBN;
+    return c >= lm::kBN ? c : 0;
 }
 
 }  // namespace cis
@@ -1022,7 +596,16 @@ CIS_API cis_status_t cis_lmhead_workspace_size(int64_t T, int64_t V, int64_t H, 
 {
     if (bytes == nullptr || T < 0 || V <= 0 || H <= 0)
         return CIS_ERR_INVALID_ARG;
-    *bytes = lm_layout(T, V, H).total;
+    *bytes = lm_layout(T, V, H, default_chunk(T, V)).total;
+    return CIS_OK;
+}
+
+CIS_API cis_status_t cis_lmhead_workspace_size_chunk(int64_t T, int64_t V, int64_t H,
+                                                     int64_t chunk, size_t *bytes)
+{
+    if (bytes == nullptr || T < 0 || V <= 0 || H <= 0 || chunk <= 0 || chunk % lm::kBN != 0)
+        return CIS_ERR_INVALID_ARG;
+    *bytes = lm_layout(T, V, H, chunk < max_chunk(V) ? chunk : max_chunk(V)).total;
     return CIS_OK;
 }
 
@@ -1037,7 +620,7 @@ CIS_API cis_status_t cis_lmhead_fused(const void *hidden, const void *weight, in
                                       double *loss_out, void *workspace, size_t workspace_bytes,
                                       void *stream)
 {
-    if (T < 0 || T > (1LL << 30) || V <= 0 || V > (1LL << 30) || H <= 0)
+    if (T < 0 || T > (1LL << 30) || V <= 0 || V > (1LL << 30) || H <= 0 || H > (1LL << 20))
         return CIS_ERR_INVALID_ARG;
     if (grad_dtype != CIS_F32 && grad_dtype != CIS_BF16)
         return CIS_ERR_INVALID_ARG;
@@ -1045,12 +628,14 @@ CIS_API cis_status_t cis_lmhead_fused(const void *hidden, const void *weight, in
         return CIS_ERR_INVALID_ARG;
     if (params->agg == CIS_AGG_SEQ_MEAN_TOKEN_MEAN && (cu_seqlens == nullptr || B < 0))
         return CIS_ERR_INVALID_ARG;
-    if (H % lm::kN2 != 0)
+    if (H % lm::kBN != 0)
         return CIS_ERR_UNSUPPORTED;  // Hd in blocks of 256 (and so of the 64-wide K blocks)
-    const LmLayout L = lm_layout(T, V, H);
-    if (workspace == nullptr || (reinterpret_cast<uintptr_t>(workspace) & 1023) ||
-        workspace_bytes < L.total)
+    if (workspace == nullptr || (reinterpret_cast<uintptr_t>(workspace) & 1023))
         return CIS_ERR_INVALID_ARG;
+    const int64_t Vc = chunk_for_bytes(T, V, H, workspace_bytes);
+    if (Vc == 0)
+        return CIS_ERR_INVALID_ARG;  // smaller than the layout for 256-column chunks
+    const LmLayout L = lm_layout(T, V, H, Vc);
     if (T > 0 && (hidden == nullptr || weight == nullptr || ids == nullptr ||
                   lp_infer == nullptr || adv == nullptr || dhidden == nullptr ||
                   dweight == nullptr))
@@ -1085,6 +670,10 @@ CIS_API cis_status_t cis_lmhead_fused(const void *hidden, const void *weight, in
     float2 *part = reinterpret_cast<float2 *>(ws + L.part);
     __nv_bfloat16 *wt = reinterpret_cast<__nv_bfloat16 *>(ws + L.wt);
     __nv_bfloat16 *ht = reinterpret_cast<__nv_bfloat16 *>(ws + L.ht);
+    uint16_t *dz = reinterpret_cast<uint16_t *>(ws + L.dz);
+    uint16_t *dzt = reinterpret_cast<uint16_t *>(ws + L.dzt);
+    float *dh_acc = grad_dtype == CIS_F32 ? static_cast<float *>(dhidden)
+                                          : reinterpret_cast<float *>(ws + L.dh);
 
     float *scale = reinterpret_cast<float *>(ws + L.base.scale);
     cudaError_t e = launch_scales(mask, T, cu_seqlens, B, P.agg, scale, a.status, s);
@@ -1093,36 +682,38 @@ CIS_API cis_status_t cis_lmhead_fused(const void *hidden, const void *weight, in
     if (T > 0) {
         const int nTt = (int)((T + lm::kBM - 1) / lm::kBM);
         const int nVt = (int)((V + lm::kBN - 1) / lm::kBN);
-        lm::Params p = {};
-        p.T = (int)T;
-        p.V = (int)V;
-        p.Hd = (int)H;
-        p.nTt = nTt;
-        p.nVt = nVt;
-        p.nK = (int)(H / lm::kBK);
-        p.ids = ids;
-        p.mask = mask;
-        p.lse = lse;
-        p.cvec = cv;
-        p.part = part;
-        p.zy = zy;
-        p.status = a.status;
+        const int nHt = (int)(H / lm::kBN);
         CUtensorMap mH, mW, mWt, mHt;
         if (!lm::make_map(&mH, hidden, H, T, H, lm::kBM) ||
             !lm::make_map(&mW, weight, H, V, H, lm::kBN) ||
-            !lm::make_map(&mWt, wt, V, H, L.vp, lm::kN2) ||
-            !lm::make_map(&mHt, ht, T, H, L.tp, lm::kN2))
+            !lm::make_map(&mWt, wt, V, H, L.vp, lm::kBN) ||
+            !lm::make_map(&mHt, ht, T, H, L.tp, lm::kBN))
             return CIS_ERR_UNSUPPORTED;
-        // FWD
-        e = lm::launch_mode<lm::kFwd>(mH, mW, mW, p,
-                                      nTt * ((nVt + lm::kFwdGroup - 1) / lm::kFwdGroup), s);
-        if (e != cudaSuccess)
+        lm::GemmArgs g = {};
+        g.T = (int)T;
+        g.V = (int)V;
+        g.ids = ids;
+        g.lse = lse;
+        g.cvec = cv;
+        g.part = part;
+        g.zy = zy;
+        g.dz = dz;
+        g.dzt = dzt;
+        g.ld_dz = Vc;
+        g.ld_dzt = L.Tp;
+        g.status = a.status;
+        // FWD: z tiles of H W^T, row statistics
+        g.nMt = nTt;
+        g.nNt = nVt;
+        g.nK = (int)(H / lm::kBK);
+        g.raster_n = 1;
+        if (lm::launch_gemm<lm::kStats>(mH, mW, g, s) != cudaSuccess)
             return CIS_ERR_CUDA;
         // per-token scalars
         lm::cis_lmhead_token_kernel<<<(unsigned)((T + 7) / 8), 256, 0, s>>>(a, part, zy, nVt, lse, cv);
         if ((e = cudaGetLastError()) != cudaSuccess)
             return CIS_ERR_CUDA;
-        // transposed copies of W and H (K-major operands of dH and dW)
+        // transposed copies of W and H (K-major B operands of DH and DW)
         dim3 tb(32, 8);
         lm::cis_lmhead_transpose_kernel<<<dim3((unsigned)((H + 31) / 32), (unsigned)((V + 31) / 32)),
                                        tb, 0, s>>>(
@@ -1132,22 +723,60 @@ CIS_API cis_status_t cis_lmhead_fused(const void *hidden, const void *weight, in
             static_cast<const __nv_bfloat16 *>(hidden), T, H, H, ht, L.tp);
         if ((e = cudaGetLastError()) != cudaSuccess)
             return CIS_ERR_CUDA;
-        // dH: A = H (token tiles), B = W (vocab tiles), B2 = W^T
-        p.out = dhidden;
-        p.out_bf16 = grad_dtype == CIS_BF16;
-        p.ld_out = H;
-        const int R = (int)(H / lm::kN2);
-        const bool clustered = lm::use_cluster_grad(H);
-        e = clustered ? lm::launch_grad<lm::kDh>(mH, mW, mWt, p, nTt, R, s)
-                      : lm::launch_mode<lm::kDh>(mH, mW, mWt, p, nTt * R, s);
-        if (e != cudaSuccess)
-            return CIS_ERR_CUDA;
-        // dW: A = W (vocab tiles), B = H (token tiles), B2 = H^T
-        p.out = dweight;
-        e = clustered ? lm::launch_grad<lm::kDw>(mW, mH, mHt, p, nVt, R, s)
-                      : lm::launch_mode<lm::kDw>(mW, mH, mHt, p, nVt * R, s);
-        if (e != cudaSuccess)
-            return CIS_ERR_CUDA;
+        for (int64_t v0 = 0; v0 < V; v0 += Vc) {
+            const int64_t w = V - v0 < Vc ? V - v0 : Vc;
+            // DZ: recompute the chunk's z tiles, write dz and dz^T
+            g.nMt = nTt;
+            g.nNt = (int)((w + lm::kBN - 1) / lm::kBN);
+            g.nK = (int)(H / lm::kBK);
+            g.raster_n = 1;
+            g.a_row0 = 0;
+            g.a_k0 = 0;
+            g.b_row0 = (int)v0;
+            g.b_k0 = 0;
+            g.col0 = (int)v0;
+            if (lm::launch_gemm<lm::kDz>(mH, mW, g, s) != cudaSuccess)
+                return CIS_ERR_CUDA;
+            CUtensorMap mDz, mDzt;
+            if (!lm::make_map(&mDz, dz, w, L.Tp, Vc, lm::kBM) ||
+                !lm::make_map(&mDzt, dzt, T, w, L.Tp, lm::kBM))
+                return CIS_ERR_UNSUPPORTED;
+            // DH (+)= dz W[chunk]: A = dz [Tp, w], B = W^T [Hd, V] from column v0
+            g.nMt = nTt;
+            g.nNt = nHt;
+            g.nK = (int)((w + lm::kBK - 1) / lm::kBK);
+            g.raster_n = 0;
+            g.a_row0 = 0;
+            g.a_k0 = 0;
+            g.b_row0 = 0;
+            g.b_k0 = (int)v0;
+            g.out = dh_acc;
+            g.out_bf16 = 0;
+            g.rows_valid = (int)T;
+            g.ld_out = H;
+            e = v0 == 0 ? lm::launch_gemm<lm::kStore>(mDz, mWt, g, s)
+                        : lm::launch_gemm<lm::kAccum>(mDz, mWt, g, s);
+            if (e != cudaSuccess)
+                return CIS_ERR_CUDA;
+            // DW[chunk] = dz^T H: A = dz^T [w, T], B = H^T [Hd, T]
+            g.nMt = (int)((w + lm::kBM - 1) / lm::kBM);
+            g.nNt = nHt;
+            g.nK = (int)((T + lm::kBK - 1) / lm::kBK);
+            g.raster_n = 0;
+            g.b_k0 = 0;
+            g.out = static_cast<uint8_t *>(dweight) +
+                    (size_t)v0 * (size_t)H * (grad_dtype == CIS_BF16 ? 2 : 4);
+            g.out_bf16 = grad_dtype == CIS_BF16;
+            g.rows_valid = (int)w;
+            if (lm::launch_gemm<lm::kStore>(mDzt, mHt, g, s) != cudaSuccess)
+                return CIS_ERR_CUDA;
+        }
+        if (grad_dtype == CIS_BF16) {
+            lm::cis_lmhead_to_bf16_kernel<<<1184, 256, 0, s>>>(
+                dh_acc, static_cast<uint16_t *>(dhidden), T * H);
+            if ((e = cudaGetLastError()) != cudaSuccess)
+                return CIS_ERR_CUDA;
+        }
     }
     return launch_reduce(a, stats_out, loss_out, s) == cudaSuccess ? CIS_OK : CIS_ERR_CUDA;
 }

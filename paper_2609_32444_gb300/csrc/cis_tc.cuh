@@ -44,21 +44,38 @@ __device__ __forceinline__ void bar_arrive(uint64_t *bar)
 {
     asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_addr(bar)) : "memory");
 }
-// Bounded wait for the phase with the given parity; false if it never came.
-__device__ __forceinline__ bool bar_wait(uint64_t *bar, uint32_t parity)
+// Bounded wait for the phase with the given parity (the barrier of this CTA,
+// completed from this CTA or, with kCluster, from others of its cluster).
+// False if it never came or, when `flag` is given, once the word it points to
+// carries kStatusTimeout: a wait elsewhere in the grid ran out, so this one
+// stops early.  The word is read every 256 polls only, off the fast path.
+template <bool kCluster = false>
+__device__ __forceinline__ bool bar_wait(uint64_t *bar, uint32_t parity,
+                                         const volatile int32_t *flag = nullptr)
 {
     const uint32_t a = smem_addr(bar);
     for (uint32_t i = 0; i < kMaxPolls; ++i) {
         uint32_t done;
-        asm volatile(
-            "{\n\t.reg .pred p;\n\t"
-            "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
-            "selp.u32 %0, 1, 0, p;\n\t}"
-            : "=r"(done)
-            : "r"(a), "r"(parity), "r"(kPollSuspendNs)
-            : "memory");
+        if (kCluster)
+            asm volatile(
+                "{\n\t.reg .pred p;\n\t"
+                "mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2, %3;\n\t"
+                "selp.u32 %0, 1, 0, p;\n\t}"
+                : "=r"(done)
+                : "r"(a), "r"(parity), "r"(kPollSuspendNs)
+                : "memory");
+        else
+            asm volatile(
+                "{\n\t.reg .pred p;\n\t"
+                "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
+                "selp.u32 %0, 1, 0, p;\n\t}"
+                : "=r"(done)
+                : "r"(a), "r"(parity), "r"(kPollSuspendNs)
+                : "memory");
         if (done)
             return true;
+        if (flag != nullptr && (i & 255) == 255 && (*flag & kStatusTimeout) != 0)
+            return false;
     }
     return false;
 }
@@ -171,22 +188,10 @@ __device__ __forceinline__ void cluster_wait()
 }
 // Bounded wait for a phase completed by another CTA of the cluster (its bulk
 // copies or its tensor cores).
-__device__ __forceinline__ bool bar_wait_cluster(uint64_t *bar, uint32_t parity)
+__device__ __forceinline__ bool bar_wait_cluster(uint64_t *bar, uint32_t parity,
+                                                 const volatile int32_t *flag = nullptr)
 {
-    const uint32_t a = smem_addr(bar);
-    for (uint32_t i = 0; i < kMaxPolls; ++i) {
-        uint32_t done;
-        asm volatile(
-            "{\n\t.reg .pred p;\n\t"
-            "mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2, %3;\n\t"
-            "selp.u32 %0, 1, 0, p;\n\t}"
-            : "=r"(done)
-            : "r"(a), "r"(parity), "r"(kPollSuspendNs)
-            : "memory");
-        if (done)
-            return true;
-    }
-    return false;
+    return bar_wait<true>(bar, parity, flag);
 }
 // Copy `bytes` of this CTA's shared memory to another CTA's shared memory
 // (addresses from map_rank); the receiver's mbarrier counts the bytes.

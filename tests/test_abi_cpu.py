@@ -86,6 +86,22 @@ def _fwd_bwd_rc(binding, **over):
                               args["ws"], args["ws_bytes"], None)
 
 
+def test_lmhead_workspace_grows_with_the_chunk(binding):
+    """4 ceil(T/128)*128 bytes per chunk column (dz and dz^T in bf16); chunks
+    wider than V (rounded up to 256) cost no more; a chunk must be a positive
+    multiple of 256."""
+    T, V, H = 1000, 5000, 512
+    s256 = binding.cis_lmhead_workspace_size_chunk(T, V, H, 256)
+    s512 = binding.cis_lmhead_workspace_size_chunk(T, V, H, 512)
+    assert s512 - s256 in range(4 * 1024 * 256, 4 * 1024 * 256 + 2049)
+    full = binding.cis_lmhead_workspace_size_chunk(T, V, H, 5120)
+    assert binding.cis_lmhead_workspace_size_chunk(T, V, H, 1 << 20) == full
+    assert binding.cis_lmhead_workspace_size(T, V, H) <= full
+    for bad in (0, -256, 100, 384):
+        with pytest.raises(RuntimeError):
+            binding.cis_lmhead_workspace_size_chunk(T, V, H, bad)
+
+
 @pytest.mark.parametrize("over", [
     dict(T=-1), dict(V=0), dict(ld=7), dict(ld_out=7), dict(dtype=5), dict(dz_dt=2),
     dict(logits=None), dict(ids=None), dict(lp_inf=None), dict(adv=None), dict(dz=None),

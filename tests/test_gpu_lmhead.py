@@ -40,12 +40,12 @@ def _bits(t):
     return bf16_tensor_bits(t)
 
 
-def _run(b, mode="cis", grad_dtype=torch.float32, lp_old=None):
+def _run(b, mode="cis", grad_dtype=torch.float32, lp_old=None, chunk=None):
     P = binding.cis_default_params(mode, lam=b.lam)
     return binding.cis_lmhead_fused(b.hidden.to(DEV), b.weight.to(DEV), b.ids.to(DEV),
                                     b.lp_infer.to(DEV), b.adv.to(DEV), P,
                                     lp_old=None if lp_old is None else lp_old.to(DEV),
-                                    mask=b.mask.to(DEV), grad_dtype=grad_dtype)
+                                    mask=b.mask.to(DEV), grad_dtype=grad_dtype, chunk=chunk)
 
 
 def _oracle(b, mode="cis", rows=None, lp_old=None):
@@ -114,6 +114,35 @@ def test_lmhead_hidden_2048(mode):
     _check_tokens(out, ref, np.arange(b.T), b, mode, full=True)
     _check_grad(out["dhidden"], ref["dhidden"], ref["dhidden_abs"], b.V, False)
     _check_grad(out["dweight"], ref["dweight"], ref["dweight_abs"], b.T, False)
+
+
+@pytest.mark.parametrize("T,V,H,chunk,grad", [(200, 1000, 512, 256, torch.float32),
+                                              (300, 4096, 2048, 1024, torch.bfloat16),
+                                              (130, 2000, 256, 768, torch.float32)])
+def test_lmhead_vocabulary_chunks(T, V, H, chunk, grad):
+    """A workspace sized for narrow vocabulary chunks: dH accumulates over the
+    chunks, dW is written chunk by chunk, the last chunk ragged; every element."""
+    b = synth.make_batch(5, T=T, V=V, H=H)
+    out = _run(b, grad_dtype=grad, chunk=chunk)
+    torch.cuda.synchronize()
+    ref = _oracle(b)
+    _check_tokens(out, ref, np.arange(T), b, "cis", full=True)
+    _check_grad(out["dhidden"], ref["dhidden"], ref["dhidden_abs"], V, grad == torch.bfloat16)
+    _check_grad(out["dweight"], ref["dweight"], ref["dweight_abs"], T, grad == torch.bfloat16)
+    assert binding.decode_stats(out["stats"])["status"] == 0
+
+
+def test_lmhead_workspace_too_small():
+    """Less workspace than 256-column chunks need is refused on the host."""
+    b = synth.make_batch(5, T=64, V=1024, H=256)
+    need = binding.cis_lmhead_workspace_size_chunk(64, 1024, 256, 256)
+    ws = torch.empty(need + 1024, dtype=torch.uint8, device=DEV)
+    off = (-ws.data_ptr()) % 1024
+    P = binding.cis_default_params("cis", lam=b.lam)
+    with pytest.raises(RuntimeError):
+        binding.cis_lmhead_fused(b.hidden.to(DEV), b.weight.to(DEV), b.ids.to(DEV),
+                                 b.lp_infer.to(DEV), b.adv.to(DEV), P, mask=b.mask.to(DEV),
+                                 workspace=ws[off:off + need - 4096], chunk=None)
 
 
 def test_lmhead_masked_tokens_and_old_logprobs():
