@@ -33,6 +33,8 @@ _lock = threading.Lock()
 _lib = None
 
 MODE_CIS, MODE_TIS, MODE_EXACT, MODE_NONE = 0, 1, 2, 3
+MODE_BAND, MODE_ICEPOP, MODE_KPOP, MODE_SEQ_TIS, MODE_SEQ_MIS = 4, 5, 6, 7, 8
+SEQ_MODES = (MODE_SEQ_TIS, MODE_SEQ_MIS)
 AGG_TOKEN_MEAN, AGG_SEQ_MEAN = 0, 1
 F32, BF16 = 0, 1
 
@@ -48,13 +50,21 @@ class OracleParams(ctypes.Structure):
         ("exact_hi", ctypes.c_double),
         ("clip_low", ctypes.c_double),
         ("clip_high", ctypes.c_double),
+        ("icepop_lo", ctypes.c_double),
+        ("icepop_hi", ctypes.c_double),
+        ("kpop_phi", ctypes.c_double),
+        ("seq_cap", ctypes.c_double),
+        ("seq_lo", ctypes.c_double),
+        ("seq_hi", ctypes.c_double),
     ]
 
 
 def params(mode=MODE_CIS, lam=2.3, kappa=5e-3, tis_cap=2.0, exact_lo=1e-6, exact_hi=1e6,
-           clip_low=0.2, clip_high=0.28, agg=AGG_TOKEN_MEAN) -> OracleParams:
+           clip_low=0.2, clip_high=0.28, agg=AGG_TOKEN_MEAN, icepop_lo=0.5, icepop_hi=5.0,
+           kpop_phi=2.0, seq_cap=2.0, seq_lo=0.5, seq_hi=2.0) -> OracleParams:
     """Hyper-parameters; defaults are the deployed values of App. C.1 / Table 8."""
-    return OracleParams(mode, agg, lam, kappa, tis_cap, exact_lo, exact_hi, clip_low, clip_high)
+    return OracleParams(mode, agg, lam, kappa, tis_cap, exact_lo, exact_hi, clip_low, clip_high,
+                        icepop_lo, icepop_hi, kpop_phi, seq_cap, seq_lo, seq_hi)
 
 
 def build(force: bool = False) -> str:
@@ -79,8 +89,9 @@ def _load():
         i64, i32, dbl = ctypes.c_int64, ctypes.c_int32, ctypes.c_double
         lib.oracle_token_logprobs.argtypes = [P, i32, i64, i64, i64, P, P, P, P, ctypes.c_int]
         lib.oracle_token_logprobs.restype = ctypes.c_int
-        lib.oracle_weights.argtypes = [P, P, P, i64, ctypes.POINTER(OracleParams), P, P, P, P]
-        lib.oracle_weights.restype = None
+        lib.oracle_weights.argtypes = [P, P, P, i64, P, i64, ctypes.POINTER(OracleParams), P, P,
+                                       P, P]
+        lib.oracle_weights.restype = ctypes.c_int
         lib.oracle_loss_scales.argtypes = [P, i64, P, i64, ctypes.c_int, P]
         lib.oracle_loss_scales.restype = None
         lib.oracle_loss_fwd_bwd.argtypes = [
@@ -142,19 +153,26 @@ def token_logprobs(logits, ids, V=None, mask=None, nthreads=0):
     return lp, lse, rc
 
 
-def weights(lp_w, lp_inf, P: OracleParams, mask=None):
-    """Algorithm 1 / Table 8 weights in fp64.  Returns (w, trunc, logk, eps)."""
+def weights(lp_w, lp_inf, P: OracleParams, mask=None, cu_seqlens=None):
+    """Algorithm 1 / Table 8 weights in fp64.  Returns (w, trunc, logk, eps).
+
+    The sequence operators (Seq-TIS, Seq-MIS) need ``cu_seqlens`` (B + 1
+    offsets of the responses)."""
     lib = _load()
     lp_w = np.ascontiguousarray(lp_w, dtype=np.float64)
     lp_inf = np.ascontiguousarray(lp_inf, dtype=np.float64)
     mask = _opt(mask, np.uint8)
+    cu = _opt(cu_seqlens, np.int32)
+    B = 0 if cu is None else cu.shape[0] - 1
     T = lp_w.shape[0]
     w = np.zeros(T, np.float64)
     tr = np.zeros(T, np.uint8)
     lk = np.zeros(T, np.float64)
     eps = np.zeros(T, np.float64)
-    lib.oracle_weights(_ptr(lp_w), _ptr(lp_inf), _ptr(mask), T, ctypes.byref(P), _ptr(w),
-                       _ptr(tr), _ptr(lk), _ptr(eps))
+    rc = lib.oracle_weights(_ptr(lp_w), _ptr(lp_inf), _ptr(mask), T, _ptr(cu), B,
+                            ctypes.byref(P), _ptr(w), _ptr(tr), _ptr(lk), _ptr(eps))
+    if rc != 0:
+        raise ValueError("a sequence operator needs cu_seqlens")
     return w, tr, lk, eps
 
 
@@ -175,7 +193,8 @@ def loss_fwd_bwd(logits, ids, lp_inf, adv, P: OracleParams, V=None, lp_old=None,
 
     ``rows``: indices of the rows whose dz is returned (None = all rows).
     Returns a dict with loss, terms, lp, lse, w, trunc, c, dz ([len(rows), V] or
-    [T, V]) and rc (0, or -1 when a valid row has an out-of-range id).
+    [T, V]) and rc (0, or -1 when a valid row has an out-of-range id).  The
+    sequence operators need ``cu_seqlens``.
     """
     lib = _load()
     a, dt = _logits_arg(logits)
@@ -200,12 +219,14 @@ def loss_fwd_bwd(logits, ids, lp_inf, adv, P: OracleParams, V=None, lp_old=None,
         _ptr(cu), B, ctypes.byref(P), _ptr(w_fixed), _ptr(rows_a), nrows if rows_a is not None
         else 0, _ptr(dz), _ptr(out["lp"]), _ptr(out["lse"]), _ptr(out["w"]), _ptr(trunc),
         _ptr(out["terms"]), _ptr(out["c"]), ctypes.byref(loss), nthreads)
+    if rc == -3:
+        raise ValueError("a sequence operator needs cu_seqlens")
     out.update(loss=loss.value, trunc=trunc, dz=dz, rc=rc)
     return out
 
 
 def lmhead_fwd_bwd(hidden, weight, ids, lp_inf, adv, P: OracleParams, lp_old=None, mask=None,
-                   rows=None, n_valid_total=None, w_fixed=None, want_dw=True):
+                   rows=None, n_valid_total=None, w_fixed=None, want_dw=True, cu_seqlens=None):
     """The token pass through the LM head, in fp64.
 
     Logits z = H W^T (Sec. 2.1; the softmax is over these logits) are formed
@@ -223,11 +244,13 @@ def lmhead_fwd_bwd(hidden, weight, ids, lp_inf, adv, P: OracleParams, lp_old=Non
         np.asarray(hidden, np.float64)
     Wf = bf16_bits_to_f64(weight) if np.asarray(weight).dtype == np.uint16 else \
         np.asarray(weight, np.float64)
+    if rows is not None and (P.mode in SEQ_MODES or cu_seqlens is not None):
+        raise ValueError("row subsets cannot take whole responses")
     idx = np.arange(Hf.shape[0]) if rows is None else np.asarray(rows, np.int64)
     sel = lambda a: None if a is None else np.asarray(a)[idx]  # noqa: E731
     Z = Hf[idx] @ Wf.T
     out = loss_fwd_bwd(Z, sel(ids), sel(lp_inf), sel(adv), P, lp_old=sel(lp_old),
-                       mask=sel(mask), w_fixed=sel(w_fixed))
+                       mask=sel(mask), w_fixed=sel(w_fixed), cu_seqlens=cu_seqlens)
     if rows is not None and n_valid_total is not None:
         if P.agg != AGG_TOKEN_MEAN:
             raise ValueError("row subsets need the token-mean normaliser")

@@ -22,8 +22,14 @@
  *   - Algorithm 1 (Sec. 3.3): p = exp(l_train), k = exp(l_train - l_infer),
  *     phi = max(1 - p, kappa), f = min{k, 1 + lambda*phi}; the estimate is
  *     (1/n) sum stopgrad(f_m) l'_m.
- *   - Table 8 (App. C.1): the other weight operators (exact ratio clamped to
- *     [1e-6, 1e6], TIS min(k, C), no correction) and their defaults.
+ *   - Table 8 (App. C.1): the other weight operators and their defaults:
+ *     exact ratio clamped to [1e-6, 1e6]; TIS min(k, C); IcePop k 1{k in
+ *     [a, b]}; KPop-dagger k 1{max(KL_B(p||q), KL_B(q||p)) <= phi}, fp64, with
+ *     p and q clamped to [1e-8, 1 - 1e-8] (App. D.5, "The KL mask and
+ *     probability saturation"); Seq-TIS min(K, C) and Seq-MIS K 1{K in [a, b]}
+ *     with K the product of k over a response; no correction.
+ *   - Sec. 4.3 / App. C.1: the two-sided band max{min{k, 1 + lambda phi},
+ *     (1 + p)/2}, the image of e^eps >= 1/2 under k = p + (1 - p) e^eps.
  *   - Lemma 3.1 / Lemma B.1: eps_t = logit p_t - logit q_t.
  *
  * Readings where the paper is silent (each also listed in the design notes):
@@ -34,7 +40,15 @@
  *   - in min(rho*A, clip(rho)*A) a tie takes the unclipped branch, so the
  *     gradient flows at rho = 1 +- c exactly;
  *   - a NaN ratio gives a NaN weight (NaN propagates; min{NaN, cap} is not
- *     read as cap).
+ *     read as cap);
+ *   - "truncated" means the operator changed the weight: capped, clamped,
+ *     lifted (band) or masked (IcePop, KPop, Seq-MIS); for the sequence
+ *     operators every token of a response gets the response's flag;
+ *   - the sequence operators take the product over the valid tokens of each
+ *     response (cu_seqlens), as a sum of log k in index order; a valid token
+ *     outside every response gets weight 0; a token with an out-of-range id
+ *     is left out of its response's product;
+ *   - KPop: 1 - p is 1 - (clamped p), and the mask is "metric > phi".
  */
 #include <math.h>
 #include <stdint.h>
@@ -46,10 +60,15 @@
 
 /* Weight operators (Table 8 of the paper, plus CIS of Algorithm 1). */
 enum {
-    OR_MODE_CIS = 0,   /* min{k, 1 + lambda*max(1-p, kappa)}      Algorithm 1 */
-    OR_MODE_TIS = 1,   /* min(k, C)                                Table 8    */
-    OR_MODE_EXACT = 2, /* k clamped to [lo, hi]                    Table 8    */
-    OR_MODE_NONE = 3   /* 1                                        Table 8    */
+    OR_MODE_CIS = 0,     /* min{k, 1 + lambda*max(1-p, kappa)}      Algorithm 1  */
+    OR_MODE_TIS = 1,     /* min(k, C)                                Table 8      */
+    OR_MODE_EXACT = 2,   /* k clamped to [lo, hi]                    Table 8      */
+    OR_MODE_NONE = 3,    /* 1                                        Table 8      */
+    OR_MODE_BAND = 4,    /* max{min{k, 1 + lambda phi}, (1 + p)/2}   Sec. 4.3     */
+    OR_MODE_ICEPOP = 5,  /* k 1{k in [a, b]}                         Table 8      */
+    OR_MODE_KPOP = 6,    /* k 1{max binary KL <= phi}                Table 8      */
+    OR_MODE_SEQ_TIS = 7, /* min(K, C), K = prod of k over a response Table 8      */
+    OR_MODE_SEQ_MIS = 8  /* K 1{K in [a, b]}                         Table 8      */
 };
 
 enum { OR_AGG_TOKEN_MEAN = 0, OR_AGG_SEQ_MEAN = 1 };
@@ -65,7 +84,18 @@ typedef struct {
     double exact_hi;
     double clip_low;  /* PPO clip range [1 - c_low, 1 + c_high], Eq. 1 */
     double clip_high;
+    double icepop_lo; /* IcePop band [a, b]                            */
+    double icepop_hi;
+    double kpop_phi;  /* KPop threshold on the binary KL               */
+    double seq_cap;   /* C of Seq-TIS                                  */
+    double seq_lo;    /* Seq-MIS band [a, b]                           */
+    double seq_hi;
 } oracle_params_t;
+
+static int is_seq_mode(int mode)
+{
+    return mode == OR_MODE_SEQ_TIS || mode == OR_MODE_SEQ_MIS;
+}
 
 /* bf16 is the top half of an IEEE binary32; the upcast is exact. */
 static double bf16_to_double(uint16_t h)
@@ -211,6 +241,45 @@ static void token_weight(double lw, double linf, const oracle_params_t *P, doubl
         tr = logk > log(P->exact_hi) || logk < log(P->exact_lo);
         break;
     }
+    case OR_MODE_BAND: {
+        /* Sec. 4.3: the CIS weight, lifted from below to (1 + p)/2. */
+        double phi = one_minus_p > P->kappa ? one_minus_p : P->kappa;
+        double cap = 1.0 + P->lambda * phi;
+        double p = exp(lw);
+        double lo = 0.5 * (1.0 + p);
+        double capped = isnan(k) ? k : (k < cap ? k : cap);
+        wt = isnan(capped) ? capped : (capped > lo ? capped : lo);
+        tr = logk > log1p(P->lambda * phi) || logk < log(lo);
+        break;
+    }
+    case OR_MODE_ICEPOP: {
+        /* Table 8: k kept on [a, b] (bounds included), else masked to 0. */
+        int out = logk < log(P->icepop_lo) || logk > log(P->icepop_hi);
+        wt = out ? 0.0 : k;
+        tr = out;
+        break;
+    }
+    case OR_MODE_KPOP: {
+        /* Table 8 / App. D.5: binary KL both ways, fp64, p and q clamped to
+         * [1e-8, 1 - 1e-8]; masked when the larger exceeds phi. */
+        const double lo = 1e-8, hi = 1.0 - 1e-8;
+        double p = exp(lw), q = exp(linf);
+        p = p < lo ? lo : (p > hi ? hi : p);
+        q = q < lo ? lo : (q > hi ? hi : q);
+        double kl_pq = p * log(p / q) + (1.0 - p) * log((1.0 - p) / (1.0 - q));
+        double kl_qp = q * log(q / p) + (1.0 - q) * log((1.0 - q) / (1.0 - p));
+        double m = kl_pq > kl_qp ? kl_pq : kl_qp;
+        int out = m > P->kpop_phi;
+        wt = out ? 0.0 : k;
+        tr = out;
+        break;
+    }
+    case OR_MODE_SEQ_TIS:
+    case OR_MODE_SEQ_MIS:
+        /* sequence operators: the weight comes from the response's product */
+        wt = 0.0;
+        tr = 0;
+        break;
     default: /* OR_MODE_NONE: weight 1. */
         wt = 1.0;
         tr = 0;
@@ -229,26 +298,81 @@ static void token_weight(double lw, double linf, const oracle_params_t *P, doubl
 }
 
 /*
- * Elementwise weights for T tokens (Algorithm 1 / Table 8).  Masked tokens get
- * w = 0, trunc = 0, logk = eps = 0.
+ * The weight of every token of a response from the response's log K =
+ * sum of log k over its valid tokens (Table 8: Seq-TIS min(K, C), Seq-MIS
+ * K 1{K in [a, b]}).
  */
-void oracle_weights(const double *lp_w, const double *lp_inf, const uint8_t *mask, int64_t T,
-                    const oracle_params_t *P, double *w_out, uint8_t *trunc_out,
-                    double *logk_out, double *eps_out)
+static void seq_weight(double logK, const oracle_params_t *P, double *w, int *trunc)
 {
+    double K = exp(logK);
+    if (P->mode == OR_MODE_SEQ_TIS) {
+        double cap = P->seq_cap;
+        *w = isnan(K) ? K : (K < cap ? K : cap);
+        *trunc = logK > log(cap);
+    } else {
+        int out = logK < log(P->seq_lo) || logK > log(P->seq_hi);
+        *w = out ? 0.0 : K;
+        *trunc = out;
+    }
+}
+
+/*
+ * Weights for T tokens (Algorithm 1 / Table 8).  Masked tokens get w = 0,
+ * trunc = 0, logk = eps = 0.  The sequence operators need cu_seqlens (B + 1
+ * offsets); `skip` (may be NULL) marks tokens left out of the products.
+ * Returns 0, or -1 for a sequence operator without cu_seqlens.
+ */
+static int weights_impl(const double *lp_w, const double *lp_inf, const uint8_t *mask,
+                        const uint8_t *skip, int64_t T, const int32_t *cu_seqlens, int64_t B,
+                        const oracle_params_t *P, double *w_out, uint8_t *trunc_out,
+                        double *logk_out, double *eps_out)
+{
+    if (is_seq_mode(P->mode) && cu_seqlens == NULL)
+        return -1;
+    double *lk = (double *)malloc(sizeof(double) * (size_t)(T > 0 ? T : 1));
+    if (!lk)
+        return -2;
     for (int64_t t = 0; t < T; ++t) {
-        double w = 0.0, lk = 0.0, e = 0.0;
+        double w = 0.0, e = 0.0;
         int tr = 0;
+        lk[t] = 0.0;
         if (row_valid(mask, t))
-            token_weight(lp_w[t], lp_inf[t], P, &w, &tr, &lk, &e);
+            token_weight(lp_w[t], lp_inf[t], P, &w, &tr, &lk[t], &e);
         w_out[t] = w;
         if (trunc_out)
             trunc_out[t] = (uint8_t)tr;
         if (logk_out)
-            logk_out[t] = lk;
+            logk_out[t] = lk[t];
         if (eps_out)
             eps_out[t] = e;
     }
+    if (is_seq_mode(P->mode)) {
+        for (int64_t i = 0; i < B; ++i) {
+            double logK = 0.0;
+            for (int64_t t = cu_seqlens[i]; t < cu_seqlens[i + 1]; ++t)
+                if (row_valid(mask, t) && !(skip && skip[t]))
+                    logK += lk[t];
+            double w;
+            int tr;
+            seq_weight(logK, P, &w, &tr);
+            for (int64_t t = cu_seqlens[i]; t < cu_seqlens[i + 1]; ++t)
+                if (row_valid(mask, t) && !(skip && skip[t])) {
+                    w_out[t] = w;
+                    if (trunc_out)
+                        trunc_out[t] = (uint8_t)tr;
+                }
+        }
+    }
+    free(lk);
+    return 0;
+}
+
+int oracle_weights(const double *lp_w, const double *lp_inf, const uint8_t *mask, int64_t T,
+                   const int32_t *cu_seqlens, int64_t B, const oracle_params_t *P,
+                   double *w_out, uint8_t *trunc_out, double *logk_out, double *eps_out)
+{
+    return weights_impl(lp_w, lp_inf, mask, NULL, T, cu_seqlens, B, P, w_out, trunc_out,
+                        logk_out, eps_out);
 }
 
 /*
@@ -306,7 +430,8 @@ void oracle_loss_scales(const uint8_t *mask, int64_t T, const int32_t *cu_seqlen
  * finite differences).  dz is written for the rows listed in `rows` (nrows of
  * them, dz_out is [nrows, V]); rows == NULL means every row (dz_out [T, V]).
  * Per-token outputs (lp, lse, w, trunc, loss_terms, c) are for all T rows.
- * Returns 0, or -1 if a valid row has an out-of-range id.
+ * Returns 0, -1 if a valid row has an out-of-range id, -3 for a sequence
+ * operator without cu_seqlens.
  */
 int oracle_loss_fwd_bwd(const void *logits, int dtype, int64_t T, int64_t V, int64_t ld,
                         const int32_t *ids, const double *lp_inf, const double *lp_old,
@@ -329,27 +454,71 @@ int oracle_loss_fwd_bwd(const void *logits, int dtype, int64_t T, int64_t V, int
         return -2;
     }
     oracle_loss_scales(mask, T, cu_seqlens, B, P->agg, s);
+    double *lpv = (double *)malloc(sizeof(double) * nT);
+    double *lwv = (double *)malloc(sizeof(double) * nT);
+    double *wv = (double *)malloc(sizeof(double) * nT);
+    uint8_t *trv = (uint8_t *)malloc(nT);
+    uint8_t *badv = (uint8_t *)malloc(nT);
+    if (!lpv || !lwv || !wv || !trv || !badv) {
+        free(s);
+        free(lse);
+        free(cc);
+        free(terms);
+        free(lpv);
+        free(lwv);
+        free(wv);
+        free(trv);
+        free(badv);
+        return -2;
+    }
     int bad = 0;
     set_threads(nthreads);
+    /* 1. log p of every valid row (Sec. 2.1) */
 #pragma omp parallel for schedule(dynamic, 4) reduction(| : bad)
     for (int64_t t = 0; t < T; ++t) {
-        double lp = 0.0, ls = 0.0, w = 0.0, term = 0.0, c = 0.0;
-        int tr = 0;
+        double lp = 0.0, ls = 0.0;
+        badv[t] = 0;
         if (row_valid(mask, t)) {
             int32_t y = ids[t];
             if (y < 0 || (int64_t)y >= V) {
                 bad = 1;
+                badv[t] = 1;
                 lp = NAN;
                 ls = NAN;
-                term = NAN;
             } else {
                 ls = row_lse(logits, dtype, ld, t, V);
                 lp = logit_at(logits, dtype, ld, t, y) - ls;
-                double lw = lp_old ? lp_old[t] : lp;
-                double lk;
-                token_weight(lw, lp_inf[t], P, &w, &tr, &lk, NULL);
-                if (w_fixed)
-                    w = w_fixed[t];
+            }
+        }
+        lse[t] = ls;
+        lpv[t] = lp;
+        lwv[t] = lp_old ? lp_old[t] : lp;
+    }
+    /* 2. the weights (Algorithm 1 / Table 8), per token or per response */
+    int rc = weights_impl(lwv, lp_inf, mask, badv, T, cu_seqlens, B, P, wv, trv, NULL, NULL);
+    if (rc != 0) {
+        free(s);
+        free(lse);
+        free(cc);
+        free(terms);
+        free(lpv);
+        free(lwv);
+        free(wv);
+        free(trv);
+        free(badv);
+        return rc == -1 ? -3 : -2;
+    }
+    /* 3. the token terms of Eq. 1 and c_t */
+    for (int64_t t = 0; t < T; ++t) {
+        double w = 0.0, term = 0.0, c = 0.0;
+        int tr = 0;
+        if (row_valid(mask, t)) {
+            if (badv[t]) {
+                term = NAN;
+            } else {
+                double lp = lpv[t];
+                w = w_fixed ? w_fixed[t] : wv[t];
+                tr = trv[t];
                 /* Eq. 1: rho = pi_theta / p_old, clipped to [1-c_low, 1+c_high]. */
                 double rho = lp_old ? exp(lp - lp_old[t]) : 1.0;
                 double A = adv[t];
@@ -366,15 +535,19 @@ int oracle_loss_fwd_bwd(const void *logits, int dtype, int64_t T, int64_t V, int
                 c = s[t] * w * A * rho * (double)g;
             }
         }
-        lse[t] = ls;
         cc[t] = c;
         terms[t] = term;
-        lp_out[t] = lp;
+        lp_out[t] = lpv[t];
         if (w_out)
             w_out[t] = w;
         if (trunc_out)
             trunc_out[t] = (uint8_t)tr;
     }
+    free(lpv);
+    free(lwv);
+    free(wv);
+    free(trv);
+    free(badv);
     /* loss = -sum_t s_t J_t, summed in index order. */
     double loss = 0.0;
     for (int64_t t = 0; t < T; ++t)

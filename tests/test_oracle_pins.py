@@ -327,7 +327,9 @@ def _fd_setup(seed, T, V):
 
 
 @pytest.mark.parametrize("V", [2, 5, 8])
-@pytest.mark.parametrize("mode", [oracle.MODE_CIS, oracle.MODE_TIS, oracle.MODE_EXACT])
+@pytest.mark.parametrize("mode", [oracle.MODE_CIS, oracle.MODE_TIS, oracle.MODE_EXACT,
+                                  oracle.MODE_BAND, oracle.MODE_ICEPOP, oracle.MODE_KPOP,
+                                  oracle.MODE_SEQ_TIS, oracle.MODE_SEQ_MIS])
 def test_gradient_matches_central_finite_differences(V, mode):
     """d loss / d z from the oracle equals central differences of its loss with
     the weight frozen (stopgrad, Algorithm 1) and log p_old fixed.  Rows cover
@@ -365,7 +367,9 @@ def test_gradient_matches_central_finite_differences(V, mode):
         assert scale > 0
         np.testing.assert_allclose(dz, fd, rtol=0, atol=1e-7 * scale)
         assert np.all(dz[1] == 0) and np.all(dz[3] == 0) and np.all(dz[5] == 0)
-        assert np.abs(dz[2]).max() > 0 and np.abs(dz[0]).max() > 0
+        for t in (0, 2):  # rows whose operator keeps a weight carry a gradient
+            assert (np.abs(dz[t]).max() > 0) == (w0[t] != 0)
+        assert np.abs(dz).max() > 0
 
 
 def test_on_policy_gradient_equals_snapshot_gradient_at_rho_one():
@@ -440,3 +444,156 @@ def test_lmhead_chain_rule_matches_finite_differences():
     scale = max(np.abs(base["dhidden"]).max(), np.abs(base["dweight"]).max())
     np.testing.assert_allclose(base["dhidden"], fdH, rtol=0, atol=1e-8 * scale)
     np.testing.assert_allclose(base["dweight"], fdW, rtol=0, atol=1e-8 * scale)
+
+
+# ---------------------------------------------- the other operators of Table 8
+def _from_p_eps(p, eps):
+    """log p and log q of tokens with training probability p and log-odds
+    displacement eps (Lemma 3.1: logit q = logit p - eps)."""
+    p = np.asarray(p, np.float64)
+    lq = -np.logaddexp(0.0, -(np.log(p) - np.log1p(-p) - eps))
+    return np.log(p), lq
+
+
+def test_new_operator_defaults_are_the_papers():
+    """Table 8 / App. D.5 hyper-parameters are the oracle's defaults."""
+    P = oracle.params()
+    assert [P.icepop_lo, P.icepop_hi] == GOLDEN["icepop_band"]["value"]
+    assert P.kpop_phi == GOLDEN["kpop_phi"]["value"]
+    assert P.seq_cap == GOLDEN["seq_tis_cap"]["value"]
+    assert [P.seq_lo, P.seq_hi] == GOLDEN["seq_mis_band"]["value"]
+
+
+def test_band_lifts_exactly_where_displacement_is_below_half():
+    """Two-sided band (Sec. 4.3): the lower bound (1 + p)/2 is the image of
+    e^eps = 1/2 under k = p + (1 - p) e^eps, so a token is lifted iff
+    e^eps < 1/2; everywhere else the band weight is the CIS weight."""
+    half = GOLDEN["band_lower_displacement"]["value"]
+    rng = _rng(41)
+    p = rng.uniform(0.01, 0.99, 4000)
+    eps = rng.uniform(-3.0, 3.0, 4000)
+    eps[np.abs(eps - math.log(half)) < 1e-6] += 1e-3  # keep clear of the boundary
+    lw, lq = _from_p_eps(p, eps)
+    wb, trb, _, _ = oracle.weights(lw, lq, oracle.params(mode=oracle.MODE_BAND))
+    wc, trc, _, _ = oracle.weights(lw, lq, oracle.params(mode=oracle.MODE_CIS))
+    lifted = np.exp(eps) < half
+    np.testing.assert_allclose(wb[lifted], (1.0 + p[lifted]) / 2.0, rtol=1e-14)
+    assert np.all(wb[~lifted] == wc[~lifted])
+    assert np.all(trb == (trc.astype(bool) | lifted))
+    assert np.all(wb >= (1.0 + p) / 2.0 * (1 - 1e-15))
+    # on the boundary e^eps = 1/2 exactly: k = (1 + p)/2, not lifted (the min ties)
+    lw1, lq1 = _from_p_eps([0.3], [math.log(half)])
+    w1, _, lk1, _ = oracle.weights(lw1, lq1, oracle.params(mode=oracle.MODE_BAND))
+    assert math.exp(lk1[0]) == pytest.approx(0.65, rel=1e-14)
+    assert w1[0] == pytest.approx(0.65, rel=1e-14)
+
+
+def test_icepop_keeps_k_inside_its_band_and_masks_outside():
+    """IcePop (Table 8): k on [0.5, 5] (bounds included), 0 outside; with a
+    band wide enough to hold every ratio it is the unclamped exact ratio."""
+    lo, hi = GOLDEN["icepop_band"]["value"]
+    rng = _rng(42)
+    lw = np.log(rng.uniform(0.01, 1.0, 3000))
+    linf = lw - rng.uniform(-3.0, 3.0, 3000)
+    k = np.exp(lw - linf)
+    w, tr, _, _ = oracle.weights(lw, linf, oracle.params(mode=oracle.MODE_ICEPOP))
+    inside = (k >= lo * (1 + 1e-12)) & (k <= hi * (1 - 1e-12))
+    outside = (k < lo * (1 - 1e-12)) | (k > hi * (1 + 1e-12))
+    np.testing.assert_allclose(w[inside], k[inside], rtol=1e-14)
+    assert np.all(w[outside] == 0.0) and np.all(tr[outside] == 1) and np.all(tr[inside] == 0)
+    # exactly on the bounds: kept
+    wb, trb, _, _ = oracle.weights(np.array([math.log(0.5), 0.0]),
+                                   np.array([0.0, -math.log(5.0)]),
+                                   oracle.params(mode=oracle.MODE_ICEPOP))
+    assert trb.tolist() == [0, 0] and wb[0] == pytest.approx(0.5) and wb[1] == pytest.approx(5.0)
+    wide, _, _, _ = oracle.weights(lw, linf, oracle.params(mode=oracle.MODE_ICEPOP,
+                                                           icepop_lo=1e-300, icepop_hi=1e300))
+    np.testing.assert_allclose(wide, k, rtol=1e-14)
+
+
+def test_kpop_mask_matches_binary_kl_from_library_entropy():
+    """KPop-dagger (Table 8, App. D.5): the binary KL both ways, recomputed with
+    scipy's relative entropy on the clamped probabilities; masked iff the
+    larger exceeds phi = 2 (decided away from the threshold)."""
+    special = pytest.importorskip("scipy.special")
+    lo, hi = GOLDEN["kpop_clamp"]["value"]
+    phi = GOLDEN["kpop_phi"]["value"]
+    rng = _rng(43)
+    n = 4000
+    lw = np.log(rng.uniform(1e-4, 1.0, n))
+    linf = np.log(rng.uniform(1e-4, 1.0, n))
+    w, tr, lk, _ = oracle.weights(lw, linf, oracle.params(mode=oracle.MODE_KPOP))
+    p = np.clip(np.exp(lw), lo, hi)
+    q = np.clip(np.exp(linf), lo, hi)
+    kl = lambda a, b: special.rel_entr(a, b) + special.rel_entr(1 - a, 1 - b)  # noqa: E731
+    m = np.maximum(kl(p, q), kl(q, p))
+    clear = np.abs(m - phi) > 1e-9
+    assert np.all((tr == 1)[clear] == (m > phi)[clear])
+    assert np.all(w[tr == 1] == 0.0)
+    keep = tr == 0
+    np.testing.assert_allclose(w[keep], np.exp(lk[keep]), rtol=1e-15)
+    assert 0 < tr.sum() < n
+    # saturation (App. D.5): probability one on both engines is kept (metric 0
+    # after the representable clamp); one on one engine only is masked when the
+    # other is far from it (q = 0.5: KL(q||p) = 0.5 log(0.5 / 1e-8) + ... > 2),
+    # kept when it is close (q = 0.999: about 0.012)
+    w2, tr2, _, _ = oracle.weights(np.array([0.0, 0.0, 0.0]),
+                                   np.array([0.0, math.log(0.5), math.log(0.999)]),
+                                   oracle.params(mode=oracle.MODE_KPOP))
+    assert tr2.tolist() == [0, 1, 0]
+    assert w2[0] == 1.0 and w2[1] == 0.0 and w2[2] == pytest.approx(1 / 0.999)
+
+
+def test_sequence_operators_use_the_product_over_each_response():
+    """Seq-TIS min(K, C) and Seq-MIS K 1{K in [0.5, 2]} (Table 8), K the
+    product of k over the valid tokens of a response: checked against the
+    product of the per-token ratios; masked tokens are left out of K and get
+    weight 0, and a token outside every response gets 0."""
+    rng = _rng(44)
+    T = 40
+    lw = np.log(rng.uniform(0.05, 1.0, T))
+    linf = lw - rng.normal(0.0, 0.3, T)
+    mask = np.ones(T, np.uint8)
+    mask[[3, 17, 30]] = 0
+    cu = np.array([0, 1, 6, 18, 25, 37], np.int32)  # tokens 37..39 in no response
+    k = np.exp(lw - linf)
+    C = GOLDEN["seq_tis_cap"]["value"]
+    lo, hi = GOLDEN["seq_mis_band"]["value"]
+    wt, trt, _, _ = oracle.weights(lw, linf, oracle.params(mode=oracle.MODE_SEQ_TIS), mask=mask,
+                                   cu_seqlens=cu)
+    wm, trm, _, _ = oracle.weights(lw, linf, oracle.params(mode=oracle.MODE_SEQ_MIS), mask=mask,
+                                   cu_seqlens=cu)
+    for i in range(len(cu) - 1):
+        sl = slice(cu[i], cu[i + 1])
+        v = mask[sl] == 1
+        K = float(np.prod(k[sl][v]))
+        assert np.allclose(wt[sl][v], min(K, C), rtol=1e-12)
+        assert np.all(trt[sl][v] == (K > C))
+        kept = lo <= K <= hi
+        assert np.allclose(wm[sl][v], K if kept else 0.0, rtol=1e-12)
+        assert np.all(trm[sl][v] == (not kept))
+        assert np.all(wt[sl][~v] == 0) and np.all(wm[sl][~v] == 0)
+    assert np.all(wt[37:] == 0) and np.all(wm[37:] == 0)
+    with pytest.raises(ValueError):
+        oracle.weights(lw, linf, oracle.params(mode=oracle.MODE_SEQ_TIS))
+
+
+def test_sequence_operators_on_one_token_responses_are_token_operators():
+    """With every response one token long, Seq-TIS is TIS with the same C and
+    Seq-MIS is IcePop with the same band."""
+    rng = _rng(45)
+    T = 500
+    lw = np.log(rng.uniform(0.01, 1.0, T))
+    linf = lw - rng.normal(0.0, 1.0, T)
+    cu = np.arange(T + 1, dtype=np.int32)
+    ws, trs, _, _ = oracle.weights(lw, linf, oracle.params(mode=oracle.MODE_SEQ_TIS),
+                                   cu_seqlens=cu)
+    wt, trt, _, _ = oracle.weights(lw, linf, oracle.params(mode=oracle.MODE_TIS))
+    np.testing.assert_allclose(ws, wt, rtol=1e-15)
+    assert np.all(trs == trt)
+    wm, trm, _, _ = oracle.weights(lw, linf, oracle.params(mode=oracle.MODE_SEQ_MIS),
+                                   cu_seqlens=cu)
+    wi, tri, _, _ = oracle.weights(lw, linf, oracle.params(mode=oracle.MODE_ICEPOP,
+                                                           icepop_lo=0.5, icepop_hi=2.0))
+    np.testing.assert_allclose(wm, wi, rtol=1e-15)
+    assert np.all(trm == tri)
