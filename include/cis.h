@@ -67,13 +67,24 @@ typedef enum {
 
 typedef enum { CIS_F32 = 0, CIS_BF16 = 1 } cis_dtype_t;
 
-/* Weight operators: CIS is Eq. 4 with the floor of Algorithm 1; the others are
- * the token-level rows of Table 8. */
+/* Weight operators: CIS is Eq. 4 with the floor of Algorithm 1; the band is
+ * the two-sided ablation of Sec. 4.3; the others are the rows of Table 8.
+ * p = exp(lp_train), k = exp(lp_train - lp_infer), phi = max(1 - p, kappa).
+ * The sequence operators use K, the product of k over the valid tokens of a
+ * response (cu_seqlens), and give every token of the response the same
+ * weight. */
 typedef enum {
-    CIS_MODE_CIS = 0,   /* w = min{k, 1 + lambda*max(1-p, kappa)}            */
-    CIS_MODE_TIS = 1,   /* w = min(k, tis_cap)                               */
-    CIS_MODE_EXACT = 2, /* w = k clamped to [exact_lo, exact_hi]             */
-    CIS_MODE_NONE = 3   /* w = 1                                             */
+    CIS_MODE_CIS = 0,     /* w = min{k, 1 + lambda*phi}                        */
+    CIS_MODE_TIS = 1,     /* w = min(k, tis_cap)                               */
+    CIS_MODE_EXACT = 2,   /* w = k clamped to [exact_lo, exact_hi]             */
+    CIS_MODE_NONE = 3,    /* w = 1                                             */
+    CIS_MODE_BAND = 4,    /* w = max{min{k, 1 + lambda*phi}, (1 + p)/2}        */
+    CIS_MODE_ICEPOP = 5,  /* w = k if k in [icepop_lo, icepop_hi], else 0      */
+    CIS_MODE_KPOP = 6,    /* w = k if max(KL_B(p||q), KL_B(q||p)) <= kpop_phi,
+                           *     else 0; fp64, p and q clamped to
+                           *     [1e-8, 1 - 1e-8] (App. D.5)                   */
+    CIS_MODE_SEQ_TIS = 7, /* w = min(K, seq_cap)                               */
+    CIS_MODE_SEQ_MIS = 8  /* w = K if K in [seq_lo, seq_hi], else 0           */
 } cis_mode_t;
 
 /* Loss normaliser: Algorithm 1 averages over the n tokens of the batch; Eq. 1
@@ -83,9 +94,10 @@ typedef enum {
     CIS_AGG_SEQ_MEAN_TOKEN_MEAN = 1/* s_t = 1/(G |y_i|) from cu_seqlens and mask */
 } cis_agg_t;
 
-/* Hyper-parameters.  Defaults (cis_default_params): the deployed CIS of
+/* Hyper-parameters.  Defaults (cis_default_params): the deployed values of
  * App. C.1 / Table 8: lambda 2.3, kappa 5e-3, TIS cap 2, exact clamp
- * [1e-6, 1e6], PPO clip (0.2, 0.28), token mean. */
+ * [1e-6, 1e6], IcePop [0.5, 5], KPop phi 2, Seq-TIS cap 2, Seq-MIS [0.5, 2],
+ * PPO clip (0.2, 0.28), token mean. */
 typedef struct {
     int32_t mode;      /* cis_mode_t                                         */
     int32_t agg;       /* cis_agg_t                                          */
@@ -96,6 +108,12 @@ typedef struct {
     double exact_hi;   /* >= exact_lo                                        */
     double clip_low;   /* in [0, 1): rho clipped below at 1 - clip_low       */
     double clip_high;  /* >= 0: rho clipped above at 1 + clip_high           */
+    double icepop_lo;  /* >= 0: IcePop band, bounds included                 */
+    double icepop_hi;  /* >= icepop_lo                                       */
+    double kpop_phi;   /* >= 0: KPop threshold on the binary KL              */
+    double seq_cap;    /* > 0: C of Seq-TIS                                  */
+    double seq_lo;     /* >= 0: Seq-MIS band, bounds included                */
+    double seq_hi;     /* >= seq_lo                                          */
 } cis_params_t;
 
 /* Reduction outputs of cis_loss_fwd_bwd, written on the device. */
@@ -103,7 +121,8 @@ typedef struct {
     double loss;          /* -sum_t s_t m_t w_t min(rho A, clip(rho) A)       */
     double trunc_excess;  /* sum over truncated tokens of (k_t - w_t)         */
     int64_t n_valid;      /* number of tokens with mask != 0                  */
-    int64_t n_truncated;  /* tokens whose weight was truncated or clamped     */
+    int64_t n_truncated;  /* tokens whose weight the operator changed: capped,
+                           * clamped, lifted (band) or masked                 */
     float max_abs_logk;   /* max over valid tokens of |log k_t|               */
     int32_t status;       /* OR of device status bits (cis_status_t)          */
 } cis_stats_t;
@@ -134,26 +153,34 @@ CIS_API cis_status_t cis_token_logprobs(const void *logits, int32_t dtype, int64
                                 void *stream);
 
 /*
- * Elementwise weights (Algorithm 1, Eq. 4, Table 8) from fp32 log-probabilities.
+ * Weights (Algorithm 1, Eq. 4, Table 8) from fp32 log-probabilities.
  *   lp_train  device float [T]: log p_t, the training-side log-probability
  *             the weight is built from (l_old when updating off the snapshot).
  *   lp_infer  device float [T]: log q_t, the raw value recorded at sampling.
  *   mask      device uint8 [T] or NULL.
+ *   cu_seqlens device int32 [B + 1] or NULL: response boundaries (non-
+ *             decreasing, cu_seqlens[B] <= T; not checked on the host).
+ *             Required by the sequence operators (CIS_ERR_INVALID_ARG
+ *             without); ignored by the others.  A valid token outside every
+ *             response gets weight 0 under a sequence operator.
  *   w_out     device float [T]: the weight (0 for masked tokens).
- *   trunc_out device uint8 [T] or NULL: 1 where the weight differs from k
- *             (CIS/TIS: k above the cap; EXACT: k outside the clamp).
+ *   trunc_out device uint8 [T] or NULL: 1 where the operator changed the
+ *             weight from k (capped, clamped, lifted or masked); under a
+ *             sequence operator, the response's flag.
  *   eps_out   device float [T] or NULL: the log-odds displacement
  *             eps = logit p - logit q (Lemma 3.1); +-inf or NaN where p or q
  *             rounds to 1 (the weight itself stays finite).
- * The truncation decision is taken as log k > log cap with log k = lp_train -
- * lp_infer evaluated exactly; fp32 arithmetic is used where its error bound
- * proves the answer and fp64 otherwise, so decisions equal those of an fp64
- * evaluation.  Errors: CIS_ERR_INVALID_ARG for NULL required pointers, T < 0
- * or parameters outside the ranges of cis_params_t.
+ * Decisions are taken on log k = lp_train - lp_infer, evaluated exactly: CIS,
+ * TIS and EXACT compare with log cap in fp32 where its error bound proves the
+ * answer and in fp64 otherwise; the band, IcePop, KPop and the sequence
+ * operators (log K summed in fp64) decide in fp64.  Errors:
+ * CIS_ERR_INVALID_ARG for NULL required pointers, T < 0, parameters outside
+ * the ranges of cis_params_t, or a sequence operator without cu_seqlens.
  */
 CIS_API cis_status_t cis_weights(const float *lp_train, const float *lp_infer, const uint8_t *mask,
-                         int64_t T, const cis_params_t *params, float *w_out,
-                         uint8_t *trunc_out, float *eps_out, void *stream);
+                         int64_t T, const int32_t *cu_seqlens, int64_t B,
+                         const cis_params_t *params, float *w_out, uint8_t *trunc_out,
+                         float *eps_out, void *stream);
 
 /* Bytes of device workspace cis_loss_fwd_bwd needs for T tokens and
  * vocabulary V.  Host only.  CIS_ERR_INVALID_ARG if bytes is NULL or T < 0. */
@@ -173,8 +200,9 @@ CIS_API cis_status_t cis_loss_workspace_size(int64_t T, int64_t V, size_t *bytes
  *   mask        device uint8 [T] or NULL.
  *   cu_seqlens  device int32 [B + 1] or NULL: response boundaries, needed for
  *               CIS_AGG_SEQ_MEAN_TOKEN_MEAN (tokens outside every response
- *               then get s_t = 0).  Must be non-decreasing with
- *               cu_seqlens[B] <= T; not checked on the host.
+ *               then get s_t = 0) and by the sequence operators.  Must be
+ *               non-decreasing with cu_seqlens[B] <= T; not checked on the
+ *               host.
  *   params      host pointer.
  *   dlogits     device, [T, ld_out] of `dlogits_dtype` (CIS_BF16 rounds to
  *               nearest even, CIS_F32); every element j < V of every row is
@@ -186,10 +214,14 @@ CIS_API cis_status_t cis_loss_workspace_size(int64_t T, int64_t V, size_t *bytes
  *               aligned; its first int32 is the device status word, zeroed
  *               by this call.
  * Sums are deterministic: the same inputs give bit-identical outputs.
+ * The sequence operators need every log p of a response before any weight:
+ * with lp_old the weights are formed first and the pass is unchanged;
+ * without it a forward pass (one more read of the logits) gives the log p.
+ * A token with an out-of-range id is left out of its response's product.
  * Errors: CIS_ERR_INVALID_ARG for NULL required pointers, T < 0, V <= 0,
  * ld < V, ld_out < V, bad parameters, a short or misaligned workspace, or
- * CIS_AGG_SEQ_MEAN_TOKEN_MEAN without cu_seqlens; CIS_ERR_CUDA if a launch
- * fails.
+ * CIS_AGG_SEQ_MEAN_TOKEN_MEAN or a sequence operator without cu_seqlens;
+ * CIS_ERR_CUDA if a launch fails.
  */
 CIS_API cis_status_t cis_loss_fwd_bwd(const void *logits, int32_t dtype, int64_t T, int64_t V,
                               int64_t ld, const int32_t *ids, const float *lp_infer,
@@ -226,7 +258,9 @@ CIS_API cis_status_t cis_loss_host_workspace_size(int64_t T, int64_t V, int32_t 
  * device (one per staging buffer and direction).  The
  * normaliser and the loss cover the whole batch, so every output equals that
  * of cis_loss_fwd_bwd.  Asynchronous on `stream`: the host outputs are valid
- * once `stream` has completed the call's work.  Errors: as cis_loss_fwd_bwd.
+ * once `stream` has completed the call's work.  Errors: as cis_loss_fwd_bwd,
+ * plus CIS_ERR_UNSUPPORTED for a sequence operator without lp_old (its
+ * weights would need every row's log p before the first chunk's dlogits).
  */
 CIS_API cis_status_t cis_loss_fwd_bwd_host(
     const void *logits, int32_t dtype, int64_t T, int64_t V, const int32_t *ids,

@@ -21,8 +21,11 @@ CIS_F32, CIS_BF16 = 0, 1
 CIS_MODE_CIS, CIS_MODE_TIS, CIS_MODE_EXACT, CIS_MODE_NONE = 0, 1, 2, 3
 CIS_AGG_TOKEN_MEAN, CIS_AGG_SEQ_MEAN_TOKEN_MEAN = 0, 1
 
+CIS_MODE_BAND, CIS_MODE_ICEPOP, CIS_MODE_KPOP, CIS_MODE_SEQ_TIS, CIS_MODE_SEQ_MIS = 4, 5, 6, 7, 8
 MODES = {"cis": CIS_MODE_CIS, "tis": CIS_MODE_TIS, "exact": CIS_MODE_EXACT,
-         "none": CIS_MODE_NONE}
+         "none": CIS_MODE_NONE, "band": CIS_MODE_BAND, "icepop": CIS_MODE_ICEPOP,
+         "kpop": CIS_MODE_KPOP, "seq_tis": CIS_MODE_SEQ_TIS, "seq_mis": CIS_MODE_SEQ_MIS}
+SEQ_MODES = ("seq_tis", "seq_mis")
 
 
 class cis_params_t(ctypes.Structure):
@@ -36,6 +39,12 @@ class cis_params_t(ctypes.Structure):
         ("exact_hi", ctypes.c_double),
         ("clip_low", ctypes.c_double),
         ("clip_high", ctypes.c_double),
+        ("icepop_lo", ctypes.c_double),
+        ("icepop_hi", ctypes.c_double),
+        ("kpop_phi", ctypes.c_double),
+        ("seq_cap", ctypes.c_double),
+        ("seq_lo", ctypes.c_double),
+        ("seq_hi", ctypes.c_double),
     ]
 
 
@@ -77,7 +86,7 @@ def lib():
     L.cis_status_string.restype = ctypes.c_char_p
     L.cis_token_logprobs.argtypes = [P, i32, i64, i64, i64, P, P, P, P, P, P]
     L.cis_token_logprobs.restype = ctypes.c_int
-    L.cis_weights.argtypes = [P, P, P, i64, ctypes.POINTER(cis_params_t), P, P, P, P]
+    L.cis_weights.argtypes = [P, P, P, i64, P, i64, ctypes.POINTER(cis_params_t), P, P, P, P]
     L.cis_weights.restype = ctypes.c_int
     L.cis_loss_workspace_size.argtypes = [i64, i64, ctypes.POINTER(ctypes.c_size_t)]
     L.cis_loss_workspace_size.restype = ctypes.c_int
@@ -155,7 +164,8 @@ def _vec(x, dtype, T, name):
 
 def cis_default_params(mode="cis", **kw) -> cis_params_t:
     """Defaults of App. C.1 / Table 8, with keyword overrides (lam, kappa, tis_cap,
-    exact_lo, exact_hi, clip_low, clip_high, agg)."""
+    exact_lo, exact_hi, clip_low, clip_high, agg, icepop_lo, icepop_hi, kpop_phi,
+    seq_cap, seq_lo, seq_hi)."""
     p = cis_params_t()
     _check(lib().cis_default_params(ctypes.byref(p)), "cis_default_params")
     p.mode = MODES[mode] if isinstance(mode, str) else int(mode)
@@ -181,19 +191,24 @@ def cis_token_logprobs(logits: torch.Tensor, ids: torch.Tensor, mask=None, V=Non
 
 
 def cis_weights(lp_train: torch.Tensor, lp_infer: torch.Tensor, params: cis_params_t,
-                mask=None, want_trunc=True, want_eps=False):
-    """Weights of Algorithm 1 / Table 8.  Returns (w, trunc or None, eps or None)."""
-    _need_cuda(lp_train, lp_infer, mask)
+                mask=None, want_trunc=True, want_eps=False, cu_seqlens=None):
+    """Weights of Algorithm 1 / Table 8 (the sequence operators need
+    cu_seqlens).  Returns (w, trunc or None, eps or None)."""
+    _need_cuda(lp_train, lp_infer, mask, cu_seqlens)
     T = lp_train.shape[0]
     _vec(lp_train, torch.float32, T, "lp_train")
     _vec(lp_infer, torch.float32, T, "lp_infer")
     _vec(mask, torch.uint8, T, "mask")
+    if cu_seqlens is not None and (cu_seqlens.dtype != torch.int32 or
+                                   not cu_seqlens.is_contiguous()):
+        raise TypeError("cu_seqlens must be contiguous int32")
+    B = 0 if cu_seqlens is None else cu_seqlens.shape[0] - 1
     dev = lp_train.device
     w = torch.empty(T, dtype=torch.float32, device=dev)
     tr = torch.empty(T, dtype=torch.uint8, device=dev) if want_trunc else None
     eps = torch.empty(T, dtype=torch.float32, device=dev) if want_eps else None
-    rc = lib().cis_weights(_ptr(lp_train), _ptr(lp_infer), _ptr(mask), T, ctypes.byref(params),
-                           _ptr(w), _ptr(tr), _ptr(eps), _stream())
+    rc = lib().cis_weights(_ptr(lp_train), _ptr(lp_infer), _ptr(mask), T, _ptr(cu_seqlens), B,
+                           ctypes.byref(params), _ptr(w), _ptr(tr), _ptr(eps), _stream())
     _check(rc, "cis_weights")
     return w, tr, eps
 

@@ -39,7 +39,7 @@ bool params_ok(const cis_params_t *p)
 {
     if (p == nullptr)
         return false;
-    if (p->mode < CIS_MODE_CIS || p->mode > CIS_MODE_NONE)
+    if (p->mode < CIS_MODE_CIS || p->mode > CIS_MODE_SEQ_MIS)
         return false;
     if (p->agg != CIS_AGG_TOKEN_MEAN && p->agg != CIS_AGG_SEQ_MEAN_TOKEN_MEAN)
         return false;
@@ -54,6 +54,14 @@ bool params_ok(const cis_params_t *p)
     if (!(p->clip_low >= 0.0 && p->clip_low < 1.0))
         return false;
     if (!finite_or_inf_nonneg(p->clip_high))
+        return false;
+    if (!(p->icepop_lo >= 0.0 && p->icepop_hi >= p->icepop_lo))
+        return false;
+    if (!finite_or_inf_nonneg(p->kpop_phi))
+        return false;
+    if (!(p->seq_cap > 0.0))
+        return false;
+    if (!(p->seq_lo >= 0.0 && p->seq_hi >= p->seq_lo))
         return false;
     return true;
 }
@@ -82,6 +90,13 @@ DevParams make_dev_params(const cis_params_t &p)
     d.log_exact_hi_f = (float)d.log_exact_hi;
     d.log_rho_lo_f = (float)d.log_rho_lo;
     d.log_rho_hi_f = (float)d.log_rho_hi;
+    d.log_icepop_lo = log(p.icepop_lo);
+    d.log_icepop_hi = log(p.icepop_hi);
+    d.kpop_phi = p.kpop_phi;
+    d.seq_cap = p.seq_cap;
+    d.log_seq_cap = log(p.seq_cap);
+    d.log_seq_lo = log(p.seq_lo);
+    d.log_seq_hi = log(p.seq_hi);
     return d;
 }
 
@@ -126,6 +141,12 @@ CIS_API cis_status_t cis_default_params(cis_params_t *out)
     out->exact_hi = 1e6;
     out->clip_low = 0.2;
     out->clip_high = 0.28;
+    out->icepop_lo = 0.5;
+    out->icepop_hi = 5.0;
+    out->kpop_phi = 2.0;
+    out->seq_cap = 2.0;
+    out->seq_lo = 0.5;
+    out->seq_hi = 2.0;
     return CIS_OK;
 }
 
@@ -169,18 +190,28 @@ CIS_API cis_status_t cis_token_logprobs(const void *logits, int32_t dtype, int64
 }
 
 CIS_API cis_status_t cis_weights(const float *lp_train, const float *lp_infer,
-                                 const uint8_t *mask, int64_t T, const cis_params_t *params,
-                                 float *w_out, uint8_t *trunc_out, float *eps_out, void *stream)
+                                 const uint8_t *mask, int64_t T, const int32_t *cu_seqlens,
+                                 int64_t B, const cis_params_t *params, float *w_out,
+                                 uint8_t *trunc_out, float *eps_out, void *stream)
 {
     if (T < 0 || !params_ok(params))
+        return CIS_ERR_INVALID_ARG;
+    const bool seq = is_seq_mode(params->mode);
+    if (seq && (cu_seqlens == nullptr || B < 0))
         return CIS_ERR_INVALID_ARG;
     if (T == 0)
         return CIS_OK;
     if (lp_train == nullptr || lp_infer == nullptr || w_out == nullptr)
         return CIS_ERR_INVALID_ARG;
     const DevParams P = make_dev_params(*params);
-    return cuda_status(launch_weights(lp_train, lp_infer, mask, T, P, w_out, trunc_out, eps_out,
-                                      (cudaStream_t)stream));
+    cudaStream_t s = (cudaStream_t)stream;
+    // per token first (a sequence operator leaves w = 0, trunc = 0 there), then
+    // the responses' weights over their valid tokens
+    cudaError_t e = launch_weights(lp_train, lp_infer, mask, T, P, w_out, trunc_out, eps_out, s);
+    if (e == cudaSuccess && seq)
+        e = launch_seq_weights(nullptr, lp_train, lp_infer, nullptr, 0, mask, cu_seqlens, B, T, P,
+                               w_out, trunc_out, s);
+    return cuda_status(e);
 }
 
 CIS_API cis_status_t cis_loss_workspace_size(int64_t T, int64_t V, size_t *bytes)
@@ -206,7 +237,8 @@ CIS_API cis_status_t cis_loss_fwd_bwd(const void *logits, int32_t dtype, int64_t
         return CIS_ERR_INVALID_ARG;
     if (!params_ok(params))
         return CIS_ERR_INVALID_ARG;
-    if (params->agg == CIS_AGG_SEQ_MEAN_TOKEN_MEAN && (cu_seqlens == nullptr || B < 0))
+    if ((params->agg == CIS_AGG_SEQ_MEAN_TOKEN_MEAN || is_seq_mode(params->mode)) &&
+        (cu_seqlens == nullptr || B < 0))
         return CIS_ERR_INVALID_ARG;
     const WsLayout L = ws_layout(T);
     if (workspace == nullptr || (reinterpret_cast<uintptr_t>(workspace) & 255) ||
@@ -252,6 +284,29 @@ CIS_API cis_status_t cis_loss_fwd_bwd(const void *logits, int32_t dtype, int64_t
                                   reinterpret_cast<float *>(ws + L.scale), a.status, s);
     if (e != cudaSuccess)
         return cuda_status(e);
+    if (T > 0 && is_seq_mode(params->mode)) {
+        // Sequence operator: every log p of a response before any weight.  The
+        // fp64 log p goes into the terms array (the pass overwrites it), the
+        // responses' weights into the weight and flag arrays, which the pass
+        // then reads (and writes back unchanged).
+        if (lp_old == nullptr) {
+            PassArgs f = a;
+            f.lp_inf = nullptr;
+            f.lp_out = nullptr;
+            f.lse_out = nullptr;
+            f.lp64_out = a.ws_terms;
+            if ((e = launch_token_logprobs(f, dtype, s)) != cudaSuccess)
+                return cuda_status(e);
+        }
+        if ((e = cudaMemsetAsync(a.ws_w, 0, 4 * (size_t)T, s)) != cudaSuccess ||
+            (e = cudaMemsetAsync(a.ws_trunc, 0, (size_t)T, s)) != cudaSuccess)
+            return cuda_status(e);
+        if ((e = launch_seq_weights(lp_old ? nullptr : a.ws_terms, lp_old, lp_infer, ids, V, mask,
+                                    cu_seqlens, B, T, a.P, a.ws_w, a.ws_trunc, s)) != cudaSuccess)
+            return cuda_status(e);
+        a.w_in = a.ws_w;
+        a.trunc_in = a.ws_trunc;
+    }
     cudaEvent_t ev0 = g_prof_begin, ev1 = g_prof_end;
     g_prof_begin = g_prof_end = nullptr;
     if (ev0 && (e = cudaEventRecord(ev0, s)) != cudaSuccess)

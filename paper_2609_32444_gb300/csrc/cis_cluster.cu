@@ -391,7 +391,11 @@ __global__ void __launch_bounds__(kThreads) cis_fused_cluster_kernel(const PassA
     if (threadIdx.x == 0) {
         const RowScalars rs = row_scalars(o, zy);
         const bool has_old = a.lp_old != nullptr;
-        const TokenWeight tw = token_weight(has_old ? (double)lold : rs.lp64, linf, a.P);
+        TokenWeight tw = token_weight(has_old ? (double)lold : rs.lp64, linf, a.P);
+        if (a.w_in) {  // a sequence operator: the response's weight
+            tw.w = a.w_in[t];
+            tw.trunc = a.trunc_in[t];
+        }
         const TokenLoss tl = token_loss(rs.lp64, has_old, lold, adv, sc, tw.w, a.P);
         if (rank == 0) {
             if (a.lp_out) a.lp_out[t] = rs.lp;

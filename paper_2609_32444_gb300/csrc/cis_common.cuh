@@ -38,7 +38,14 @@ struct DevParams {
     float log_tis_cap_f, log_exact_lo_f, log_exact_hi_f, log_rho_lo_f, log_rho_hi_f;
     double lam, kappa;
     double log_tis_cap, log_exact_lo, log_exact_hi, log_rho_lo, log_rho_hi;
+    double log_icepop_lo, log_icepop_hi, kpop_phi;
+    double seq_cap, log_seq_cap, log_seq_lo, log_seq_hi;
 };
+
+__host__ __device__ __forceinline__ bool is_seq_mode(int32_t mode)
+{
+    return mode == CIS_MODE_SEQ_TIS || mode == CIS_MODE_SEQ_MIS;
+}
 
 // Device status bits (cis_status_t values that can only be seen on the GPU).
 constexpr int32_t kStatusTimeout = CIS_ERR_DEVICE_TIMEOUT;
@@ -145,8 +152,64 @@ __device__ __forceinline__ TokenWeight token_weight(double lw, float linf, const
         r.w = hi ? P.exact_hi_f : (lo ? P.exact_lo_f : expf(logk));
         break;
     }
+    case CIS_MODE_BAND: {
+        // Sec. 4.3: the CIS weight, lifted from below to (1 + p)/2 (the image
+        // of e^eps = 1/2); both decisions in fp64
+        const double phi = fmax(-expm1(lw), P.kappa);
+        const double lo = 0.5 * (1.0 + exp(lw));
+        const bool up = logk64 > log1p(P.lam * phi);
+        const bool low = logk64 < log(lo);
+        r.trunc = up || low;
+        r.w = up ? (float)(1.0 + P.lam * phi) : (low ? (float)lo : expf(logk));
+        break;
+    }
+    case CIS_MODE_ICEPOP: {
+        // Table 8: k on [lo, hi] (bounds included), else masked
+        const bool out = logk64 < P.log_icepop_lo || logk64 > P.log_icepop_hi;
+        r.trunc = out;
+        r.w = out ? 0.0f : expf(logk);
+        break;
+    }
+    case CIS_MODE_KPOP: {
+        // Table 8 / App. D.5: binary KL both ways in fp64 on probabilities
+        // clamped to [1e-8, 1 - 1e-8]; masked when the larger exceeds phi
+        const double lo = 1e-8, hi = 1.0 - 1e-8;
+        double p = exp(lw), q = exp((double)linf);
+        p = p < lo ? lo : (p > hi ? hi : p);
+        q = q < lo ? lo : (q > hi ? hi : q);
+        const double kl_pq = p * log(p / q) + (1.0 - p) * log((1.0 - p) / (1.0 - q));
+        const double kl_qp = q * log(q / p) + (1.0 - q) * log((1.0 - q) / (1.0 - p));
+        const double m = kl_pq > kl_qp ? kl_pq : kl_qp;
+        const bool out = m > P.kpop_phi;
+        r.trunc = out;
+        r.w = out ? 0.0f : expf(logk);
+        break;
+    }
+    case CIS_MODE_SEQ_TIS:
+    case CIS_MODE_SEQ_MIS:
+        // the weight is the response's (seq_weight); callers pass it in
+        r.w = 0.0f;
+        break;
     default:
         break;
+    }
+    return r;
+}
+
+// The weight of every token of a response from log K, the sum of log k over
+// its valid tokens (Table 8: Seq-TIS min(K, C), Seq-MIS K 1{K in [lo, hi]}).
+__device__ __forceinline__ TokenWeight seq_weight(double logK, const DevParams &P)
+{
+    TokenWeight r;
+    r.logk = (float)logK;
+    if (P.mode == CIS_MODE_SEQ_TIS) {
+        const bool tr = logK > P.log_seq_cap;
+        r.trunc = tr;
+        r.w = tr ? (float)P.seq_cap : (float)exp(logK);
+    } else {
+        const bool out = logK < P.log_seq_lo || logK > P.log_seq_hi;
+        r.trunc = out;
+        r.w = out ? 0.0f : (float)exp(logK);
     }
     return r;
 }

@@ -119,8 +119,13 @@ CIS_API cis_status_t cis_loss_fwd_bwd_host(
         return CIS_ERR_INVALID_ARG;
     if (!params_ok(params))
         return CIS_ERR_INVALID_ARG;
-    if (params->agg == CIS_AGG_SEQ_MEAN_TOKEN_MEAN && (cu_seqlens == nullptr || B < 0))
+    if ((params->agg == CIS_AGG_SEQ_MEAN_TOKEN_MEAN || is_seq_mode(params->mode)) &&
+        (cu_seqlens == nullptr || B < 0))
         return CIS_ERR_INVALID_ARG;
+    // a sequence operator's weights need every row's log p before the first
+    // chunk's dlogits unless they come from lp_old
+    if (is_seq_mode(params->mode) && lp_old == nullptr && T > 0)
+        return CIS_ERR_UNSUPPORTED;
     const int isz = dbytes(dtype), osz = dbytes(dlogits_dtype);
     const HostLayout L = host_layout(T, V, isz, osz, chunk_tokens, B < 0 ? 0 : B);
     if (workspace == nullptr || (reinterpret_cast<uintptr_t>(workspace) & 255) ||
@@ -178,6 +183,15 @@ CIS_API cis_status_t cis_loss_fwd_bwd_host(
     a.P = make_dev_params(*params);
     const int32_t *cu_dev = cu_seqlens ? reinterpret_cast<const int32_t *>(dptr(L.cu)) : nullptr;
     CIS_TRY(launch_scales(a.mask, T, cu_dev, B, params->agg, scale, a.status, sc));
+    if (T > 0 && is_seq_mode(params->mode)) {
+        // the responses' weights from lp_old, read by every chunk's pass
+        CIS_TRY(cudaMemsetAsync(a.ws_w, 0, 4 * n, sc));
+        CIS_TRY(cudaMemsetAsync(a.ws_trunc, 0, n, sc));
+        CIS_TRY(launch_seq_weights(nullptr, a.lp_old, a.lp_inf, a.ids, V, a.mask, cu_dev, B, T,
+                                   a.P, a.ws_w, a.ws_trunc, sc));
+        a.w_in = a.ws_w;
+        a.trunc_in = a.ws_trunc;
+    }
 
     const int64_t nchunks = (T + chunk_tokens - 1) / chunk_tokens;
     std::vector<cudaEvent_t> ev;  // per chunk: copied in, computed, copied out
@@ -237,6 +251,8 @@ CIS_API cis_status_t cis_loss_fwd_bwd_host(
             c.ws_trunc = a.ws_trunc + r0;
             c.ws_logk = a.ws_logk + r0;
             c.ws_terms = a.ws_terms + r0;
+            c.w_in = a.w_in ? a.w_in + r0 : nullptr;
+            c.trunc_in = a.trunc_in ? a.trunc_in + r0 : nullptr;
             cudaError_t ke = cluster_path_applies(c, dtype, dlogits_dtype)
                                  ? launch_cluster_fwd_bwd(c, dtype, dlogits_dtype, sc)
                                  : launch_rowwise_fwd_bwd(c, dtype, dlogits_dtype, sc);

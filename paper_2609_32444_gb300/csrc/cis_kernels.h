@@ -31,6 +31,11 @@ struct PassArgs {
     double *ws_terms;
     int32_t *status;
     DevParams P;
+    // sequence operators: weights formed beforehand (seq_weight); the pass
+    // uses them instead of token_weight's
+    const float *w_in;
+    const uint8_t *trunc_in;
+    double *lp64_out;      // forward-only kernel: log p in fp64 (may be null)
 };
 
 // Host-side parameter checks and the kernels' copy of the parameters.
@@ -42,6 +47,16 @@ struct WsLayout {
     size_t status, scale, terms, logk, w, trunc, total;
 };
 WsLayout ws_layout(int64_t T);
+
+// Sequence operators: w[t], trunc[t] for the valid tokens of each response
+// from the fp64 sum of log k = lw - lp_inf over its valid tokens with an id
+// in [0, V) (lw64 if given, else lw32); other tokens are not written.
+// Response ranges are clamped to [0, T), so bad offsets cannot reach memory
+// outside the T-long arrays.
+cudaError_t launch_seq_weights(const double *lw64, const float *lw32, const float *lp_inf,
+                               const int32_t *ids, int64_t V, const uint8_t *mask,
+                               const int32_t *cu_seqlens, int64_t B, int64_t T,
+                               const DevParams &P, float *w, uint8_t *trunc, cudaStream_t s);
 
 // Forward-only: lp (and lse) of the sampled token, one CTA per row.
 cudaError_t launch_token_logprobs(const PassArgs &a, int dtype, cudaStream_t s);

@@ -423,9 +423,20 @@ __global__ void cis_lmhead_token_kernel(const PassArgs a, const float2 *part, co
     o = warp_ms(o);
     if (lane == 0) {
         const RowScalars rs = row_scalars(o, zy[t]);
+        if (is_seq_mode(a.P.mode) && a.w_in == nullptr) {
+            // sequence operator, first sweep: log p only (the response's
+            // weight needs every token of the response)
+            if (a.lp64_out)
+                a.lp64_out[t] = rs.lp64;
+            return;
+        }
         const bool has_old = a.lp_old != nullptr;
         const float lold = has_old ? a.lp_old[t] : 0.0f;
-        const TokenWeight tw = token_weight(has_old ? (double)lold : rs.lp64, a.lp_inf[t], a.P);
+        TokenWeight tw = token_weight(has_old ? (double)lold : rs.lp64, a.lp_inf[t], a.P);
+        if (a.w_in) {
+            tw.w = a.w_in[t];
+            tw.trunc = a.trunc_in[t];
+        }
         const TokenLoss tl = token_loss(rs.lp64, has_old, lold, a.adv[t], a.scale[t], tw.w, a.P);
         if (a.lp_out) a.lp_out[t] = rs.lp;
         if (a.w_out) a.w_out[t] = tw.w;
@@ -626,7 +637,8 @@ CIS_API cis_status_t cis_lmhead_fused(const void *hidden, const void *weight, in
         return CIS_ERR_INVALID_ARG;
     if (!params_ok(params))
         return CIS_ERR_INVALID_ARG;
-    if (params->agg == CIS_AGG_SEQ_MEAN_TOKEN_MEAN && (cu_seqlens == nullptr || B < 0))
+    if ((params->agg == CIS_AGG_SEQ_MEAN_TOKEN_MEAN || is_seq_mode(params->mode)) &&
+        (cu_seqlens == nullptr || B < 0))
         return CIS_ERR_INVALID_ARG;
     if (H % lm::kBN != 0)
         return CIS_ERR_UNSUPPORTED;  // Hd in blocks of 256 (and so of the 64-wide K blocks)
@@ -710,6 +722,27 @@ CIS_API cis_status_t cis_lmhead_fused(const void *hidden, const void *weight, in
         if (lm::launch_gemm<lm::kStats>(mH, mW, g, s) != cudaSuccess)
             return CIS_ERR_CUDA;
         // per-token scalars
+        if (is_seq_mode(P.mode)) {
+            // sequence operator: log p of every token (fp64, into the terms
+            // array, which the second sweep then overwrites), the responses'
+            // weights, then the token scalars with those weights
+            if (lp_old == nullptr) {
+                PassArgs f = a;
+                f.lp64_out = a.ws_terms;
+                lm::cis_lmhead_token_kernel<<<(unsigned)((T + 7) / 8), 256, 0, s>>>(f, part, zy, nVt,
+                                                                                lse, cv);
+                if ((e = cudaGetLastError()) != cudaSuccess)
+                    return CIS_ERR_CUDA;
+            }
+            if (cudaMemsetAsync(a.ws_w, 0, 4 * (size_t)T, s) != cudaSuccess ||
+                cudaMemsetAsync(a.ws_trunc, 0, (size_t)T, s) != cudaSuccess)
+                return CIS_ERR_CUDA;
+            if (launch_seq_weights(lp_old ? nullptr : a.ws_terms, lp_old, lp_infer, ids, V, mask,
+                                   cu_seqlens, B, T, a.P, a.ws_w, a.ws_trunc, s) != cudaSuccess)
+                return CIS_ERR_CUDA;
+            a.w_in = a.ws_w;
+            a.trunc_in = a.ws_trunc;
+        }
         lm::cis_lmhead_token_kernel<<<(unsigned)((T + 7) / 8), 256, 0, s>>>(a, part, zy, nVt, lse, cv);
         if ((e = cudaGetLastError()) != cudaSuccess)
             return CIS_ERR_CUDA;

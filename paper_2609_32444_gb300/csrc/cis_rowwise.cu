@@ -129,6 +129,7 @@ __global__ void __launch_bounds__(kRowThreads) cis_fused_row_kernel(const PassAr
                 set_status(a.status, kStatusBadId);
             if (a.lp_out) a.lp_out[t] = lp;
             if (a.lse_out) a.lse_out[t] = lp;
+            if (!kBwd && a.lp64_out) a.lp64_out[t] = lp;
             if (kBwd) {
                 if (a.w_out) a.w_out[t] = 0.0f;
                 if (a.trunc_out) a.trunc_out[t] = 0;
@@ -146,10 +147,15 @@ __global__ void __launch_bounds__(kRowThreads) cis_fused_row_kernel(const PassAr
         const RowScalars rs = row_scalars(o, to_f32(row[y]));
         if (a.lp_out) a.lp_out[t] = rs.lp;
         if (a.lse_out) a.lse_out[t] = rs.lse;
+        if (!kBwd && a.lp64_out) a.lp64_out[t] = rs.lp64;
         if (kBwd) {
             const bool has_old = a.lp_old != nullptr;
             const double lw = has_old ? (double)a.lp_old[t] : rs.lp64;
-            const TokenWeight tw = token_weight(lw, a.lp_inf[t], a.P);
+            TokenWeight tw = token_weight(lw, a.lp_inf[t], a.P);
+            if (a.w_in) {  // a sequence operator: the response's weight
+                tw.w = a.w_in[t];
+                tw.trunc = a.trunc_in[t];
+            }
             const TokenLoss tl = token_loss(rs.lp64, has_old, has_old ? a.lp_old[t] : 0.0f,
                                             a.adv[t], a.scale[t], tw.w, a.P);
             if (a.w_out) a.w_out[t] = tw.w;

@@ -13,6 +13,7 @@ namespace cis {
 namespace {
 
 constexpr int kSmallThreads = 1024;
+constexpr int kSeqThreads = 256;  // one CTA per response
 constexpr int kMaxSeqInShared = 12000;
 
 __device__ __forceinline__ bool is_valid(const uint8_t *mask, int64_t t)
@@ -114,6 +115,43 @@ __global__ void cis_weights_kernel(const float *lp_w, const float *lp_inf, const
     }
 }
 
+// One CTA per response: the fp64 sum of log k over its valid tokens in a
+// fixed order (thread-strided partial sums, then a tree), then the response's
+// weight for each of them (seq_weight, Table 8).
+__global__ void __launch_bounds__(kSeqThreads)
+    cis_seq_weights_kernel(const double *lw64, const float *lw32, const float *lp_inf,
+                           const int32_t *ids, int64_t V, const uint8_t *mask,
+                           const int32_t *cu, int64_t T, const DevParams P, float *w,
+                           uint8_t *trunc)
+{
+    __shared__ double red[kSeqThreads];
+    const int64_t i = blockIdx.x;
+    int64_t b = cu[i], e = cu[i + 1];
+    b = b < 0 ? 0 : (b > T ? T : b);
+    e = e < b ? b : (e > T ? T : e);
+    auto used = [&](int64_t t) {
+        return is_valid(mask, t) && (ids == nullptr || (ids[t] >= 0 && (int64_t)ids[t] < V));
+    };
+    double acc = 0.0;
+    for (int64_t t = b + threadIdx.x; t < e; t += kSeqThreads)
+        if (used(t))
+            acc += (lw64 ? lw64[t] : (double)lw32[t]) - (double)lp_inf[t];
+    red[threadIdx.x] = acc;
+    __syncthreads();
+    for (int off = kSeqThreads / 2; off > 0; off >>= 1) {
+        if (threadIdx.x < off)
+            red[threadIdx.x] += red[threadIdx.x + off];
+        __syncthreads();
+    }
+    const TokenWeight tw = seq_weight(red[0], P);
+    for (int64_t t = b + threadIdx.x; t < e; t += kSeqThreads)
+        if (used(t)) {
+            w[t] = tw.w;
+            if (trunc)
+                trunc[t] = tw.trunc;
+        }
+}
+
 struct RedPart {
     double loss, excess;
     long long nvalid, ntrunc;
@@ -201,4 +239,19 @@ cudaError_t launch_reduce(const PassArgs &a, cis_stats_t *stats, double *loss, c
     return cudaGetLastError();
 }
 
+cudaError_t launch_seq_weights(const double *lw64, const float *lw32, const float *lp_inf,
+                               const int32_t *ids, int64_t V, const uint8_t *mask,
+                               const int32_t *cu_seqlens, int64_t B, int64_t T,
+                               const DevParams &P, float *w, uint8_t *trunc, cudaStream_t s)
+{
+    if (B <= 0 || T <= 0)
+        return cudaSuccess;
+    if (B > 0x7fffffffLL)
+        return cudaErrorInvalidValue;
+    cis_seq_weights_kernel<<<(unsigned)B, kSeqThreads, 0, s>>>(lw64, lw32, lp_inf, ids, V, mask,
+                                                                cu_seqlens, T, P, w, trunc);
+    return cudaGetLastError();
+}
+
 }  // namespace cis
+

@@ -124,11 +124,43 @@ def test_other_entry_points_reject_bad_arguments(binding):
     assert L.cis_token_logprobs(None, 1, 4, 8, 8, fake, None, fake, None, None, None) == 1
     assert L.cis_token_logprobs(fake, 1, 0, 8, 8, None, None, None, None, None, None) == 0
     p.kappa = 2.0
-    assert L.cis_weights(fake, fake, None, 4, ctypes.byref(p), fake, None, None, None) == 1
+    assert L.cis_weights(fake, fake, None, 4, None, 0, ctypes.byref(p), fake, None, None,
+                         None) == 1
     p.kappa = 5e-3
-    assert L.cis_weights(None, fake, None, 4, ctypes.byref(p), fake, None, None, None) == 1
-    assert L.cis_weights(None, None, None, 0, ctypes.byref(p), None, None, None, None) == 0
+    assert L.cis_weights(None, fake, None, 4, None, 0, ctypes.byref(p), fake, None, None,
+                         None) == 1
+    assert L.cis_weights(None, None, None, 0, None, 0, ctypes.byref(p), None, None, None,
+                         None) == 0
     assert L.cis_default_params(None) == 1
+
+
+@pytest.mark.parametrize("field,value", [("icepop_lo", 6.0), ("icepop_lo", -1.0),
+                                         ("kpop_phi", -0.5), ("seq_cap", 0.0),
+                                         ("seq_hi", 0.1), ("mode", 9)])
+def test_new_operator_parameters_are_validated(binding, field, value):
+    """Bands with lo > hi or lo < 0, a negative KPop threshold, a zero Seq-TIS
+    cap and an unknown mode are refused before any GPU work."""
+    L = binding.lib()
+    fake = ctypes.c_void_p(0x10000)
+    p = binding.cis_default_params("icepop")
+    setattr(p, field, value)
+    assert L.cis_weights(fake, fake, None, 4, None, 0, ctypes.byref(p), fake, None, None,
+                         None) == 1
+
+
+def test_sequence_operators_need_responses(binding):
+    """Seq-TIS / Seq-MIS without cu_seqlens: CIS_ERR_INVALID_ARG before any
+    GPU work, from the weights, the fused pass, the host path and the LM head."""
+    L = binding.lib()
+    fake = ctypes.c_void_p(0x10000)
+    for mode in ("seq_tis", "seq_mis"):
+        p = binding.cis_default_params(mode)
+        assert L.cis_weights(fake, fake, None, 4, None, 0, ctypes.byref(p), fake, None, None,
+                             None) == 1
+        assert _fwd_bwd_rc(binding, params={"mode": binding.MODES[mode]}) == 1
+    d = binding.cis_default_params()
+    assert (d.icepop_lo, d.icepop_hi, d.kpop_phi) == (0.5, 5.0, 2.0)
+    assert (d.seq_cap, d.seq_lo, d.seq_hi) == (2.0, 0.5, 2.0)
 
 
 def test_binding_refuses_cpu_tensors(binding):

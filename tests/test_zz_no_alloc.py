@@ -87,3 +87,29 @@ def test_noalloc_rejects_more_tokens_than_its_scratch(noalloc):
                  None, 0, ctypes.byref(P), ctypes.c_void_p(0x4000000), binding.CIS_BF16, 8,
                  None, None, None, None, None, None)
     assert rc == binding.CIS_ERR_UNSUPPORTED
+
+
+def test_noalloc_sequence_operator(noalloc):
+    """Seq-MIS through the no-allocation entry point (forward pass, response
+    weights, then the pass, all in the static array) equals the workspace
+    entry point."""
+    b = synth.make_batch(1)
+    g = {k: v.cuda() for k, v in dict(logits=b.logits, ids=b.ids, lp=b.lp_infer, adv=b.adv,
+                                       mask=b.mask, cu=b.cu_seqlens).items()}
+    P = binding.cis_default_params("seq_mis", lam=b.lam)
+    T, V = b.T, b.V
+    dev = g["logits"].device
+    dz = torch.empty((T, V), dtype=torch.float32, device=dev)
+    w = torch.empty(T, device=dev)
+    loss = torch.empty(1, dtype=torch.float64, device=dev)
+    ptr = lambda t: ctypes.c_void_p(t.data_ptr())  # noqa: E731
+    rc = noalloc(ptr(g["logits"]), binding.CIS_F32, T, V, V, ptr(g["ids"]), ptr(g["lp"]), None,
+                 ptr(g["adv"]), ptr(g["mask"]), ptr(g["cu"]), b.cu_seqlens.shape[0] - 1,
+                 ctypes.byref(P), ptr(dz), binding.CIS_F32, V, None, ptr(w), None, None,
+                 ptr(loss), ctypes.c_void_p(torch.cuda.current_stream().cuda_stream))
+    assert rc == 0
+    ref = binding.cis_loss_fwd_bwd(g["logits"], g["ids"], g["lp"], g["adv"], P, mask=g["mask"],
+                                   cu_seqlens=g["cu"], dlogits_dtype=torch.float32)
+    torch.cuda.synchronize()
+    assert torch.equal(w, ref["w"]) and torch.equal(loss, ref["loss"])
+    assert torch.equal(dz, ref["dlogits"])
