@@ -98,6 +98,8 @@ def _load():
             P, i32, i64, i64, i64, P, P, P, P, P, P, i64, ctypes.POINTER(OracleParams), P,
             P, i64, P, P, P, P, P, P, P, P, ctypes.c_int]
         lib.oracle_loss_fwd_bwd.restype = ctypes.c_int
+        lib.oracle_token_entropy.argtypes = [P, i32, i64, i64, i64, P, P, ctypes.c_int]
+        lib.oracle_token_entropy.restype = None
         lib.oracle_max_threads.argtypes = []
         lib.oracle_max_threads.restype = ctypes.c_int
         _ = dbl
@@ -151,6 +153,18 @@ def token_logprobs(logits, ids, V=None, mask=None, nthreads=0):
     rc = lib.oracle_token_logprobs(_ptr(a), dt, T, V, ld, _ptr(ids), _ptr(mask), _ptr(lp),
                                    _ptr(lse), nthreads)
     return lp, lse, rc
+
+
+def token_entropy(logits, V=None, mask=None, nthreads=0):
+    """H_t = -sum_j p_tj log p_tj of each row's softmax in fp64 (App. D)."""
+    lib = _load()
+    a, dt = _logits_arg(logits)
+    T, ld = a.shape
+    V = ld if V is None else V
+    mask = _opt(mask, np.uint8)
+    h = np.zeros(T, np.float64)
+    lib.oracle_token_entropy(_ptr(a), dt, T, V, ld, _ptr(mask), _ptr(h), nthreads)
+    return h
 
 
 def weights(lp_w, lp_inf, P: OracleParams, mask=None, cu_seqlens=None):

@@ -31,6 +31,8 @@
  *   - Sec. 4.3 / App. C.1: the two-sided band max{min{k, 1 + lambda phi},
  *     (1 + p)/2}, the image of e^eps >= 1/2 under k = p + (1 - p) e^eps.
  *   - Lemma 3.1 / Lemma B.1: eps_t = logit p_t - logit q_t.
+ *   - App. D (training statistics): the entropy of the training policy,
+ *     -sum_j p_j log p_j per token.
  *
  * Readings where the paper is silent (each also listed in the design notes):
  *   - the truncation flag is "k > cap", decided in fp64 in the log domain:
@@ -196,6 +198,31 @@ int oracle_token_logprobs(const void *logits, int dtype, int64_t T, int64_t V, i
             lse_out[t] = lse;
     }
     return bad ? -1 : 0;
+}
+
+/*
+ * Entropy of each row's softmax, H_t = -sum_j p_tj log p_tj with
+ * log p_tj = z_tj - lse_t (the training-side entropy the paper logs, App. D);
+ * entries with p = 0 add nothing (0 log 0 = 0).  Masked rows get 0.
+ */
+void oracle_token_entropy(const void *logits, int dtype, int64_t T, int64_t V, int64_t ld,
+                          const uint8_t *mask, double *h_out, int nthreads)
+{
+    set_threads(nthreads);
+#pragma omp parallel for schedule(dynamic, 4)
+    for (int64_t t = 0; t < T; ++t) {
+        double h = 0.0;
+        if (row_valid(mask, t)) {
+            double lse = row_lse(logits, dtype, ld, t, V);
+            for (int64_t j = 0; j < V; ++j) {
+                double lpj = logit_at(logits, dtype, ld, t, j) - lse;
+                double pj = exp(lpj);
+                if (pj != 0.0 || isnan(pj))
+                    h -= pj * lpj;
+            }
+        }
+        h_out[t] = h;
+    }
 }
 
 /*

@@ -597,3 +597,38 @@ def test_sequence_operators_on_one_token_responses_are_token_operators():
                                                            icepop_lo=0.5, icepop_hi=2.0))
     np.testing.assert_allclose(wm, wi, rtol=1e-15)
     assert np.all(trm == tri)
+
+
+# ---------------------------------------------------------------- entropy
+def test_entropy_closed_forms():
+    """Uniform rows give log V, one-hot rows 0, two-point rows the binary
+    entropy; every row lies in [0, log V]; masked rows give 0."""
+    V = 7
+    z = np.zeros((4, V))
+    z[1, 1:] = -np.inf                     # one-hot
+    z[2, 2:] = -np.inf                     # two-point, p = 1/(1 + e^-1.5)
+    z[2, 1] = -1.5
+    z[3] = np.random.default_rng(7).standard_normal(V) * 3
+    h = oracle.token_entropy(z, mask=np.array([1, 1, 1, 1], np.uint8))
+    assert h[0] == pytest.approx(math.log(V), rel=1e-15)
+    assert h[1] == 0.0
+    p = 1.0 / (1.0 + math.exp(-1.5))
+    assert h[2] == pytest.approx(-p * math.log(p) - (1 - p) * math.log(1 - p), rel=1e-14)
+    assert 0.0 < h[3] < math.log(V)
+    hm = oracle.token_entropy(z, mask=np.array([1, 0, 1, 0], np.uint8))
+    assert hm[1] == 0.0 and hm[3] == 0.0 and hm[0] == h[0]
+
+
+@pytest.mark.parametrize("V", [2, 5, 8])
+def test_entropy_matches_50_digit_brute_force_and_is_shift_invariant(V):
+    rng = np.random.default_rng(50 + V)
+    z = rng.standard_normal((6, V)) * 4
+    h = oracle.token_entropy(z)
+    mpmath.mp.dps = 50
+    for t in range(6):
+        zs = [mpmath.mpf(float(x)) for x in z[t]]
+        S = mpmath.fsum(mpmath.exp(x) for x in zs)
+        ref = -mpmath.fsum((mpmath.exp(x) / S) * (x - mpmath.log(S)) for x in zs)
+        assert abs(h[t] - float(ref)) <= 1e-14 * max(1.0, float(ref))
+    h2 = oracle.token_entropy(z + 123.25)
+    np.testing.assert_allclose(h2, h, rtol=1e-12, atol=1e-13)
