@@ -125,6 +125,10 @@ typedef struct {
                            * clamped, lifted (band) or masked                 */
     float max_abs_logk;   /* max over valid tokens of |log k_t|               */
     int32_t status;       /* OR of device status bits (cis_status_t)          */
+    double entropy_sum;   /* sum over valid tokens of the softmax entropy H_t
+                           * when the call writes entropy_out, else 0; the
+                           * batch entropy the paper logs is entropy_sum /
+                           * n_valid                                          */
 } cis_stats_t;
 
 /* Fills *out with the defaults above.  Host only.  CIS_ERR_INVALID_ARG if out
@@ -142,6 +146,9 @@ CIS_API const char *cis_status_string(int32_t status);
  *   mask       device uint8 [T] or NULL.
  *   lp_out     device float [T].
  *   lse_out    device float [T] or NULL: logsumexp of each row.
+ *   entropy_out device float [T] or NULL: entropy of each row's softmax,
+ *              H_t = -sum_j p_tj log p_tj (the training-side entropy the
+ *              paper logs, App. D); 0 for masked rows.
  *   dev_status device int32 [1] or NULL: device status bits are OR-ed in
  *              (the caller zeroes it first).
  * Errors: CIS_ERR_INVALID_ARG for NULL required pointers, T < 0, V <= 0,
@@ -149,8 +156,8 @@ CIS_API const char *cis_status_string(int32_t status);
  */
 CIS_API cis_status_t cis_token_logprobs(const void *logits, int32_t dtype, int64_t T, int64_t V,
                                 int64_t ld, const int32_t *ids, const uint8_t *mask,
-                                float *lp_out, float *lse_out, int32_t *dev_status,
-                                void *stream);
+                                float *lp_out, float *lse_out, float *entropy_out,
+                                int32_t *dev_status, void *stream);
 
 /*
  * Weights (Algorithm 1, Eq. 4, Table 8) from fp32 log-probabilities.
@@ -208,6 +215,10 @@ CIS_API cis_status_t cis_loss_workspace_size(int64_t T, int64_t V, size_t *bytes
  *               nearest even, CIS_F32); every element j < V of every row is
  *               written.  May not overlap the logits.
  *   lp_out, w_out, trunc_out  device per-token outputs or NULL.
+ *   entropy_out device float [T] or NULL: each row's softmax entropy, taken
+ *               in the same pass (a variant of the kernel that keeps one more
+ *               sum per row; without it the pass does no entropy work), and
+ *               summed into stats_out->entropy_sum.
  *   stats_out   device cis_stats_t* or NULL.
  *   loss_out    device double [1] or NULL: the loss (also in stats_out).
  *   workspace   device, >= cis_loss_workspace_size(T, V) bytes, 256-byte
@@ -229,9 +240,9 @@ CIS_API cis_status_t cis_loss_fwd_bwd(const void *logits, int32_t dtype, int64_t
                               const int32_t *cu_seqlens, int64_t B,
                               const cis_params_t *params, void *dlogits,
                               int32_t dlogits_dtype, int64_t ld_out, float *lp_out,
-                              float *w_out, uint8_t *trunc_out, cis_stats_t *stats_out,
-                              double *loss_out, void *workspace, size_t workspace_bytes,
-                              void *stream);
+                              float *w_out, uint8_t *trunc_out, float *entropy_out,
+                              cis_stats_t *stats_out, double *loss_out, void *workspace,
+                              size_t workspace_bytes, void *stream);
 
 /*
  * Bytes of device workspace cis_loss_fwd_bwd_host needs for T tokens of V
@@ -246,7 +257,7 @@ CIS_API cis_status_t cis_loss_host_workspace_size(int64_t T, int64_t V, int32_t 
  * cis_loss_fwd_bwd for callers whose buffers are in host memory.
  *   Every tensor argument is a HOST pointer: logits [T, V] and dlogits [T, V]
  *   (contiguous rows), ids, lp_infer, lp_old, adv, mask, cu_seqlens, and the
- *   outputs lp_out, w_out, trunc_out, stats_out, loss_out.  Page-locked
+ *   outputs lp_out, w_out, trunc_out, entropy_out, stats_out, loss_out.  Page-locked
  *   (pinned) memory lets the copies overlap; pageable memory works but the
  *   copies then serialise.
  *   workspace is DEVICE memory of cis_loss_host_workspace_size(...) bytes,
@@ -266,7 +277,7 @@ CIS_API cis_status_t cis_loss_fwd_bwd_host(
     const void *logits, int32_t dtype, int64_t T, int64_t V, const int32_t *ids,
     const float *lp_infer, const float *lp_old, const float *adv, const uint8_t *mask,
     const int32_t *cu_seqlens, int64_t B, const cis_params_t *params, void *dlogits,
-    int32_t dlogits_dtype, float *lp_out, float *w_out, uint8_t *trunc_out,
+    int32_t dlogits_dtype, float *lp_out, float *w_out, uint8_t *trunc_out, float *entropy_out,
     cis_stats_t *stats_out, double *loss_out, int64_t chunk_tokens, void *workspace,
     size_t workspace_bytes, void *stream);
 
@@ -304,7 +315,9 @@ CIS_API cis_status_t cis_lmhead_workspace_size_chunk(int64_t T, int64_t V, int64
  *   dhidden     device [T, H] of grad_dtype (CIS_F32 or CIS_BF16), written.
  *   dweight     device [V, H] of grad_dtype, written (rows of tokens that are
  *               masked contribute nothing).
- *   lp_out, w_out, trunc_out, stats_out, loss_out: as for cis_loss_fwd_bwd.
+ *   lp_out, w_out, trunc_out, entropy_out, stats_out, loss_out: as for
+ *               cis_loss_fwd_bwd (the entropy comes from the forward sweep's
+ *               tiles).
  *   workspace   device, 1024-byte aligned; its first int32 is the device
  *               status word.  workspace_bytes picks the chunk: the widest
  *               multiple of 256 columns whose cis_lmhead_workspace_size_chunk
@@ -321,9 +334,9 @@ CIS_API cis_status_t cis_lmhead_fused(const void *hidden, const void *weight, in
                                       const int32_t *cu_seqlens, int64_t B,
                                       const cis_params_t *params, void *dhidden, void *dweight,
                                       int32_t grad_dtype, float *lp_out, float *w_out,
-                                      uint8_t *trunc_out, cis_stats_t *stats_out,
-                                      double *loss_out, void *workspace, size_t workspace_bytes,
-                                      void *stream);
+                                      uint8_t *trunc_out, float *entropy_out,
+                                      cis_stats_t *stats_out, double *loss_out, void *workspace,
+                                      size_t workspace_bytes, void *stream);
 
 /*
  * Largest T that cis_loss_fwd_bwd_noalloc accepts.
@@ -359,8 +372,8 @@ CIS_API cis_status_t cis_loss_fwd_bwd_noalloc(const void *logits, int32_t dtype,
                                               const cis_params_t *params, void *dlogits,
                                               int32_t dlogits_dtype, int64_t ld_out,
                                               float *lp_out, float *w_out, uint8_t *trunc_out,
-                                              cis_stats_t *stats_out, double *loss_out,
-                                              void *stream);
+                                              float *entropy_out, cis_stats_t *stats_out,
+                                              double *loss_out, void *stream);
 
 /*
  * Profiling aid.  The next cis_loss_fwd_bwd call made from the calling host

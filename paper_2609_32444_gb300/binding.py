@@ -56,6 +56,7 @@ class cis_stats_t(ctypes.Structure):
         ("n_truncated", ctypes.c_int64),
         ("max_abs_logk", ctypes.c_float),
         ("status", ctypes.c_int32),
+        ("entropy_sum", ctypes.c_double),
     ]
 
 
@@ -84,7 +85,7 @@ def lib():
     L.cis_default_params.restype = ctypes.c_int
     L.cis_status_string.argtypes = [i32]
     L.cis_status_string.restype = ctypes.c_char_p
-    L.cis_token_logprobs.argtypes = [P, i32, i64, i64, i64, P, P, P, P, P, P]
+    L.cis_token_logprobs.argtypes = [P, i32, i64, i64, i64, P, P, P, P, P, P, P]
     L.cis_token_logprobs.restype = ctypes.c_int
     L.cis_weights.argtypes = [P, P, P, i64, P, i64, ctypes.POINTER(cis_params_t), P, P, P, P]
     L.cis_weights.restype = ctypes.c_int
@@ -92,7 +93,7 @@ def lib():
     L.cis_loss_workspace_size.restype = ctypes.c_int
     L.cis_loss_fwd_bwd.argtypes = [P, i32, i64, i64, i64, P, P, P, P, P, P, i64,
                                    ctypes.POINTER(cis_params_t), P, i32, i64, P, P, P, P, P, P,
-                                   ctypes.c_size_t, P]
+                                   P, ctypes.c_size_t, P]
     L.cis_loss_fwd_bwd.restype = ctypes.c_int
     L.cis_lmhead_workspace_size.argtypes = [i64, i64, i64, ctypes.POINTER(ctypes.c_size_t)]
     L.cis_lmhead_workspace_size.restype = ctypes.c_int
@@ -101,13 +102,13 @@ def lib():
     L.cis_lmhead_workspace_size_chunk.restype = ctypes.c_int
     L.cis_lmhead_fused.argtypes = [P, P, i64, i64, i64, P, P, P, P, P, P, i64,
                                    ctypes.POINTER(cis_params_t), P, P, i32, P, P, P, P, P, P,
-                                   ctypes.c_size_t, P]
+                                   P, ctypes.c_size_t, P]
     L.cis_lmhead_fused.restype = ctypes.c_int
     L.cis_loss_host_workspace_size.argtypes = [i64, i64, i32, i32, i64, i64,
                                                ctypes.POINTER(ctypes.c_size_t)]
     L.cis_loss_host_workspace_size.restype = ctypes.c_int
     L.cis_loss_fwd_bwd_host.argtypes = [P, i32, i64, i64, P, P, P, P, P, P, i64,
-                                        ctypes.POINTER(cis_params_t), P, i32, P, P, P, P, P,
+                                        ctypes.POINTER(cis_params_t), P, i32, P, P, P, P, P, P,
                                         i64, P, ctypes.c_size_t, P]
     L.cis_loss_fwd_bwd_host.restype = ctypes.c_int
     L.cis_profile_next_call.argtypes = [P, P]
@@ -175,8 +176,10 @@ def cis_default_params(mode="cis", **kw) -> cis_params_t:
 
 
 def cis_token_logprobs(logits: torch.Tensor, ids: torch.Tensor, mask=None, V=None,
-                       want_lse=False, dev_status=None):
-    """log p of the sampled tokens (fp32) -- and the row logsumexp if asked."""
+                       want_lse=False, dev_status=None, want_entropy=False):
+    """log p of the sampled tokens (fp32) -- and the row logsumexp and the
+    softmax entropy if asked: returns lp, or a tuple (lp, lse, entropy) with
+    None for what was not asked when either is."""
     _need_cuda(logits, ids, mask)
     T, ld = _rows(logits)
     V = logits.shape[1] if V is None else V
@@ -184,9 +187,13 @@ def cis_token_logprobs(logits: torch.Tensor, ids: torch.Tensor, mask=None, V=Non
     _vec(mask, torch.uint8, T, "mask")
     lp = torch.empty(T, dtype=torch.float32, device=logits.device)
     lse = torch.empty(T, dtype=torch.float32, device=logits.device) if want_lse else None
+    ent = torch.empty(T, dtype=torch.float32, device=logits.device) if want_entropy else None
     rc = lib().cis_token_logprobs(_ptr(logits), _dtype_code(logits.dtype), T, V, ld, _ptr(ids),
-                                  _ptr(mask), _ptr(lp), _ptr(lse), _ptr(dev_status), _stream())
+                                  _ptr(mask), _ptr(lp), _ptr(lse), _ptr(ent), _ptr(dev_status),
+                                  _stream())
     _check(rc, "cis_token_logprobs")
+    if want_entropy:
+        return lp, lse, ent
     return (lp, lse) if want_lse else lp
 
 
@@ -222,10 +229,11 @@ def cis_loss_workspace_size(T: int, V: int) -> int:
 def cis_loss_fwd_bwd(logits: torch.Tensor, ids: torch.Tensor, lp_infer: torch.Tensor,
                      adv: torch.Tensor, params: cis_params_t, lp_old=None, mask=None,
                      cu_seqlens=None, dlogits=None, dlogits_dtype=None, V=None,
-                     want_lp=True, want_w=True, want_trunc=True, workspace=None):
+                     want_lp=True, want_w=True, want_trunc=True, workspace=None,
+                     want_entropy=False):
     """Fused forward + backward token pass.  Returns a dict with dlogits, lp, w,
-    trunc, loss (device fp64 [1]), stats (device bytes of cis_stats_t) and the
-    workspace (its first int32 is the device status word)."""
+    trunc, entropy (if asked), loss (device fp64 [1]), stats (device bytes of
+    cis_stats_t) and the workspace (its first int32 is the device status word)."""
     _need_cuda(logits, ids, lp_infer, adv, lp_old, mask, cu_seqlens, dlogits)
     T, ld = _rows(logits)
     V = logits.shape[1] if V is None else V
@@ -248,6 +256,7 @@ def cis_loss_fwd_bwd(logits: torch.Tensor, ids: torch.Tensor, lp_infer: torch.Te
     lp = torch.empty(T, dtype=torch.float32, device=dev) if want_lp else None
     w = torch.empty(T, dtype=torch.float32, device=dev) if want_w else None
     tr = torch.empty(T, dtype=torch.uint8, device=dev) if want_trunc else None
+    ent = torch.empty(T, dtype=torch.float32, device=dev) if want_entropy else None
     stats = torch.empty(ctypes.sizeof(cis_stats_t), dtype=torch.uint8, device=dev)
     loss = torch.empty(1, dtype=torch.float64, device=dev)
     nws = cis_loss_workspace_size(T, V)
@@ -257,10 +266,10 @@ def cis_loss_fwd_bwd(logits: torch.Tensor, ids: torch.Tensor, lp_infer: torch.Te
         _ptr(logits), _dtype_code(logits.dtype), T, V, ld, _ptr(ids), _ptr(lp_infer),
         _ptr(lp_old), _ptr(adv), _ptr(mask), _ptr(cu_seqlens), B, ctypes.byref(params),
         _ptr(dlogits), _dtype_code(dlogits.dtype), ld_out, _ptr(lp), _ptr(w), _ptr(tr),
-        _ptr(stats), _ptr(loss), _ptr(workspace), workspace.numel(), _stream())
+        _ptr(ent), _ptr(stats), _ptr(loss), _ptr(workspace), workspace.numel(), _stream())
     _check(rc, "cis_loss_fwd_bwd")
-    return {"dlogits": dlogits, "lp": lp, "w": w, "trunc": tr, "loss": loss, "stats": stats,
-            "workspace": workspace}
+    return {"dlogits": dlogits, "lp": lp, "w": w, "trunc": tr, "entropy": ent, "loss": loss,
+            "stats": stats, "workspace": workspace}
 
 
 def cis_loss_host_workspace_size(T, V, dtype, dlogits_dtype, chunk_tokens, B=0) -> int:
@@ -274,7 +283,7 @@ def cis_loss_host_workspace_size(T, V, dtype, dlogits_dtype, chunk_tokens, B=0) 
 def cis_loss_fwd_bwd_host(logits: torch.Tensor, ids: torch.Tensor, lp_infer: torch.Tensor,
                           adv: torch.Tensor, params: cis_params_t, dlogits: torch.Tensor,
                           lp_old=None, mask=None, cu_seqlens=None, chunk_tokens=2048,
-                          workspace=None, outputs=None):
+                          workspace=None, outputs=None, want_entropy=False):
     """The fused pass with every tensor in HOST memory (pinned for overlap);
     rows stream through the GPU in chunks.  ``outputs``: optional dict of host
     tensors lp, w, trunc, stats, loss to fill.  Returns that dict; it is valid
@@ -290,6 +299,8 @@ def cis_loss_fwd_bwd_host(logits: torch.Tensor, ids: torch.Tensor, lp_infer: tor
     out.setdefault("lp", torch.empty(T, dtype=torch.float32).pin_memory())
     out.setdefault("w", torch.empty(T, dtype=torch.float32).pin_memory())
     out.setdefault("trunc", torch.empty(T, dtype=torch.uint8).pin_memory())
+    if want_entropy:
+        out.setdefault("entropy", torch.empty(T, dtype=torch.float32).pin_memory())
     out.setdefault("stats", torch.empty(ctypes.sizeof(cis_stats_t), dtype=torch.uint8).pin_memory())
     out.setdefault("loss", torch.empty(1, dtype=torch.float64).pin_memory())
     nws = cis_loss_host_workspace_size(T, V, logits.dtype, dlogits.dtype, chunk_tokens, B)
@@ -299,7 +310,8 @@ def cis_loss_fwd_bwd_host(logits: torch.Tensor, ids: torch.Tensor, lp_infer: tor
         _ptr(logits), _dtype_code(logits.dtype), T, V, _ptr(ids), _ptr(lp_infer), _ptr(lp_old),
         _ptr(adv), _ptr(mask), _ptr(cu_seqlens), B, ctypes.byref(params), _ptr(dlogits),
         _dtype_code(dlogits.dtype), _ptr(out["lp"]), _ptr(out["w"]), _ptr(out["trunc"]),
-        _ptr(out["stats"]), _ptr(out["loss"]), chunk_tokens, _ptr(workspace), workspace.numel(),
+        _ptr(out.get("entropy")), _ptr(out["stats"]), _ptr(out["loss"]), chunk_tokens,
+        _ptr(workspace), workspace.numel(),
         _stream())
     _check(rc, "cis_loss_fwd_bwd_host")
     out["workspace"] = workspace
@@ -323,7 +335,7 @@ def cis_lmhead_workspace_size_chunk(T: int, V: int, H: int, chunk: int) -> int:
 def cis_lmhead_fused(hidden: torch.Tensor, weight: torch.Tensor, ids: torch.Tensor,
                      lp_infer: torch.Tensor, adv: torch.Tensor, params: cis_params_t,
                      lp_old=None, mask=None, cu_seqlens=None, grad_dtype=torch.float32,
-                     workspace=None, chunk=None):
+                     workspace=None, chunk=None, want_entropy=False):
     """Token pass through the LM head (logits never stored).  `chunk` (a
     multiple of 256) sizes the workspace for vocabulary chunks of that many
     columns; by default the library's choice.  Returns a dict with dhidden,
@@ -348,6 +360,7 @@ def cis_lmhead_fused(hidden: torch.Tensor, weight: torch.Tensor, ids: torch.Tens
     lp = torch.empty(T, dtype=torch.float32, device=dev)
     w = torch.empty(T, dtype=torch.float32, device=dev)
     tr = torch.empty(T, dtype=torch.uint8, device=dev)
+    ent = torch.empty(T, dtype=torch.float32, device=dev) if want_entropy else None
     stats = torch.empty(ctypes.sizeof(cis_stats_t), dtype=torch.uint8, device=dev)
     loss = torch.empty(1, dtype=torch.float64, device=dev)
     if workspace is None:  # else the caller's, as given (the library checks its size)
@@ -361,11 +374,11 @@ def cis_lmhead_fused(hidden: torch.Tensor, weight: torch.Tensor, ids: torch.Tens
     rc = lib().cis_lmhead_fused(
         _ptr(hidden), _ptr(weight), T, H, V, _ptr(ids), _ptr(lp_infer), _ptr(lp_old),
         _ptr(adv), _ptr(mask), _ptr(cu_seqlens), B, ctypes.byref(params), _ptr(dh), _ptr(dw),
-        _dtype_code(grad_dtype), _ptr(lp), _ptr(w), _ptr(tr), _ptr(stats), _ptr(loss),
-        _ptr(ws), ws.numel(), _stream())
+        _dtype_code(grad_dtype), _ptr(lp), _ptr(w), _ptr(tr), _ptr(ent), _ptr(stats),
+        _ptr(loss), _ptr(ws), ws.numel(), _stream())
     _check(rc, "cis_lmhead_fused")
-    return {"dhidden": dh, "dweight": dw, "lp": lp, "w": w, "trunc": tr, "loss": loss,
-            "stats": stats, "workspace": ws}
+    return {"dhidden": dh, "dweight": dw, "lp": lp, "w": w, "trunc": tr, "entropy": ent,
+            "loss": loss, "stats": stats, "workspace": ws}
 
 
 def cis_profile_next_call(begin: "torch.cuda.Event | None", end: "torch.cuda.Event | None"):

@@ -167,8 +167,8 @@ CIS_API const char *cis_status_string(int32_t status)
 
 CIS_API cis_status_t cis_token_logprobs(const void *logits, int32_t dtype, int64_t T, int64_t V,
                                         int64_t ld, const int32_t *ids, const uint8_t *mask,
-                                        float *lp_out, float *lse_out, int32_t *dev_status,
-                                        void *stream)
+                                        float *lp_out, float *lse_out, float *entropy_out,
+                                        int32_t *dev_status, void *stream)
 {
     if (!shape_ok(T, V, ld) || !dtype_ok(dtype))
         return CIS_ERR_INVALID_ARG;
@@ -185,6 +185,7 @@ CIS_API cis_status_t cis_token_logprobs(const void *logits, int32_t dtype, int64
     a.mask = mask;
     a.lp_out = lp_out;
     a.lse_out = lse_out;
+    a.entropy_out = entropy_out;
     a.status = dev_status;
     return cuda_status(launch_token_logprobs(a, dtype, (cudaStream_t)stream));
 }
@@ -229,8 +230,8 @@ CIS_API cis_status_t cis_loss_fwd_bwd(const void *logits, int32_t dtype, int64_t
                                       const uint8_t *mask, const int32_t *cu_seqlens, int64_t B,
                                       const cis_params_t *params, void *dlogits,
                                       int32_t dlogits_dtype, int64_t ld_out, float *lp_out,
-                                      float *w_out, uint8_t *trunc_out, cis_stats_t *stats_out,
-                                      double *loss_out, void *workspace,
+                                      float *w_out, uint8_t *trunc_out, float *entropy_out,
+                                      cis_stats_t *stats_out, double *loss_out, void *workspace,
                                       size_t workspace_bytes, void *stream)
 {
     if (!shape_ok(T, V, ld) || ld_out < V || !dtype_ok(dtype) || !dtype_ok(dlogits_dtype))
@@ -273,6 +274,7 @@ CIS_API cis_status_t cis_loss_fwd_bwd(const void *logits, int32_t dtype, int64_t
     a.lp_out = lp_out;
     a.w_out = w_out;
     a.trunc_out = trunc_out;
+    a.entropy_out = entropy_out;
     a.ws_w = reinterpret_cast<float *>(ws + L.w);
     a.ws_trunc = ws + L.trunc;
     a.ws_logk = reinterpret_cast<float *>(ws + L.logk);
@@ -294,6 +296,7 @@ CIS_API cis_status_t cis_loss_fwd_bwd(const void *logits, int32_t dtype, int64_t
             f.lp_inf = nullptr;
             f.lp_out = nullptr;
             f.lse_out = nullptr;
+            f.entropy_out = nullptr;  // the fused pass writes it
             f.lp64_out = a.ws_terms;
             if ((e = launch_token_logprobs(f, dtype, s)) != cudaSuccess)
                 return cuda_status(e);

@@ -178,6 +178,22 @@ __device__ __forceinline__ float sum8_exp2_off(const float (&z)[8], float off)
     return ((e[0] + e[1]) + (e[2] + e[3])) + ((e[4] + e[5]) + (e[6] + e[7]));
 }
 
+// The same, also accumulating u += e_i x_i with x_i = z_i log2e - off (the
+// exponent): the entropy term, in log2 units before the offset correction.
+// Entries whose exponential flushes to 0 (x_i <= -126) add nothing; x_i is
+// clamped so that -inf entries (e_i = 0) give 0, not NaN.
+__device__ __forceinline__ float sum8_exp2_off_u(const float (&z)[8], float off, float &u)
+{
+    float e[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+        const float x = fmaf(z[i], kLog2e, -off);
+        e[i] = ex2_ftz(x);
+        u = fmaf(e[i], fmaxf(x, -1024.0f), u);
+    }
+    return ((e[0] + e[1]) + (e[2] + e[3])) + ((e[4] + e[5]) + (e[6] + e[7]));
+}
+
 // 8 results to global memory with streaming (evict-first) 16-byte stores.
 template <typename OutT> __device__ __forceinline__ void store8(OutT *dst, const float (&v)[8]);
 template <>
@@ -200,11 +216,19 @@ __device__ __forceinline__ void store8<float>(float *dst, const float (&v)[8])
 
 constexpr int kChunks = 4;  // the slice is copied in this many pieces
 
-struct ClusterShared {
+// kEnt: the entropy variant exchanges (m, s, u) instead of (m, s).
+template <bool kEnt> struct ClusterShared {
     alignas(8) uint64_t bar[kChunks];  // completion of each copy chunk
     alignas(8) uint64_t xbar;          // arrival of the cluster's (m, s) pairs
     float2 part[kMaxCluster];
     MaxSum red[512 / 32];
+    float c, cs, B, lp;
+};
+template <> struct ClusterShared<true> {
+    alignas(8) uint64_t bar[kChunks];
+    alignas(8) uint64_t xbar;          // arrival of the cluster's (m, s, u) triples
+    float4 part[kMaxCluster];
+    MaxSumU red[512 / 32];
     float c, cs, B, lp;
 };
 
@@ -221,6 +245,17 @@ __device__ __forceinline__ void st_async_pair(uint32_t dst, float m, float s, ui
     asm volatile(
         "st.async.shared::cluster.mbarrier::complete_tx::bytes.v2.f32 [%0], {%1, %2}, [%3];"
         ::"r"(dst), "f"(m), "f"(s), "r"(bar)
+        : "memory");
+}
+
+// Store (m, s, u, 0) into another CTA's shared memory, counted like the pair.
+__device__ __forceinline__ void st_async_quad(uint32_t dst, float m, float s, float u,
+                                              uint32_t bar)
+{
+    asm volatile(
+        "st.async.shared::cluster.mbarrier::complete_tx::bytes.v4.f32 [%0], {%1, %2, %3, %4}, "
+        "[%5];" ::"r"(dst),
+        "f"(m), "f"(s), "f"(u), "f"(0.0f), "r"(bar)
         : "memory");
 }
 
@@ -255,11 +290,11 @@ __device__ __forceinline__ void wait_or_flag(uint32_t bar, bool cluster_scope, i
     }
 }
 
-template <typename InT, typename OutT, int kThreads>
+template <typename InT, typename OutT, int kThreads, bool kEnt>
 __global__ void __launch_bounds__(kThreads) cis_fused_cluster_kernel(const PassArgs a, int64_t slice)
 {
     extern __shared__ __align__(128) uint8_t dyn_smem[];
-    __shared__ ClusterShared sh;
+    __shared__ ClusterShared<kEnt> sh;
     // the bulk copy needs a 16-byte aligned destination; 128 bytes of slack
     // are allocated so the slab can start on a 128-byte boundary
     uint8_t *slab = dyn_smem + ((128 - (smem_u32(dyn_smem) & 127)) & 127);
@@ -285,6 +320,7 @@ __global__ void __launch_bounds__(kThreads) cis_fused_cluster_kernel(const PassA
             if (valid)
                 set_status(a.status, kStatusBadId);
             if (a.lp_out) a.lp_out[t] = lp;
+            if (kEnt) a.entropy_out[t] = lp;
             if (a.w_out) a.w_out[t] = 0.0f;
             if (a.trunc_out) a.trunc_out[t] = 0;
             a.ws_w[t] = 0.0f;
@@ -303,7 +339,7 @@ __global__ void __launch_bounds__(kThreads) cis_fused_cluster_kernel(const PassA
             mbar_init(smem_u32(&sh.bar[c]), 1);
         mbar_init(xbar, 1);
         // the one local arrival on xbar; the peers' stores bring the bytes
-        mbar_expect_tx(xbar, (uint32_t)(cs * sizeof(float2)));
+        mbar_expect_tx(xbar, (uint32_t)(cs * (kEnt ? sizeof(float4) : sizeof(float2))));
         const uint8_t *src = reinterpret_cast<const uint8_t *>(a.logits) +
                              (t * a.ld + v0) * (int64_t)sizeof(InT);
         for (int c = 0; c < kChunks; ++c) {
@@ -359,7 +395,7 @@ __global__ void __launch_bounds__(kThreads) cis_fused_cluster_kernel(const PassA
     // 2^{(z - m) log2e} is formed with one FMA as 2^{z log2e - cm}, cm = fl(m log2e);
     // the rounding residual of cm is exact (an FMA) and is taken out once at
     // the end, so the sum equals the one over (z - m) log2e.
-    float s = 0.0f;
+    float s = 0.0f, u = 0.0f;
     if (m != -INFINITY) {
         const float cm = m * kLog2e;
         const float cm_err = fmaf(m, kLog2e, -cm);  // m log2e - cm, exactly
@@ -367,29 +403,52 @@ __global__ void __launch_bounds__(kThreads) cis_fused_cluster_kernel(const PassA
         for (int g = threadIdx.x; g < ng; g += kThreads) {
             float z[8];
             load8<InT>(slab, g, z);
-            s += sum8_exp2_off(z, cm);
+            if (kEnt)
+                s += sum8_exp2_off_u(z, cm, u);
+            else
+                s += sum8_exp2_off(z, cm);
         }
-        s *= ex2_ftz(-cm_err);
+        const float f = ex2_ftz(-cm_err);
+        if (kEnt)  // sum e (z - m) = f ln2 (sum e x - cm_err sum e)
+            u = f * kLn2 * fmaf(-cm_err, s, u);
+        s *= f;
     }
-    const MaxSum mine = block_ms<kThreads, false>(MaxSum{m, s}, sh.red);
-
-    // Exchange the CTA pairs: lane r of warp 0 stores this CTA's pair into
-    // slot [rank] of CTA r, counted on CTA r's xbar.
-    cluster_wait();
-    if (threadIdx.x < cs)
-        st_async_pair(map_rank(smem_u32(&sh.part[rank]), threadIdx.x), mine.m, mine.s,
-                      map_rank(xbar, threadIdx.x));
+    // Exchange the CTA pairs (triples): lane r of warp 0 stores this CTA's
+    // values into slot [rank] of CTA r, counted on CTA r's xbar.
+    if constexpr (kEnt) {
+        const MaxSumU mine = block_msu<kThreads, false>(MaxSumU{m, s, u}, sh.red);
+        cluster_wait();
+        if (threadIdx.x < cs)
+            st_async_quad(map_rank(smem_u32(&sh.part[rank]), threadIdx.x), mine.m, mine.s,
+                          mine.u, map_rank(xbar, threadIdx.x));
+    } else {
+        const MaxSum mine = block_ms<kThreads, false>(MaxSum{m, s}, sh.red);
+        cluster_wait();
+        if (threadIdx.x < cs)
+            st_async_pair(map_rank(smem_u32(&sh.part[rank]), threadIdx.x), mine.m, mine.s,
+                          map_rank(xbar, threadIdx.x));
+    }
     wait_or_flag(xbar, true, a.status);
     // Everything addressed to this CTA has landed; tell the cluster, and wait
     // for the others' word only at exit (so no CTA leaves while stores into
     // its shared memory may be in flight).
     cluster_arrive_relaxed();
     MaxSum o{sh.part[0].x, sh.part[0].y};
-    for (unsigned r = 1; r < cs; ++r)
-        o = ms_combine(o, MaxSum{sh.part[r].x, sh.part[r].y});
+    MaxSumU ou{0.0f, 0.0f, 0.0f};
+    if constexpr (kEnt) {
+        ou = MaxSumU{sh.part[0].x, sh.part[0].y, sh.part[0].z};
+        for (unsigned r = 1; r < cs; ++r)
+            ou = msu_combine(ou, MaxSumU{sh.part[r].x, sh.part[r].y, sh.part[r].z});
+        o = MaxSum{ou.m, ou.s};
+    } else {
+        for (unsigned r = 1; r < cs; ++r)
+            o = ms_combine(o, MaxSum{sh.part[r].x, sh.part[r].y});
+    }
 
     if (threadIdx.x == 0) {
         const RowScalars rs = row_scalars(o, zy);
+        if (kEnt && rank == 0)
+            a.entropy_out[t] = row_entropy(ou, zy, rs.lp);
         const bool has_old = a.lp_old != nullptr;
         TokenWeight tw = token_weight(has_old ? (double)lold : rs.lp64, linf, a.P);
         if (a.w_in) {  // a sequence operator: the response's weight
@@ -512,10 +571,10 @@ int cluster_threads()
     return v;
 }
 
-template <typename InT, typename OutT, int NT>
+template <typename InT, typename OutT, int NT, bool kEnt = false>
 cudaError_t launch_cluster_nt(const PassArgs &a, const Plan &p, cudaStream_t s)
 {
-    auto kern = cis_fused_cluster_kernel<InT, OutT, NT>;
+    auto kern = cis_fused_cluster_kernel<InT, OutT, NT, kEnt>;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          (int)p.smem);
     if (e != cudaSuccess)
@@ -538,6 +597,8 @@ cudaError_t launch_cluster_nt(const PassArgs &a, const Plan &p, cudaStream_t s)
 template <typename InT, typename OutT>
 cudaError_t launch_cluster_t(const PassArgs &a, const Plan &p, cudaStream_t s)
 {
+    if (a.entropy_out)  // the entropy variant is built for 256 threads only
+        return launch_cluster_nt<InT, OutT, 256, true>(a, p, s);
     switch (cluster_threads()) {
     case 512: return launch_cluster_nt<InT, OutT, 512>(a, p, s);
     case 384: return launch_cluster_nt<InT, OutT, 384>(a, p, s);

@@ -26,6 +26,7 @@
 namespace cis {
 
 constexpr float kLog2e = 1.4426950408889634f;
+constexpr float kLn2 = 0.6931471805599453f;
 
 // Hyper-parameters as the kernels use them: fp32 copies for the fast path and
 // fp64 values (with logs taken on the host) for the certified fallback.
@@ -302,6 +303,60 @@ __device__ __forceinline__ MaxSum block_ms(MaxSum v, MaxSum *sh)
     return r;
 }
 
+// Row statistics with the entropy term: (m, s, u) over a set of entries, with
+// s = sum e^{z_j - m} and u = sum e^{z_j - m} (z_j - m).  Moving to a larger
+// offset m' scales both by f = e^{m - m'} and shifts u by (m - m') s.
+struct MaxSumU {
+    float m;
+    float s;
+    float u;
+};
+
+// (m, s) comes from ms_combine itself, so the entropy variants of the kernels
+// reduce (m, s) exactly as the others do; u follows the same offsets.
+__device__ __forceinline__ MaxSumU msu_combine(MaxSumU a, MaxSumU b)
+{
+    const MaxSum r = ms_combine(MaxSum{a.m, a.s}, MaxSum{b.m, b.s});
+    const float m = r.m;
+    if (m == -INFINITY)
+        return {m, r.s, a.u + b.u};
+    const float ua = a.m == -INFINITY ? a.u * 0.0f
+                                      : fmaf(a.m - m, a.s, a.u) * ex2_ftz((a.m - m) * kLog2e);
+    const float ub = b.m == -INFINITY ? b.u * 0.0f
+                                      : fmaf(b.m - m, b.s, b.u) * ex2_ftz((b.m - m) * kLog2e);
+    return {m, r.s, ua + ub};
+}
+
+__device__ __forceinline__ MaxSumU warp_msu(MaxSumU v)
+{
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        MaxSumU w;
+        w.m = __shfl_xor_sync(0xffffffffu, v.m, o);
+        w.s = __shfl_xor_sync(0xffffffffu, v.s, o);
+        w.u = __shfl_xor_sync(0xffffffffu, v.u, o);
+        v = msu_combine(v, w);
+    }
+    return v;
+}
+
+template <int NT, bool kReuse = true>
+__device__ __forceinline__ MaxSumU block_msu(MaxSumU v, MaxSumU *sh)
+{
+    v = warp_msu(v);
+    const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+    if (lane == 0)
+        sh[wid] = v;
+    __syncthreads();
+    MaxSumU r = sh[0];
+#pragma unroll
+    for (int i = 1; i < NT / 32; ++i)
+        r = msu_combine(r, sh[i]);
+    if (kReuse)
+        __syncthreads();
+    return r;
+}
+
 // Per-row scalars from (m', s') over j != y and z_y.  With the log-odds
 //   d = z_y - log sum_{j != y} e^{z_j} = (z_y - m') - log s',
 // log p = -softplus(-d) is accurate for p near 0 and near 1 (Sec. 3.3 notes
@@ -348,6 +403,28 @@ __device__ __forceinline__ RowScalars row_scalars(MaxSum o, float zy)
     r.m = o.m;
     r.bias_log2 = lse_m * kLog2e;
     return r;
+}
+
+// Entropy of the row's softmax, H = -sum_j p_j log p_j (the training-side
+// entropy the paper logs, App. D), from (m', s', u') over j != y and z_y.
+// With p the sampled token's probability and q_j = e^{z_j - m'} / s' the
+// distribution over the other entries,
+//   H = -p log p - (1 - p) log(1 - p) + (1 - p) H_q,   H_q = log s' - u'/s',
+// which has no cancellation when p is close to 0 or to 1; log p and
+// log(1 - p) both come from the log-odds d = (z_y - m') - log s'.
+__device__ __forceinline__ float row_entropy(MaxSumU o, float zy, float lp)
+{
+    if (o.m == -INFINITY && o.s == 0.0f)
+        return zy != zy ? zy : 0.0f;  // every other entry is -inf: p = 1
+    const float ls = logf(o.s);
+    const float d = (float)(((double)zy - (double)o.m) - (double)ls);
+    // log(1 - p) = -softplus(d)
+    const float l1mp = d > 0.0f ? -(d + log1pf(expf(-d))) : -log1pf(expf(d));
+    const float p = expf(lp), q = expf(l1mp);
+    const float hq = ls - o.u / o.s;
+    const float plp = p == 0.0f ? 0.0f : p * lp;      // 0 log 0 = 0
+    const float qlq = q == 0.0f ? 0.0f : q * l1mp;
+    return -plp - qlq + (q == 0.0f ? 0.0f : q * hq);
 }
 
 }  // namespace cis

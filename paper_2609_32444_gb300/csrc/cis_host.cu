@@ -53,7 +53,8 @@ cudaError_t streams_for_device(HostStreams **out)
 
 struct HostLayout {
     WsLayout base;
-    size_t ids, lpi, lpo, adv, mask, cu, lp, w, tr, stats, loss, in[kBufs], out[kBufs], total;
+    size_t ids, lpi, lpo, adv, mask, cu, lp, w, tr, ent, stats, loss, in[kBufs], out[kBufs],
+        total;
 };
 
 HostLayout host_layout(int64_t T, int64_t V, int isz, int osz, int64_t chunk, int64_t B)
@@ -72,6 +73,7 @@ HostLayout host_layout(int64_t T, int64_t V, int isz, int osz, int64_t chunk, in
     L.lp = o; o = up(o + 4 * n);
     L.w = o; o = up(o + 4 * n);
     L.tr = o; o = up(o + n);
+    L.ent = o; o = up(o + 4 * n);
     L.stats = o; o = up(o + sizeof(cis_stats_t));
     L.loss = o; o = up(o + 8);
     for (int b = 0; b < kBufs; ++b) {
@@ -109,7 +111,7 @@ CIS_API cis_status_t cis_loss_fwd_bwd_host(
     const void *logits, int32_t dtype, int64_t T, int64_t V, const int32_t *ids,
     const float *lp_infer, const float *lp_old, const float *adv, const uint8_t *mask,
     const int32_t *cu_seqlens, int64_t B, const cis_params_t *params, void *dlogits,
-    int32_t dlogits_dtype, float *lp_out, float *w_out, uint8_t *trunc_out,
+    int32_t dlogits_dtype, float *lp_out, float *w_out, uint8_t *trunc_out, float *entropy_out,
     cis_stats_t *stats_out, double *loss_out, int64_t chunk_tokens, void *workspace,
     size_t workspace_bytes, void *stream)
 {
@@ -175,6 +177,7 @@ CIS_API cis_status_t cis_loss_fwd_bwd_host(
     a.lp_out = reinterpret_cast<float *>(dptr(L.lp));
     a.w_out = reinterpret_cast<float *>(dptr(L.w));
     a.trunc_out = dptr(L.tr);
+    a.entropy_out = entropy_out ? reinterpret_cast<float *>(dptr(L.ent)) : nullptr;
     a.ws_w = reinterpret_cast<float *>(dptr(L.base.w));
     a.ws_trunc = dptr(L.base.trunc);
     a.ws_logk = reinterpret_cast<float *>(dptr(L.base.logk));
@@ -247,6 +250,7 @@ CIS_API cis_status_t cis_loss_fwd_bwd_host(
             c.lp_out = a.lp_out + r0;
             c.w_out = a.w_out + r0;
             c.trunc_out = a.trunc_out + r0;
+            c.entropy_out = a.entropy_out ? a.entropy_out + r0 : nullptr;
             c.ws_w = a.ws_w + r0;
             c.ws_trunc = a.ws_trunc + r0;
             c.ws_logk = a.ws_logk + r0;
@@ -280,6 +284,8 @@ CIS_API cis_status_t cis_loss_fwd_bwd_host(
                 cudaMemcpyAsync(w_out, a.w_out, 4 * n, cudaMemcpyDeviceToHost, sc);
             if (st == CIS_OK && trunc_out)
                 cudaMemcpyAsync(trunc_out, a.trunc_out, n, cudaMemcpyDeviceToHost, sc);
+            if (st == CIS_OK && entropy_out)
+                cudaMemcpyAsync(entropy_out, a.entropy_out, 4 * n, cudaMemcpyDeviceToHost, sc);
             if (st == CIS_OK && stats_out)
                 cudaMemcpyAsync(stats_out, stats_dev, sizeof(cis_stats_t),
                                 cudaMemcpyDeviceToHost, sc);

@@ -36,6 +36,7 @@ struct PassArgs {
     const float *w_in;
     const uint8_t *trunc_in;
     double *lp64_out;      // forward-only kernel: log p in fp64 (may be null)
+    float *entropy_out;    // per-token entropy of the softmax (may be null)
 };
 
 // Host-side parameter checks and the kernels' copy of the parameters.

@@ -87,6 +87,7 @@ struct GemmArgs {
     const int32_t *ids;
     const float *lse, *cvec;
     float2 *part;     // kStats: [nNt, T] (max, sum) over j != y
+    float *part_u;    // kStats: [nNt, T] sum e^{z - max} (z - max), or null (no entropy)
     float *zy;        // kStats: z at the sampled token
     uint16_t *dz;     // kDz: bf16 [Tp, ld_dz], column = chunk-local vocabulary index
     uint16_t *dzt;    // kDz: bf16 [chunk, ld_dzt], column = token
@@ -254,7 +255,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (EPI == kStats) {
                 const int row = m * kBM + r;  // token
                 const int y_r = row < g.T ? g.ids[row] : -1;
-                float mx = -INFINITY, s = 0.0f, zyv = 0.0f;
+                const bool ent = g.part_u != nullptr;
+                float mx = -INFINITY, s = 0.0f, u = 0.0f, zyv = 0.0f;
                 bool got_y = false;
                 for (int c0 = 0; c0 < kBN; c0 += 32) {
                     float v[32];
@@ -275,19 +277,38 @@ __global__ void __launch_bounds__(kThreads, 1)
                         cm = fmaxf(cm, v[q]);
                     }
                     if (cm > mx) {
-                        s = mx == -INFINITY ? 0.0f : s * ex2_ftz((mx - cm) * kLog2e);
+                        if (mx == -INFINITY) {
+                            s = 0.0f;
+                            u = 0.0f;
+                        } else {
+                            const float d = mx - cm, f = ex2_ftz(d * kLog2e);
+                            u = fmaf(d, s, u) * f;
+                            s *= f;
+                        }
                         mx = cm;
                     }
                     if (mx != -INFINITY) {
-                        float a = 0.0f;
+                        float a = 0.0f, au = 0.0f;
+                        if (ent) {  // the entropy term, e (z - max)
 #pragma unroll
-                        for (int q = 0; q < 32; ++q)
-                            a += ex2_ftz((v[q] - mx) * kLog2e);
+                            for (int q = 0; q < 32; ++q) {
+                                const float d = v[q] - mx, e = ex2_ftz(d * kLog2e);
+                                a += e;
+                                au = fmaf(e, fmaxf(d, -1024.0f), au);
+                            }
+                        } else {
+#pragma unroll
+                            for (int q = 0; q < 32; ++q)
+                                a += ex2_ftz((v[q] - mx) * kLog2e);
+                        }
                         s += a;
+                        u += au;
                     }
                 }
                 if (row < g.T) {
                     g.part[(int64_t)n * g.T + row] = make_float2(mx, s);
+                    if (ent)
+                        g.part_u[(int64_t)n * g.T + row] = u;
                     if (got_y)
                         g.zy[row] = zyv;
                 }
@@ -388,8 +409,8 @@ __global__ void cis_lmhead_to_bf16_kernel(const float *src, uint16_t *dst, int64
 }
 
 // Per token: combine the FWD pairs, then log p, weight, loss, c_t (one warp).
-__global__ void cis_lmhead_token_kernel(const PassArgs a, const float2 *part, const float *zy,
-                                        int nVt, float *lse_out, float *c_out)
+__global__ void cis_lmhead_token_kernel(const PassArgs a, const float2 *part, const float *part_u,
+                                        const float *zy, int nVt, float *lse_out, float *c_out)
 {
     const int64_t t = blockIdx.x * (int64_t)(blockDim.x / 32) + (threadIdx.x >> 5);
     const int lane = threadIdx.x & 31;
@@ -410,19 +431,32 @@ __global__ void cis_lmhead_token_kernel(const PassArgs a, const float2 *part, co
             a.ws_trunc[t] = 0;
             a.ws_logk[t] = 0.0f;
             a.ws_terms[t] = valid ? (double)NAN : 0.0;
+            if (a.entropy_out) a.entropy_out[t] = lp;
             lse_out[t] = 0.0f;
             c_out[t] = 0.0f;
         }
         return;
     }
     MaxSum o{-INFINITY, 0.0f};
-    for (int j = lane; j < nVt; j += 32) {
-        const float2 q = part[(int64_t)j * a.T + t];
-        o = ms_combine(o, MaxSum{q.x, q.y});
+    MaxSumU ou{-INFINITY, 0.0f, 0.0f};
+    if (part_u) {
+        for (int j = lane; j < nVt; j += 32) {
+            const float2 q = part[(int64_t)j * a.T + t];
+            ou = msu_combine(ou, MaxSumU{q.x, q.y, part_u[(int64_t)j * a.T + t]});
+        }
+        ou = warp_msu(ou);
+        o = MaxSum{ou.m, ou.s};
+    } else {
+        for (int j = lane; j < nVt; j += 32) {
+            const float2 q = part[(int64_t)j * a.T + t];
+            o = ms_combine(o, MaxSum{q.x, q.y});
+        }
+        o = warp_ms(o);
     }
-    o = warp_ms(o);
     if (lane == 0) {
         const RowScalars rs = row_scalars(o, zy[t]);
+        if (part_u && a.entropy_out)
+            a.entropy_out[t] = row_entropy(ou, zy[t], rs.lp);
         if (is_seq_mode(a.P.mode) && a.w_in == nullptr) {
             // sequence operator, first sweep: log p only (the response's
             // weight needs every token of the response)
@@ -530,7 +564,7 @@ cudaError_t launch_gemm(const CUtensorMap &a, const CUtensorMap &b, const GemmAr
 // for vocabulary chunks of Vc columns (a multiple of 256).
 struct LmLayout {
     WsLayout base;
-    size_t lse, c, zy, part, wt, ht, dh, dz, dzt, total;
+    size_t lse, c, zy, part, part_u, wt, ht, dh, dz, dzt, total;
     int64_t vp, tp, Tp, Vc;
 };
 
@@ -555,6 +589,8 @@ LmLayout lm_layout(int64_t T, int64_t V, int64_t Hd, int64_t Vc)
     o = up(o + 4 * (size_t)T);
     L.part = o;
     o = up(o + 8 * (size_t)T * (size_t)nVt);
+    L.part_u = o;
+    o = up(o + 4 * (size_t)T * (size_t)nVt);
     L.wt = o;
     o = up(o + 2 * (size_t)Hd * (size_t)L.vp);
     L.ht = o;
@@ -627,9 +663,9 @@ CIS_API cis_status_t cis_lmhead_fused(const void *hidden, const void *weight, in
                                       const int32_t *cu_seqlens, int64_t B,
                                       const cis_params_t *params, void *dhidden, void *dweight,
                                       int32_t grad_dtype, float *lp_out, float *w_out,
-                                      uint8_t *trunc_out, cis_stats_t *stats_out,
-                                      double *loss_out, void *workspace, size_t workspace_bytes,
-                                      void *stream)
+                                      uint8_t *trunc_out, float *entropy_out,
+                                      cis_stats_t *stats_out, double *loss_out, void *workspace,
+                                      size_t workspace_bytes, void *stream)
 {
     if (T < 0 || T > (1LL << 30) || V <= 0 || V > (1LL << 30) || H <= 0 || H > (1LL << 20))
         return CIS_ERR_INVALID_ARG;
@@ -670,6 +706,7 @@ CIS_API cis_status_t cis_lmhead_fused(const void *hidden, const void *weight, in
     a.lp_out = lp_out;
     a.w_out = w_out;
     a.trunc_out = trunc_out;
+    a.entropy_out = entropy_out;
     a.ws_w = reinterpret_cast<float *>(ws + L.base.w);
     a.ws_trunc = ws + L.base.trunc;
     a.ws_logk = reinterpret_cast<float *>(ws + L.base.logk);
@@ -680,6 +717,7 @@ CIS_API cis_status_t cis_lmhead_fused(const void *hidden, const void *weight, in
     float *cv = reinterpret_cast<float *>(ws + L.c);
     float *zy = reinterpret_cast<float *>(ws + L.zy);
     float2 *part = reinterpret_cast<float2 *>(ws + L.part);
+    float *part_u = entropy_out ? reinterpret_cast<float *>(ws + L.part_u) : nullptr;
     __nv_bfloat16 *wt = reinterpret_cast<__nv_bfloat16 *>(ws + L.wt);
     __nv_bfloat16 *ht = reinterpret_cast<__nv_bfloat16 *>(ws + L.ht);
     uint16_t *dz = reinterpret_cast<uint16_t *>(ws + L.dz);
@@ -708,6 +746,7 @@ CIS_API cis_status_t cis_lmhead_fused(const void *hidden, const void *weight, in
         g.lse = lse;
         g.cvec = cv;
         g.part = part;
+        g.part_u = part_u;
         g.zy = zy;
         g.dz = dz;
         g.dzt = dzt;
@@ -729,8 +768,8 @@ CIS_API cis_status_t cis_lmhead_fused(const void *hidden, const void *weight, in
             if (lp_old == nullptr) {
                 PassArgs f = a;
                 f.lp64_out = a.ws_terms;
-                lm::cis_lmhead_token_kernel<<<(unsigned)((T + 7) / 8), 256, 0, s>>>(f, part, zy, nVt,
-                                                                                lse, cv);
+                lm::cis_lmhead_token_kernel<<<(unsigned)((T + 7) / 8), 256, 0, s>>>(
+                    f, part, part_u, zy, nVt, lse, cv);
                 if ((e = cudaGetLastError()) != cudaSuccess)
                     return CIS_ERR_CUDA;
             }
@@ -743,7 +782,8 @@ CIS_API cis_status_t cis_lmhead_fused(const void *hidden, const void *weight, in
             a.w_in = a.ws_w;
             a.trunc_in = a.ws_trunc;
         }
-        lm::cis_lmhead_token_kernel<<<(unsigned)((T + 7) / 8), 256, 0, s>>>(a, part, zy, nVt, lse, cv);
+        lm::cis_lmhead_token_kernel<<<(unsigned)((T + 7) / 8), 256, 0, s>>>(a, part, part_u, zy,
+                                                                            nVt, lse, cv);
         if ((e = cudaGetLastError()) != cudaSuccess)
             return CIS_ERR_CUDA;
         // transposed copies of W and H (K-major B operands of DH and DW)

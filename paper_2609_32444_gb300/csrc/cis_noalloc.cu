@@ -65,7 +65,7 @@ extern "C" CIS_API cis_status_t cis_loss_fwd_bwd_noalloc(
     const float *lp_infer, const float *lp_old, const float *adv, const uint8_t *mask,
     const int32_t *cu_seqlens, int64_t B, const cis_params_t *params, void *dlogits,
     int32_t dlogits_dtype, int64_t ld_out, float *lp_out, float *w_out, uint8_t *trunc_out,
-    cis_stats_t *stats_out, double *loss_out, void *stream)
+    float *entropy_out, cis_stats_t *stats_out, double *loss_out, void *stream)
 {
     if (T > kMaxTokens)
         return CIS_ERR_UNSUPPORTED;
@@ -77,5 +77,6 @@ extern "C" CIS_API cis_status_t cis_loss_fwd_bwd_noalloc(
         return st;
     return cis_loss_fwd_bwd(logits, dtype, T, V, ld, ids, lp_infer, lp_old, adv, mask,
                             cu_seqlens, B, params, dlogits, dlogits_dtype, ld_out, lp_out, w_out,
-                            trunc_out, stats_out, loss_out, scratch, kScratchBytes, stream);
+                            trunc_out, entropy_out, stats_out, loss_out, scratch, kScratchBytes,
+                            stream);
 }

@@ -59,6 +59,36 @@ __device__ __forceinline__ void ms_update(MaxSum &acc, const float (&z)[EV], int
     }
 }
 
+// The same for (m, s, u): (m, s) by the update above, so that it is the same
+// bit for bit; u = sum e^{z - m} (z - m) follows the offset.
+template <int EV>
+__device__ __forceinline__ void ms_update(MaxSumU &acc, const float (&z)[EV], int skip)
+{
+    const float m0 = acc.m, s0 = acc.s;
+    MaxSum ms{acc.m, acc.s};
+    ms_update<EV>(ms, z, skip);
+    float u = acc.u;
+    if (!(ms.m == m0)) {  // the offset moved (or became NaN)
+        if (m0 == -INFINITY) {
+            u = u * 0.0f;
+        } else {
+            const float d = m0 - ms.m;
+            u = fmaf(d, s0, u) * ex2_ftz(d * kLog2e);
+        }
+    }
+    if (ms.m != -INFINITY) {
+#pragma unroll
+        for (int i = 0; i < EV; ++i) {
+            const float d = z[i] - ms.m;
+            const float e = i == skip ? 0.0f : ex2_ftz(d * kLog2e);
+            u = fmaf(e, fmaxf(d, -1024.0f), u);
+        }
+    }
+    acc.m = ms.m;
+    acc.s = ms.s;
+    acc.u = u;
+}
+
 template <typename InT, bool kStream>
 __device__ __forceinline__ uint4 load16(const uint4 *p)
 {
@@ -79,12 +109,13 @@ __device__ __forceinline__ void unpack(uint4 q, float (&z)[4])
     z[2] = __uint_as_float(q.z); z[3] = __uint_as_float(q.w);
 }
 
-// This thread's (m, s) over entries j != y of one row.
-template <typename InT, bool kStream>
-__device__ MaxSum row_stats(const InT *row, int64_t V, int64_t y)
+// This thread's (m, s) -- or (m, s, u) -- over entries j != y of one row.
+template <typename InT, bool kStream, typename Acc = MaxSum>
+__device__ Acc row_stats(const InT *row, int64_t V, int64_t y)
 {
     constexpr int EV = 16 / sizeof(InT);
-    MaxSum acc{-INFINITY, 0.0f};
+    Acc acc{};
+    acc.m = -INFINITY;
     int64_t j0 = 0;
     if ((reinterpret_cast<uintptr_t>(row) & 15) == 0) {
         const int64_t nvec = V / EV;
@@ -104,15 +135,19 @@ __device__ MaxSum row_stats(const InT *row, int64_t V, int64_t y)
     return acc;
 }
 
-struct RowShared {
+template <bool kEnt> struct RowShared {
     MaxSum red[kRowThreads / 32];
     float c, m, bias, lp;
 };
+template <> struct RowShared<true> {
+    MaxSumU red[kRowThreads / 32];
+    float c, m, bias, lp;
+};
 
-template <typename InT, typename OutT, bool kBwd>
+template <typename InT, typename OutT, bool kBwd, bool kEnt>
 __global__ void __launch_bounds__(kRowThreads) cis_fused_row_kernel(const PassArgs a)
 {
-    __shared__ RowShared sh;
+    __shared__ RowShared<kEnt> sh;
     const int64_t t = blockIdx.x;
     const bool valid = a.mask == nullptr || a.mask[t] != 0;
     const int64_t y = a.ids[t];
@@ -130,6 +165,7 @@ __global__ void __launch_bounds__(kRowThreads) cis_fused_row_kernel(const PassAr
             if (a.lp_out) a.lp_out[t] = lp;
             if (a.lse_out) a.lse_out[t] = lp;
             if (!kBwd && a.lp64_out) a.lp64_out[t] = lp;
+            if (kEnt) a.entropy_out[t] = lp;
             if (kBwd) {
                 if (a.w_out) a.w_out[t] = 0.0f;
                 if (a.trunc_out) a.trunc_out[t] = 0;
@@ -142,9 +178,18 @@ __global__ void __launch_bounds__(kRowThreads) cis_fused_row_kernel(const PassAr
         return;
     }
     const InT *row = reinterpret_cast<const InT *>(a.logits) + t * a.ld;
-    const MaxSum o = block_ms<kRowThreads>(row_stats<InT, !kBwd>(row, a.V, y), sh.red);
+    MaxSum o;
+    MaxSumU ou{0.0f, 0.0f, 0.0f};
+    if constexpr (kEnt) {
+        ou = block_msu<kRowThreads>(row_stats<InT, !kBwd, MaxSumU>(row, a.V, y), sh.red);
+        o = MaxSum{ou.m, ou.s};
+    } else {
+        o = block_ms<kRowThreads>(row_stats<InT, !kBwd>(row, a.V, y), sh.red);
+    }
     if (threadIdx.x == 0) {
         const RowScalars rs = row_scalars(o, to_f32(row[y]));
+        if (kEnt)
+            a.entropy_out[t] = row_entropy(ou, to_f32(row[y]), rs.lp);
         if (a.lp_out) a.lp_out[t] = rs.lp;
         if (a.lse_out) a.lse_out[t] = rs.lse;
         if (!kBwd && a.lp64_out) a.lp64_out[t] = rs.lp64;
@@ -188,7 +233,10 @@ cudaError_t launch_row(const PassArgs &a, cudaStream_t s)
 {
     if (a.T == 0)
         return cudaSuccess;
-    cis_fused_row_kernel<InT, OutT, kBwd><<<(unsigned)a.T, kRowThreads, 0, s>>>(a);
+    if (a.entropy_out)
+        cis_fused_row_kernel<InT, OutT, kBwd, true><<<(unsigned)a.T, kRowThreads, 0, s>>>(a);
+    else
+        cis_fused_row_kernel<InT, OutT, kBwd, false><<<(unsigned)a.T, kRowThreads, 0, s>>>(a);
     return cudaGetLastError();
 }
 

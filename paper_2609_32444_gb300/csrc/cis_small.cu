@@ -153,19 +153,51 @@ __global__ void __launch_bounds__(kSeqThreads)
 }
 
 struct RedPart {
-    double loss, excess;
+    double loss, excess, ent;
     long long nvalid, ntrunc;
     float maxlk;
 };
 
-// One CTA: thread i sums tokens i, i + 1024, ... in order, then a fixed tree.
+__device__ __forceinline__ RedPart red_add(RedPart a, const RedPart &b)
+{
+    a.loss += b.loss;
+    a.excess += b.excess;
+    a.ent += b.ent;
+    a.nvalid += b.nvalid;
+    a.ntrunc += b.ntrunc;
+    a.maxlk = fmaxf(a.maxlk, b.maxlk);
+    return a;
+}
+
+__device__ __forceinline__ RedPart red_shfl(const RedPart &v, int o)
+{
+    RedPart r;
+    r.loss = __shfl_xor_sync(0xffffffffu, v.loss, o);
+    r.excess = __shfl_xor_sync(0xffffffffu, v.excess, o);
+    r.ent = __shfl_xor_sync(0xffffffffu, v.ent, o);
+    r.nvalid = __shfl_xor_sync(0xffffffffu, v.nvalid, o);
+    r.ntrunc = __shfl_xor_sync(0xffffffffu, v.ntrunc, o);
+    r.maxlk = __shfl_xor_sync(0xffffffffu, v.maxlk, o);
+    return r;
+}
+
+__device__ __forceinline__ RedPart red_warp(RedPart v)
+{
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1)
+        v = red_add(v, red_shfl(v, o));
+    return v;
+}
+
+// One CTA: thread i sums tokens i, i + 1024, ... in order, then a fixed tree
+// (within each warp, then over the 32 warps), so the sums are deterministic.
 __global__ void __launch_bounds__(kSmallThreads)
     cis_reduce_kernel(const uint8_t *mask, int64_t T, const double *terms, const float *logk,
-                  const float *w, const uint8_t *trunc, const int32_t *status,
-                  cis_stats_t *stats, double *loss_out)
+                  const float *w, const uint8_t *trunc, const float *entropy,
+                  const int32_t *status, cis_stats_t *stats, double *loss_out)
 {
-    __shared__ RedPart sh[kSmallThreads];
-    RedPart p{0.0, 0.0, 0, 0, 0.0f};
+    __shared__ RedPart sh[kSmallThreads / 32];
+    RedPart p{0.0, 0.0, 0.0, 0, 0, 0.0f};
     for (int64_t t = threadIdx.x; t < T; t += kSmallThreads) {
         p.loss += terms[t];
         if (!is_valid(mask, t))
@@ -177,32 +209,28 @@ __global__ void __launch_bounds__(kSmallThreads)
             p.ntrunc += 1;
             p.excess += exp((double)lk) - (double)w[t];
         }
+        if (entropy)
+            p.ent += (double)entropy[t];
     }
-    sh[threadIdx.x] = p;
+    p = red_warp(p);
+    const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+    if (lane == 0)
+        sh[wid] = p;
     __syncthreads();
-    for (int stride = kSmallThreads / 2; stride > 0; stride >>= 1) {
-        if (threadIdx.x < stride) {
-            RedPart &a = sh[threadIdx.x];
-            const RedPart &b = sh[threadIdx.x + stride];
-            a.loss += b.loss;
-            a.excess += b.excess;
-            a.nvalid += b.nvalid;
-            a.ntrunc += b.ntrunc;
-            a.maxlk = fmaxf(a.maxlk, b.maxlk);
-        }
-        __syncthreads();
-    }
-    if (threadIdx.x == 0) {
-        const RedPart &r = sh[0];
-        if (loss_out)
-            *loss_out = r.loss;
-        if (stats) {
-            stats->loss = r.loss;
-            stats->trunc_excess = r.excess;
-            stats->n_valid = r.nvalid;
-            stats->n_truncated = r.ntrunc;
-            stats->max_abs_logk = r.maxlk;
-            stats->status = status ? *status : 0;
+    if (wid == 0) {
+        p = red_warp(sh[lane]);
+        if (lane == 0) {
+            if (loss_out)
+                *loss_out = p.loss;
+            if (stats) {
+                stats->loss = p.loss;
+                stats->trunc_excess = p.excess;
+                stats->n_valid = p.nvalid;
+                stats->n_truncated = p.ntrunc;
+                stats->max_abs_logk = p.maxlk;
+                stats->status = status ? *status : 0;
+                stats->entropy_sum = p.ent;
+            }
         }
     }
 }
@@ -235,7 +263,7 @@ cudaError_t launch_weights(const float *lp_w, const float *lp_inf, const uint8_t
 cudaError_t launch_reduce(const PassArgs &a, cis_stats_t *stats, double *loss, cudaStream_t s)
 {
     cis_reduce_kernel<<<1, kSmallThreads, 0, s>>>(a.mask, a.T, a.ws_terms, a.ws_logk, a.ws_w,
-                                               a.ws_trunc, a.status, stats, loss);
+                                               a.ws_trunc, a.entropy_out, a.status, stats, loss);
     return cudaGetLastError();
 }
 

@@ -82,7 +82,7 @@ def _fwd_bwd_rc(binding, **over):
     return L.cis_loss_fwd_bwd(args["logits"], args["dtype"], args["T"], args["V"], args["ld"],
                               args["ids"], args["lp_inf"], args["lp_old"], args["adv"],
                               args["mask"], args["cu"], args["B"], ctypes.byref(p), args["dz"],
-                              args["dz_dt"], args["ld_out"], None, None, None, None, None,
+                              args["dz_dt"], args["ld_out"], None, None, None, None, None, None,
                               args["ws"], args["ws_bytes"], None)
 
 
@@ -120,9 +120,12 @@ def test_other_entry_points_reject_bad_arguments(binding):
     L = binding.lib()
     fake = ctypes.c_void_p(0x10000)
     p = binding.cis_default_params()
-    assert L.cis_token_logprobs(fake, 1, 4, 8, 7, fake, None, fake, None, None, None) == 1
-    assert L.cis_token_logprobs(None, 1, 4, 8, 8, fake, None, fake, None, None, None) == 1
-    assert L.cis_token_logprobs(fake, 1, 0, 8, 8, None, None, None, None, None, None) == 0
+    assert L.cis_token_logprobs(fake, 1, 4, 8, 7, fake, None, fake, None, None, None,
+                                None) == 1
+    assert L.cis_token_logprobs(None, 1, 4, 8, 8, fake, None, fake, None, None, None,
+                                None) == 1
+    assert L.cis_token_logprobs(fake, 1, 0, 8, 8, None, None, None, None, None, None,
+                                None) == 0
     p.kappa = 2.0
     assert L.cis_weights(fake, fake, None, 4, None, 0, ctypes.byref(p), fake, None, None,
                          None) == 1

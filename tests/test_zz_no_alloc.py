@@ -30,7 +30,7 @@ def noalloc():
     P, i32, i64 = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64
     f = L.cis_loss_fwd_bwd_noalloc
     f.argtypes = [P, i32, i64, i64, i64, P, P, P, P, P, P, i64,
-                  ctypes.POINTER(binding.cis_params_t), P, i32, i64, P, P, P, P, P, P]
+                  ctypes.POINTER(binding.cis_params_t), P, i32, i64, P, P, P, P, P, P, P]
     f.restype = ctypes.c_int
     return f
 
@@ -47,7 +47,7 @@ def _call(f, g, P, T, V):
     ptr = lambda t: ctypes.c_void_p(t.data_ptr())  # noqa: E731
     rc = f(ptr(g["logits"]), binding.CIS_BF16, T, V, V, ptr(g["ids"]), ptr(g["lp"]), None,
            ptr(g["adv"]), ptr(g["mask"]), None, 0, ctypes.byref(P), ptr(out["dz"]),
-           binding.CIS_BF16, V, ptr(out["lp"]), ptr(out["w"]), ptr(out["trunc"]),
+           binding.CIS_BF16, V, ptr(out["lp"]), ptr(out["w"]), ptr(out["trunc"]), None,
            ptr(out["stats"]), ptr(out["loss"]),
            ctypes.c_void_p(torch.cuda.current_stream().cuda_stream))
     return rc, out
@@ -85,7 +85,7 @@ def test_noalloc_rejects_more_tokens_than_its_scratch(noalloc):
     fake = ctypes.c_void_p(0x10000)
     rc = noalloc(fake, binding.CIS_BF16, MAX_TOKENS + 1, 8, 8, fake, fake, None, fake, None,
                  None, 0, ctypes.byref(P), ctypes.c_void_p(0x4000000), binding.CIS_BF16, 8,
-                 None, None, None, None, None, None)
+                 None, None, None, None, None, None, None)
     assert rc == binding.CIS_ERR_UNSUPPORTED
 
 
@@ -105,7 +105,7 @@ def test_noalloc_sequence_operator(noalloc):
     ptr = lambda t: ctypes.c_void_p(t.data_ptr())  # noqa: E731
     rc = noalloc(ptr(g["logits"]), binding.CIS_F32, T, V, V, ptr(g["ids"]), ptr(g["lp"]), None,
                  ptr(g["adv"]), ptr(g["mask"]), ptr(g["cu"]), b.cu_seqlens.shape[0] - 1,
-                 ctypes.byref(P), ptr(dz), binding.CIS_F32, V, None, ptr(w), None, None,
+                 ctypes.byref(P), ptr(dz), binding.CIS_F32, V, None, ptr(w), None, None, None,
                  ptr(loss), ctypes.c_void_p(torch.cuda.current_stream().cuda_stream))
     assert rc == 0
     ref = binding.cis_loss_fwd_bwd(g["logits"], g["ids"], g["lp"], g["adv"], P, mask=g["mask"],
