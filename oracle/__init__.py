@@ -100,6 +100,10 @@ def _load():
         lib.oracle_loss_fwd_bwd.restype = ctypes.c_int
         lib.oracle_token_entropy.argtypes = [P, i32, i64, i64, i64, P, P, ctypes.c_int]
         lib.oracle_token_entropy.restype = None
+        lib.oracle_mismatch_diagnostics.argtypes = [P, P, i32, i64, i64, i64, P, P,
+                                                    ctypes.POINTER(OracleParams), P, P, P, P, P,
+                                                    ctypes.c_int]
+        lib.oracle_mismatch_diagnostics.restype = ctypes.c_int
         lib.oracle_max_threads.argtypes = []
         lib.oracle_max_threads.restype = ctypes.c_int
         _ = dbl
@@ -165,6 +169,30 @@ def token_entropy(logits, V=None, mask=None, nthreads=0):
     h = np.zeros(T, np.float64)
     lib.oracle_token_entropy(_ptr(a), dt, T, V, ld, _ptr(mask), _ptr(h), nthreads)
     return h
+
+
+def mismatch_diagnostics(z_train, z_infer, ids, P: OracleParams, mask=None, nthreads=0):
+    """Per-position mismatch diagnostics in fp64 (App. A.5, Sec. 4.3 Fig. 5c-d):
+    eps (Lemma 3.1's definition, normalised gauge), log k and p of the sampled
+    token, and over y ~ q the squared bias ||E[(f - k) grad log p]||^2 and the
+    variance increase of f grad log p over grad log p.  O(V^2) per position:
+    small V only.  Returns a dict of [T] arrays."""
+    lib = _load()
+    a, dt = _logits_arg(z_train)
+    b, dt2 = _logits_arg(z_infer)
+    if dt != dt2 or a.shape != b.shape:
+        raise ValueError("both logit tensors must have the same type and shape")
+    T, V = a.shape
+    ids = np.ascontiguousarray(ids, dtype=np.int32)
+    mask = _opt(mask, np.uint8)
+    out = {k: np.zeros(T, np.float64) for k in ("eps", "logk", "p", "bias2", "dvar")}
+    rc = lib.oracle_mismatch_diagnostics(_ptr(a), _ptr(b), dt, T, V, V, _ptr(ids), _ptr(mask),
+                                         ctypes.byref(P), _ptr(out["eps"]), _ptr(out["logk"]),
+                                         _ptr(out["p"]), _ptr(out["bias2"]), _ptr(out["dvar"]),
+                                         nthreads)
+    if rc != 0:
+        raise ValueError("the diagnostics take a token operator")
+    return out
 
 
 def weights(lp_w, lp_inf, P: OracleParams, mask=None, cu_seqlens=None):

@@ -614,3 +614,101 @@ int oracle_loss_fwd_bwd(const void *logits, int dtype, int64_t T, int64_t V, int
     free(terms);
     return bad ? -1 : 0;
 }
+
+/*
+ * Mismatch diagnostics from the two engines' full logits (App. A.5 and
+ * Sec. 4.3, Fig. 5c-d).  Per position t, with p = softmax(z_train),
+ * q = softmax(z_infer), the normalised gauge delta_j = log q_j - log p_j
+ * (App. A.5, "Gauge convention") and the sampled token y:
+ *   eps_t   = -delta_y + log sum_{j != y} w_j exp(delta_j),
+ *             w_j = e^{z_j} / sum_{j' != y} e^{z_j'}   (Lemma 3.1's definition)
+ *   logk_t  = log p_y - log q_y,  p_t = p_y
+ * and, for the weight operator f of `P` (a token operator) applied to every
+ * candidate token j (k_j = p_j / q_j), with g_j = e_j - p the gradient of
+ * log p_j with respect to the logits and expectations over y ~ q:
+ *   bias2_t = || E_q[(f_y - k_y) g_y] ||^2
+ *   dvar_t  = (E_q ||f_y g_y||^2 - ||E_q f_y g_y||^2) - (E_q ||g_y||^2 - ||E_q g_y||^2)
+ * Both vectors are formed explicitly (a V-vector per position), not from a
+ * closed form.  Masked rows get 0.  Returns 0, or -1 for a sequence operator
+ * (the candidates of one position have no response to share).
+ */
+int oracle_mismatch_diagnostics(const void *z_train, const void *z_infer, int dtype, int64_t T,
+                                int64_t V, int64_t ld, const int32_t *ids, const uint8_t *mask,
+                                const oracle_params_t *P, double *eps_out, double *logk_out,
+                                double *p_out, double *bias2_out, double *dvar_out, int nthreads)
+{
+    if (is_seq_mode(P->mode))
+        return -1;
+    set_threads(nthreads);
+#pragma omp parallel for schedule(dynamic, 1)
+    for (int64_t t = 0; t < T; ++t) {
+        double eps = 0.0, lk = 0.0, pt = 0.0, bias2 = 0.0, dvar = 0.0;
+        if (row_valid(mask, t)) {
+            const int64_t y = ids[t];
+            const double lse = row_lse(z_train, dtype, ld, t, V);
+            const double lsei = row_lse(z_infer, dtype, ld, t, V);
+            double *lp = (double *)malloc(sizeof(double) * (size_t)V);
+            double *lq = (double *)malloc(sizeof(double) * (size_t)V);
+            double *bvec = (double *)malloc(sizeof(double) * (size_t)V);
+            double *fvec = (double *)malloc(sizeof(double) * (size_t)V);
+            double *gvec = (double *)malloc(sizeof(double) * (size_t)V);
+            for (int64_t j = 0; j < V; ++j) {
+                lp[j] = logit_at(z_train, dtype, ld, t, j) - lse;
+                lq[j] = logit_at(z_infer, dtype, ld, t, j) - lsei;
+            }
+            /* eps by Lemma 3.1's definition, in the normalised gauge */
+            double Sy = 0.0, acc = 0.0;
+            for (int64_t j = 0; j < V; ++j)
+                if (j != y)
+                    Sy += exp(lp[j]);
+            for (int64_t j = 0; j < V; ++j)
+                if (j != y)
+                    acc += exp(lp[j]) / Sy * exp(lq[j] - lp[j]);
+            eps = -(lq[y] - lp[y]) + log(acc);
+            lk = lp[y] - lq[y];
+            pt = exp(lp[y]);
+            /* E_q[(f - k) g], E_q[f g], E_q[g] as V-vectors; second moments */
+            double e_f2g2 = 0.0, e_g2 = 0.0;
+            for (int64_t j = 0; j < V; ++j)
+                bvec[j] = fvec[j] = gvec[j] = 0.0;
+            for (int64_t yy = 0; yy < V; ++yy) {
+                const double qy = exp(lq[yy]);
+                if (qy == 0.0)
+                    continue;
+                double f, dummy_e;
+                int tr;
+                token_weight(lp[yy], lq[yy], P, &f, &tr, NULL, &dummy_e);
+                const double ky = exp(lp[yy] - lq[yy]);
+                double g2 = 0.0;
+                for (int64_t j = 0; j < V; ++j) {
+                    const double gj = (j == yy ? 1.0 : 0.0) - exp(lp[j]);
+                    bvec[j] += qy * (f - ky) * gj;
+                    fvec[j] += qy * f * gj;
+                    gvec[j] += qy * gj;
+                    g2 += gj * gj;
+                }
+                e_f2g2 += qy * f * f * g2;
+                e_g2 += qy * g2;
+            }
+            double nb = 0.0, nf = 0.0, ng = 0.0;
+            for (int64_t j = 0; j < V; ++j) {
+                nb += bvec[j] * bvec[j];
+                nf += fvec[j] * fvec[j];
+                ng += gvec[j] * gvec[j];
+            }
+            bias2 = nb;
+            dvar = (e_f2g2 - nf) - (e_g2 - ng);
+            free(lp);
+            free(lq);
+            free(bvec);
+            free(fvec);
+            free(gvec);
+        }
+        eps_out[t] = eps;
+        logk_out[t] = lk;
+        p_out[t] = pt;
+        bias2_out[t] = bias2;
+        dvar_out[t] = dvar;
+    }
+    return 0;
+}

@@ -632,3 +632,62 @@ def test_entropy_matches_50_digit_brute_force_and_is_shift_invariant(V):
         assert abs(h[t] - float(ref)) <= 1e-14 * max(1.0, float(ref))
     h2 = oracle.token_entropy(z + 123.25)
     np.testing.assert_allclose(h2, h, rtol=1e-12, atol=1e-13)
+
+
+# ------------------------------------------------------- mismatch diagnostics
+def _softmax64(z):
+    z = np.asarray(z, np.float64)
+    e = np.exp(z - z.max(axis=1, keepdims=True))
+    return e / e.sum(axis=1, keepdims=True)
+
+
+def _diag_inputs(seed, T=5, V=9, sd=0.4):
+    rng = np.random.default_rng(seed)
+    z = rng.standard_normal((T, V)) * 2.0
+    zi = z + rng.standard_normal((T, V)) * sd
+    ids = rng.integers(0, V, T).astype(np.int32)
+    return z, zi, ids
+
+
+@pytest.mark.parametrize("mode", [oracle.MODE_CIS, oracle.MODE_TIS, oracle.MODE_EXACT,
+                                  oracle.MODE_NONE, oracle.MODE_BAND, oracle.MODE_ICEPOP,
+                                  oracle.MODE_KPOP])
+def test_diagnostics_vanish_when_engines_agree(mode):
+    """Identical logits: eps = log k = 0, and every operator has f(1) = 1, so
+    the bias and the variance increase are 0."""
+    z, _, ids = _diag_inputs(60)
+    d = oracle.mismatch_diagnostics(z, z, ids, oracle.params(mode=mode))
+    for k in ("eps", "logk", "bias2", "dvar"):
+        assert np.all(np.abs(d[k]) < 1e-13), k
+
+
+def test_diagnostics_eps_is_the_log_odds_displacement():
+    """eps from Lemma 3.1's w_j definition in the normalised gauge equals
+    logit p - logit q (App. A.5) and satisfies k = p + (1 - p) e^eps."""
+    z, zi, ids = _diag_inputs(61, T=8)
+    d = oracle.mismatch_diagnostics(z, zi, ids, oracle.params())
+    p = _softmax64(z)[np.arange(8), ids]
+    q = _softmax64(zi)[np.arange(8), ids]
+    np.testing.assert_allclose(d["eps"], np.log(p / (1 - p)) - np.log(q / (1 - q)), atol=1e-12)
+    np.testing.assert_allclose(np.exp(d["logk"]), p + (1 - p) * np.exp(d["eps"]), rtol=1e-12)
+    np.testing.assert_allclose(d["p"], p, rtol=1e-13)
+
+
+def test_diagnostics_closed_forms_for_no_correction_and_exact_ratio():
+    """E_q[k grad log p] = sum_y p_y (e_y - p) = 0, so with no correction the
+    bias vector is E_q[grad log p] = q - p and the variance is unchanged;
+    the exact ratio (clamp inactive) is unbiased (Sec. 4.3) and its variance
+    increase is sum_y (p_y^2 / q_y)(1 - 2 p_y + |p|^2) - (1 - |q|^2)."""
+    z, zi, ids = _diag_inputs(62, T=6, V=11)
+    P_, Q_ = _softmax64(z), _softmax64(zi)
+    none = oracle.mismatch_diagnostics(z, zi, ids, oracle.params(mode=oracle.MODE_NONE))
+    np.testing.assert_allclose(none["bias2"], ((Q_ - P_) ** 2).sum(axis=1), rtol=1e-11)
+    assert np.all(np.abs(none["dvar"]) < 1e-13)
+    ex = oracle.mismatch_diagnostics(z, zi, ids, oracle.params(mode=oracle.MODE_EXACT))
+    assert np.all(ex["bias2"] < 1e-26)
+    p2 = (P_ ** 2).sum(axis=1, keepdims=True)
+    dv = ((P_ ** 2 / Q_) * (1 - 2 * P_ + p2)).sum(axis=1) - (1 - (Q_ ** 2).sum(axis=1))
+    np.testing.assert_allclose(ex["dvar"], dv, rtol=1e-10)
+    # a truncating operator is biased and adds less variance than the exact ratio
+    cis = oracle.mismatch_diagnostics(z, zi, ids, oracle.params(mode=oracle.MODE_CIS, lam=0.2))
+    assert np.all(cis["bias2"] >= 0) and np.all(cis["dvar"] <= ex["dvar"] + 1e-15)
