@@ -50,7 +50,7 @@ def parse_args():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--mode", choices=["cis", "tis", "exact", "none"], default="cis")
-    ap.add_argument("--workload", type=int, default=3, choices=[2, 3, 4, 5])
+    ap.add_argument("--workload", type=int, default=3, choices=[2, 3, 4, 5, 6])
     ap.add_argument("--dlogits", choices=["bf16", "f32"], default="bf16")
     ap.add_argument("--e2e-steps", type=int, default=10)
     ap.add_argument("--e2e-chunk", type=int, default=2048)
@@ -492,6 +492,83 @@ def run_lmhead(args, rank, world, local):
         print(json.dumps(line), flush=True)
 
 
+def run_diag(args, rank, world, local):
+    """Workload 6: the mismatch diagnostics over both engines' logits."""
+    import numpy as np
+    import torch
+    from paper_2609_32444_gb300 import binding, build, synth
+
+    build.build()
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    spec = synth.WORKLOADS[6]
+    b = synth.make_batch(6, device=dev, seed=1006 + 7919 * rank, T=args.tokens)
+    T, V = b.T, b.V
+    zi = b.extra["logits_infer"]
+    P = binding.cis_default_params(args.mode, lam=b.lam)
+
+    def step():
+        return binding.cis_mismatch_diagnostics(b.logits, zi, b.ids, P, mask=b.mask)
+
+    for _ in range(max(3, args.warmup)):
+        out = step()
+    torch.cuda.synchronize()
+    barrier(world)
+    stream = torch.cuda.current_stream()
+    clocks = ClockSampler(physical_gpu_index(local))
+    time.sleep(0.5)
+    start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize()
+    barrier(world)
+    h0 = time.time()
+    start.record(stream)
+    for _ in range(args.steps):
+        out = step()
+    end.record(stream)
+    torch.cuda.synchronize()
+    h1 = time.time()
+    barrier(world)
+    clocks.mark(h0, h1)
+    ms = max_over_ranks(start.elapsed_time(end), world) / args.steps
+    # one launch per call: both tensors read once (the second pass is meant to
+    # hit L2), ids and mask read, five floats written per position
+    alg_bytes = 2 * T * V * b.logits.element_size() + T * (4 + 1) + 5 * 4 * T
+    peak, peak_src = measured_peaks()
+    achieved = alg_bytes / (ms / 1e3) / 1e9
+    cpu = None
+    if rank == 0 and not args.no_cpu_baseline:
+        import oracle
+        rows = [0]
+        zt_h = b.logits[rows].cpu().contiguous().view(torch.int16).numpy().view(np.uint16)
+        zi_h = zi[rows].cpu().contiguous().view(torch.int16).numpy().view(np.uint16)
+        t0 = time.perf_counter()
+        oracle.mismatch_diagnostics(zt_h, zi_h, b.ids[rows].cpu().numpy(),
+                                    oracle.params(mode={"cis": 0, "tis": 1, "exact": 2,
+                                                        "none": 3}[args.mode], lam=b.lam))
+        el = time.perf_counter() - t0
+        cpu = {"value": len(rows) / el, "unit": "positions/s", "cores": 1, "kind": "oracle",
+               "sample": f"{len(rows)} position of V={V}: explicit fp64 expectation vectors "
+                         f"(O(V^2) per position), one host thread"}
+    if rank == 0:
+        line = {
+            "metric": "CIS mismatch diagnostics positions/s at V=151936 bf16 (two logit tensors)",
+            "value": T * world / (ms / 1e3), "unit": "positions/s", "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+            "data": "synthetic",
+            "config": {"workload": spec["name"], "T": T, "V": V, "mode": args.mode,
+                       "io_dtype": "bf16",
+                       "l2": "no flush: the 9.96 GB of logits per step exceed the L2"},
+            "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
+                         "frac": achieved / peak, "traffic": None,
+                         "kernel": "cis_mismatch_kernel<bf16> (two passes over both rows)",
+                         "algorithmic_bytes_per_launch": alg_bytes, "peak_source": peak_src},
+            "cpu_baseline": cpu, "e2e": None, "gpu_launches": args.steps,
+            "clocks": clocks.summary(),
+        }
+        print(json.dumps(line), flush=True)
+
+
 def main():
     args = parse_args()
     rank, world, local = dist_setup()
@@ -499,6 +576,8 @@ def main():
         run_reference(args, rank, world)
     elif args.workload == 5:
         run_lmhead(args, rank, world, local)
+    elif args.workload == 6:
+        run_diag(args, rank, world, local)
     else:
         run_ours(args, rank, world, local)
     if world > 1:

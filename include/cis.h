@@ -339,6 +339,39 @@ CIS_API cis_status_t cis_lmhead_fused(const void *hidden, const void *weight, in
                                       size_t workspace_bytes, void *stream);
 
 /*
+ * Mismatch diagnostics from both engines' full logits (App. A.5; Sec. 4.3,
+ * Fig. 5c-d), one row per position.  With p = softmax(logits_train),
+ * q = softmax(logits_infer), y the sampled token and f the weight operator of
+ * params (a token operator) applied to every candidate j (k_j = p_j / q_j):
+ *   eps_out   [T] the log-odds displacement of y: -delta_y + log sum_{j != y}
+ *             w_j e^{delta_j} with w_j = e^{z_j} / sum_{j' != y} e^{z_j'} and
+ *             delta in the normalised gauge log q - log p (Lemma 3.1), which
+ *             equals logit p_y - logit q_y.
+ *   logk_out  [T] or NULL: log k_y = log p_y - log q_y.
+ *   p_out     [T] or NULL: p_y.
+ *   bias2_out [T] or NULL: || E_{y~q}[(f_y - k_y) g_y] ||^2, g_y = e_y - p the
+ *             gradient of log p_y with respect to the logits.
+ *   dvar_out  [T] or NULL: the variance increase of f_y g_y over g_y under
+ *             y ~ q (trace of the covariance).
+ * All outputs are device float arrays; masked rows get 0, valid rows with an
+ * id outside [0, V) get NaN and set CIS_ERR_BAD_TOKEN_ID in dev_status
+ * (device int32 or NULL).  logits_* are device [T, ld_*] of dtype (CIS_F32 or
+ * CIS_BF16).  The expectations over y ~ q are exact sums over the V
+ * candidates; the operator's weight is taken in fp32 per candidate.  Two
+ * streaming passes over both tensors.  Errors: CIS_ERR_INVALID_ARG for NULL
+ * required pointers, T < 0, V <= 0, ld < V, an unknown dtype, bad parameters
+ * or a sequence operator.
+ */
+CIS_API cis_status_t cis_mismatch_diagnostics(const void *logits_train, const void *logits_infer,
+                                              int32_t dtype, int64_t T, int64_t V,
+                                              int64_t ld_train, int64_t ld_infer,
+                                              const int32_t *ids, const uint8_t *mask,
+                                              const cis_params_t *params, float *eps_out,
+                                              float *logk_out, float *p_out, float *bias2_out,
+                                              float *dvar_out, int32_t *dev_status,
+                                              void *stream);
+
+/*
  * Largest T that cis_loss_fwd_bwd_noalloc accepts.
  */
 #define CIS_NOALLOC_MAX_TOKENS 65536

@@ -111,6 +111,9 @@ def lib():
                                         ctypes.POINTER(cis_params_t), P, i32, P, P, P, P, P, P,
                                         i64, P, ctypes.c_size_t, P]
     L.cis_loss_fwd_bwd_host.restype = ctypes.c_int
+    L.cis_mismatch_diagnostics.argtypes = [P, P, i32, i64, i64, i64, i64, P, P,
+                                           ctypes.POINTER(cis_params_t), P, P, P, P, P, P, P]
+    L.cis_mismatch_diagnostics.restype = ctypes.c_int
     L.cis_profile_next_call.argtypes = [P, P]
     L.cis_profile_next_call.restype = ctypes.c_int
     _lib = L
@@ -379,6 +382,31 @@ def cis_lmhead_fused(hidden: torch.Tensor, weight: torch.Tensor, ids: torch.Tens
     _check(rc, "cis_lmhead_fused")
     return {"dhidden": dh, "dweight": dw, "lp": lp, "w": w, "trunc": tr, "entropy": ent,
             "loss": loss, "stats": stats, "workspace": ws}
+
+
+def cis_mismatch_diagnostics(logits_train: torch.Tensor, logits_infer: torch.Tensor,
+                             ids: torch.Tensor, params: cis_params_t, mask=None, V=None,
+                             dev_status=None):
+    """Per-position mismatch diagnostics (App. A.5; Sec. 4.3, Fig. 5c-d): a dict
+    of device float [T] tensors eps, logk, p, bias2, dvar."""
+    _need_cuda(logits_train, logits_infer, ids, mask)
+    if logits_train.dtype != logits_infer.dtype:
+        raise TypeError("both logit tensors must have the same type")
+    T, ld_t = _rows(logits_train)
+    Ti, ld_i = _rows(logits_infer)
+    if Ti != T:
+        raise ValueError("both logit tensors must have T rows")
+    V = min(logits_train.shape[1], logits_infer.shape[1]) if V is None else V
+    _vec(ids, torch.int32, T, "ids")
+    _vec(mask, torch.uint8, T, "mask")
+    out = {k: torch.empty(T, dtype=torch.float32, device=logits_train.device)
+           for k in ("eps", "logk", "p", "bias2", "dvar")}
+    rc = lib().cis_mismatch_diagnostics(
+        _ptr(logits_train), _ptr(logits_infer), _dtype_code(logits_train.dtype), T, V, ld_t, ld_i,
+        _ptr(ids), _ptr(mask), ctypes.byref(params), _ptr(out["eps"]), _ptr(out["logk"]),
+        _ptr(out["p"]), _ptr(out["bias2"]), _ptr(out["dvar"]), _ptr(dev_status), _stream())
+    _check(rc, "cis_mismatch_diagnostics")
+    return out
 
 
 def cis_profile_next_call(begin: "torch.cuda.Event | None", end: "torch.cuda.Event | None"):

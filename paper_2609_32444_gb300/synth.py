@@ -50,6 +50,8 @@ WORKLOADS = {
     4: dict(name="c4_t65536_v151936_bf16_masked40", T=65536, V=151936, dtype="bf16", lam=2.3),
     5: dict(name="c5_lmhead_t16384_h2048_v151936_bf16", T=16384, V=151936, H=2048,
             dtype="bf16", lam=2.3),
+    # the mismatch diagnostics: workload 3's recipe, keeping both engines' logits
+    6: dict(name="c6_mismatch_t16384_v151936_bf16", T=16384, V=151936, dtype="bf16", lam=2.3),
 }
 
 
@@ -146,8 +148,17 @@ def _tempered_rows(n: int, V: int, pstar: torch.Tensor, g: torch.Generator, devi
 
 
 def make_batch(cfg: int, device="cpu", seed: int | None = None, T: int | None = None,
-               V: int | None = None, chunk_rows: int = 1024, H: int | None = None) -> Batch:
-    """Draw the synthetic batch of workload ``cfg`` (see module docstring)."""
+               V: int | None = None, chunk_rows: int = 1024, H: int | None = None,
+               keep_infer: bool = False) -> Batch:
+    """Draw the synthetic batch of workload ``cfg`` (see module docstring).
+    ``keep_infer`` (workloads 1-4; always for 6) also returns the inference
+    engine's logits, rounded to the batch's logit type, as
+    ``extra["logits_infer"]``."""
+    if cfg == 6:
+        b = make_batch(3, device, 1006 if seed is None else seed, T, V, chunk_rows,
+                       keep_infer=True)
+        b.cfg = 6
+        return b
     spec = WORKLOADS[cfg]
     T = spec["T"] if T is None else T
     V = spec["V"] if V is None else V
@@ -169,8 +180,9 @@ def make_batch(cfg: int, device="cpu", seed: int | None = None, T: int | None = 
         L = T // nseq
         signs = torch.tensor([1.0, -1.0] * (nseq // 2))[torch.randperm(nseq, generator=gcpu)]
         cu, mask, adv = _pack([L] * nseq, T, signs, device)
+        extra = {"logits_infer": zi.float().contiguous()} if keep_infer else {}
         return Batch(cfg, T, V, z.float().contiguous(), ids.int(), lp_inf, adv, mask, cu,
-                     spec["lam"])
+                     spec["lam"], extra=extra)
 
     if cfg == 2:
         z = torch.randn((T, V), generator=g, device=device) * 3.0
@@ -194,7 +206,9 @@ def make_batch(cfg: int, device="cpu", seed: int | None = None, T: int | None = 
         lengths = raw if sum(raw) <= T else _scale_lengths(raw, T)
         rewards = (torch.rand(nseq, generator=gcpu) < 0.4).float()
         cu, mask, adv = _pack(lengths, T, _group_advantages(rewards, 8), device)
-        return Batch(cfg, T, V, z.contiguous(), ids.int(), lp_inf, adv, mask, cu, spec["lam"])
+        extra = {"logits_infer": zi.to(torch.bfloat16).contiguous()} if keep_infer else {}
+        return Batch(cfg, T, V, z.contiguous(), ids.int(), lp_inf, adv, mask, cu, spec["lam"],
+                     extra=extra)
 
     if cfg in (3, 4, 5):
         if cfg == 4:
@@ -230,6 +244,7 @@ def make_batch(cfg: int, device="cpu", seed: int | None = None, T: int | None = 
         pstar = torch.exp(lo + (hi - lo) * torch.rand(T, generator=g, device=device,
                                                       dtype=torch.float64)).float()
         spike = torch.zeros(T, dtype=torch.bool, device=device)
+        infer = torch.empty((T, V), dtype=torch.bfloat16, device=device) if keep_infer else None
         if cfg == 4:
             valid = torch.nonzero(mask.cpu()).view(-1)
             n_sp = round(0.01 * valid.numel())
@@ -246,8 +261,13 @@ def make_batch(cfg: int, device="cpu", seed: int | None = None, T: int | None = 
                 rr = torch.nonzero(sp).view(-1)
                 zi[rr, y[rr]] -= 6.0
             lp_inf[r0:r1] = _engine_logprob(zi, y)
+            if infer is not None:
+                infer[r0:r1] = zi.to(torch.bfloat16)
+        extra = {"pstar": pstar, "spike": spike}
+        if infer is not None:
+            extra["logits_infer"] = infer
         return Batch(cfg, T, V, logits, ids.int(), lp_inf, adv, mask, cu, spec["lam"],
-                     extra={"pstar": pstar, "spike": spike})
+                     extra=extra)
 
     raise ValueError(f"unknown workload {cfg}")
 

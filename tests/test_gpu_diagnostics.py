@@ -1,0 +1,128 @@
+"""GPU parity of the mismatch diagnostics (App. A.5; Sec. 4.3, Fig. 5c-d)
+against the fp64 oracle, and at full vocabulary size against closed forms.
+
+Tolerances, from the arithmetic: eps and log k come from fp32 row sums (as log
+p does in the token pass: 2e-5 plus 4 ulps).  The bias and the variance
+increase are fp64 combinations of per-candidate fp32 terms of size O(1) (the
+variances themselves are at most 1), summed in fp32 per thread: their error
+is absolute, about V_thread 2^-24 with V_thread = V / 512 terms per thread.
+They are held to 1e-3 of their own size plus an absolute 2e-6 (small V) or
+2e-5 (V = 151936).
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from _util import logits_for_oracle
+from paper_2609_32444_gb300 import binding, synth
+
+pytestmark = [pytest.mark.gpu,
+              pytest.mark.skipif(not torch.cuda.is_available(), reason="needs a CUDA GPU")]
+
+DEV = torch.device("cuda")
+OMODE = {"cis": oracle.MODE_CIS, "tis": oracle.MODE_TIS, "exact": oracle.MODE_EXACT,
+         "none": oracle.MODE_NONE, "band": oracle.MODE_BAND, "icepop": oracle.MODE_ICEPOP,
+         "kpop": oracle.MODE_KPOP}
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    from paper_2609_32444_gb300 import build
+    build.build()
+    binding.lib()
+
+
+def _rows(seed, T, V, dtype, sd=0.3):
+    g = torch.Generator().manual_seed(seed)
+    z = torch.randn((T, V), generator=g) * 2.5
+    zi = z + torch.randn((T, V), generator=g) * sd
+    ids = torch.randint(0, V, (T,), generator=g).int()
+    return z.to(dtype), zi.to(dtype), ids
+
+
+def _compare(out, ref, mask=None, abs_tol=2e-6):
+    m = np.ones(len(ref["eps"]), bool) if mask is None else mask.astype(bool)
+    got = {k: v.cpu().numpy().astype(np.float64) for k, v in out.items()}
+    for k in ("eps", "logk"):
+        tol = 2e-5 + 2.0 ** -21 * np.abs(ref[k][m])
+        assert np.all(np.abs(got[k][m] - ref[k][m]) <= tol), k
+    assert np.all(np.abs(got["p"][m] - ref["p"][m]) <= 1e-5 * ref["p"][m] + 1e-30)
+    for k in ("bias2", "dvar"):
+        err = np.abs(got[k][m] - ref[k][m])
+        tol = 1e-3 * np.abs(ref[k][m]) + abs_tol
+        assert np.all(err <= tol), f"{k}: worst excess {np.max(err - tol):.2e}"
+    for k in got:
+        assert np.all(got[k][~m] == 0), k
+
+
+@pytest.mark.parametrize("dtype", [torch.float32, torch.bfloat16])
+@pytest.mark.parametrize("mode", list(OMODE))
+def test_diagnostics_match_oracle_small_rows(mode, dtype):
+    """T=24 rows of V=64 (and a ragged V=61 for fp32): every output, every token operator."""
+    V = 61 if dtype == torch.float32 else 64
+    z, zi, ids = _rows(3, 24, V, dtype)
+    out = binding.cis_mismatch_diagnostics(z.to(DEV), zi.to(DEV), ids.to(DEV),
+                                           binding.cis_default_params(mode))
+    torch.cuda.synchronize()
+    ref = oracle.mismatch_diagnostics(logits_for_oracle(z), logits_for_oracle(zi), ids.numpy(),
+                                      oracle.params(mode=OMODE[mode]))
+    _compare(out, ref)
+
+
+@pytest.mark.parametrize("mode", ["cis", "tis", "exact"])
+def test_diagnostics_v1024_recipe(mode):
+    """The V=1024 recipe's two engines (noise 0.05 plus spikes of +4), masked rows included."""
+    b = synth.make_batch(1, keep_infer=True)
+    zi = b.extra["logits_infer"]
+    m = b.mask.clone()
+    m[::7] = 0
+    out = binding.cis_mismatch_diagnostics(b.logits.to(DEV), zi.to(DEV), b.ids.to(DEV),
+                                           binding.cis_default_params(mode), mask=m.to(DEV))
+    torch.cuda.synchronize()
+    ref = oracle.mismatch_diagnostics(b.logits.numpy(), zi.numpy(), b.ids.numpy(),
+                                      oracle.params(mode=OMODE[mode]), mask=m.numpy())
+    _compare(out, ref, m.numpy())
+
+
+def test_diagnostics_full_vocabulary_closed_forms():
+    """V=151936 (workload 6's recipe, 24 rows): eps = logit p - logit q (App. A.5),
+    and with fp64 softmaxes from torch: no correction has bias ||q - p||^2 and
+    no added variance; the exact ratio (clamp inactive here) is unbiased and
+    adds sum_y (p_y^2/q_y)(1 - 2 p_y + |p|^2) - (1 - |q|^2)."""
+    b = synth.make_batch(6, device=DEV, T=24)
+    z, zi = b.logits, b.extra["logits_infer"]
+    Pd = torch.softmax(z.double(), dim=1)
+    Qd = torch.softmax(zi.double(), dim=1)
+    y = b.ids.long()
+    p = Pd[torch.arange(24), y]
+    q = Qd[torch.arange(24), y]
+    none = binding.cis_mismatch_diagnostics(z, zi, b.ids, binding.cis_default_params("none"))
+    ex = binding.cis_mismatch_diagnostics(z, zi, b.ids, binding.cis_default_params("exact"))
+    torch.cuda.synchronize()
+    eps = (torch.log(p) - torch.log1p(-p)) - (torch.log(q) - torch.log1p(-q))
+    assert torch.all((none["eps"].double() - eps).abs() <= 2e-5 + 2.0 ** -21 * eps.abs())
+    b2 = ((Qd - Pd) ** 2).sum(dim=1)
+    assert torch.all((none["bias2"].double() - b2).abs() <= 1e-3 * b2 + 2e-5)
+    assert torch.all(none["dvar"].double().abs() <= 2e-5)
+    kmax = (Pd / Qd).max().item()
+    assert 1e-6 < (Pd / Qd).min().item() and kmax < 1e6  # the clamp is inactive
+    assert torch.all(ex["bias2"].double() <= 2e-5)
+    p2 = (Pd ** 2).sum(dim=1, keepdim=True)
+    dv = ((Pd ** 2 / Qd) * (1 - 2 * Pd + p2)).sum(dim=1) - (1 - (Qd ** 2).sum(dim=1))
+    assert torch.all((ex["dvar"].double() - dv).abs() <= 1e-3 * dv.abs() + 2e-5)
+    cis = binding.cis_mismatch_diagnostics(z, zi, b.ids, binding.cis_default_params("cis"))
+    torch.cuda.synchronize()
+    assert torch.all(cis["dvar"] <= ex["dvar"] + 2e-5)
+
+
+def test_diagnostics_bad_id_and_status():
+    z, zi, ids = _rows(4, 8, 64, torch.float32)
+    ids[3] = 64
+    st = torch.zeros(1, dtype=torch.int32, device=DEV)
+    out = binding.cis_mismatch_diagnostics(z.to(DEV), zi.to(DEV), ids.to(DEV),
+                                           binding.cis_default_params(), dev_status=st)
+    torch.cuda.synchronize()
+    assert int(st.item()) & binding.CIS_ERR_BAD_TOKEN_ID
+    assert all(torch.isnan(out[k][3]).item() for k in out)
+    assert not any(torch.isnan(out[k][:3]).any().item() for k in out)
