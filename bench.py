@@ -547,8 +547,9 @@ def run_diag(args, rank, world, local):
                                                         "none": 3}[args.mode], lam=b.lam))
         el = time.perf_counter() - t0
         cpu = {"value": len(rows) / el, "unit": "positions/s", "cores": 1, "kind": "oracle",
-               "sample": f"{len(rows)} position of V={V}: explicit fp64 expectation vectors "
-                         f"(O(V^2) per position), one host thread"}
+               "sample": f"{len(rows)} position of V={V} ({el:.0f} s): explicit fp64 "
+                         f"expectation vectors (O(V^2) per position), one host thread; one "
+                         f"position is the smallest sample"}
     if rank == 0:
         line = {
             "metric": "CIS mismatch diagnostics positions/s at V=151936 bf16 (two logit tensors)",

@@ -12,14 +12,15 @@
 //             P2 = sum p^2,  R2 = sum r^2,  RP = sum r p    (r = q f - p)
 //             C1 = sum q (f^2 - 1)(1 - 2p),  C2 = sum q (f^2 - 1),
 //             C3 = sum q (f - 1),  C4 = sum q^2 (f^2 - 1),
-//             C5 = sum q (f - 1) p,  C6 = sum q (f + 1) p.
+//             C5 = sum q (f - 1) p,  QP = sum q p.
 // With sum q = sum p = 1 the expectations reduce to these sums:
 //   E_q[(f - k) g]_j = r_j - p_j C3, so bias2 = R2 - 2 C3 RP + C3^2 P2;
-//   Var(f g) - Var(g) = C1 + P2 C2 - [C4 - (2 + C3) C5 - C3 C6 + C3 (2 + C3) P2].
+//   Var(f g) - Var(g) = C1 + P2 C2 - [C4 - (2 + C3) C5 - C3 C6 + C3 (2 + C3) P2]
+//   with C6 = sum q (f + 1) p = C5 + 2 QP.
 // Every term but P2 is proportional to f - 1 or to q f - p, so neither result
 // is a small difference of O(1) numbers.  Per-thread sums are fp32, the block
-// sums fp64.  The second pass reads the rows again (mostly from L2: a row pair
-// is at most 2 V 4 bytes and only one row per SM is in flight).
+// sums fp64.  The second pass reads the rows again, from L2 where they are
+// still resident.
 #include "cis_kernels.h"
 #include "cis_rowops.cuh"
 
@@ -30,26 +31,33 @@ constexpr int kDiagThreads = 512;
 constexpr int kNSums = 9;
 
 // The operator's weight for one candidate j in fp32 (a statistic: no fp64
-// decision fallback), from log p_j, log q_j, p_j, k_j.
-__device__ __forceinline__ float elem_weight(float lp, float lq, float p, float k,
+// decision fallback), from the exponents xp = log2 p_j, xq = log2 q_j, p_j and
+// k_j = 2^{xp - xq}; MODE is a compile-time cis_mode_t, so the per-candidate
+// loop has no branch on it.
+template <int MODE>
+__device__ __forceinline__ float elem_weight(float xp, float xq, float p, float k,
                                              const DevParams &P)
 {
-    switch (P.mode) {
-    case CIS_MODE_CIS:
-        return fminf(k, 1.0f + P.lam_f * fmaxf(1.0f - p, P.kappa_f));
-    case CIS_MODE_TIS:
+    if (MODE == CIS_MODE_CIS)
+        return fminf(k, fmaf(P.lam_f, fmaxf(1.0f - p, P.kappa_f), 1.0f));
+    if (MODE == CIS_MODE_TIS)
         return fminf(k, P.tis_cap_f);
-    case CIS_MODE_EXACT:
+    if (MODE == CIS_MODE_EXACT)
         return fminf(fmaxf(k, P.exact_lo_f), P.exact_hi_f);
-    case CIS_MODE_BAND:
-        return fmaxf(fminf(k, 1.0f + P.lam_f * fmaxf(1.0f - p, P.kappa_f)), 0.5f * (1.0f + p));
-    case CIS_MODE_ICEPOP: {
-        const float lk = lp - lq;
-        return (lk < (float)P.log_icepop_lo || lk > (float)P.log_icepop_hi) ? 0.0f : k;
+    if (MODE == CIS_MODE_BAND)
+        return fmaxf(fminf(k, fmaf(P.lam_f, fmaxf(1.0f - p, P.kappa_f), 1.0f)),
+                     0.5f * (1.0f + p));
+    if (MODE == CIS_MODE_ICEPOP) {  // log k against the band, in log2 units
+        const float lk2 = xp - xq;
+        return (lk2 < (float)(P.log_icepop_lo * 1.4426950408889634) ||
+                lk2 > (float)(P.log_icepop_hi * 1.4426950408889634))
+                   ? 0.0f
+                   : k;
     }
-    case CIS_MODE_KPOP: {
+    if (MODE == CIS_MODE_KPOP) {
         // binary KL both ways with p, q clamped to [1e-8, 1 - 1e-8], in the
         // log domain so that 1 - 1e-8 stays representable
+        const float lp = xp * kLn2, lq = xq * kLn2;
         const float lo = -18.420680743952367f;  // log 1e-8
         const float hi = -1e-8f;                // log(1 - 1e-8)
         const float l1p = logf(-expm1f(lp)), l1q = logf(-expm1f(lq));
@@ -60,9 +68,7 @@ __device__ __forceinline__ float elem_weight(float lp, float lq, float p, float 
         const float kqp = qb * (b - a) + qb1 * (b1 - a1);
         return fmaxf(kpq, kqp) > (float)P.kpop_phi ? 0.0f : k;
     }
-    default:
-        return 1.0f;
-    }
+    return 1.0f;  // CIS_MODE_NONE
 }
 
 struct DiagShared {
@@ -71,7 +77,7 @@ struct DiagShared {
     float lse_p, lse_q;
 };
 
-template <typename InT>
+template <typename InT, int MODE>
 __global__ void __launch_bounds__(kDiagThreads)
     cis_mismatch_kernel(const InT *zt, const InT *zi, int64_t T, int64_t V, int64_t ld_t,
                         int64_t ld_i, const int32_t *ids, const uint8_t *mask,
@@ -117,25 +123,30 @@ __global__ void __launch_bounds__(kDiagThreads)
         sh.lse_q = si.lse;
     }
     __syncthreads();
-    const float lse_p = sh.lse_p, lse_q = sh.lse_q;
+    // the exponents in log2 units, x = z log2e - lse log2e (one FMA each);
+    // probabilities that flush to 0 add nothing measurable to the sums
+    const float op = sh.lse_p * kLog2e, oq = sh.lse_q * kLog2e;
     // pass 2: the sums over every candidate j
     float acc[kNSums] = {0, 0, 0, 0, 0, 0, 0, 0, 0};
     auto add = [&](float a, float b) {
-        const float lp = a - lse_p, lq = b - lse_q;
-        const float p = ex2_full(lp * kLog2e), q = ex2_full(lq * kLog2e);
-        const float k = ex2_full((lp - lq) * kLog2e);
-        const float f = q > 0.0f ? elem_weight(lp, lq, p, k, P) : 1.0f;
-        const float fm1 = f - 1.0f, f2m1 = fm1 * (f + 1.0f);
+        const float xp = fmaf(a, kLog2e, -op), xq = fmaf(b, kLog2e, -oq);
+        const float p = ex2_ftz(xp), q = ex2_ftz(xq);
+        const float k = ex2_ftz(xp - xq);
+        // a candidate with q = 0 is never drawn: only r = -p counts, so f = 1
+        const float f = q > 0.0f ? elem_weight<MODE>(xp, xq, p, k, P) : 1.0f;
+        const float fm1 = f - 1.0f;
+        const float t1 = q * (fm1 * (f + 1.0f));   // q (f^2 - 1)
+        const float t2 = q * fm1;                  // q (f - 1)
         const float r = fmaf(q, f, -p);
-        acc[0] = fmaf(p, p, acc[0]);                            // P2
-        acc[1] = fmaf(r, r, acc[1]);                            // R2
-        acc[2] = fmaf(r, p, acc[2]);                            // RP
-        acc[3] = fmaf(q * f2m1, fmaf(-2.0f, p, 1.0f), acc[3]);  // C1
-        acc[4] = fmaf(q, f2m1, acc[4]);                         // C2
-        acc[5] = fmaf(q, fm1, acc[5]);                          // C3
-        acc[6] = fmaf(q * q, f2m1, acc[6]);                     // C4
-        acc[7] = fmaf(q * fm1, p, acc[7]);                      // C5
-        acc[8] = fmaf(q * (f + 1.0f), p, acc[8]);               // C6
+        acc[0] = fmaf(p, p, acc[0]);                       // P2
+        acc[1] = fmaf(r, r, acc[1]);                       // R2
+        acc[2] = fmaf(r, p, acc[2]);                       // RP
+        acc[3] = fmaf(t1, fmaf(-2.0f, p, 1.0f), acc[3]);   // C1
+        acc[4] += t1;                                      // C2
+        acc[5] += t2;                                      // C3
+        acc[6] = fmaf(t1, q, acc[6]);                      // C4
+        acc[7] = fmaf(t2, p, acc[7]);                      // C5
+        acc[8] = fmaf(q, p, acc[8]);                       // QP
     };
     constexpr int EV = 16 / sizeof(InT);
     int64_t j0 = 0;
@@ -179,12 +190,49 @@ __global__ void __launch_bounds__(kDiagThreads)
                 S[i] += sh.sums[w][i];
         }
         const double P2 = S[0], R2 = S[1], RP = S[2], C1 = S[3], C2 = S[4], C3 = S[5],
-                     C4 = S[6], C5 = S[7], C6 = S[8];
+                     C4 = S[6], C5 = S[7], C6 = C5 + 2.0 * S[8];
         const double bias2 = R2 - 2.0 * C3 * RP + C3 * C3 * P2;
         const double dvar = C1 + P2 * C2 - (C4 - (2.0 + C3) * C5 - C3 * C6 + C3 * (2.0 + C3) * P2);
         if (bias2_out) bias2_out[t] = (float)bias2;
         if (dvar_out) dvar_out[t] = (float)dvar;
     }
+}
+
+
+template <typename InT, int MODE>
+void launch_mode(const void *zt, const void *zi, int64_t T, int64_t V, int64_t ld_t,
+                 int64_t ld_i, const int32_t *ids, const uint8_t *mask, const DevParams &P,
+                 float *eps, float *logk, float *p, float *bias2, float *dvar, int32_t *status,
+                 cudaStream_t s)
+{
+    cis_mismatch_kernel<InT, MODE><<<(unsigned)T, kDiagThreads, 0, s>>>(
+        static_cast<const InT *>(zt), static_cast<const InT *>(zi), T, V, ld_t, ld_i, ids, mask,
+        P, eps, logk, p, bias2, dvar, status);
+}
+
+template <typename InT>
+void launch_type(const void *zt, const void *zi, int64_t T, int64_t V, int64_t ld_t,
+                 int64_t ld_i, const int32_t *ids, const uint8_t *mask, const DevParams &P,
+                 float *eps, float *logk, float *p, float *bias2, float *dvar, int32_t *status,
+                 cudaStream_t s)
+{
+#define CIS_DIAG_CASE(M)                                                                          \
+    case M:                                                                                      \
+        launch_mode<InT, M>(zt, zi, T, V, ld_t, ld_i, ids, mask, P, eps, logk, p, bias2, dvar,    \
+                            status, s);                                                          \
+        break;
+    switch (P.mode) {
+        CIS_DIAG_CASE(CIS_MODE_CIS)
+        CIS_DIAG_CASE(CIS_MODE_TIS)
+        CIS_DIAG_CASE(CIS_MODE_EXACT)
+        CIS_DIAG_CASE(CIS_MODE_BAND)
+        CIS_DIAG_CASE(CIS_MODE_ICEPOP)
+        CIS_DIAG_CASE(CIS_MODE_KPOP)
+    default:
+        launch_mode<InT, CIS_MODE_NONE>(zt, zi, T, V, ld_t, ld_i, ids, mask, P, eps, logk, p,
+                                        bias2, dvar, status, s);
+    }
+#undef CIS_DIAG_CASE
 }
 
 }  // namespace
@@ -197,13 +245,11 @@ cudaError_t launch_mismatch(const void *zt, const void *zi, int dtype, int64_t T
     if (T == 0)
         return cudaSuccess;
     if (dtype == CIS_BF16)
-        cis_mismatch_kernel<__nv_bfloat16><<<(unsigned)T, kDiagThreads, 0, s>>>(
-            static_cast<const __nv_bfloat16 *>(zt), static_cast<const __nv_bfloat16 *>(zi), T, V,
-            ld_t, ld_i, ids, mask, P, eps, logk, p, bias2, dvar, status);
+        launch_type<__nv_bfloat16>(zt, zi, T, V, ld_t, ld_i, ids, mask, P, eps, logk, p, bias2,
+                                   dvar, status, s);
     else
-        cis_mismatch_kernel<float><<<(unsigned)T, kDiagThreads, 0, s>>>(
-            static_cast<const float *>(zt), static_cast<const float *>(zi), T, V, ld_t, ld_i, ids,
-            mask, P, eps, logk, p, bias2, dvar, status);
+        launch_type<float>(zt, zi, T, V, ld_t, ld_i, ids, mask, P, eps, logk, p, bias2, dvar,
+                           status, s);
     return cudaGetLastError();
 }
 
