@@ -25,8 +25,9 @@
 // accumulators in TMEM so that the epilogue of one tile overlaps the main loop
 // of the next; persistent CTAs take tiles i, i + grid, i + 2 grid, ...  Warp
 // roles: warp 0 issues TMA loads, warp 1 issues tcgen05.mma (one thread) and
-// owns TMEM, warps 2..5 are the epilogue (one TMEM lane = one tile row per
-// thread).  All waits are bounded: a wait that runs out sets
+// owns TMEM, warps 2..9 are the epilogue: two warps per TMEM lane quadrant
+// (one tile row per thread), each taking one 128-column half of the tile, so
+// that a tile's epilogue fits in the next tile's main loop.  All waits are bounded: a wait that runs out sets
 // CIS_ERR_DEVICE_TIMEOUT, and the CTA drains its own loads and MMAs and runs
 // to its end, so that TMEM is always released.
 #include <cuda.h>
@@ -46,27 +47,41 @@ constexpr int kStages = 4;
 constexpr int kStageA = kBM * kBK * 2;  // 16 KB
 constexpr int kStageB = kBN * kBK * 2;  // 32 KB
 constexpr int kStageBytes = kStageA + kStageB;
-constexpr int kThreads = 192;
+constexpr int kEpiWarps = 8;            // two per TMEM lane quadrant, one per column half
+constexpr int kEpiThreads = 32 * kEpiWarps;
+constexpr int kThreads = 64 + kEpiThreads;
+constexpr int kHalf = kBN / 2;          // columns per epilogue half
 constexpr uint32_t kTmemCols = 2 * kBN;  // two accumulators
 constexpr size_t kSmemBytes = (size_t)kStages * kStageBytes + 1024;
+// kDz stages dz^T through shared memory: per 32-column chunk two boxes of 64
+// tokens x 32 vocabulary rows (128-byte swizzle), double-buffered per half.
+constexpr int kDztBox = 64 * 32 * 2;                     // 4 KB
+constexpr int kDztBuf = 2 * kDztBox;                     // one chunk: 128 tokens
+constexpr size_t kSmemBytesDz = kSmemBytes + 2 * 2 * kDztBuf;
 // dz + dz^T of one chunk take 4 Tp bytes per vocabulary column; the default
 // chunk keeps them within this many bytes.
 constexpr int64_t kDefaultChunkBytes = 1ll << 30;
 
 enum Epi { kStats = 0, kDz = 1, kStore = 2, kAccum = 3 };
 
-// OR of `pred` over the 128 epilogue threads (named barrier 1), so that the
-// four epilogue warps leave their loop together.
+// OR of `pred` over the epilogue threads (named barrier 1), so that the
+// epilogue warps leave their loop together.
 __device__ __forceinline__ int __syncthreads_or_epi(int pred)
 {
     int r;
     asm volatile(
         "{\n\t.reg .pred p, q;\n\tsetp.ne.s32 p, %1, 0;\n\t"
-        "bar.red.or.pred q, 1, 128, p;\n\tselp.s32 %0, 1, 0, q;\n\t}"
+        "bar.red.or.pred q, 1, %2, p;\n\tselp.s32 %0, 1, 0, q;\n\t}"
         : "=r"(r)
-        : "r"(pred)
+        : "r"(pred), "n"(kEpiThreads)
         : "memory");
     return r;
+}
+
+// Barrier of the 128 threads of one epilogue half (named barriers 2 and 3).
+__device__ __forceinline__ void half_sync(int half)
+{
+    asm volatile("bar.sync %0, 128;" ::"r"(2 + half) : "memory");
 }
 
 __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi)
@@ -86,8 +101,8 @@ struct GemmArgs {
     int T, V, col0;
     const int32_t *ids;
     const float *lse, *cvec;
-    float2 *part;     // kStats: [nNt, T] (max, sum) over j != y
-    float *part_u;    // kStats: [nNt, T] sum e^{z - max} (z - max), or null (no entropy)
+    float2 *part;     // kStats: [2 nNt, T] (max, sum) over j != y per 128-column half
+    float *part_u;    // kStats: [2 nNt, T] sum e^{z - max} (z - max), or null (no entropy)
     float *zy;        // kStats: z at the sampled token
     uint16_t *dz;     // kDz: bf16 [Tp, ld_dz], column = chunk-local vocabulary index
     uint16_t *dzt;    // kDz: bf16 [chunk, ld_dzt], column = token
@@ -125,11 +140,20 @@ struct Abort {
     }
 };
 
+// Tile order.  raster_n: groups of kGroupN vocabulary tiles, token tiles
+// inside a group, so that the tiles in flight at one time (one per SM) share
+// about 152 / kGroupN token tiles of A and kGroupN tiles of B in L2;
+// otherwise m-major (the nNt column blocks of a row block together).
+constexpr int kGroupN = 8;
 __device__ __forceinline__ void tile_mn(const GemmArgs &g, int i, int &m, int &n)
 {
     if (g.raster_n) {
-        n = i / g.nMt;
-        m = i - n * g.nMt;
+        const int per = kGroupN * g.nMt;
+        const int grp = i / per, j = i - grp * per;
+        const int n0 = grp * kGroupN;
+        const int gw = g.nNt - n0 < kGroupN ? g.nNt - n0 : kGroupN;
+        m = j / gw;
+        n = n0 + (j - m * gw);
     } else {
         m = i / g.nNt;
         n = i - m * g.nNt;
@@ -139,10 +163,12 @@ __device__ __forceinline__ void tile_mn(const GemmArgs &g, int i, int &m, int &n
 template <int EPI>
 __global__ void __launch_bounds__(kThreads, 1)
     cis_lmhead_gemm_kernel(const __grid_constant__ CUtensorMap tmA,
-                           const __grid_constant__ CUtensorMap tmB, const GemmArgs g)
+                           const __grid_constant__ CUtensorMap tmB,
+                           const __grid_constant__ CUtensorMap tmDzt, const GemmArgs g)
 {
     extern __shared__ __align__(1024) uint8_t dsm[];
     uint8_t *ring = dsm + ((1024 - (tc::smem_addr(dsm) & 1023)) & 1023);
+    uint8_t *stage_dzt = ring + kStages * kStageBytes;  // kDz only
     __shared__ __align__(8) Barriers bars;
     __shared__ uint32_t tmem_base;
     __shared__ int aborted;
@@ -158,7 +184,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         for (int b = 0; b < 2; ++b) {
             tc::bar_init(&bars.accfull[b], 1);
-            tc::bar_init(&bars.accempty[b], 128);
+            tc::bar_init(&bars.accempty[b], kEpiThreads);
         }
         tc::bar_init(&bars.done, 1);
         tc::bar_init_fence();
@@ -239,10 +265,16 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
     } else {
         // ---------------------------------------------------------- epilogue
-        const int lg = warp & 3;  // TMEM lane quadrant of this warp
+        // warps 2..9: TMEM lane quadrant warp % 4 (one tile row per thread),
+        // column half (warp - 2) / 4 of the 256-column tile
+        const int lg = warp & 3;
+        const int half = (warp - 2) >> 2;
         const int r = lg * 32 + lane;
         const uint32_t lane_off = (uint32_t)(lg * 32) << 16;
+        const int cbeg = half * kHalf;
+        const bool leader = r == 0;  // issues this half's dz^T stores
         int i = 0;
+        uint32_t nchunk = 0;  // kDz: chunks this half staged so far (selects the buffer)
         for (int t = blockIdx.x; t < nTiles; t += gridDim.x, ++i) {
             if (__syncthreads_or_epi(ab.on()))
                 break;
@@ -258,7 +290,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const bool ent = g.part_u != nullptr;
                 float mx = -INFINITY, s = 0.0f, u = 0.0f, zyv = 0.0f;
                 bool got_y = false;
-                for (int c0 = 0; c0 < kBN; c0 += 32) {
+                for (int c0 = cbeg; c0 < cbeg + kHalf; c0 += 32) {
                     float v[32];
                     tc::tmem_ld32(taddr + c0, v);
                     const int base = g.col0 + n * kBN + c0;
@@ -305,10 +337,11 @@ __global__ void __launch_bounds__(kThreads, 1)
                         u += au;
                     }
                 }
-                if (row < g.T) {
-                    g.part[(int64_t)n * g.T + row] = make_float2(mx, s);
+                if (row < g.T) {  // one (max, sum) per 128-column half
+                    const int64_t pi = (int64_t)(2 * n + half) * g.T + row;
+                    g.part[pi] = make_float2(mx, s);
                     if (ent)
-                        g.part_u[(int64_t)n * g.T + row] = u;
+                        g.part_u[pi] = u;
                     if (got_y)
                         g.zy[row] = zyv;
                 }
@@ -321,7 +354,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const float lse_r = live ? g.lse[row] : 0.0f;
                 const int y_r = live ? g.ids[row] : -1;
                 const int cl0 = n * kBN;  // chunk-local column of the tile
-                for (int c0 = 0; c0 < kBN; c0 += 32) {
+                for (int c0 = cbeg; c0 < cbeg + kHalf; c0 += 32) {
                     float v[32];
                     tc::tmem_ld32(taddr + c0, v);
                     const int gc0 = g.col0 + cl0 + c0;  // vocabulary index of v[0]
@@ -341,20 +374,38 @@ __global__ void __launch_bounds__(kThreads, 1)
                     }
                     uint4 *drow = reinterpret_cast<uint4 *>(g.dz + (int64_t)row * g.ld_dz + cl0 + c0);
 #pragma unroll
-                    for (int q = 0; q < 4; ++q)
-                        drow[q] = make_uint4(w[4 * q], w[4 * q + 1], w[4 * q + 2], w[4 * q + 3]);
-                    // dz^T: the warp's 32 consecutive tokens make one 64-byte run per column
-                    uint16_t *dcol = g.dzt + (int64_t)(cl0 + c0) * g.ld_dzt + row;
+                    for (int q = 0; q < 4; ++q)  // streaming: read back only by the next launch
+                        __stcs(drow + q, make_uint4(w[4 * q], w[4 * q + 1], w[4 * q + 2], w[4 * q + 3]));
+                    // dz^T through shared memory: this chunk's 32 vocabulary rows x
+                    // 128 tokens as two TMA boxes of 64 tokens (128-byte swizzle).
+                    // Buffer nchunk & 1 was last read by the stores of chunk
+                    // nchunk - 2: at most one group (chunk nchunk - 1) may still read.
+                    uint8_t *buf = stage_dzt + (2 * half + (nchunk & 1)) * kDztBuf;
+                    if (leader)
+                        tc::bulk_wait_read<1>();
+                    half_sync(half);
+                    {
+                        uint8_t *box = buf + (r >> 6) * kDztBox;
+                        const int tq = (r & 63) >> 3, tb = (r & 7) * 2;
 #pragma unroll
-                    for (int q = 0; q < 32; ++q)
-                        dcol[(int64_t)q * g.ld_dzt] =
-                            (uint16_t)((q & 1) ? (w[q >> 1] >> 16) : (w[q >> 1] & 0xFFFFu));
+                        for (int q = 0; q < 32; ++q)
+                            *reinterpret_cast<uint16_t *>(box + tc::sw128_offset(q, tq) + tb) =
+                                (uint16_t)((q & 1) ? (w[q >> 1] >> 16) : (w[q >> 1] & 0xFFFFu));
+                    }
+                    tc::fence_proxy_async_smem();
+                    half_sync(half);
+                    if (leader) {
+                        tc::tma_store_2d_evict_first(&tmDzt, m * kBM, cl0 + c0, buf);
+                        tc::tma_store_2d_evict_first(&tmDzt, m * kBM + 64, cl0 + c0, buf + kDztBox);
+                        tc::bulk_commit();
+                    }
+                    ++nchunk;
                 }
             } else {
                 const int lr = m * kBM + r;  // row of the output block
                 const bool live = lr < g.rows_valid;
                 const int64_t o = (int64_t)lr * g.ld_out + (int64_t)n * kBN;
-                for (int c0 = 0; c0 < kBN; c0 += 32) {
+                for (int c0 = cbeg; c0 < cbeg + kHalf; c0 += 32) {
                     float v[32];
                     tc::tmem_ld32(taddr + c0, v);
                     if (!live)
@@ -363,11 +414,11 @@ __global__ void __launch_bounds__(kThreads, 1)
                         uint4 *dst = reinterpret_cast<uint4 *>(
                             reinterpret_cast<uint16_t *>(g.out) + o + c0);
 #pragma unroll
-                        for (int q = 0; q < 4; ++q)
-                            dst[q] = make_uint4(pack_bf16x2(v[8 * q + 0], v[8 * q + 1]),
-                                                pack_bf16x2(v[8 * q + 2], v[8 * q + 3]),
-                                                pack_bf16x2(v[8 * q + 4], v[8 * q + 5]),
-                                                pack_bf16x2(v[8 * q + 6], v[8 * q + 7]));
+                        for (int q = 0; q < 4; ++q)  // streaming: outputs are not re-read here
+                            __stcs(dst + q, make_uint4(pack_bf16x2(v[8 * q + 0], v[8 * q + 1]),
+                                                       pack_bf16x2(v[8 * q + 2], v[8 * q + 3]),
+                                                       pack_bf16x2(v[8 * q + 4], v[8 * q + 5]),
+                                                       pack_bf16x2(v[8 * q + 6], v[8 * q + 7])));
                     } else {
                         float4 *dst = reinterpret_cast<float4 *>(
                             reinterpret_cast<float *>(g.out) + o + c0);
@@ -382,7 +433,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                                 x.z += old.z;
                                 x.w += old.w;
                             }
-                            dst[q] = x;
+                            __stcs(dst + q, x);
                         }
                     }
                 }
@@ -390,6 +441,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             tc::fence_before_sync();
             tc::bar_arrive(&bars.accempty[acc]);
         }
+        if (EPI == kDz && leader)
+            tc::bulk_wait_all();  // the dz^T stores have read shared memory and landed
     }
     __syncwarp();
     tc::fence_before_sync();
@@ -539,14 +592,17 @@ bool make_map(CUtensorMap *m, const void *ptr, int64_t inner, int64_t outer, int
 
 template <int EPI>
 cudaError_t launch_gemm(const CUtensorMap &a, const CUtensorMap &b, const GemmArgs &g,
-                        cudaStream_t s)
+                        cudaStream_t s, const CUtensorMap *dzt = nullptr)
 {
     const int tiles = g.nMt * g.nNt;
     if (tiles <= 0 || g.nK <= 0)
         return cudaSuccess;
+    if (EPI == kDz && dzt == nullptr)
+        return cudaErrorInvalidValue;
     auto k = cis_lmhead_gemm_kernel<EPI>;
+    const size_t smem = EPI == kDz ? kSmemBytesDz : kSmemBytes;
     cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         (int)kSmemBytes);
+                                         (int)smem);
     if (e != cudaSuccess)
         return e;
     int dev = 0, sms = 0;
@@ -554,7 +610,7 @@ cudaError_t launch_gemm(const CUtensorMap &a, const CUtensorMap &b, const GemmAr
         (e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess)
         return e;
     const int grid = tiles < sms ? tiles : sms;
-    k<<<grid, kThreads, kSmemBytes, s>>>(a, b, g);
+    k<<<grid, kThreads, smem, s>>>(a, b, dzt ? *dzt : a, g);
     return cudaGetLastError();
 }
 
@@ -587,10 +643,10 @@ LmLayout lm_layout(int64_t T, int64_t V, int64_t Hd, int64_t Vc)
     o = up(o + 4 * (size_t)T);
     L.zy = o;
     o = up(o + 4 * (size_t)T);
-    L.part = o;
-    o = up(o + 8 * (size_t)T * (size_t)nVt);
+    L.part = o;  // one (max, sum) per 128-column half tile
+    o = up(o + 8 * (size_t)T * (size_t)(2 * nVt));
     L.part_u = o;
-    o = up(o + 4 * (size_t)T * (size_t)nVt);
+    o = up(o + 4 * (size_t)T * (size_t)(2 * nVt));
     L.wt = o;
     o = up(o + 2 * (size_t)Hd * (size_t)L.vp);
     L.ht = o;
@@ -769,7 +825,7 @@ CIS_API cis_status_t cis_lmhead_fused(const void *hidden, const void *weight, in
                 PassArgs f = a;
                 f.lp64_out = a.ws_terms;
                 lm::cis_lmhead_token_kernel<<<(unsigned)((T + 7) / 8), 256, 0, s>>>(
-                    f, part, part_u, zy, nVt, lse, cv);
+                    f, part, part_u, zy, 2 * nVt, lse, cv);
                 if ((e = cudaGetLastError()) != cudaSuccess)
                     return CIS_ERR_CUDA;
             }
@@ -783,7 +839,7 @@ CIS_API cis_status_t cis_lmhead_fused(const void *hidden, const void *weight, in
             a.trunc_in = a.ws_trunc;
         }
         lm::cis_lmhead_token_kernel<<<(unsigned)((T + 7) / 8), 256, 0, s>>>(a, part, part_u, zy,
-                                                                            nVt, lse, cv);
+                                                                            2 * nVt, lse, cv);
         if ((e = cudaGetLastError()) != cudaSuccess)
             return CIS_ERR_CUDA;
         // transposed copies of W and H (K-major B operands of DH and DW)
@@ -808,9 +864,12 @@ CIS_API cis_status_t cis_lmhead_fused(const void *hidden, const void *weight, in
             g.b_row0 = (int)v0;
             g.b_k0 = 0;
             g.col0 = (int)v0;
-            if (lm::launch_gemm<lm::kDz>(mH, mW, g, s) != cudaSuccess)
+            CUtensorMap mDz, mDzt, mDztStore;
+            // dz^T as the DZ epilogue stores it: boxes of 64 tokens x 32 rows
+            if (!lm::make_map(&mDztStore, dzt, L.Tp, Vc, L.Tp, 32))
+                return CIS_ERR_UNSUPPORTED;
+            if (lm::launch_gemm<lm::kDz>(mH, mW, g, s, &mDztStore) != cudaSuccess)
                 return CIS_ERR_CUDA;
-            CUtensorMap mDz, mDzt;
             if (!lm::make_map(&mDz, dz, w, L.Tp, Vc, lm::kBM) ||
                 !lm::make_map(&mDzt, dzt, T, w, L.Tp, lm::kBM))
                 return CIS_ERR_UNSUPPORTED;
