@@ -34,13 +34,21 @@ sys.path.insert(0, ROOT)
 METRIC = "CIS loss fwd+bwd tokens/s at V=151936 bf16; achieved % of HBM roofline"
 FALLBACK_HBM_GBS = 6800.0
 NOMINAL_HBM_GBS = 8000.0
+# the sources of each profiled kernel: a summary's traffic figure is used only
+# while their hash matches the one recorded with it
+FUSED_SOURCES = ["paper_2609_32444_gb300/csrc/cis_cluster.cu",
+                 "paper_2609_32444_gb300/csrc/cis_dsmem.cuh",
+                 "paper_2609_32444_gb300/csrc/cis_common.cuh"]
+DIAG_SOURCES = ["paper_2609_32444_gb300/csrc/cis_diag.cu",
+                "paper_2609_32444_gb300/csrc/cis_dsmem.cuh",
+                "paper_2609_32444_gb300/csrc/cis_common.cuh"]
 # committed ncu summaries that carry the full-size DRAM traffic per workload
 PROFILE_SUMMARIES = {
-    3: os.path.join(ROOT, "profiles", "fused_pass_t16384_v151936_bf16.md"),
-    4: os.path.join(ROOT, "profiles", "fused_pass_t65536_v151936_bf16_masked40.md"),
+    3: (os.path.join(ROOT, "profiles", "fused_pass_t16384_v151936_bf16.md"), FUSED_SOURCES),
+    4: (os.path.join(ROOT, "profiles", "fused_pass_t65536_v151936_bf16_masked40.md"),
+        FUSED_SOURCES),
+    6: (os.path.join(ROOT, "profiles", "mismatch_t16384_v151936_bf16.md"), DIAG_SOURCES),
 }
-KERNEL_SOURCES = ["paper_2609_32444_gb300/csrc/cis_cluster.cu",
-                  "paper_2609_32444_gb300/csrc/cis_common.cuh"]
 
 
 def parse_args():
@@ -99,9 +107,9 @@ def measured_peaks():
     return FALLBACK_HBM_GBS, "fallback 6.8 TB/s (no MEASURED_PEAKS.json)"
 
 
-def kernel_source_hash() -> str:
+def kernel_source_hash(sources=FUSED_SOURCES) -> str:
     h = hashlib.sha256()
-    for rel in KERNEL_SOURCES:
+    for rel in sources:
         with open(os.path.join(ROOT, rel), "rb") as f:
             h.update(f.read())
     return h.hexdigest()[:16]
@@ -110,13 +118,14 @@ def kernel_source_hash() -> str:
 def profiled_traffic(workload: int = 3, tokens=None):
     """DRAM bytes per launch of the main kernel from the committed ncu summary
     of this workload, if it was taken on the current kernel source (else None)."""
-    path = PROFILE_SUMMARIES.get(workload)
-    if tokens is not None or path is None or not os.path.exists(path):
+    entry = PROFILE_SUMMARIES.get(workload)
+    if tokens is not None or entry is None or not os.path.exists(entry[0]):
         return None
+    path, sources = entry
     txt = open(path).read()
     m = re.search(r"traffic_bytes_per_launch:\s*(\d+)", txt)
     s = re.search(r"kernel_source_sha256_16:\s*([0-9a-f]+)", txt)
-    if not m or not s or s.group(1) != kernel_source_hash():
+    if not m or not s or s.group(1) != kernel_source_hash(sources):
         return None
     return int(m.group(1))
 
@@ -530,8 +539,9 @@ def run_diag(args, rank, world, local):
     barrier(world)
     clocks.mark(h0, h1)
     ms = max_over_ranks(start.elapsed_time(end), world) / args.steps
-    # one launch per call: both tensors read once (the second pass is meant to
-    # hit L2), ids and mask read, five floats written per position
+    # one launch per call: both tensors read once from HBM (the second pass
+    # re-reads each row from L2), ids and mask read, five floats written per
+    # position
     alg_bytes = 2 * T * V * b.logits.element_size() + T * (4 + 1) + 5 * 4 * T
     peak, peak_src = measured_peaks()
     achieved = alg_bytes / (ms / 1e3) / 1e9
@@ -561,8 +571,9 @@ def run_diag(args, rank, world, local):
                        "io_dtype": "bf16",
                        "l2": "no flush: the 9.96 GB of logits per step exceed the L2"},
             "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
-                         "frac": achieved / peak, "traffic": None,
-                         "kernel": "cis_mismatch_kernel<bf16> (two passes over both rows)",
+                         "frac": achieved / peak, "traffic": profiled_traffic(6, args.tokens),
+                         "kernel": "cis_mismatch_stream_kernel<cis, 24 warps> (both rows "
+                                   "streamed through shared memory twice, HBM once)",
                          "algorithmic_bytes_per_launch": alg_bytes, "peak_source": peak_src},
             "cpu_baseline": cpu, "e2e": None, "gpu_launches": args.steps,
             "clocks": clocks.summary(),

@@ -89,6 +89,14 @@ __device__ __forceinline__ float ex2_full(float x)
     return y;
 }
 
+// max with NaN propagation (fmaxf drops a NaN operand).
+__device__ __forceinline__ float max_nan(float a, float b)
+{
+    float r;
+    asm("max.NaN.f32 %0, %1, %2;" : "=f"(r) : "f"(a), "f"(b));
+    return r;
+}
+
 // +1: a > b for certain; -1: a < b for certain (a <= b in the fp64 sense);
 // 0: too close to call from fp32 values with relative errors below ~1e-6.
 __device__ __forceinline__ int certain_cmp(float a, float b)

@@ -5,9 +5,9 @@
 // variance increase of f g over g, with g = e_y - p the gradient of log p_y
 // with respect to the logits and f the weight operator.
 //
-// One CTA of 512 threads per row, two streaming passes over both rows:
-//   pass 1: (max, sum) over j != y of each engine's logits (cis_rowops.cuh),
-//           giving log p, log q, their log-odds d_p, d_q, and lse of each;
+// Per position, two passes over both engines' rows:
+//   pass 1: (max, sum) over j != y of each engine's logits, giving log p,
+//           log q, their log-odds d_p, d_q, and lse of each;
 //   pass 2: p_j, q_j, k_j and f_j for every candidate j, accumulating
 //             P2 = sum p^2,  R2 = sum r^2,  RP = sum r p    (r = q f - p)
 //             C1 = sum q (f^2 - 1)(1 - 2p),  C2 = sum q (f^2 - 1),
@@ -18,9 +18,22 @@
 //   Var(f g) - Var(g) = C1 + P2 C2 - [C4 - (2 + C3) C5 - C3 C6 + C3 (2 + C3) P2]
 //   with C6 = sum q (f + 1) p = C5 + 2 QP.
 // Every term but P2 is proportional to f - 1 or to q f - p, so neither result
-// is a small difference of O(1) numbers.  Per-thread sums are fp32, the block
-// sums fp64.  The second pass reads the rows again, from L2 where they are
-// still resident.
+// is a small difference of O(1) numbers.  Per-thread sums are fp32; the
+// one-CTA kernel adds the threads' sums in fp64, the streaming kernel adds a
+// warp's in fp32 and the warps' in fp64.
+//
+// Two kernels compute this:
+//   - cis_mismatch_stream_kernel (bf16 rows, V a multiple of 8, 16-byte
+//     aligned rows): one CTA per SM walking its rows, a producer warp
+//     streaming both rows through a shared-memory ring with bulk copies, once
+//     per pass (HBM reads each row once: the second copy comes from L2); pass
+//     2 forms two candidates per instruction with the packed f32x2 FMA, add
+//     and multiply;
+//   - cis_mismatch_kernel (any row): one CTA per position streaming both rows
+//     from global memory with vector loads, twice.
+#include <stdlib.h>
+
+#include "cis_dsmem.cuh"
 #include "cis_kernels.h"
 #include "cis_rowops.cuh"
 
@@ -199,6 +212,487 @@ __global__ void __launch_bounds__(kDiagThreads)
 }
 
 
+// ---------------------------------------------------------------------------
+// Streaming kernel.
+
+// The operator's weight for two candidates at once (f32x2 where the
+// arithmetic allows it); the same values as elem_weight lane by lane.  Where
+// q = 0 the candidate is never drawn and only r = -p counts: every operator
+// here but IcePop and KPop gives a finite f there, so q (f - 1) = 0 without a
+// test; those two can return k = inf and keep the explicit guard.
+template <int MODE>
+__device__ __forceinline__ float2 elem_weight2(float2 xp, float2 xq, float2 p, float2 q, float2 k,
+                                               const DevParams &P)
+{
+    const float2 one = make_float2(1.0f, 1.0f);
+    if (MODE == CIS_MODE_CIS || MODE == CIS_MODE_BAND) {
+        float2 c = __ffma2_rn(p, make_float2(-1.0f, -1.0f), one);  // 1 - p
+        c = make_float2(fmaxf(c.x, P.kappa_f), fmaxf(c.y, P.kappa_f));
+        c = __ffma2_rn(c, make_float2(P.lam_f, P.lam_f), one);     // 1 + lam max(1 - p, kappa)
+        float2 f = make_float2(fminf(k.x, c.x), fminf(k.y, c.y));
+        if (MODE == CIS_MODE_BAND) {  // lower edge (1 + p) / 2
+            const float2 lo = __ffma2_rn(p, make_float2(0.5f, 0.5f), make_float2(0.5f, 0.5f));
+            f = make_float2(fmaxf(f.x, lo.x), fmaxf(f.y, lo.y));
+        }
+        return f;
+    }
+    if (MODE == CIS_MODE_TIS)
+        return make_float2(fminf(k.x, P.tis_cap_f), fminf(k.y, P.tis_cap_f));
+    if (MODE == CIS_MODE_EXACT)
+        return make_float2(fminf(fmaxf(k.x, P.exact_lo_f), P.exact_hi_f),
+                           fminf(fmaxf(k.y, P.exact_lo_f), P.exact_hi_f));
+    if (MODE == CIS_MODE_ICEPOP || MODE == CIS_MODE_KPOP)
+        return make_float2(q.x > 0.0f ? elem_weight<MODE>(xp.x, xq.x, p.x, k.x, P) : 1.0f,
+                           q.y > 0.0f ? elem_weight<MODE>(xp.y, xq.y, p.y, k.y, P) : 1.0f);
+    return one;  // CIS_MODE_NONE
+}
+
+// Pass 2 for two candidates (zp: training logits, zq: inference logits), with
+// nop = -lse_p log2e and noq = -lse_q log2e.  The sums are kept in the signs
+// that need no negation:
+//   acc = [P2, R2, -RP, D = sum T1 p, -C2, -C3, -C4, -C5, QP]
+// with T2 = q (1 - f) = -q (f - 1), T1 = T2 (1 + f) = -q (f^2 - 1) and
+// r' = p - q f = -r; then C1 = sum q (f^2 - 1)(1 - 2p) = C2 + 2 D.
+template <int MODE>
+__device__ __forceinline__ void diag_pair(float2 zp, float2 zq, float2 nop, float2 noq,
+                                          const DevParams &P, float2 (&acc)[kNSums])
+{
+    const float2 l2e = make_float2(kLog2e, kLog2e);
+    const float2 one = make_float2(1.0f, 1.0f), m1 = make_float2(-1.0f, -1.0f);
+    const float2 xp = __ffma2_rn(zp, l2e, nop), xq = __ffma2_rn(zq, l2e, noq);
+    const float2 p = make_float2(ex2_ftz(xp.x), ex2_ftz(xp.y));
+    const float2 q = make_float2(ex2_ftz(xq.x), ex2_ftz(xq.y));
+    const float2 d = __ffma2_rn(xq, m1, xp);  // xp - xq, rounded once
+    const float2 k = make_float2(ex2_ftz(d.x), ex2_ftz(d.y));
+    const float2 f = elem_weight2<MODE>(xp, xq, p, q, k, P);
+    const float2 g = __ffma2_rn(f, m1, one);  // 1 - f (exact for f in [1/2, 2])
+    const float2 h = __fadd2_rn(f, one);      // 1 + f
+    const float2 T2 = __fmul2_rn(q, g);
+    const float2 T1 = __fmul2_rn(T2, h);
+    const float2 r = __ffma2_rn(__fmul2_rn(q, f), m1, p);  // p - q f
+    acc[0] = __ffma2_rn(p, p, acc[0]);
+    acc[1] = __ffma2_rn(r, r, acc[1]);
+    acc[2] = __ffma2_rn(r, p, acc[2]);
+    acc[3] = __ffma2_rn(T1, p, acc[3]);
+    acc[4] = __fadd2_rn(T1, acc[4]);
+    acc[5] = __fadd2_rn(T2, acc[5]);
+    acc[6] = __ffma2_rn(T1, q, acc[6]);
+    acc[7] = __ffma2_rn(T2, p, acc[7]);
+    acc[8] = __ffma2_rn(q, p, acc[8]);
+}
+
+__device__ __forceinline__ float2 bf16_pair(uint32_t w)
+{
+    return make_float2(bf16_lo(w), bf16_hi(w));
+}
+
+// Sum of 2^{z log2e + noff} over one 8-entry bf16 group, into a packed pair.
+__device__ __forceinline__ float2 sum8_exp2_pk(uint4 w, float2 noff, float2 acc)
+{
+    const float2 l2e = make_float2(kLog2e, kLog2e);
+    const uint32_t ws[4] = {w.x, w.y, w.z, w.w};
+    float2 e[4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const float2 x = __ffma2_rn(bf16_pair(ws[i]), l2e, noff);
+        e[i] = make_float2(ex2_ftz(x.x), ex2_ftz(x.y));
+    }
+    return __fadd2_rn(acc, __fadd2_rn(__fadd2_rn(e[0], e[1]), __fadd2_rn(e[2], e[3])));
+}
+
+struct DiagArgs {
+    const __nv_bfloat16 *zt, *zi;
+    int64_t T, V, ld_t, ld_i;
+    const int32_t *ids;
+    const uint8_t *mask;
+    DevParams P;
+    float *eps, *logk, *p, *bias2, *dvar;
+    int32_t *status;
+};
+
+// The layout for NW consumer warps (plus one producer warp): a ring slot
+// holds two groups per consumer thread of each row, as many slots as fit in
+// about 200 KB of shared memory.
+template <int NW> struct StreamCfg {
+    static constexpr int kConsThreads = NW * 32;
+    static constexpr int kThreads = kConsThreads + 32;
+    static constexpr int kSlotGroups = 2 * kConsThreads;  // 8-entry groups of each row per slot
+    static constexpr int kSlotBytes = 2 * kSlotGroups * 16;
+    static constexpr int kRing = (200 * 1024) / kSlotBytes < 8 ? (200 * 1024) / kSlotBytes : 8;
+    static constexpr size_t kSmem = (size_t)kRing * kSlotBytes + 128;
+};
+constexpr int kMaxRing = 8;
+constexpr int kMaxConsWarps = 32;
+
+struct StreamShared {
+    alignas(8) uint64_t full[kMaxRing];   // a slot's two copies have landed
+    alignas(8) uint64_t empty[kMaxRing];  // every consumer warp is done with a slot
+    MaxSum red[2][kMaxConsWarps];
+    float wsum[kMaxConsWarps][kNSums];
+    double total[kNSums];
+    float op, oq;
+    int aborted;
+};
+
+// The consumer warps' own barrier (the producer warp never joins it).
+template <int NT> __device__ __forceinline__ void cons_sync()
+{
+    asm volatile("bar.sync 1, %0;" ::"n"(NT) : "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive(uint32_t bar)
+{
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+
+// Bulk copy whose lines L2 may evict first (their last read).
+__device__ __forceinline__ void bulk_g2s_evict_first(uint32_t dst, const void *src, uint32_t bytes,
+                                                     uint32_t bar)
+{
+    asm volatile(
+        "{\n\t.reg .b64 pol;\n\t"
+        "createpolicy.fractional.L2::evict_first.b64 pol, 1.0;\n\t"
+        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint"
+        " [%0], [%1], %2, [%3], pol;\n\t}" ::"r"(dst),
+        "l"(src), "r"(bytes), "r"(bar)
+        : "memory");
+}
+
+// A wait that runs out marks the CTA as aborted (and the status word): every
+// later wait then returns at once, so each role finishes its loops without
+// waiting again and the consumers still meet at every barrier.
+struct StreamAbort {
+    volatile int *flag;
+    int32_t *status;
+    __device__ __forceinline__ bool on() const { return *flag != 0; }
+    __device__ __forceinline__ void wait(uint32_t bar, uint32_t parity) const
+    {
+        if (*flag)
+            return;
+        if (!mbar_wait(bar, parity)) {
+            *flag = 1;
+            set_status(status, kStatusTimeout);
+        }
+    }
+};
+
+// The sampled entry of a group set to -inf (pass 1 sums over j != y).
+__device__ __forceinline__ uint4 drop_entry(uint4 w, int i)
+{
+    const uint32_t keep = (i & 1) ? 0x0000ffffu : 0xffff0000u;
+    const uint32_t ninf = (i & 1) ? 0xff800000u : 0x0000ff80u;
+    const int k = i >> 1;
+    w.x = k == 0 ? ((w.x & keep) | ninf) : w.x;
+    w.y = k == 1 ? ((w.y & keep) | ninf) : w.y;
+    w.z = k == 2 ? ((w.z & keep) | ninf) : w.z;
+    w.w = k == 3 ? ((w.w & keep) | ninf) : w.w;
+    return w;
+}
+
+// Running (max, sum) of one row over 8 more entries: the exact maximum of
+// the group (bf16 pairs compared packed, NaN propagating); when it rises the
+// sum is rescaled; the exponentials are 2^{z log2e - cm} with cm = fl(m log2e),
+// the residual m log2e - cm being taken out once per thread at the end.
+__device__ __forceinline__ void pass1_update(uint4 w, float &m, float &cm, float2 &s)
+{
+    const __nv_bfloat162 *h = reinterpret_cast<const __nv_bfloat162 *>(&w);
+    const __nv_bfloat162 a = __hmax2_nan(__hmax2_nan(h[0], h[1]), __hmax2_nan(h[2], h[3]));
+    const float lm = max_nan(__low2float(a), __high2float(a));
+    if (lm > m || lm != lm) {
+        const float ncm = lm * kLog2e;
+        const float f = ex2_ftz(cm - ncm);
+        s = __fmul2_rn(s, make_float2(f, f));
+        m = lm;
+        cm = ncm;
+    }
+    s = sum8_exp2_pk(w, make_float2(-cm, -cm), s);
+}
+
+// One CTA per SM walks rows t = blockIdx.x, blockIdx.x + gridDim.x, ...  Per
+// row, a producer thread streams both rows through a ring of kRing shared-
+// memory slots twice (bulk copies of sg groups per row per slot): once for
+// pass 1 (from HBM) and once for pass 2 (the same bytes again, mostly from L2,
+// where pass 1 left them microseconds earlier; these copies mark the lines
+// evict-first).  The consumer warps:
+//   pass 1: per thread a running (max, sum) of each row over its groups;
+//           warp, then CTA combination; lanes 0 and 16 of warp 0 form the two
+//           rows' scalars (log p, log q, lse; eps, log k, p for the output);
+//   pass 2: the nine sums, two candidates per packed instruction;
+//           warp sums in fp32, CTA sums in fp64 by warp 0, which also forms
+//           bias2 and dvar while the other warps start the next row.
+template <int MODE, int NW>
+__global__ void __launch_bounds__(StreamCfg<NW>::kThreads, 1)
+    cis_mismatch_stream_kernel(const DiagArgs a, int sg)
+{
+    using C = StreamCfg<NW>;
+    constexpr int kConsWarps = NW, kConsThreads = C::kConsThreads, kRing = C::kRing;
+    constexpr int kSlotGroups = C::kSlotGroups, kSlotBytes = C::kSlotBytes;
+    extern __shared__ __align__(128) uint8_t dyn_smem[];
+    __shared__ StreamShared sh;
+    uint8_t *ring = dyn_smem + ((128 - (smem_u32(dyn_smem) & 127)) & 127);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int ng = (int)(a.V / 8);
+    const int nst = (ng + sg - 1) / sg;
+    if (threadIdx.x == 0) {
+        for (int i = 0; i < kRing; ++i) {
+            mbar_init(smem_u32(&sh.full[i]), 1);
+            mbar_init(smem_u32(&sh.empty[i]), kConsWarps);
+        }
+        sh.aborted = 0;
+    }
+    __syncthreads();
+    const StreamAbort ab{&sh.aborted, a.status};
+
+    if (warp == kConsWarps) {  // producer
+        if (lane != 0)
+            return;
+        uint32_t k = 0;
+        for (int64_t t = blockIdx.x; t < a.T && !ab.on(); t += gridDim.x) {
+            const int64_t y = a.ids[t];
+            if ((a.mask != nullptr && a.mask[t] == 0) || y < 0 || y >= a.V)
+                continue;
+            const uint8_t *rp = reinterpret_cast<const uint8_t *>(a.zt + t * a.ld_t);
+            const uint8_t *rq = reinterpret_cast<const uint8_t *>(a.zi + t * a.ld_i);
+            for (int pass = 0; pass < 2 && !ab.on(); ++pass)
+                for (int st = 0; st < nst; ++st, ++k) {
+                    const uint32_t s = k % kRing, u = k / kRing;
+                    if (u > 0)
+                        ab.wait(smem_u32(&sh.empty[s]), (u - 1) & 1);
+                    if (ab.on())
+                        break;
+                    const int g0 = st * sg, n = min(sg, ng - g0);
+                    const uint32_t bytes = (uint32_t)n * 16;
+                    const uint32_t full = smem_u32(&sh.full[s]);
+                    const uint32_t dst = smem_u32(ring + (size_t)s * kSlotBytes);
+                    mbar_expect_tx(full, 2 * bytes);
+                    if (pass == 0) {
+                        bulk_g2s(dst, rp + (int64_t)g0 * 16, bytes, full);
+                        bulk_g2s(dst + kSlotGroups * 16, rq + (int64_t)g0 * 16, bytes, full);
+                    } else {
+                        bulk_g2s_evict_first(dst, rp + (int64_t)g0 * 16, bytes, full);
+                        bulk_g2s_evict_first(dst + kSlotGroups * 16, rq + (int64_t)g0 * 16, bytes,
+                                             full);
+                    }
+                }
+        }
+        // copies still in flight land before the CTA may exit: the last
+        // use of each slot (k counts the uses issued)
+        for (uint32_t j = k > (uint32_t)kRing ? k - kRing : 0; j < k; ++j)
+            mbar_wait(smem_u32(&sh.full[j % kRing]), (j / kRing) & 1);
+        return;
+    }
+
+    // consumers
+    const int ct = threadIdx.x;
+    uint32_t k = 0;
+    for (int64_t t = blockIdx.x; t < a.T; t += gridDim.x) {
+        const bool valid = a.mask == nullptr || a.mask[t] != 0;
+        const int64_t y = a.ids[t];
+        if (!valid || y < 0 || y >= a.V) {
+            if (ct == 0) {
+                const float v = valid ? NAN : 0.0f;
+                if (valid)
+                    set_status(a.status, kStatusBadId);
+                a.eps[t] = v;
+                if (a.logk) a.logk[t] = v;
+                if (a.p) a.p[t] = v;
+                if (a.bias2) a.bias2[t] = v;
+                if (a.dvar) a.dvar[t] = v;
+            }
+            continue;
+        }
+        // the sampled entries, read early (used after pass 1)
+        float zy = 0.0f;
+        if (warp == 0 && (lane == 0 || lane == 16))
+            zy = to_f32(lane == 0 ? a.zt[t * a.ld_t + y] : a.zi[t * a.ld_i + y]);
+        const int gy = (int)(y >> 3), iy = (int)(y & 7);
+
+        // pass 1
+        float m_p = -INFINITY, m_q = -INFINITY, cm_p = 0.0f, cm_q = 0.0f;
+        float2 s_p = make_float2(0.0f, 0.0f), s_q = make_float2(0.0f, 0.0f);
+        for (int st = 0; st < nst; ++st, ++k) {
+            const uint32_t s = k % kRing;
+            ab.wait(smem_u32(&sh.full[s]), (k / kRing) & 1);
+            const uint4 *slot = reinterpret_cast<const uint4 *>(ring + (size_t)s * kSlotBytes);
+            const int g0 = st * sg, n = min(sg, ng - g0);
+#pragma unroll 1
+            for (int j = ct; j < n; j += kConsThreads) {
+                uint4 u = slot[j], v = slot[kSlotGroups + j];
+                if (g0 + j == gy) {
+                    u = drop_entry(u, iy);
+                    v = drop_entry(v, iy);
+                }
+                pass1_update(u, m_p, cm_p, s_p);
+                pass1_update(v, m_q, cm_q, s_q);
+            }
+            __syncwarp();
+            if (lane == 0)
+                mbar_arrive(smem_u32(&sh.empty[s]));
+        }
+        MaxSum rp{m_p, s_p.x + s_p.y}, rq{m_q, s_q.x + s_q.y};
+        if (m_p != -INFINITY)
+            rp.s *= ex2_ftz(-fmaf(m_p, kLog2e, -cm_p));
+        if (m_q != -INFINITY)
+            rq.s *= ex2_ftz(-fmaf(m_q, kLog2e, -cm_q));
+        rp = warp_ms(rp);
+        rq = warp_ms(rq);
+        if (lane == 0) {
+            sh.red[0][warp] = rp;
+            sh.red[1][warp] = rq;
+        }
+        cons_sync<kConsThreads>();
+        if (warp == 0) {
+            // lanes 0-15 combine the training row's warp pairs, 16-31 the
+            // inference row's (lane l takes warps l, l + 16, ...), then a
+            // fixed tree over the 16 lanes
+            const int r = lane >> 4;
+            MaxSum o = sh.red[r][lane & 15];
+            for (int w = (lane & 15) + 16; w < kConsWarps; w += 16)
+                o = ms_combine(o, sh.red[r][w]);
+#pragma unroll
+            for (int off = 8; off > 0; off >>= 1) {
+                MaxSum x;
+                x.m = __shfl_xor_sync(0xffffffffu, o.m, off);
+                x.s = __shfl_xor_sync(0xffffffffu, o.s, off);
+                o = ms_combine(o, x);
+            }
+            const RowScalars rs = row_scalars(o, zy);
+            // lane 0 gets the inference row's values from lane 16
+            const double lp64_q = __shfl_sync(0xffffffffu, rs.lp64, 16);
+            const float lse_q = __shfl_sync(0xffffffffu, rs.lse, 16);
+            const float om_q = __shfl_sync(0xffffffffu, o.m, 16);
+            const float os_q = __shfl_sync(0xffffffffu, o.s, 16);
+            const float zy_q = __shfl_sync(0xffffffffu, zy, 16);
+            if (lane == 0) {
+                // eps = logit p - logit q: Lemma 3.1's -delta_y + log sum_{j != y}
+                // w_j e^{delta_j} in the normalised gauge, from the log-odds
+                const double dp = ((double)zy - (double)o.m) - (double)logf(o.s);
+                const double dq = ((double)zy_q - (double)om_q) - (double)logf(os_q);
+                a.eps[t] = (float)(dp - dq);
+                if (a.logk) a.logk[t] = (float)(rs.lp64 - lp64_q);
+                if (a.p) a.p[t] = expf(rs.lp);
+                sh.op = rs.lse * kLog2e;
+                sh.oq = lse_q * kLog2e;
+            }
+        }
+        cons_sync<kConsThreads>();
+
+        // pass 2
+        float2 acc[kNSums];
+#pragma unroll
+        for (int i = 0; i < kNSums; ++i)
+            acc[i] = make_float2(0.0f, 0.0f);
+        const float2 nop = make_float2(-sh.op, -sh.op), noq = make_float2(-sh.oq, -sh.oq);
+        for (int st = 0; st < nst; ++st, ++k) {
+            const uint32_t s = k % kRing;
+            ab.wait(smem_u32(&sh.full[s]), (k / kRing) & 1);
+            const uint4 *slot = reinterpret_cast<const uint4 *>(ring + (size_t)s * kSlotBytes);
+            const int n = min(sg, ng - st * sg);
+#pragma unroll 1
+            for (int j = ct; j < n; j += kConsThreads) {
+                const uint4 u = slot[j], v = slot[kSlotGroups + j];
+                diag_pair<MODE>(bf16_pair(u.x), bf16_pair(v.x), nop, noq, a.P, acc);
+                diag_pair<MODE>(bf16_pair(u.y), bf16_pair(v.y), nop, noq, a.P, acc);
+                diag_pair<MODE>(bf16_pair(u.z), bf16_pair(v.z), nop, noq, a.P, acc);
+                diag_pair<MODE>(bf16_pair(u.w), bf16_pair(v.w), nop, noq, a.P, acc);
+            }
+            __syncwarp();
+            if (lane == 0)
+                mbar_arrive(smem_u32(&sh.empty[s]));
+        }
+        // warp sums in fp32 (fp64 arithmetic is scarce on this part), the
+        // CTA's in fp64 by lanes 0-8 of warp 0, in warp order
+#pragma unroll
+        for (int i = 0; i < kNSums; ++i) {
+            float v = acc[i].x + acc[i].y;
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1)
+                v += __shfl_xor_sync(0xffffffffu, v, o);
+            if (lane == 0)
+                sh.wsum[warp][i] = v;
+        }
+        cons_sync<kConsThreads>();
+        if (warp == 0) {
+            if (lane < kNSums) {
+                double v = sh.wsum[0][lane];
+                for (int w = 1; w < kConsWarps; ++w)
+                    v += sh.wsum[w][lane];
+                sh.total[lane] = v;
+            }
+            __syncwarp();
+            if (lane == 0) {
+                const double *S = sh.total;
+                const double P2 = S[0], R2 = S[1], RP = -S[2], D = S[3], C2 = -S[4], C3 = -S[5],
+                             C4 = -S[6], C5 = -S[7], QP = S[8];
+                const double C1 = C2 + 2.0 * D, C6 = C5 + 2.0 * QP;
+                const double bias2 = R2 - 2.0 * C3 * RP + C3 * C3 * P2;
+                const double dvar =
+                    C1 + P2 * C2 - (C4 - (2.0 + C3) * C5 - C3 * C6 + C3 * (2.0 + C3) * P2);
+                if (a.bias2) a.bias2[t] = (float)bias2;
+                if (a.dvar) a.dvar[t] = (float)dvar;
+            }
+        }
+    }
+}
+
+// Groups per slot (CIS_DIAG_SLOT_GROUPS, read at each call: small values
+// make short rows span several slots in tests), and whether the streaming
+// kernel applies at all (CIS_DIAG_KERNEL=row selects the one-CTA kernel).
+int diag_slot_groups(int max_groups)
+{
+    const char *e = getenv("CIS_DIAG_SLOT_GROUPS");
+    const long v = e ? atol(e) : max_groups;
+    return v < 1 ? 1 : (v > max_groups ? max_groups : (int)v);
+}
+
+// Consumer warps (CIS_DIAG_WARPS, for tuning sweeps: 16 or 24; 24 measured
+// faster at V=151936: six warps per scheduler hide more of the dependent
+// latencies than four).
+int diag_warps()
+{
+    const char *e = getenv("CIS_DIAG_WARPS");
+    return (e && atoi(e) == 16) ? 16 : 24;
+}
+
+bool diag_stream_applies(const void *zt, const void *zi, int dtype, int64_t V, int64_t ld_t,
+                         int64_t ld_i)
+{
+    if (dtype != CIS_BF16 || V % 8 != 0)
+        return false;
+    if ((reinterpret_cast<uintptr_t>(zt) & 15) || (reinterpret_cast<uintptr_t>(zi) & 15) ||
+        (ld_t * 2) % 16 || (ld_i * 2) % 16)
+        return false;
+    const char *e = getenv("CIS_DIAG_KERNEL");
+    return !(e && e[0] == 'r');
+}
+
+template <int MODE, int NW>
+cudaError_t launch_stream_nw(const DiagArgs &a, cudaStream_t s)
+{
+    using C = StreamCfg<NW>;
+    auto kern = cis_mismatch_stream_kernel<MODE, NW>;
+    cudaError_t e =
+        cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)C::kSmem);
+    if (e != cudaSuccess)
+        return e;
+    int dev = 0, sms = 0;
+    if ((e = cudaGetDevice(&dev)) != cudaSuccess ||
+        (e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess)
+        return e;
+    const int64_t grid = a.T < sms ? a.T : sms;
+    kern<<<(unsigned)grid, C::kThreads, C::kSmem, s>>>(a, diag_slot_groups(C::kSlotGroups));
+    return cudaGetLastError();
+}
+
+template <int MODE>
+cudaError_t launch_stream_mode(const DiagArgs &a, cudaStream_t s)
+{
+    return diag_warps() == 24 ? launch_stream_nw<MODE, 24>(a, s) : launch_stream_nw<MODE, 16>(a, s);
+}
+
+// ---------------------------------------------------------------------------
+// Dispatch on the operator (a template parameter of both kernels).
+
 template <typename InT, int MODE>
 void launch_mode(const void *zt, const void *zi, int64_t T, int64_t V, int64_t ld_t,
                  int64_t ld_i, const int32_t *ids, const uint8_t *mask, const DevParams &P,
@@ -209,6 +703,14 @@ void launch_mode(const void *zt, const void *zi, int64_t T, int64_t V, int64_t l
         static_cast<const InT *>(zt), static_cast<const InT *>(zi), T, V, ld_t, ld_i, ids, mask,
         P, eps, logk, p, bias2, dvar, status);
 }
+
+#define CIS_DIAG_MODES(X)  \
+    X(CIS_MODE_CIS)        \
+    X(CIS_MODE_TIS)        \
+    X(CIS_MODE_EXACT)      \
+    X(CIS_MODE_BAND)       \
+    X(CIS_MODE_ICEPOP)     \
+    X(CIS_MODE_KPOP)
 
 template <typename InT>
 void launch_type(const void *zt, const void *zi, int64_t T, int64_t V, int64_t ld_t,
@@ -222,18 +724,25 @@ void launch_type(const void *zt, const void *zi, int64_t T, int64_t V, int64_t l
                             status, s);                                                          \
         break;
     switch (P.mode) {
-        CIS_DIAG_CASE(CIS_MODE_CIS)
-        CIS_DIAG_CASE(CIS_MODE_TIS)
-        CIS_DIAG_CASE(CIS_MODE_EXACT)
-        CIS_DIAG_CASE(CIS_MODE_BAND)
-        CIS_DIAG_CASE(CIS_MODE_ICEPOP)
-        CIS_DIAG_CASE(CIS_MODE_KPOP)
+        CIS_DIAG_MODES(CIS_DIAG_CASE)
     default:
         launch_mode<InT, CIS_MODE_NONE>(zt, zi, T, V, ld_t, ld_i, ids, mask, P, eps, logk, p,
                                         bias2, dvar, status, s);
     }
 #undef CIS_DIAG_CASE
 }
+
+cudaError_t launch_stream(const DiagArgs &a, cudaStream_t s)
+{
+#define CIS_DIAG_SCASE(M) \
+    case M: return launch_stream_mode<M>(a, s);
+    switch (a.P.mode) {
+        CIS_DIAG_MODES(CIS_DIAG_SCASE)
+    default: return launch_stream_mode<CIS_MODE_NONE>(a, s);
+    }
+#undef CIS_DIAG_SCASE
+}
+#undef CIS_DIAG_MODES
 
 }  // namespace
 
@@ -244,6 +753,12 @@ cudaError_t launch_mismatch(const void *zt, const void *zi, int dtype, int64_t T
 {
     if (T == 0)
         return cudaSuccess;
+    if (diag_stream_applies(zt, zi, dtype, V, ld_t, ld_i)) {
+        const DiagArgs a{static_cast<const __nv_bfloat16 *>(zt),
+                         static_cast<const __nv_bfloat16 *>(zi),
+                         T, V, ld_t, ld_i, ids, mask, P, eps, logk, p, bias2, dvar, status};
+        return launch_stream(a, s);
+    }
     if (dtype == CIS_BF16)
         launch_type<__nv_bfloat16>(zt, zi, T, V, ld_t, ld_i, ids, mask, P, eps, logk, p, bias2,
                                    dvar, status, s);

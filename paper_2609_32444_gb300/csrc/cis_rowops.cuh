@@ -9,13 +9,6 @@
 namespace cis {
 namespace {
 
-__device__ __forceinline__ float max_nan(float a, float b)
-{
-    float r;
-    asm("max.NaN.f32 %0, %1, %2;" : "=f"(r) : "f"(a), "f"(b));
-    return r;
-}
-
 // Add EV values to a running (m, s), leaving out position `skip` (-1: none).
 template <int EV>
 __device__ __forceinline__ void ms_update(MaxSum &acc, const float (&z)[EV], int skip)

@@ -1,6 +1,11 @@
 """GPU parity of the mismatch diagnostics (App. A.5; Sec. 4.3, Fig. 5c-d)
 against the fp64 oracle, and at full vocabulary size against closed forms.
 
+Both kernels are covered: the streaming kernel (bf16 rows with V a multiple
+of 8; CIS_DIAG_SLOT_GROUPS shrinks its ring slots so that short rows still
+span many slots, wrap the ring and end in a partial slot) and the one-CTA
+kernel (fp32 or ragged rows, or bf16 with CIS_DIAG_KERNEL=row).
+
 Tolerances, from the arithmetic: eps and log k come from fp32 row sums (as log
 p does in the token pass: 2e-5 plus 4 ulps).  The bias and the variance
 increase are fp64 combinations of per-candidate fp32 terms of size O(1) (the
@@ -45,8 +50,10 @@ def _compare(out, ref, mask=None, abs_tol=2e-6):
     m = np.ones(len(ref["eps"]), bool) if mask is None else mask.astype(bool)
     got = {k: v.cpu().numpy().astype(np.float64) for k, v in out.items()}
     for k in ("eps", "logk"):
-        tol = 2e-5 + 2.0 ** -21 * np.abs(ref[k][m])
-        assert np.all(np.abs(got[k][m] - ref[k][m]) <= tol), k
+        fin = np.isfinite(ref[k][m])
+        assert np.array_equal(got[k][m][~fin], ref[k][m][~fin]), k  # equal infinities
+        tol = 2e-5 + 2.0 ** -21 * np.abs(ref[k][m][fin])
+        assert np.all(np.abs(got[k][m][fin] - ref[k][m][fin]) <= tol), k
     assert np.all(np.abs(got["p"][m] - ref["p"][m]) <= 1e-5 * ref["p"][m] + 1e-30)
     for k in ("bias2", "dvar"):
         err = np.abs(got[k][m] - ref[k][m])
@@ -56,10 +63,15 @@ def _compare(out, ref, mask=None, abs_tol=2e-6):
         assert np.all(got[k][~m] == 0), k
 
 
+@pytest.mark.parametrize("kernel", ["stream", "row"])
 @pytest.mark.parametrize("dtype", [torch.float32, torch.bfloat16])
 @pytest.mark.parametrize("mode", list(OMODE))
-def test_diagnostics_match_oracle_small_rows(mode, dtype):
+def test_diagnostics_match_oracle_small_rows(mode, dtype, kernel, monkeypatch):
     """T=24 rows of V=64 (and a ragged V=61 for fp32): every output, every token operator."""
+    if kernel == "row":
+        monkeypatch.setenv("CIS_DIAG_KERNEL", "row")
+    elif dtype == torch.float32:
+        pytest.skip("the streaming kernel takes bf16 rows")
     V = 61 if dtype == torch.float32 else 64
     z, zi, ids = _rows(3, 24, V, dtype)
     out = binding.cis_mismatch_diagnostics(z.to(DEV), zi.to(DEV), ids.to(DEV),
@@ -116,9 +128,95 @@ def test_diagnostics_full_vocabulary_closed_forms():
     assert torch.all(cis["dvar"] <= ex["dvar"] + 2e-5)
 
 
-def test_diagnostics_bad_id_and_status():
-    z, zi, ids = _rows(4, 8, 64, torch.float32)
-    ids[3] = 64
+@pytest.mark.parametrize("mode", list(OMODE))
+def test_diagnostics_stream_ragged_slots(mode, monkeypatch):
+    """The streaming kernel with 64-group slots (V=2056: four full slots and a
+    one-group slot per pass), sampled ids on slot edges, masked rows, and
+    more rows than SMs per CTA only through the row loop (T=24)."""
+    monkeypatch.setenv("CIS_DIAG_SLOT_GROUPS", "64")
+    V, T = 2056, 24
+    z, zi, ids = _rows(11, T, V, torch.bfloat16, sd=0.5)
+    ids[:8] = torch.tensor([0, V - 1, 511, 512, 1023, 1024, 2047, 2048], dtype=torch.int32)
+    m = torch.ones(T, dtype=torch.uint8)
+    m[[5, 17]] = 0
+    out = binding.cis_mismatch_diagnostics(z.to(DEV), zi.to(DEV), ids.to(DEV),
+                                           binding.cis_default_params(mode), mask=m.to(DEV))
+    torch.cuda.synchronize()
+    ref = oracle.mismatch_diagnostics(logits_for_oracle(z), logits_for_oracle(zi), ids.numpy(),
+                                      oracle.params(mode=OMODE[mode]), mask=m.numpy())
+    _compare(out, ref, m.numpy())
+
+
+def test_diagnostics_slot_sizes_agree(monkeypatch):
+    """The same bf16 rows (V=24576: 3072 groups, so every consumer warp holds
+    groups in a full slot) through ring slots of 16 and 24 warps, of 64, 7
+    and 1 groups (the last wraps the ring hundreds of times per pass) and the
+    one-CTA kernel: results differ by summation order only."""
+    V, T = 24576, 16
+    z, zi, ids = _rows(12, T, V, torch.bfloat16)
+    P = binding.cis_default_params("cis")
+    outs = []
+    for warps, sg in [("16", None), ("24", None), ("16", "64"), ("16", "7"), ("24", "1")]:
+        monkeypatch.setenv("CIS_DIAG_WARPS", warps)
+        if sg is None:
+            monkeypatch.delenv("CIS_DIAG_SLOT_GROUPS", raising=False)
+        else:
+            monkeypatch.setenv("CIS_DIAG_SLOT_GROUPS", sg)
+        outs.append(binding.cis_mismatch_diagnostics(z.to(DEV), zi.to(DEV), ids.to(DEV), P))
+    monkeypatch.setenv("CIS_DIAG_KERNEL", "row")
+    outs.append(binding.cis_mismatch_diagnostics(z.to(DEV), zi.to(DEV), ids.to(DEV), P))
+    torch.cuda.synchronize()
+    # each result carries the fp32 summation error that the oracle tolerance
+    # allows (slots of 1 group put all 4096 candidates in one thread's sums)
+    base = {k: v.double().cpu() for k, v in outs[0].items()}
+    for o in outs[1:]:
+        for k, v in o.items():
+            d = (v.double().cpu() - base[k]).abs()
+            assert torch.all(d <= 2e-3 * base[k].abs() + 4e-6), k
+
+
+def test_diagnostics_many_rows_per_cta():
+    """T=700 rows of V=1024 (several rows per CTA on any GPU), every fifth
+    masked: each row matches the oracle."""
+    V, T = 1024, 700
+    z, zi, ids = _rows(14, T, V, torch.bfloat16)
+    m = torch.ones(T, dtype=torch.uint8)
+    m[::5] = 0
+    out = binding.cis_mismatch_diagnostics(z.to(DEV), zi.to(DEV), ids.to(DEV),
+                                           binding.cis_default_params("cis"), mask=m.to(DEV))
+    torch.cuda.synchronize()
+    ref = oracle.mismatch_diagnostics(logits_for_oracle(z), logits_for_oracle(zi), ids.numpy(),
+                                      oracle.params(mode=oracle.MODE_CIS), mask=m.numpy())
+    _compare(out, ref, m.numpy())
+
+
+def test_diagnostics_all_other_entries_neg_inf(monkeypatch):
+    """A row whose entries other than y are -inf for the training engine
+    (p = 1, every other candidate has k = f = 0).  logit p is infinite there:
+    eps is not finite on either side (the kernel's log-odds give +inf, the
+    oracle's definition NaN); the other outputs agree."""
+    monkeypatch.setenv("CIS_DIAG_SLOT_GROUPS", "64")
+    V, T = 2056, 4
+    z, zi, ids = _rows(13, T, V, torch.bfloat16)
+    z[0, :] = float("-inf")
+    z[0, ids[0]] = 1.0
+    out = binding.cis_mismatch_diagnostics(z.to(DEV), zi.to(DEV), ids.to(DEV),
+                                           binding.cis_default_params("cis"))
+    torch.cuda.synchronize()
+    ref = oracle.mismatch_diagnostics(logits_for_oracle(z), logits_for_oracle(zi), ids.numpy(),
+                                      oracle.params(mode=oracle.MODE_CIS))
+    assert not np.isfinite(out["eps"][0].item()) and not np.isfinite(ref["eps"][0])
+    assert out["p"][0].item() == 1.0
+    out["eps"][0] = 0.0
+    ref["eps"][0] = 0.0
+    _compare(out, ref)
+
+
+@pytest.mark.parametrize("dtype,V", [(torch.float32, 64), (torch.bfloat16, 2056)])
+def test_diagnostics_bad_id_and_status(dtype, V, monkeypatch):
+    monkeypatch.setenv("CIS_DIAG_SLOT_GROUPS", "64")
+    z, zi, ids = _rows(4, 8, V, dtype)
+    ids[3] = V
     st = torch.zeros(1, dtype=torch.int32, device=DEV)
     out = binding.cis_mismatch_diagnostics(z.to(DEV), zi.to(DEV), ids.to(DEV),
                                            binding.cis_default_params(), dev_status=st)
