@@ -424,12 +424,12 @@ def run_lmhead(args, rank, world, local):
     nws = binding.cis_lmhead_workspace_size(T, V, H)
     wbuf = torch.empty(nws + 1024, dtype=torch.uint8, device=dev)
     ws = wbuf[(-wbuf.data_ptr()) % 1024:][:nws]
-    # the library's default vocabulary chunk (dz and dz^T of a chunk within 1 GiB)
+    # the library's default vocabulary chunk (dz of a chunk within 1 GiB)
     tp = -(-T // 128) * 128
-    chunk = min(-(-V // 256) * 256, max(256, (1 << 30) // (4 * tp) // 256 * 256))
+    chunk = min(-(-V // 256) * 256, max(256, (1 << 30) // (2 * tp) // 256 * 256))
     n_chunks = -(-V // chunk)
-    # scales, FWD, token, 2 transposes, (DZ, DH, DW) per chunk, reduce
-    launches_per_call = 5 + 3 * n_chunks + 1
+    # scales, FWD, token, (DZ, DH, DW) per chunk, reduce
+    launches_per_call = 3 + 3 * n_chunks + 1
 
     def step():
         return binding.cis_lmhead_fused(b.hidden, b.weight, b.ids, b.lp_infer, b.adv, P,

@@ -12,13 +12,19 @@
 //        logits entry points; gives lse_t and c_t.
 //   then for each vocabulary chunk [v0, v0 + w):
 //   DZ   recompute the chunk's z tiles, form dz = c (softmax - onehot) in bf16
-//        and write it twice, as dz [T, w] and as dz^T [w, T];
+//        and write it as dz [Tp, w];
 //   DH   dH (+)= dz W[v0 : v0 + w]   (K = w, fp32 accumulator);
 //   DW   dW[v0 : v0 + w] = dz^T H    (K = T).
 //
 // dz exists one chunk at a time (the chunk width follows the workspace the
-// caller gives); z never exists outside TMEM.  Every MMA operand is K-major:
-// DH reads W^T and DW reads H^T, which the call writes into its workspace.
+// caller gives); z never exists outside TMEM.  Every operand is read where
+// it lies: FWD and DZ take H and W K-major; DH takes dz K-major and W
+// MN-major (its columns are the output's); DW takes dz and H MN-major (the
+// contraction runs over their rows, the tokens).  An MN-major operand tile
+// arrives as boxes of 64 MN entries x 64 K rows (128-byte swizzle): the
+// canonical MN-major layout of the shared-memory descriptor, with LBO the
+// stride between 64-entry MN blocks and SBO the stride between 8-row K
+// groups; the instruction descriptor marks it transposed (bits 15, 16).
 //
 // The GEMM kernel: 128 x 256 tiles, K blocks of 64 (one 128-byte swizzled row
 // of bf16), a 4-stage ring of 48 KB (A 16 KB + B 32 KB), two 256-column fp32
@@ -53,13 +59,9 @@ constexpr int kThreads = 64 + kEpiThreads;
 constexpr int kHalf = kBN / 2;          // columns per epilogue half
 constexpr uint32_t kTmemCols = 2 * kBN;  // two accumulators
 constexpr size_t kSmemBytes = (size_t)kStages * kStageBytes + 1024;
-// kDz stages dz^T through shared memory: per 32-column chunk two boxes of 64
-// tokens x 32 vocabulary rows (128-byte swizzle), double-buffered per half.
-constexpr int kDztBox = 64 * 32 * 2;                     // 4 KB
-constexpr int kDztBuf = 2 * kDztBox;                     // one chunk: 128 tokens
-constexpr size_t kSmemBytesDz = kSmemBytes + 2 * 2 * kDztBuf;
-// dz + dz^T of one chunk take 4 Tp bytes per vocabulary column; the default
-// chunk keeps them within this many bytes.
+constexpr int kMnBox = 64 * kBK * 2;     // one MN-major box: 64 MN entries x 64 K rows, 8 KB
+// dz of one chunk takes 2 Tp bytes per vocabulary column; the default chunk
+// keeps it within this many bytes.
 constexpr int64_t kDefaultChunkBytes = 1ll << 30;
 
 enum Epi { kStats = 0, kDz = 1, kStore = 2, kAccum = 3 };
@@ -78,12 +80,6 @@ __device__ __forceinline__ int __syncthreads_or_epi(int pred)
     return r;
 }
 
-// Barrier of the 128 threads of one epilogue half (named barriers 2 and 3).
-__device__ __forceinline__ void half_sync(int half)
-{
-    asm volatile("bar.sync %0, 128;" ::"r"(2 + half) : "memory");
-}
-
 __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi)
 {
     __nv_bfloat162 h = __floats2bfloat162_rn(lo, hi);
@@ -91,8 +87,10 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi)
 }
 
 // One launch of the GEMM kernel: C[M, N] = A[M, K] B[N, K]^T over tiles
-// (m, n) of 128 x 256, with TMA coordinates offset by (a_k0, a_row0) and
-// (b_k0, b_row0).
+// (m, n) of 128 x 256, with TMA coordinates offset by a_row0 / b_row0 along
+// M / N and a_k0 / b_k0 along K.  Whether an operand's tensor map runs along
+// M / N in its inner dimension (MN-major) rather than along K is a template
+// parameter of the kernel (A_MN, B_MN).
 struct GemmArgs {
     int nMt, nNt, nK;
     int raster_n;  // 1: tile i -> (m = i % nMt, n = i / nMt); 0: (m = i / nNt, n = i % nNt)
@@ -105,8 +103,7 @@ struct GemmArgs {
     float *part_u;    // kStats: [2 nNt, T] sum e^{z - max} (z - max), or null (no entropy)
     float *zy;        // kStats: z at the sampled token
     uint16_t *dz;     // kDz: bf16 [Tp, ld_dz], column = chunk-local vocabulary index
-    uint16_t *dzt;    // kDz: bf16 [chunk, ld_dzt], column = token
-    int64_t ld_dz, ld_dzt;
+    int64_t ld_dz;
     // kStore, kAccum: rows m 128 + r < rows_valid of out [., ld_out]
     void *out;
     int out_bf16, rows_valid;
@@ -160,15 +157,13 @@ __device__ __forceinline__ void tile_mn(const GemmArgs &g, int i, int &m, int &n
     }
 }
 
-template <int EPI>
+template <int EPI, bool A_MN, bool B_MN>
 __global__ void __launch_bounds__(kThreads, 1)
     cis_lmhead_gemm_kernel(const __grid_constant__ CUtensorMap tmA,
-                           const __grid_constant__ CUtensorMap tmB,
-                           const __grid_constant__ CUtensorMap tmDzt, const GemmArgs g)
+                           const __grid_constant__ CUtensorMap tmB, const GemmArgs g)
 {
     extern __shared__ __align__(1024) uint8_t dsm[];
     uint8_t *ring = dsm + ((1024 - (tc::smem_addr(dsm) & 1023)) & 1023);
-    uint8_t *stage_dzt = ring + kStages * kStageBytes;  // kDz only
     __shared__ __align__(8) Barriers bars;
     __shared__ uint32_t tmem_base;
     __shared__ int aborted;
@@ -213,10 +208,24 @@ __global__ void __launch_bounds__(kThreads, 1)
                     used |= 1u << stage;
                     last = (last & ~(1u << stage)) | (phase << stage);
                     uint8_t *st = ring + stage * kStageBytes;
-                    tc::tma_load_2d(st, &tmA, g.a_k0 + kb * kBK, g.a_row0 + m * kBM,
-                                    &bars.full[stage]);
-                    tc::tma_load_2d(st + kStageA, &tmB, g.b_k0 + kb * kBK, g.b_row0 + n * kBN,
-                                    &bars.full[stage]);
+                    const int ka = g.a_k0 + kb * kBK, kbb = g.b_k0 + kb * kBK;
+                    if (A_MN) {  // MN-major: boxes of 64 rows of M along the inner dimension
+#pragma unroll
+                        for (int i = 0; i < kBM / 64; ++i)
+                            tc::tma_load_2d(st + i * kMnBox, &tmA, g.a_row0 + m * kBM + 64 * i, ka,
+                                            &bars.full[stage]);
+                    } else {
+                        tc::tma_load_2d(st, &tmA, ka, g.a_row0 + m * kBM, &bars.full[stage]);
+                    }
+                    if (B_MN) {
+#pragma unroll
+                        for (int i = 0; i < kBN / 64; ++i)
+                            tc::tma_load_2d(st + kStageA + i * kMnBox, &tmB,
+                                            g.b_row0 + n * kBN + 64 * i, kbb, &bars.full[stage]);
+                    } else {
+                        tc::tma_load_2d(st + kStageA, &tmB, kbb, g.b_row0 + n * kBN,
+                                        &bars.full[stage]);
+                    }
                     if (++stage == kStages) {
                         stage = 0;
                         phase ^= 1;
@@ -231,7 +240,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     } else if (warp == 1) {
         // ---------------------------------------------------------- MMA issue
         if (lane == 0) {
-            constexpr uint32_t kId = tc::idesc_bf16(kBM, kBN);
+            constexpr uint32_t kId = tc::idesc_bf16(kBM, kBN) | ((uint32_t)A_MN << 15) |
+                                     ((uint32_t)B_MN << 16);
+            // a K step of 16: 32 bytes along a K-major row, 16 rows (2 K
+            // groups) of an MN-major tile
+            constexpr uint32_t a_step = A_MN ? 16 * 128 : 32, b_step = B_MN ? 16 * 128 : 32;
             int stage = 0;
             uint32_t phase = 0;
             int i = 0;
@@ -248,9 +261,13 @@ __global__ void __launch_bounds__(kThreads, 1)
                     const uint32_t sa = tc::smem_addr(ring + stage * kStageBytes);
                     const uint32_t sb = sa + kStageA;
 #pragma unroll
-                    for (int kk = 0; kk < kBK / 16; ++kk)
-                        tc::mma_bf16(d, tc::desc_sw128(sa + kk * 32), tc::desc_sw128(sb + kk * 32),
-                                     kId, (kb | kk) != 0);
+                    for (int kk = 0; kk < kBK / 16; ++kk) {
+                        const uint64_t da = A_MN ? tc::desc_sw128_mn(sa + kk * a_step, kMnBox)
+                                                 : tc::desc_sw128(sa + kk * a_step);
+                        const uint64_t db = B_MN ? tc::desc_sw128_mn(sb + kk * b_step, kMnBox)
+                                                 : tc::desc_sw128(sb + kk * b_step);
+                        tc::mma_bf16(d, da, db, kId, (kb | kk) != 0);
+                    }
                     tc::mma_commit(&bars.empty[stage]);
                     if (++stage == kStages) {
                         stage = 0;
@@ -272,9 +289,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int r = lg * 32 + lane;
         const uint32_t lane_off = (uint32_t)(lg * 32) << 16;
         const int cbeg = half * kHalf;
-        const bool leader = r == 0;  // issues this half's dz^T stores
         int i = 0;
-        uint32_t nchunk = 0;  // kDz: chunks this half staged so far (selects the buffer)
         for (int t = blockIdx.x; t < nTiles; t += gridDim.x, ++i) {
             if (__syncthreads_or_epi(ab.on()))
                 break;
@@ -374,32 +389,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                     }
                     uint4 *drow = reinterpret_cast<uint4 *>(g.dz + (int64_t)row * g.ld_dz + cl0 + c0);
 #pragma unroll
-                    for (int q = 0; q < 4; ++q)  // streaming: read back only by the next launch
-                        __stcs(drow + q, make_uint4(w[4 * q], w[4 * q + 1], w[4 * q + 2], w[4 * q + 3]));
-                    // dz^T through shared memory: this chunk's 32 vocabulary rows x
-                    // 128 tokens as two TMA boxes of 64 tokens (128-byte swizzle).
-                    // Buffer nchunk & 1 was last read by the stores of chunk
-                    // nchunk - 2: at most one group (chunk nchunk - 1) may still read.
-                    uint8_t *buf = stage_dzt + (2 * half + (nchunk & 1)) * kDztBuf;
-                    if (leader)
-                        tc::bulk_wait_read<1>();
-                    half_sync(half);
-                    {
-                        uint8_t *box = buf + (r >> 6) * kDztBox;
-                        const int tq = (r & 63) >> 3, tb = (r & 7) * 2;
-#pragma unroll
-                        for (int q = 0; q < 32; ++q)
-                            *reinterpret_cast<uint16_t *>(box + tc::sw128_offset(q, tq) + tb) =
-                                (uint16_t)((q & 1) ? (w[q >> 1] >> 16) : (w[q >> 1] & 0xFFFFu));
-                    }
-                    tc::fence_proxy_async_smem();
-                    half_sync(half);
-                    if (leader) {
-                        tc::tma_store_2d_evict_first(&tmDzt, m * kBM, cl0 + c0, buf);
-                        tc::tma_store_2d_evict_first(&tmDzt, m * kBM + 64, cl0 + c0, buf + kDztBox);
-                        tc::bulk_commit();
-                    }
-                    ++nchunk;
+                    for (int q = 0; q < 4; ++q)  // read back by the next two launches (DH, DW)
+                        drow[q] = make_uint4(w[4 * q], w[4 * q + 1], w[4 * q + 2], w[4 * q + 3]);
                 }
             } else {
                 const int lr = m * kBM + r;  // row of the output block
@@ -441,8 +432,6 @@ __global__ void __launch_bounds__(kThreads, 1)
             tc::fence_before_sync();
             tc::bar_arrive(&bars.accempty[acc]);
         }
-        if (EPI == kDz && leader)
-            tc::bulk_wait_all();  // the dz^T stores have read shared memory and landed
     }
     __syncwarp();
     tc::fence_before_sync();
@@ -537,25 +526,6 @@ __global__ void cis_lmhead_token_kernel(const PassArgs a, const float2 *part, co
     }
 }
 
-// out[c, r] = in[r, c] for a bf16 [rows, cols] matrix (row stride ld_in).
-__global__ void cis_lmhead_transpose_kernel(const __nv_bfloat16 *in, int64_t rows, int64_t cols,
-                                            int64_t ld_in, __nv_bfloat16 *out, int64_t ld_out)
-{
-    __shared__ __nv_bfloat16 tile[32][33];
-    const int64_t r0 = (int64_t)blockIdx.y * 32, c0 = (int64_t)blockIdx.x * 32;
-    for (int i = threadIdx.y; i < 32; i += blockDim.y) {
-        const int64_t r = r0 + i, c = c0 + threadIdx.x;
-        if (r < rows && c < cols)
-            tile[i][threadIdx.x] = in[r * ld_in + c];
-    }
-    __syncthreads();
-    for (int i = threadIdx.y; i < 32; i += blockDim.y) {
-        const int64_t c = c0 + i, r = r0 + threadIdx.x;
-        if (c < cols && r < rows)
-            out[c * ld_out + r] = tile[threadIdx.x][i];
-    }
-}
-
 // ------------------------------------------------------------------ host side
 PFN_cuTensorMapEncodeTiled_v12000 encoder()
 {
@@ -590,17 +560,15 @@ bool make_map(CUtensorMap *m, const void *ptr, int64_t inner, int64_t outer, int
                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-template <int EPI>
+template <int EPI, bool A_MN = false, bool B_MN = false>
 cudaError_t launch_gemm(const CUtensorMap &a, const CUtensorMap &b, const GemmArgs &g,
-                        cudaStream_t s, const CUtensorMap *dzt = nullptr)
+                        cudaStream_t s)
 {
     const int tiles = g.nMt * g.nNt;
     if (tiles <= 0 || g.nK <= 0)
         return cudaSuccess;
-    if (EPI == kDz && dzt == nullptr)
-        return cudaErrorInvalidValue;
-    auto k = cis_lmhead_gemm_kernel<EPI>;
-    const size_t smem = EPI == kDz ? kSmemBytesDz : kSmemBytes;
+    auto k = cis_lmhead_gemm_kernel<EPI, A_MN, B_MN>;
+    const size_t smem = kSmemBytes;
     cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          (int)smem);
     if (e != cudaSuccess)
@@ -610,7 +578,7 @@ cudaError_t launch_gemm(const CUtensorMap &a, const CUtensorMap &b, const GemmAr
         (e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess)
         return e;
     const int grid = tiles < sms ? tiles : sms;
-    k<<<grid, kThreads, smem, s>>>(a, b, dzt ? *dzt : a, g);
+    k<<<grid, kThreads, smem, s>>>(a, b, g);
     return cudaGetLastError();
 }
 
@@ -620,8 +588,8 @@ cudaError_t launch_gemm(const CUtensorMap &a, const CUtensorMap &b, const GemmAr
 // for vocabulary chunks of Vc columns (a multiple of 256).
 struct LmLayout {
     WsLayout base;
-    size_t lse, c, zy, part, part_u, wt, ht, dh, dz, dzt, total;
-    int64_t vp, tp, Tp, Vc;
+    size_t lse, c, zy, part, part_u, dh, dz, total;
+    int64_t Tp, Vc;
 };
 
 static int64_t round_up(int64_t x, int64_t m) { return (x + m - 1) / m * m; }
@@ -632,8 +600,6 @@ LmLayout lm_layout(int64_t T, int64_t V, int64_t Hd, int64_t Vc)
     LmLayout L;
     L.base = ws_layout(T);
     const int64_t nVt = (V + lm::kBN - 1) / lm::kBN;
-    L.vp = round_up(V, 8);
-    L.tp = round_up(T, 8);
     L.Tp = round_up(T, lm::kBM);
     L.Vc = Vc;
     size_t o = up(L.base.total);
@@ -647,16 +613,10 @@ LmLayout lm_layout(int64_t T, int64_t V, int64_t Hd, int64_t Vc)
     o = up(o + 8 * (size_t)T * (size_t)(2 * nVt));
     L.part_u = o;
     o = up(o + 4 * (size_t)T * (size_t)(2 * nVt));
-    L.wt = o;
-    o = up(o + 2 * (size_t)Hd * (size_t)L.vp);
-    L.ht = o;
-    o = up(o + 2 * (size_t)Hd * (size_t)L.tp);
     L.dh = o;
     o = up(o + 4 * (size_t)T * (size_t)Hd);
     L.dz = o;
     o = up(o + 2 * (size_t)L.Tp * (size_t)Vc);
-    L.dzt = o;
-    o = up(o + 2 * (size_t)Vc * (size_t)L.Tp);
     L.total = o;
     return L;
 }
@@ -664,11 +624,11 @@ LmLayout lm_layout(int64_t T, int64_t V, int64_t Hd, int64_t Vc)
 // The widest chunk: every vocabulary column at once.
 static int64_t max_chunk(int64_t V) { return round_up(V, lm::kBN); }
 
-// The default chunk: dz and dz^T within kDefaultChunkBytes.
+// The default chunk: dz within kDefaultChunkBytes.
 static int64_t default_chunk(int64_t T, int64_t V)
 {
     const int64_t Tp = round_up(T, lm::kBM);
-    int64_t c = Tp > 0 ? lm::kDefaultChunkBytes / (4 * Tp) / lm::kBN * lm::kBN : max_chunk(V);
+    int64_t c = Tp > 0 ? lm::kDefaultChunkBytes / (2 * Tp) / lm::kBN * lm::kBN : max_chunk(V);
     if (c < lm::kBN)
         c = lm::kBN;
     return c < max_chunk(V) ? c : max_chunk(V);
@@ -680,7 +640,7 @@ static int64_t chunk_for_bytes(int64_t T, int64_t V, int64_t Hd, size_t bytes)
     const size_t fixed = lm_layout(T, V, Hd, 0).total;
     if (bytes < fixed)
         return 0;
-    const size_t per = 4 * (size_t)round_up(T, lm::kBM);
+    const size_t per = 2 * (size_t)round_up(T, lm::kBM);
     int64_t c = per > 0 ? (int64_t)((bytes - fixed) / per) / lm::kBN * lm::kBN : max_chunk(V);
     if (c > max_chunk(V))
         c = max_chunk(V);
@@ -774,10 +734,7 @@ CIS_API cis_status_t cis_lmhead_fused(const void *hidden, const void *weight, in
     float *zy = reinterpret_cast<float *>(ws + L.zy);
     float2 *part = reinterpret_cast<float2 *>(ws + L.part);
     float *part_u = entropy_out ? reinterpret_cast<float *>(ws + L.part_u) : nullptr;
-    __nv_bfloat16 *wt = reinterpret_cast<__nv_bfloat16 *>(ws + L.wt);
-    __nv_bfloat16 *ht = reinterpret_cast<__nv_bfloat16 *>(ws + L.ht);
     uint16_t *dz = reinterpret_cast<uint16_t *>(ws + L.dz);
-    uint16_t *dzt = reinterpret_cast<uint16_t *>(ws + L.dzt);
     float *dh_acc = grad_dtype == CIS_F32 ? static_cast<float *>(dhidden)
                                           : reinterpret_cast<float *>(ws + L.dh);
 
@@ -789,11 +746,13 @@ CIS_API cis_status_t cis_lmhead_fused(const void *hidden, const void *weight, in
         const int nTt = (int)((T + lm::kBM - 1) / lm::kBM);
         const int nVt = (int)((V + lm::kBN - 1) / lm::kBN);
         const int nHt = (int)(H / lm::kBN);
-        CUtensorMap mH, mW, mWt, mHt;
+        // K-major maps of H and W (FWD, DZ) and MN-major ones (boxes of 64
+        // rows: W as DH's B operand, H as DW's)
+        CUtensorMap mH, mW, mWmn, mHmn;
         if (!lm::make_map(&mH, hidden, H, T, H, lm::kBM) ||
             !lm::make_map(&mW, weight, H, V, H, lm::kBN) ||
-            !lm::make_map(&mWt, wt, V, H, L.vp, lm::kBN) ||
-            !lm::make_map(&mHt, ht, T, H, L.tp, lm::kBN))
+            !lm::make_map(&mWmn, weight, H, V, H, 64) ||
+            !lm::make_map(&mHmn, hidden, H, T, H, 64))
             return CIS_ERR_UNSUPPORTED;
         lm::GemmArgs g = {};
         g.T = (int)T;
@@ -805,9 +764,7 @@ CIS_API cis_status_t cis_lmhead_fused(const void *hidden, const void *weight, in
         g.part_u = part_u;
         g.zy = zy;
         g.dz = dz;
-        g.dzt = dzt;
         g.ld_dz = Vc;
-        g.ld_dzt = L.Tp;
         g.status = a.status;
         // FWD: z tiles of H W^T, row statistics
         g.nMt = nTt;
@@ -842,19 +799,9 @@ CIS_API cis_status_t cis_lmhead_fused(const void *hidden, const void *weight, in
                                                                             2 * nVt, lse, cv);
         if ((e = cudaGetLastError()) != cudaSuccess)
             return CIS_ERR_CUDA;
-        // transposed copies of W and H (K-major B operands of DH and DW)
-        dim3 tb(32, 8);
-        lm::cis_lmhead_transpose_kernel<<<dim3((unsigned)((H + 31) / 32), (unsigned)((V + 31) / 32)),
-                                       tb, 0, s>>>(
-            static_cast<const __nv_bfloat16 *>(weight), V, H, H, wt, L.vp);
-        lm::cis_lmhead_transpose_kernel<<<dim3((unsigned)((H + 31) / 32), (unsigned)((T + 31) / 32)),
-                                       tb, 0, s>>>(
-            static_cast<const __nv_bfloat16 *>(hidden), T, H, H, ht, L.tp);
-        if ((e = cudaGetLastError()) != cudaSuccess)
-            return CIS_ERR_CUDA;
         for (int64_t v0 = 0; v0 < V; v0 += Vc) {
             const int64_t w = V - v0 < Vc ? V - v0 : Vc;
-            // DZ: recompute the chunk's z tiles, write dz and dz^T
+            // DZ: recompute the chunk's z tiles, write dz
             g.nMt = nTt;
             g.nNt = (int)((w + lm::kBN - 1) / lm::kBN);
             g.nK = (int)(H / lm::kBK);
@@ -864,16 +811,16 @@ CIS_API cis_status_t cis_lmhead_fused(const void *hidden, const void *weight, in
             g.b_row0 = (int)v0;
             g.b_k0 = 0;
             g.col0 = (int)v0;
-            CUtensorMap mDz, mDzt, mDztStore;
-            // dz^T as the DZ epilogue stores it: boxes of 64 tokens x 32 rows
-            if (!lm::make_map(&mDztStore, dzt, L.Tp, Vc, L.Tp, 32))
-                return CIS_ERR_UNSUPPORTED;
-            if (lm::launch_gemm<lm::kDz>(mH, mW, g, s, &mDztStore) != cudaSuccess)
+            if (lm::launch_gemm<lm::kDz>(mH, mW, g, s) != cudaSuccess)
                 return CIS_ERR_CUDA;
+            // dz K-major (DH's A: rows are tokens) and MN-major (DW's A: its
+            // M runs along dz's columns; rows past T read as zeros)
+            CUtensorMap mDz, mDzmn;
             if (!lm::make_map(&mDz, dz, w, L.Tp, Vc, lm::kBM) ||
-                !lm::make_map(&mDzt, dzt, T, w, L.Tp, lm::kBM))
+                !lm::make_map(&mDzmn, dz, w, T, Vc, 64))
                 return CIS_ERR_UNSUPPORTED;
-            // DH (+)= dz W[chunk]: A = dz [Tp, w], B = W^T [Hd, V] from column v0
+            // DH (+)= dz W[chunk]: A = dz [Tp, w] K-major, B = W rows v0 .. v0 + w
+            // MN-major (N along Hd, K along the vocabulary)
             g.nMt = nTt;
             g.nNt = nHt;
             g.nK = (int)((w + lm::kBK - 1) / lm::kBK);
@@ -886,11 +833,12 @@ CIS_API cis_status_t cis_lmhead_fused(const void *hidden, const void *weight, in
             g.out_bf16 = 0;
             g.rows_valid = (int)T;
             g.ld_out = H;
-            e = v0 == 0 ? lm::launch_gemm<lm::kStore>(mDz, mWt, g, s)
-                        : lm::launch_gemm<lm::kAccum>(mDz, mWt, g, s);
+            e = v0 == 0 ? lm::launch_gemm<lm::kStore, false, true>(mDz, mWmn, g, s)
+                        : lm::launch_gemm<lm::kAccum, false, true>(mDz, mWmn, g, s);
             if (e != cudaSuccess)
                 return CIS_ERR_CUDA;
-            // DW[chunk] = dz^T H: A = dz^T [w, T], B = H^T [Hd, T]
+            // DW[chunk] = dz^T H: A = dz MN-major (M along the chunk's columns,
+            // K along the tokens), B = H MN-major (N along Hd, K along tokens)
             g.nMt = (int)((w + lm::kBM - 1) / lm::kBM);
             g.nNt = nHt;
             g.nK = (int)((T + lm::kBK - 1) / lm::kBK);
@@ -900,7 +848,7 @@ CIS_API cis_status_t cis_lmhead_fused(const void *hidden, const void *weight, in
                     (size_t)v0 * (size_t)H * (grad_dtype == CIS_BF16 ? 2 : 4);
             g.out_bf16 = grad_dtype == CIS_BF16;
             g.rows_valid = (int)w;
-            if (lm::launch_gemm<lm::kStore>(mDzt, mHt, g, s) != cudaSuccess)
+            if (lm::launch_gemm<lm::kStore, true, true>(mDzmn, mHmn, g, s) != cudaSuccess)
                 return CIS_ERR_CUDA;
         }
         if (grad_dtype == CIS_BF16) {

@@ -1,13 +1,16 @@
 // cis_tc.cuh -- sm_103a tensor-core plumbing for the fused LM-head kernels:
 // mbarriers, TMA tile loads, tcgen05 MMA / TMEM, shared-memory descriptors.
 //
-// Operand tiles are K-major with the 128-byte swizzle: a tile of R rows and 64
+// K-major operand tiles use the 128-byte swizzle: a tile of R rows and 64
 // bf16 along K occupies R x 128 bytes, rows in groups of 8 (1024 bytes) in
 // which the 16-byte chunk c of row r sits at chunk position c ^ (r % 8).  TMA
 // with CU_TENSOR_MAP_SWIZZLE_128B writes exactly this layout when the box is
 // 64 elements wide, and tcgen05.mma reads it through a descriptor whose stride
 // between 8-row groups is 1024 bytes.  Successive K=16 steps inside the
 // 64-wide block advance the descriptor's start address by 32 bytes.
+// MN-major tiles (desc_sw128_mn) are the same swizzled rows with the roles
+// exchanged: each 128-byte row holds 64 entries along M or N for one K index,
+// 8 rows form a 1024-byte group, and a K=16 step is 16 rows (2048 bytes).
 #pragma once
 
 #include <cuda.h>
@@ -44,34 +47,23 @@ __device__ __forceinline__ void bar_arrive(uint64_t *bar)
 {
     asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_addr(bar)) : "memory");
 }
-// Bounded wait for the phase with the given parity (the barrier of this CTA,
-// completed from this CTA or, with kCluster, from others of its cluster).
-// False if it never came or, when `flag` is given, once the word it points to
-// carries kStatusTimeout: a wait elsewhere in the grid ran out, so this one
-// stops early.  The word is read every 256 polls only, off the fast path.
-template <bool kCluster = false>
+// Bounded wait for the phase with the given parity.  False if it never came
+// or, when `flag` is given, once the word it points to carries
+// kStatusTimeout: a wait elsewhere in the grid ran out, so this one stops
+// early.  The word is read every 256 polls only, off the fast path.
 __device__ __forceinline__ bool bar_wait(uint64_t *bar, uint32_t parity,
                                          const volatile int32_t *flag = nullptr)
 {
     const uint32_t a = smem_addr(bar);
     for (uint32_t i = 0; i < kMaxPolls; ++i) {
         uint32_t done;
-        if (kCluster)
-            asm volatile(
-                "{\n\t.reg .pred p;\n\t"
-                "mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2, %3;\n\t"
-                "selp.u32 %0, 1, 0, p;\n\t}"
-                : "=r"(done)
-                : "r"(a), "r"(parity), "r"(kPollSuspendNs)
-                : "memory");
-        else
-            asm volatile(
-                "{\n\t.reg .pred p;\n\t"
-                "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
-                "selp.u32 %0, 1, 0, p;\n\t}"
-                : "=r"(done)
-                : "r"(a), "r"(parity), "r"(kPollSuspendNs)
-                : "memory");
+        asm volatile(
+            "{\n\t.reg .pred p;\n\t"
+            "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
+            "selp.u32 %0, 1, 0, p;\n\t}"
+            : "=r"(done)
+            : "r"(a), "r"(parity), "r"(kPollSuspendNs)
+            : "memory");
         if (done)
             return true;
         if (flag != nullptr && (i & 255) == 255 && (*flag & kStatusTimeout) != 0)
@@ -90,37 +82,6 @@ __device__ __forceinline__ void tma_load_2d(void *dst, const CUtensorMap *map, i
         "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(smem_addr(bar))
         : "memory");
 }
-
-// Tile of `map` at (x, y) from shared memory to global memory (bulk async
-// group of the issuing thread).
-__device__ __forceinline__ void tma_store_2d(const CUtensorMap *map, int x, int y, const void *src)
-{
-    asm volatile("cp.async.bulk.tensor.2d.global.shared::cta.bulk_group [%0, {%1, %2}], [%3];" ::"l"(
-                     reinterpret_cast<uint64_t>(map)),
-                 "r"(x), "r"(y), "r"(smem_addr(src))
-                 : "memory");
-}
-// The same with an L2 policy that evicts the written lines first (data that
-// is not read again soon, so that it does not push operands out of L2).
-__device__ __forceinline__ void tma_store_2d_evict_first(const CUtensorMap *map, int x, int y,
-                                                         const void *src)
-{
-    asm volatile(
-        "{\n\t.reg .b64 pol;\n\t"
-        "createpolicy.fractional.L2::evict_first.b64 pol, 1.0;\n\t"
-        "cp.async.bulk.tensor.2d.global.shared::cta.bulk_group.L2::cache_hint"
-        " [%0, {%1, %2}], [%3], pol;\n\t}" ::"l"(reinterpret_cast<uint64_t>(map)),
-        "r"(x), "r"(y), "r"(smem_addr(src))
-        : "memory");
-}
-__device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
-// Wait until at most N of this thread's bulk groups still read shared memory.
-template <int N> __device__ __forceinline__ void bulk_wait_read()
-{
-    asm volatile("cp.async.bulk.wait_group.read %0;" ::"n"(N) : "memory");
-}
-// Wait until all of this thread's bulk groups are complete.
-__device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
 
 // ------------------------------------------------------------------ tcgen05
 __device__ __forceinline__ void tmem_alloc(uint32_t *dst_smem, uint32_t ncols)
@@ -144,12 +105,6 @@ __device__ __forceinline__ void fence_after_sync()
 {
     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
 }
-// Generic-proxy shared-memory writes become visible to the tensor cores.
-__device__ __forceinline__ void fence_proxy_async_smem()
-{
-    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-}
-
 // D[tmem] (+)= A[smem] * B[smem]^T, bf16 inputs, fp32 accumulate.
 __device__ __forceinline__ void mma_bf16(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc,
                                          uint32_t idesc, bool accumulate)
@@ -182,6 +137,15 @@ __device__ __forceinline__ uint64_t desc_sw128(uint32_t saddr)
            ((uint64_t)1 << 46) | ((uint64_t)2 << 61);
 }
 
+// Descriptor of an MN-major, 128-byte-swizzled operand tile starting at
+// saddr: 64-entry MN blocks (128-byte rows, one per K index) `mn_block`
+// bytes apart (LBO), 8-row K groups 1024 bytes apart (SBO).
+__device__ __forceinline__ uint64_t desc_sw128_mn(uint32_t saddr, uint32_t mn_block)
+{
+    return (uint64_t)((saddr & 0x3FFFF) >> 4) | ((uint64_t)((mn_block >> 4) & 0x3FFF) << 16) |
+           ((uint64_t)64 << 32) | ((uint64_t)1 << 46) | ((uint64_t)2 << 61);
+}
+
 // 32 consecutive fp32 columns of this thread's TMEM lane.
 __device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32])
 {
@@ -200,65 +164,6 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32])
 #pragma unroll
     for (int i = 0; i < 32; ++i)
         v[i] = __uint_as_float(r[i]);
-}
-
-// ------------------------------------------------------------------ cluster
-__device__ __forceinline__ uint32_t map_rank(uint32_t saddr, uint32_t rank)
-{
-    uint32_t r;
-    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(saddr), "r"(rank));
-    return r;
-}
-__device__ __forceinline__ void cluster_arrive()
-{
-    asm volatile("barrier.cluster.arrive.release.aligned;" ::: "memory");
-}
-__device__ __forceinline__ void cluster_wait()
-{
-    asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory");
-}
-// Bounded wait for a phase completed by another CTA of the cluster (its bulk
-// copies or its tensor cores).
-__device__ __forceinline__ bool bar_wait_cluster(uint64_t *bar, uint32_t parity,
-                                                 const volatile int32_t *flag = nullptr)
-{
-    return bar_wait<true>(bar, parity, flag);
-}
-// Copy `bytes` of this CTA's shared memory to another CTA's shared memory
-// (addresses from map_rank); the receiver's mbarrier counts the bytes.
-__device__ __forceinline__ void bulk_s2s(uint32_t dst_cluster, uint32_t src_cta, uint32_t bytes,
-                                         uint32_t bar_cluster)
-{
-    asm volatile(
-        "cp.async.bulk.shared::cluster.shared::cta.mbarrier::complete_tx::bytes"
-        " [%0], [%1], %2, [%3];" ::"r"(dst_cluster),
-        "r"(src_cta), "r"(bytes), "r"(bar_cluster)
-        : "memory");
-}
-// Once every MMA issued so far by this thread is done, arrive on the mbarrier
-// at the same shared-memory offset in each CTA of `cta_mask`.
-__device__ __forceinline__ void mma_commit_multicast(uint64_t *bar, uint16_t cta_mask)
-{
-    asm volatile(
-        "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64"
-        " [%0], %1;" ::"r"(smem_addr(bar)),
-        "h"(cta_mask)
-        : "memory");
-}
-
-// max(*addr, v) on a 32-bit word of a CTA of the cluster (address from map_rank).
-__device__ __forceinline__ void red_max_cluster(uint32_t addr_cluster, int v)
-{
-    asm volatile("red.relaxed.cluster.shared::cluster.max.s32 [%0], %1;" ::"r"(addr_cluster),
-                 "r"(v)
-                 : "memory");
-}
-
-// Byte offset of 16-byte chunk q (0..7) of row r inside a 128-byte-swizzled
-// K-major block (the layout TMA SWIZZLE_128B produces).
-__device__ __forceinline__ uint32_t sw128_offset(int r, int q)
-{
-    return (uint32_t)((r >> 3) * 1024 + (r & 7) * 128 + ((q ^ (r & 7)) << 4));
 }
 
 }  // namespace tc

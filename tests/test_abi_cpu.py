@@ -87,13 +87,13 @@ def _fwd_bwd_rc(binding, **over):
 
 
 def test_lmhead_workspace_grows_with_the_chunk(binding):
-    """4 ceil(T/128)*128 bytes per chunk column (dz and dz^T in bf16); chunks
-    wider than V (rounded up to 256) cost no more; a chunk must be a positive
+    """2 ceil(T/128)*128 bytes per chunk column (dz in bf16); chunks wider
+    than V (rounded up to 256) cost no more; a chunk must be a positive
     multiple of 256."""
     T, V, H = 1000, 5000, 512
     s256 = binding.cis_lmhead_workspace_size_chunk(T, V, H, 256)
     s512 = binding.cis_lmhead_workspace_size_chunk(T, V, H, 512)
-    assert s512 - s256 in range(4 * 1024 * 256, 4 * 1024 * 256 + 2049)
+    assert s512 - s256 in range(2 * 1024 * 256, 2 * 1024 * 256 + 1025)
     full = binding.cis_lmhead_workspace_size_chunk(T, V, H, 5120)
     assert binding.cis_lmhead_workspace_size_chunk(T, V, H, 1 << 20) == full
     assert binding.cis_lmhead_workspace_size(T, V, H) <= full
