@@ -338,11 +338,14 @@ def cis_lmhead_workspace_size_chunk(T: int, V: int, H: int, chunk: int) -> int:
 def cis_lmhead_fused(hidden: torch.Tensor, weight: torch.Tensor, ids: torch.Tensor,
                      lp_infer: torch.Tensor, adv: torch.Tensor, params: cis_params_t,
                      lp_old=None, mask=None, cu_seqlens=None, grad_dtype=torch.float32,
-                     workspace=None, chunk=None, want_entropy=False):
+                     workspace=None, chunk=None, want_entropy=False, dhidden=None,
+                     dweight=None):
     """Token pass through the LM head (logits never stored).  `chunk` (a
     multiple of 256) sizes the workspace for vocabulary chunks of that many
-    columns; by default the library's choice.  Returns a dict with dhidden,
-    dweight, lp, w, trunc, loss, stats and the workspace."""
+    columns; by default the library's choice.  `dhidden` [T, H] and `dweight`
+    [V, H] (contiguous, `grad_dtype`, 16-byte aligned) receive the gradients
+    if given.  Returns a dict with dhidden, dweight, lp, w, trunc, loss, stats
+    and the workspace."""
     _need_cuda(hidden, weight, ids, lp_infer, adv, lp_old, mask, cu_seqlens)
     if hidden.dtype != torch.bfloat16 or weight.dtype != torch.bfloat16:
         raise TypeError("hidden and weight must be bfloat16")
@@ -358,8 +361,16 @@ def cis_lmhead_fused(hidden: torch.Tensor, weight: torch.Tensor, ids: torch.Tens
                       (mask, torch.uint8, "mask")):
         _vec(x, dt, T, nm)
     B = 0 if cu_seqlens is None else cu_seqlens.shape[0] - 1
-    dh = torch.empty((T, H), dtype=grad_dtype, device=dev)
-    dw = torch.empty((V, H), dtype=grad_dtype, device=dev)
+    def _out(x, shape, nm):
+        if x is None:
+            return torch.empty(shape, dtype=grad_dtype, device=dev)
+        if x.dtype != grad_dtype or tuple(x.shape) != shape or not x.is_contiguous():
+            raise ValueError(f"{nm} must be a contiguous {grad_dtype} tensor of shape {shape}")
+        _need_cuda(x)
+        return x
+
+    dh = _out(dhidden, (T, H), "dhidden")
+    dw = _out(dweight, (V, H), "dweight")
     lp = torch.empty(T, dtype=torch.float32, device=dev)
     w = torch.empty(T, dtype=torch.float32, device=dev)
     tr = torch.empty(T, dtype=torch.uint8, device=dev)

@@ -80,6 +80,30 @@ __device__ __forceinline__ int __syncthreads_or_epi(int pred)
     return r;
 }
 
+// 32-byte global accesses (sm_100 and later): one full sector per thread, so
+// that a warp's store into 32 rows writes 32 whole sectors.  The address must
+// be 32-byte aligned.
+__device__ __forceinline__ void st_v8(void *p, const uint32_t *w)
+{
+    asm volatile("st.global.v8.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8};" ::"l"(p), "r"(w[0]),
+                 "r"(w[1]), "r"(w[2]), "r"(w[3]), "r"(w[4]), "r"(w[5]), "r"(w[6]), "r"(w[7])
+                 : "memory");
+}
+// The same with the streaming (evict-first) hint.
+__device__ __forceinline__ void st_v8_cs(void *p, const uint32_t *w)
+{
+    asm volatile("st.global.cs.v8.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8};" ::"l"(p), "r"(w[0]),
+                 "r"(w[1]), "r"(w[2]), "r"(w[3]), "r"(w[4]), "r"(w[5]), "r"(w[6]), "r"(w[7])
+                 : "memory");
+}
+__device__ __forceinline__ void ld_v8(const void *p, float *r)
+{
+    asm volatile("ld.global.v8.f32 {%0, %1, %2, %3, %4, %5, %6, %7}, [%8];"
+                 : "=f"(r[0]), "=f"(r[1]), "=f"(r[2]), "=f"(r[3]), "=f"(r[4]), "=f"(r[5]),
+                   "=f"(r[6]), "=f"(r[7])
+                 : "l"(p));
+}
+
 __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi)
 {
     __nv_bfloat162 h = __floats2bfloat162_rn(lo, hi);
@@ -104,9 +128,10 @@ struct GemmArgs {
     float *zy;        // kStats: z at the sampled token
     uint16_t *dz;     // kDz: bf16 [Tp, ld_dz], column = chunk-local vocabulary index
     int64_t ld_dz;
-    // kStore, kAccum: rows m 128 + r < rows_valid of out [., ld_out]
+    // kStore, kAccum: rows m 128 + r < rows_valid of out [., ld_out]; out_v8:
+    // out is 32-byte aligned (32-byte accesses), else 16-byte ones
     void *out;
-    int out_bf16, rows_valid;
+    int out_bf16, rows_valid, out_v8;
     int64_t ld_out;
     int32_t *status;
 };
@@ -387,10 +412,11 @@ __global__ void __launch_bounds__(kThreads, 1)
                         }
                         w[q >> 1] = pack_bf16x2(d[0], d[1]);
                     }
-                    uint4 *drow = reinterpret_cast<uint4 *>(g.dz + (int64_t)row * g.ld_dz + cl0 + c0);
-#pragma unroll
-                    for (int q = 0; q < 4; ++q)  // read back by the next two launches (DH, DW)
-                        drow[q] = make_uint4(w[4 * q], w[4 * q + 1], w[4 * q + 2], w[4 * q + 3]);
+                    // 64 bytes of the row in two full-sector stores (read back by
+                    // the next two launches, DH and DW)
+                    uint16_t *drow = g.dz + (int64_t)row * g.ld_dz + cl0 + c0;
+                    st_v8(drow, w);
+                    st_v8(drow + 16, w + 8);
                 }
             } else {
                 const int lr = m * kBM + r;  // row of the output block
@@ -402,14 +428,38 @@ __global__ void __launch_bounds__(kThreads, 1)
                     if (!live)
                         continue;
                     if (g.out_bf16) {
-                        uint4 *dst = reinterpret_cast<uint4 *>(
-                            reinterpret_cast<uint16_t *>(g.out) + o + c0);
+                        uint32_t w[16];
 #pragma unroll
-                        for (int q = 0; q < 4; ++q)  // streaming: outputs are not re-read here
-                            __stcs(dst + q, make_uint4(pack_bf16x2(v[8 * q + 0], v[8 * q + 1]),
-                                                       pack_bf16x2(v[8 * q + 2], v[8 * q + 3]),
-                                                       pack_bf16x2(v[8 * q + 4], v[8 * q + 5]),
-                                                       pack_bf16x2(v[8 * q + 6], v[8 * q + 7])));
+                        for (int q = 0; q < 16; ++q)
+                            w[q] = pack_bf16x2(v[2 * q], v[2 * q + 1]);
+                        uint16_t *dst = reinterpret_cast<uint16_t *>(g.out) + o + c0;
+                        if (g.out_v8) {  // streaming: outputs are not re-read here
+                            st_v8_cs(dst, w);
+                            st_v8_cs(dst + 16, w + 8);
+                        } else {
+                            uint4 *d4 = reinterpret_cast<uint4 *>(dst);
+#pragma unroll
+                            for (int q = 0; q < 4; ++q)
+                                __stcs(d4 + q, make_uint4(w[4 * q], w[4 * q + 1], w[4 * q + 2],
+                                                          w[4 * q + 3]));
+                        }
+                    } else if (g.out_v8) {
+                        float *dst = reinterpret_cast<float *>(g.out) + o + c0;
+#pragma unroll
+                        for (int q = 0; q < 4; ++q) {
+                            float x[8];
+#pragma unroll
+                            for (int e = 0; e < 8; ++e)
+                                x[e] = v[8 * q + e];
+                            if (EPI == kAccum) {
+                                float old[8];
+                                ld_v8(dst + 8 * q, old);
+#pragma unroll
+                                for (int e = 0; e < 8; ++e)
+                                    x[e] += old[e];
+                            }
+                            st_v8_cs(dst + 8 * q, reinterpret_cast<const uint32_t *>(x));
+                        }
                     } else {
                         float4 *dst = reinterpret_cast<float4 *>(
                             reinterpret_cast<float *>(g.out) + o + c0);
@@ -831,6 +881,7 @@ CIS_API cis_status_t cis_lmhead_fused(const void *hidden, const void *weight, in
             g.b_k0 = (int)v0;
             g.out = dh_acc;
             g.out_bf16 = 0;
+            g.out_v8 = (reinterpret_cast<uintptr_t>(dh_acc) & 31) == 0;
             g.rows_valid = (int)T;
             g.ld_out = H;
             e = v0 == 0 ? lm::launch_gemm<lm::kStore, false, true>(mDz, mWmn, g, s)
@@ -847,6 +898,7 @@ CIS_API cis_status_t cis_lmhead_fused(const void *hidden, const void *weight, in
             g.out = static_cast<uint8_t *>(dweight) +
                     (size_t)v0 * (size_t)H * (grad_dtype == CIS_BF16 ? 2 : 4);
             g.out_bf16 = grad_dtype == CIS_BF16;
+            g.out_v8 = (reinterpret_cast<uintptr_t>(g.out) & 31) == 0;
             g.rows_valid = (int)w;
             if (lm::launch_gemm<lm::kStore, true, true>(mDzmn, mHmn, g, s) != cudaSuccess)
                 return CIS_ERR_CUDA;

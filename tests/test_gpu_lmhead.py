@@ -132,6 +132,34 @@ def test_lmhead_vocabulary_chunks(T, V, H, chunk, grad):
     assert binding.decode_stats(out["stats"])["status"] == 0
 
 
+@pytest.mark.parametrize("grad", [torch.float32, torch.bfloat16])
+def test_lmhead_outputs_16_byte_aligned(grad):
+    """Gradient buffers that are 16-byte but not 32-byte aligned take the
+    16-byte store path; the results equal those of aligned buffers bit for
+    bit (the same arithmetic, only the store width differs)."""
+    b = synth.make_batch(5, T=200, V=1000, H=256)
+    T, H, V = 200, 256, 1000
+    es = torch.empty((), dtype=grad).element_size()
+    pad = 16 // es
+    dh_buf = torch.empty(T * H + pad, dtype=grad, device=DEV)
+    dw_buf = torch.empty(V * H + pad, dtype=grad, device=DEV)
+    dh = dh_buf[pad:].view(T, H)
+    dw = dw_buf[pad:].view(V, H)
+    assert dh.data_ptr() % 32 == 16 and dw.data_ptr() % 32 == 16
+    P = binding.cis_default_params("cis", lam=b.lam)
+    args = (b.hidden.to(DEV), b.weight.to(DEV), b.ids.to(DEV), b.lp_infer.to(DEV),
+            b.adv.to(DEV), P)
+    kw = dict(mask=b.mask.to(DEV), grad_dtype=grad, chunk=256)
+    odd = binding.cis_lmhead_fused(*args, dhidden=dh, dweight=dw, **kw)
+    ref = binding.cis_lmhead_fused(*args, **kw)
+    torch.cuda.synchronize()
+    assert ref["dhidden"].data_ptr() % 32 == 0 and ref["dweight"].data_ptr() % 32 == 0
+    assert torch.equal(odd["dhidden"].view(torch.int16 if es == 2 else torch.int32),
+                       ref["dhidden"].view(torch.int16 if es == 2 else torch.int32))
+    assert torch.equal(odd["dweight"].view(torch.int16 if es == 2 else torch.int32),
+                       ref["dweight"].view(torch.int16 if es == 2 else torch.int32))
+
+
 def test_lmhead_workspace_too_small():
     """Less workspace than 256-column chunks need is refused on the host."""
     b = synth.make_batch(5, T=64, V=1024, H=256)
