@@ -418,6 +418,33 @@ CIS_API cis_status_t cis_loss_fwd_bwd_noalloc(const void *logits, int32_t dtype,
  */
 CIS_API cis_status_t cis_profile_next_call(void *begin_event, void *end_event);
 
+/*
+ * Self-test of the failure detection of the kernels' waits.
+ *
+ * Every wait inside the library's kernels (for bulk copies, tensor-core work
+ * or other CTAs of a cluster) polls its mbarrier a bounded number of times,
+ * each poll suspending for at most 1 µs (about 2 s in all), then sets
+ * CIS_ERR_DEVICE_TIMEOUT in the call's device status word and lets the
+ * kernel run to its end, so that the CUDA context stays usable and the host
+ * reads the error after a synchronisation.  This call runs one CTA that
+ * waits on an mbarrier which nothing ever completes, through the same wait
+ * code with a poll limit of `max_polls` (1 .. 2^21), and reports the
+ * timeout the same way.
+ *
+ * Arguments:
+ *   - max_polls: the poll limit (each poll waits at most about 1 µs).
+ *   - cluster_scope: 0 for the CTA-scope wait (bulk copies into this CTA),
+ *     1 for the cluster-scope wait (data from other CTAs of a cluster).
+ *   - dev_status: device int32, OR-ed with CIS_ERR_DEVICE_TIMEOUT; the
+ *     caller clears and reads it.
+ *   - stream: cudaStream_t (NULL: the default stream); asynchronous.
+ *
+ * CIS_ERR_INVALID_ARG for a null status, a limit out of range or a scope
+ * other than 0 or 1.
+ */
+CIS_API cis_status_t cis_selftest_bounded_wait(uint32_t max_polls, int32_t cluster_scope,
+                                               int32_t *dev_status, void *stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -114,6 +114,8 @@ def lib():
     L.cis_mismatch_diagnostics.argtypes = [P, P, i32, i64, i64, i64, i64, P, P,
                                            ctypes.POINTER(cis_params_t), P, P, P, P, P, P, P]
     L.cis_mismatch_diagnostics.restype = ctypes.c_int
+    L.cis_selftest_bounded_wait.argtypes = [ctypes.c_uint32, i32, P, P]
+    L.cis_selftest_bounded_wait.restype = ctypes.c_int
     L.cis_profile_next_call.argtypes = [P, P]
     L.cis_profile_next_call.restype = ctypes.c_int
     _lib = L
@@ -418,6 +420,20 @@ def cis_mismatch_diagnostics(logits_train: torch.Tensor, logits_infer: torch.Ten
         _ptr(out["p"]), _ptr(out["bias2"]), _ptr(out["dvar"]), _ptr(dev_status), _stream())
     _check(rc, "cis_mismatch_diagnostics")
     return out
+
+
+def cis_selftest_bounded_wait(max_polls: int, cluster_scope: bool = False,
+                              dev_status: "torch.Tensor | None" = None) -> torch.Tensor:
+    """Run the bounded-wait self-test (a wait that nothing completes, with a
+    limit of max_polls polls); returns the device status word (int32 [1]),
+    which then carries CIS_ERR_DEVICE_TIMEOUT."""
+    if dev_status is None:
+        dev_status = torch.zeros(1, dtype=torch.int32, device="cuda")
+    _need_cuda(dev_status)
+    _check(lib().cis_selftest_bounded_wait(int(max_polls), int(bool(cluster_scope)),
+                                           _ptr(dev_status), _stream()),
+           "cis_selftest_bounded_wait")
+    return dev_status
 
 
 def cis_profile_next_call(begin: "torch.cuda.Event | None", end: "torch.cuda.Event | None"):

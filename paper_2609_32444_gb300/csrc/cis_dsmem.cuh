@@ -39,10 +39,11 @@ __device__ __forceinline__ void bulk_g2s(uint32_t dst, const void *src, uint32_t
         : "memory");
 }
 
-// Bounded wait on phase `parity` of an mbarrier; false if it never completed.
-__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity)
+// Bounded wait on phase `parity` of an mbarrier: at most max_polls polls,
+// each suspending for up to kPollSuspendNs; false if it never completed.
+__device__ __forceinline__ bool mbar_wait_n(uint32_t bar, uint32_t parity, uint32_t max_polls)
 {
-    for (uint32_t i = 0; i < kMaxPolls; ++i) {
+    for (uint32_t i = 0; i < max_polls; ++i) {
         uint32_t done;
         asm volatile(
             "{\n\t.reg .pred p;\n\t"
@@ -55,6 +56,10 @@ __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity)
             return true;
     }
     return false;
+}
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity)
+{
+    return mbar_wait_n(bar, parity, kMaxPolls);
 }
 
 __device__ __forceinline__ void cluster_arrive_relaxed()
@@ -195,9 +200,10 @@ __device__ __forceinline__ void st_async_quad(uint32_t dst, float m, float s, fl
 }
 
 // Bounded wait for data written by other CTAs of the cluster.
-__device__ __forceinline__ bool mbar_wait_cluster(uint32_t bar, uint32_t parity)
+__device__ __forceinline__ bool mbar_wait_cluster_n(uint32_t bar, uint32_t parity,
+                                                    uint32_t max_polls)
 {
-    for (uint32_t i = 0; i < kMaxPolls; ++i) {
+    for (uint32_t i = 0; i < max_polls; ++i) {
         uint32_t done;
         asm volatile(
             "{\n\t.reg .pred p;\n\t"
@@ -210,6 +216,10 @@ __device__ __forceinline__ bool mbar_wait_cluster(uint32_t bar, uint32_t parity)
             return true;
     }
     return false;
+}
+__device__ __forceinline__ bool mbar_wait_cluster(uint32_t bar, uint32_t parity)
+{
+    return mbar_wait_cluster_n(bar, parity, kMaxPolls);
 }
 
 __device__ __forceinline__ void wait_or_flag(uint32_t bar, bool cluster_scope, int32_t *status)

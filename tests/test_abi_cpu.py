@@ -171,3 +171,14 @@ def test_binding_refuses_cpu_tensors(binding):
     x = torch.zeros(2, 8)
     with pytest.raises(ValueError):
         binding.cis_token_logprobs(x, torch.zeros(2, dtype=torch.int32))
+
+
+def test_selftest_bounded_wait_rejects_bad_arguments(binding):
+    """The wait self-test validates on the host: a status word is required,
+    the poll limit is 1 .. 2^21 and the scope 0 or 1 (no launch happens)."""
+    L = binding.lib()
+    dummy = ctypes.c_void_p(0x1000)  # never dereferenced: rejected first
+    assert L.cis_selftest_bounded_wait(100, 0, None, None) == binding.CIS_ERR_INVALID_ARG
+    assert L.cis_selftest_bounded_wait(0, 0, dummy, None) == binding.CIS_ERR_INVALID_ARG
+    assert L.cis_selftest_bounded_wait((1 << 21) + 1, 0, dummy, None) == binding.CIS_ERR_INVALID_ARG
+    assert L.cis_selftest_bounded_wait(100, 2, dummy, None) == binding.CIS_ERR_INVALID_ARG
