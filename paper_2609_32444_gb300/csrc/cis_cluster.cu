@@ -4,7 +4,7 @@
 // CTA's shared memory.  A cluster of CS CTAs (1 <= CS <= 8) therefore
 // splits each row into CS contiguous slices.  Per row:
 //   1. each CTA copies its slice from HBM into shared memory with bulk
-//      asynchronous copies (cp.async.bulk, four chunks, each completing on its
+//      asynchronous copies (cp.async.bulk, two chunks, each completing on its
 //      own mbarrier so that pass 1 starts on the first chunk; no multicast);
 //   2. pass 1 over shared memory: per thread the exact maximum of its entries
 //      (j != y; bf16 pairs compared packed), then the sum of e^{z - max}; a
@@ -116,8 +116,9 @@ __global__ void __launch_bounds__(kThreads) cis_fused_cluster_kernel(const PassA
     const uint32_t xbar = smem_u32(&sh.xbar);
     if (threadIdx.x == 0) {
         for (int c = 0; c < kChunks; ++c)
-            mbar_init(smem_u32(&sh.bar[c]), 1);
-        mbar_init(xbar, 1);
+            mbar_init_only(smem_u32(&sh.bar[c]), 1);
+        mbar_init_only(xbar, 1);
+        mbar_init_fence();
         // the one local arrival on xbar; the peers' stores bring the bytes
         mbar_expect_tx(xbar, (uint32_t)(cs * (kEnt ? sizeof(float4) : sizeof(float2))));
         const uint8_t *src = reinterpret_cast<const uint8_t *>(a.logits) +
@@ -247,16 +248,23 @@ __global__ void __launch_bounds__(kThreads) cis_fused_cluster_kernel(const PassA
         }
         // Pass 2 forms c softmax_j as cs 2^{z_j log2e - B}: with the power-of-two
         // scale K = clamp(ilogb(c) + 25, 0, 127) (below), B = fl(m log2e + bias
-        // - K), and the rounding residual of B folded into cs.
+        // - K), and the rounding residual of B folded into cs.  The residual is
+        // exact: the product's error from an FMA, the two sums' errors from
+        // two-sums (fp32 throughout: fp64 operations take 64 cycles each here).
         const float c = tl.c;
         const int kexp = (int)((__float_as_uint(c) >> 23) & 0xff) - 127 + 25;
         const int K = kexp < 0 ? 0 : (kexp > 127 ? 127 : kexp);
         float cs = ldexpf(c, -K);
         float B = INFINITY;
         if (rs.bias_log2 != INFINITY) {
-            const double Bd = (double)rs.m * (double)kLog2e + ((double)rs.bias_log2 - K);
-            B = (float)Bd;
-            cs *= ex2_ftz((float)((double)B - Bd));
+            const float p = rs.m * kLog2e, pe = fmaf(rs.m, kLog2e, -p);  // p + pe = m log2e
+            const float a = rs.bias_log2, k = -(float)K;
+            const float q = a + k, qv = q - a;
+            const float qe = (a - (q - qv)) + (k - qv);  // q + qe = bias - K
+            B = p + q;
+            const float bv = B - p;
+            const float se = (p - (B - bv)) + (q - bv);  // B + se = p + q
+            cs *= ex2_ftz(-(se + pe + qe));
         }
         sh.c = c;
         sh.cs = cs;

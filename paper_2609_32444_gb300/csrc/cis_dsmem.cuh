@@ -11,7 +11,7 @@ namespace cis {
 namespace {
 
 constexpr int kMaxCluster = 8;
-constexpr int kChunks = 4;  // a slice is copied in this many pieces
+constexpr int kChunks = 2;  // a slice is copied in this many pieces (1 to 8 measured: 2 is fastest)
 
 __device__ __forceinline__ uint32_t smem_u32(const void *p)
 {
@@ -21,6 +21,16 @@ __device__ __forceinline__ uint32_t smem_u32(const void *p)
 __device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count)
 {
     asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+}
+// Several initialisations, then one fence that makes all of them visible to
+// the cluster (and to the async proxy).
+__device__ __forceinline__ void mbar_init_only(uint32_t bar, uint32_t count)
+{
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
+}
+__device__ __forceinline__ void mbar_init_fence()
+{
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
 }
 
