@@ -311,12 +311,14 @@ struct DiagArgs {
 };
 
 // The layout for NW consumer warps (plus one producer warp): a ring slot
-// holds two groups per consumer thread of each row, as many slots as fit in
-// about 200 KB of shared memory.
+// holds four groups per consumer thread of each row, as many slots as fit in
+// about 200 KB of shared memory (3 for 16 warps).  Each slot costs every warp
+// a wait, an arrive and the loop set-up; four groups a thread amortise that
+// (two, three, five and six measured slower).
 template <int NW> struct StreamCfg {
     static constexpr int kConsThreads = NW * 32;
     static constexpr int kThreads = kConsThreads + 32;
-    static constexpr int kSlotGroups = 2 * kConsThreads;  // 8-entry groups of each row per slot
+    static constexpr int kSlotGroups = 4 * kConsThreads;  // 8-entry groups of each row per slot
     static constexpr int kSlotBytes = 2 * kSlotGroups * 16;
     static constexpr int kRing = (200 * 1024) / kSlotBytes < 8 ? (200 * 1024) / kSlotBytes : 8;
     static constexpr size_t kSmem = (size_t)kRing * kSlotBytes + 128;
@@ -645,13 +647,13 @@ int diag_slot_groups(int max_groups)
     return v < 1 ? 1 : (v > max_groups ? max_groups : (int)v);
 }
 
-// Consumer warps (CIS_DIAG_WARPS, for tuning sweeps: 16 or 24; 24 measured
-// faster at V=151936: six warps per scheduler hide more of the dependent
-// latencies than four).
+// Consumer warps (CIS_DIAG_WARPS, for tuning sweeps: 16 or 24; 16 measured
+// faster at V=151936 with four groups a thread per slot: 3 slots of 64 KB
+// against 2 of 96 KB for 24 warps).
 int diag_warps()
 {
     const char *e = getenv("CIS_DIAG_WARPS");
-    return (e && atoi(e) == 16) ? 16 : 24;
+    return (e && atoi(e) == 24) ? 24 : 16;
 }
 
 bool diag_stream_applies(const void *zt, const void *zi, int dtype, int64_t V, int64_t ld_t,
