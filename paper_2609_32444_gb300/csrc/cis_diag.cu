@@ -226,9 +226,12 @@ __device__ __forceinline__ float2 elem_weight2(float2 xp, float2 xq, float2 p, f
 {
     const float2 one = make_float2(1.0f, 1.0f);
     if (MODE == CIS_MODE_CIS || MODE == CIS_MODE_BAND) {
-        float2 c = __ffma2_rn(p, make_float2(-1.0f, -1.0f), one);  // 1 - p
-        c = make_float2(fmaxf(c.x, P.kappa_f), fmaxf(c.y, P.kappa_f));
-        c = __ffma2_rn(c, make_float2(P.lam_f, P.lam_f), one);     // 1 + lam max(1 - p, kappa)
+        // 1 + lam max(1 - p, kappa) = max((1 + lam) - lam p, 1 + lam kappa) for
+        // lam >= 0: one packed FMA and two maxima per pair
+        float2 c = __ffma2_rn(p, make_float2(-P.lam_f, -P.lam_f),
+                              make_float2(1.0f + P.lam_f, 1.0f + P.lam_f));
+        const float lo = fmaf(P.lam_f, P.kappa_f, 1.0f);
+        c = make_float2(fmaxf(c.x, lo), fmaxf(c.y, lo));
         float2 f = make_float2(fminf(k.x, c.x), fminf(k.y, c.y));
         if (MODE == CIS_MODE_BAND) {  // lower edge (1 + p) / 2
             const float2 lo = __ffma2_rn(p, make_float2(0.5f, 0.5f), make_float2(0.5f, 0.5f));
