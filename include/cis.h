@@ -283,7 +283,7 @@ CIS_API cis_status_t cis_loss_fwd_bwd_host(
 
 /*
  * Bytes of device workspace cis_lmhead_fused needs with its default
- * vocabulary chunk (dz and dz^T of one chunk within about 1 GiB).  Host only.
+ * vocabulary chunk (dz of one chunk within about 1 GiB).  Host only.
  * CIS_ERR_INVALID_ARG if bytes is NULL, T < 0, V <= 0 or H <= 0.
  */
 CIS_API cis_status_t cis_lmhead_workspace_size(int64_t T, int64_t V, int64_t H, size_t *bytes);
@@ -291,7 +291,7 @@ CIS_API cis_status_t cis_lmhead_workspace_size(int64_t T, int64_t V, int64_t H, 
 /*
  * Bytes of device workspace for vocabulary chunks of `chunk` columns (a
  * positive multiple of 256; wider than V rounded up to 256 counts as that).
- * The workspace grows by 4 * ceil(T / 128) * 128 bytes per chunk column.
+ * The workspace grows by 2 * ceil(T / 128) * 128 bytes per chunk column.
  * Host only.  CIS_ERR_INVALID_ARG for a NULL bytes, T < 0, V <= 0, H <= 0 or
  * a chunk that is not a positive multiple of 256.
  */
@@ -306,15 +306,17 @@ CIS_API cis_status_t cis_lmhead_workspace_size_chunk(int64_t T, int64_t V, int64
  *   dhidden = dz W,   dweight = dz^T hidden,   dz = c (softmax - onehot).
  * The forward sweep keeps per-token softmax statistics only; the gradient
  * sweep recomputes z one vocabulary chunk at a time and holds that chunk's dz
- * (bf16, twice: [T, chunk] and [chunk, T]) in the workspace.
+ * (bf16 [ceil(T / 128) * 128, chunk]) in the workspace, read by both
+ * gradient products where it lies.
  *   hidden      device bf16 [T, H], contiguous rows, 16-byte aligned.
  *   weight      device bf16 [V, H], contiguous rows, 16-byte aligned.
  *   H           hidden size; a multiple of 256 (else CIS_ERR_UNSUPPORTED).
  *   ids, lp_infer, lp_old, adv, mask, cu_seqlens, B, params: as for
  *               cis_loss_fwd_bwd.
- *   dhidden     device [T, H] of grad_dtype (CIS_F32 or CIS_BF16), written.
+ *   dhidden     device [T, H] of grad_dtype (CIS_F32 or CIS_BF16), written;
+ *               16-byte aligned (32-byte aligned buffers take the wider stores).
  *   dweight     device [V, H] of grad_dtype, written (rows of tokens that are
- *               masked contribute nothing).
+ *               masked contribute nothing); alignment as for dhidden.
  *   lp_out, w_out, trunc_out, entropy_out, stats_out, loss_out: as for
  *               cis_loss_fwd_bwd (the entropy comes from the forward sweep's
  *               tiles).
