@@ -114,6 +114,16 @@ typedef struct {
     double seq_cap;    /* > 0: C of Seq-TIS                                  */
     double seq_lo;     /* >= 0: Seq-MIS band, bounds included                */
     double seq_hi;     /* >= seq_lo                                          */
+    /* Token-sharded data parallelism (the rows of one batch split across
+     * GPUs at response boundaries): a DEVICE pointer to two int64 values
+     * {N, G}, the batch's number of valid tokens and of responses with a
+     * valid token, i.e. the sum over shards of what cis_count_valid writes.
+     * When set, the loss normaliser uses them (token mean: s_t = 1/N;
+     * sequence mean: s_t = 1/(G |y_i|), each response lying in one shard),
+     * so that the shards' losses add up to the batch loss and each shard's
+     * dlogits are the batch's rows.  NULL (the default): this call's own
+     * counts.  Read on the device by the call's first kernel.              */
+    const int64_t *global_counts;
 } cis_params_t;
 
 /* Reduction outputs of cis_loss_fwd_bwd, written on the device. */
@@ -134,6 +144,21 @@ typedef struct {
 /* Fills *out with the defaults above.  Host only.  CIS_ERR_INVALID_ARG if out
  * is NULL. */
 CIS_API cis_status_t cis_default_params(cis_params_t *out);
+
+/*
+ * This call's share of the loss normaliser, for token-sharded runs: writes
+ * counts_out[0] = N, the number of tokens with mask != 0 (all T when mask is
+ * NULL), and counts_out[1] = G, the number of responses [cu_seqlens[i],
+ * cu_seqlens[i+1]) with at least one valid token (0 when cu_seqlens is
+ * NULL).  Summed over the shards (an all-reduce of the int64 pair) they are
+ * what cis_params_t.global_counts points to.
+ *   mask        device uint8 [T] or NULL;  cu_seqlens device int32 [B + 1] or
+ *               NULL;  counts_out device int64 [2], written.
+ * Asynchronous on `stream`.  CIS_ERR_INVALID_ARG for T < 0, B < 0 or a NULL
+ * counts_out; CIS_ERR_UNSUPPORTED for more than 12000 responses.
+ */
+CIS_API cis_status_t cis_count_valid(const uint8_t *mask, int64_t T, const int32_t *cu_seqlens,
+                                     int64_t B, int64_t *counts_out, void *stream);
 
 /* Human-readable name of a status value (static string, never NULL). */
 CIS_API const char *cis_status_string(int32_t status);

@@ -56,15 +56,21 @@ class OracleParams(ctypes.Structure):
         ("seq_cap", ctypes.c_double),
         ("seq_lo", ctypes.c_double),
         ("seq_hi", ctypes.c_double),
+        ("n_global", ctypes.c_int64),
+        ("g_global", ctypes.c_int64),
     ]
 
 
 def params(mode=MODE_CIS, lam=2.3, kappa=5e-3, tis_cap=2.0, exact_lo=1e-6, exact_hi=1e6,
            clip_low=0.2, clip_high=0.28, agg=AGG_TOKEN_MEAN, icepop_lo=0.5, icepop_hi=5.0,
-           kpop_phi=2.0, seq_cap=2.0, seq_lo=0.5, seq_hi=2.0) -> OracleParams:
-    """Hyper-parameters; defaults are the deployed values of App. C.1 / Table 8."""
+           kpop_phi=2.0, seq_cap=2.0, seq_lo=0.5, seq_hi=2.0, n_global=0,
+           g_global=0) -> OracleParams:
+    """Hyper-parameters; defaults are the deployed values of App. C.1 / Table 8.
+    n_global / g_global (> 0): the batch's valid tokens / responses with a
+    valid token when the rows passed are one shard of that batch."""
     return OracleParams(mode, agg, lam, kappa, tis_cap, exact_lo, exact_hi, clip_low, clip_high,
-                        icepop_lo, icepop_hi, kpop_phi, seq_cap, seq_lo, seq_hi)
+                        icepop_lo, icepop_hi, kpop_phi, seq_cap, seq_lo, seq_hi, n_global,
+                        g_global)
 
 
 def build(force: bool = False) -> str:

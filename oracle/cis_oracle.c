@@ -92,6 +92,10 @@ typedef struct {
     double seq_cap;   /* C of Seq-TIS                                  */
     double seq_lo;    /* Seq-MIS band [a, b]                           */
     double seq_hi;
+    int64_t n_global; /* > 0: the batch's valid tokens, when these rows
+                       * are one shard of it (token mean); 0: these rows' */
+    int64_t g_global; /* > 0: the batch's responses with a valid token
+                       * (sequence mean); 0: these rows'                */
 } oracle_params_t;
 
 static int is_seq_mode(int mode)
@@ -409,9 +413,13 @@ int oracle_weights(const double *lp_w, const double *lp_inf, const uint8_t *mask
  *                             i, |y_i| = valid tokens of i, G = responses with
  *                             at least one valid token.  Tokens outside every
  *                             response get 0.
+ * n and G are counts over the whole batch (Algorithm 1's 1/n, Eq. 1's 1/G):
+ * when these T rows are one shard of a batch, n_global / g_global (> 0) give
+ * the batch's counts; 0 means these rows are the batch.
  */
-void oracle_loss_scales(const uint8_t *mask, int64_t T, const int32_t *cu_seqlens, int64_t B,
-                        int agg, double *s_out)
+void oracle_loss_scales_global(const uint8_t *mask, int64_t T, const int32_t *cu_seqlens,
+                               int64_t B, int agg, int64_t n_global, int64_t g_global,
+                               double *s_out)
 {
     if (agg == OR_AGG_SEQ_MEAN && cu_seqlens != NULL) {
         int64_t G = 0;
@@ -421,6 +429,8 @@ void oracle_loss_scales(const uint8_t *mask, int64_t T, const int32_t *cu_seqlen
                 n += row_valid(mask, t);
             G += n > 0;
         }
+        if (g_global > 0)
+            G = g_global;
         for (int64_t t = 0; t < T; ++t)
             s_out[t] = 0.0;
         for (int64_t i = 0; i < B; ++i) {
@@ -435,8 +445,16 @@ void oracle_loss_scales(const uint8_t *mask, int64_t T, const int32_t *cu_seqlen
     int64_t n = 0;
     for (int64_t t = 0; t < T; ++t)
         n += row_valid(mask, t);
+    if (n_global > 0)
+        n = n_global;
     for (int64_t t = 0; t < T; ++t)
         s_out[t] = (n > 0 && row_valid(mask, t)) ? 1.0 / (double)n : 0.0;
+}
+
+void oracle_loss_scales(const uint8_t *mask, int64_t T, const int32_t *cu_seqlens, int64_t B,
+                        int agg, double *s_out)
+{
+    oracle_loss_scales_global(mask, T, cu_seqlens, B, agg, 0, 0, s_out);
 }
 
 /*
@@ -480,7 +498,7 @@ int oracle_loss_fwd_bwd(const void *logits, int dtype, int64_t T, int64_t V, int
         free(terms);
         return -2;
     }
-    oracle_loss_scales(mask, T, cu_seqlens, B, P->agg, s);
+    oracle_loss_scales_global(mask, T, cu_seqlens, B, P->agg, P->n_global, P->g_global, s);
     double *lpv = (double *)malloc(sizeof(double) * nT);
     double *lwv = (double *)malloc(sizeof(double) * nT);
     double *wv = (double *)malloc(sizeof(double) * nT);

@@ -45,6 +45,7 @@ class cis_params_t(ctypes.Structure):
         ("seq_cap", ctypes.c_double),
         ("seq_lo", ctypes.c_double),
         ("seq_hi", ctypes.c_double),
+        ("global_counts", ctypes.c_void_p),  # device int64 {N, G} of a sharded batch, or NULL
     ]
 
 
@@ -114,6 +115,8 @@ def lib():
     L.cis_mismatch_diagnostics.argtypes = [P, P, i32, i64, i64, i64, i64, P, P,
                                            ctypes.POINTER(cis_params_t), P, P, P, P, P, P, P]
     L.cis_mismatch_diagnostics.restype = ctypes.c_int
+    L.cis_count_valid.argtypes = [P, i64, P, i64, P, P]
+    L.cis_count_valid.restype = ctypes.c_int
     L.cis_selftest_bounded_wait.argtypes = [ctypes.c_uint32, i32, P, P]
     L.cis_selftest_bounded_wait.restype = ctypes.c_int
     L.cis_profile_next_call.argtypes = [P, P]
@@ -178,6 +181,34 @@ def cis_default_params(mode="cis", **kw) -> cis_params_t:
     for k, v in kw.items():
         setattr(p, k, v)
     return p
+
+
+def cis_count_valid(T: int, mask=None, cu_seqlens=None, out=None) -> torch.Tensor:
+    """This shard's {N, G} as a device int64 [2] tensor: valid tokens, and
+    responses with a valid token (what a token-sharded run all-reduces)."""
+    _need_cuda(mask, cu_seqlens)
+    _vec(mask, torch.uint8, T, "mask")
+    B = 0 if cu_seqlens is None else cu_seqlens.shape[0] - 1
+    if out is None:
+        dev = mask.device if mask is not None else (
+            cu_seqlens.device if cu_seqlens is not None else torch.device("cuda"))
+        out = torch.empty(2, dtype=torch.int64, device=dev)
+    _need_cuda(out)
+    _check(lib().cis_count_valid(_ptr(mask), T, _ptr(cu_seqlens), B, _ptr(out), _stream()),
+           "cis_count_valid")
+    return out
+
+
+def with_global_counts(params: cis_params_t, counts: torch.Tensor) -> cis_params_t:
+    """A copy of params whose normaliser uses the batch-wide {N, G} in
+    `counts` (device int64 [2], kept alive by the caller until the call's
+    kernels have run)."""
+    _need_cuda(counts)
+    if counts.dtype != torch.int64 or counts.numel() != 2 or not counts.is_contiguous():
+        raise ValueError("counts must be a contiguous device int64 tensor of 2 elements")
+    q = cis_params_t.from_buffer_copy(params)
+    q.global_counts = counts.data_ptr()
+    return q
 
 
 def cis_token_logprobs(logits: torch.Tensor, ids: torch.Tensor, mask=None, V=None,

@@ -147,7 +147,19 @@ CIS_API cis_status_t cis_default_params(cis_params_t *out)
     out->seq_cap = 2.0;
     out->seq_lo = 0.5;
     out->seq_hi = 2.0;
+    out->global_counts = nullptr;
     return CIS_OK;
+}
+
+CIS_API cis_status_t cis_count_valid(const uint8_t *mask, int64_t T, const int32_t *cu_seqlens,
+                                     int64_t B, int64_t *counts_out, void *stream)
+{
+    if (T < 0 || B < 0 || counts_out == nullptr || (cu_seqlens == nullptr && B > 0))
+        return CIS_ERR_INVALID_ARG;
+    const cudaError_t e = launch_count_valid(mask, T, cu_seqlens, B, counts_out,
+                                             (cudaStream_t)stream);
+    return e == cudaSuccess ? CIS_OK
+                            : (e == cudaErrorNotSupported ? CIS_ERR_UNSUPPORTED : CIS_ERR_CUDA);
 }
 
 CIS_API const char *cis_status_string(int32_t status)
@@ -283,7 +295,8 @@ CIS_API cis_status_t cis_loss_fwd_bwd(const void *logits, int32_t dtype, int64_t
     a.P = make_dev_params(*params);
 
     cudaError_t e = launch_scales(mask, T, cu_seqlens, B, params->agg,
-                                  reinterpret_cast<float *>(ws + L.scale), a.status, s);
+                                  reinterpret_cast<float *>(ws + L.scale), a.status, s,
+                                  params->global_counts);
     if (e != cudaSuccess)
         return cuda_status(e);
     if (T > 0 && is_seq_mode(params->mode)) {

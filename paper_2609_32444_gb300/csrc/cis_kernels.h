@@ -74,8 +74,11 @@ cudaError_t launch_cluster_fwd_bwd(const PassArgs &a, int dtype, int out_dtype,
 bool cluster_path_applies(const PassArgs &a, int dtype, int out_dtype);
 
 // Loss scales s_t (and clears the status word).
+cudaError_t launch_count_valid(const uint8_t *mask, int64_t T, const int32_t *cu_seqlens,
+                               int64_t B, int64_t *counts, cudaStream_t s);
 cudaError_t launch_scales(const uint8_t *mask, int64_t T, const int32_t *cu_seqlens, int64_t B,
-                          int agg, float *scale, int32_t *status, cudaStream_t s);
+                          int agg, float *scale, int32_t *status, cudaStream_t s,
+                          const int64_t *global_counts = nullptr);
 
 // Elementwise weights (cis_weights).
 cudaError_t launch_weights(const float *lp_w, const float *lp_inf, const uint8_t *mask,

@@ -30,9 +30,11 @@ __device__ __forceinline__ T warp_sum(T v)
     return v;
 }
 
+// The loss normaliser.  global_counts (device {N, G}, or null): the batch's
+// counts over every shard, used in place of this call's own.
 __global__ void __launch_bounds__(kSmallThreads)
     cis_scales_kernel(const uint8_t *mask, int64_t T, const int32_t *cu, int64_t B, int agg,
-                  float *scale, int32_t *status)
+                  float *scale, int32_t *status, const int64_t *global_counts)
 {
     __shared__ long long part[kSmallThreads / 32];
     __shared__ int cnt[kMaxSeqInShared];
@@ -65,6 +67,8 @@ __global__ void __launch_bounds__(kSmallThreads)
         long long G = 0;
         for (int i = 0; i < kSmallThreads / 32; ++i)
             G += part[i];
+        if (global_counts)
+            G = global_counts[1];
         for (int64_t i = wid; i < B; i += kSmallThreads / 32) {
             int64_t lo = cu[i], hi = cu[i + 1];
             lo = lo < 0 ? 0 : (lo > T ? T : lo);
@@ -86,9 +90,53 @@ __global__ void __launch_bounds__(kSmallThreads)
     long long N = 0;
     for (int i = 0; i < kSmallThreads / 32; ++i)
         N += part[i];
+    if (global_counts)
+        N = global_counts[0];
     const float s = N > 0 ? (float)(1.0 / (double)N) : 0.0f;
     for (int64_t t = threadIdx.x; t < T; t += kSmallThreads)
         scale[t] = is_valid(mask, t) ? s : 0.0f;
+}
+
+// This call's {N, G}: valid tokens, and responses with a valid token (one
+// warp per response), for the all-reduce of a token-sharded run.
+__global__ void __launch_bounds__(kSmallThreads)
+    cis_count_kernel(const uint8_t *mask, int64_t T, const int32_t *cu, int64_t B,
+                     int64_t *counts)
+{
+    __shared__ long long part[2][kSmallThreads / 32];
+    const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+    long long n = 0, g = 0;
+    for (int64_t t = threadIdx.x; t < T; t += kSmallThreads)
+        n += is_valid(mask, t);
+    if (cu != nullptr) {
+        for (int64_t i = wid; i < B; i += kSmallThreads / 32) {
+            int64_t lo = cu[i], hi = cu[i + 1];
+            lo = lo < 0 ? 0 : (lo > T ? T : lo);
+            hi = hi < lo ? lo : (hi > T ? T : hi);
+            int c = 0;
+            for (int64_t t = lo + lane; t < hi; t += 32)
+                c += is_valid(mask, t);
+            c = warp_sum(c);
+            if (lane == 0)
+                g += c > 0;
+        }
+    }
+    n = warp_sum(n);
+    g = warp_sum(g);
+    if (lane == 0) {
+        part[0][wid] = n;
+        part[1][wid] = g;
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        long long N = 0, G = 0;
+        for (int i = 0; i < kSmallThreads / 32; ++i) {
+            N += part[0][i];
+            G += part[1][i];
+        }
+        counts[0] = N;
+        counts[1] = G;
+    }
 }
 
 __global__ void cis_weights_kernel(const float *lp_w, const float *lp_inf, const uint8_t *mask,
@@ -238,11 +286,22 @@ __global__ void __launch_bounds__(kSmallThreads)
 }  // namespace
 
 cudaError_t launch_scales(const uint8_t *mask, int64_t T, const int32_t *cu_seqlens, int64_t B,
-                          int agg, float *scale, int32_t *status, cudaStream_t s)
+                          int agg, float *scale, int32_t *status, cudaStream_t s,
+                          const int64_t *global_counts)
 {
     if (agg == CIS_AGG_SEQ_MEAN_TOKEN_MEAN && B > kMaxSeqInShared)
         return cudaErrorNotSupported;
-    cis_scales_kernel<<<1, kSmallThreads, 0, s>>>(mask, T, cu_seqlens, B, agg, scale, status);
+    cis_scales_kernel<<<1, kSmallThreads, 0, s>>>(mask, T, cu_seqlens, B, agg, scale, status,
+                                                  global_counts);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_count_valid(const uint8_t *mask, int64_t T, const int32_t *cu_seqlens,
+                               int64_t B, int64_t *counts, cudaStream_t s)
+{
+    if (B > kMaxSeqInShared)
+        return cudaErrorNotSupported;
+    cis_count_kernel<<<1, kSmallThreads, 0, s>>>(mask, T, cu_seqlens, B, counts);
     return cudaGetLastError();
 }
 
