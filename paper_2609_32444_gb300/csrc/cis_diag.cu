@@ -405,7 +405,11 @@ __device__ __forceinline__ void pass1_update(uint4 w, float &m, float &cm, float
     const float lm = max_nan(__low2float(a), __high2float(a));
     if (lm > m || lm != lm) {
         const float ncm = lm * kLog2e;
-        const float f = ex2_ftz(cm - ncm);
+        // cm - ncm < 0 once m is finite (the maximum only rises); while the
+        // sum is still empty (m = -inf, cm = 0) a very negative first maximum
+        // would make 2^{0 - ncm} overflow and 0 x inf = NaN: the clamp keeps
+        // the factor finite there (and changes nothing otherwise)
+        const float f = ex2_ftz(fminf(cm - ncm, 0.0f));
         s = __fmul2_rn(s, make_float2(f, f));
         m = lm;
         cm = ncm;

@@ -212,6 +212,62 @@ def test_diagnostics_all_other_entries_neg_inf(monkeypatch):
     _compare(out, ref)
 
 
+@pytest.mark.parametrize("kernel", ["stream", "row"])
+def test_diagnostics_huge_magnitude_logits(kernel, monkeypatch):
+    """Rows at near-zero temperature: logits of magnitude ~1e4 in bf16, so a
+    thread's first groups can all lie thousands below zero (a running sum
+    started there must stay 0, not 0 x inf), with ties at the top and the
+    sampled token among them in some rows."""
+    if kernel == "row":
+        monkeypatch.setenv("CIS_DIAG_KERNEL", "row")
+    monkeypatch.setenv("CIS_DIAG_SLOT_GROUPS", "64")
+    V, T = 4096, 12
+    g = torch.Generator().manual_seed(21)
+    z = (torch.randn((T, V), generator=g) * 4e3).to(torch.bfloat16)
+    ids = torch.randint(0, V, (T,), generator=g).int()
+    top = z.float().argmax(dim=1)
+    for t in range(0, T, 2):  # a tie at the top, y one of the two
+        z[t, (top[t] + 1) % V] = z[t, top[t]]
+        ids[t] = top[t]
+    zi = z.clone()
+    zi[1::2] = (z[1::2].float() + torch.randn((T // 2, V), generator=g) * 300.0).to(torch.bfloat16)
+    out = binding.cis_mismatch_diagnostics(z.to(DEV), zi.to(DEV), ids.to(DEV),
+                                           binding.cis_default_params("cis"))
+    torch.cuda.synchronize()
+    ref = oracle.mismatch_diagnostics(logits_for_oracle(z), logits_for_oracle(zi), ids.numpy(),
+                                      oracle.params(mode=oracle.MODE_CIS))
+    for k in out:
+        assert not torch.isnan(out[k]).any(), k
+    # rows with p = 1 exactly have an infinite (kernel) or undefined (oracle) eps
+    fin = np.isfinite(ref["eps"])
+    sel = torch.from_numpy(fin).to(DEV)
+    _compare({k: v[sel] for k, v in out.items()}, {k: v[fin] for k, v in ref.items()})
+
+
+def test_diagnostics_full_vocabulary_low_temperature_rows():
+    """Rows 12040, 13614, 14810 and 15007 of workload 6 as generated on the
+    GPU (V=151936): near-zero temperature, a tie or a single token at the top
+    (p = 0.5 or ~1) and logits far below it.  A pass-1 running sum started on
+    a group thousands below zero once overflowed its rescale (0 x inf = NaN)
+    here; the outputs must be finite (eps may be infinite) and match fp64
+    closed forms, as in the closed-form test above."""
+    b = synth.make_batch(6, device=DEV, T=16384)
+    rows = torch.tensor([12040, 13614, 14810, 15007], device=DEV)
+    z, zi = b.logits[rows].contiguous(), b.extra["logits_infer"][rows].contiguous()
+    ids = b.ids[rows].contiguous()
+    none = binding.cis_mismatch_diagnostics(z, zi, ids, binding.cis_default_params("none"))
+    torch.cuda.synchronize()
+    for k in none:
+        assert torch.isfinite(none[k]).all() or k == "eps", (k, none[k])
+    Pd = torch.softmax(z.double(), dim=1)
+    Qd = torch.softmax(zi.double(), dim=1)
+    p = Pd[torch.arange(4), ids.long()]
+    assert torch.all((none["p"].double() - p).abs() <= 1e-5 * p + 1e-30)
+    b2 = ((Qd - Pd) ** 2).sum(dim=1)
+    assert torch.all((none["bias2"].double() - b2).abs() <= 1e-3 * b2 + 2e-5)
+    assert torch.all(none["dvar"].double().abs() <= 2e-5)
+
+
 @pytest.mark.parametrize("dtype,V", [(torch.float32, 64), (torch.bfloat16, 2056)])
 def test_diagnostics_bad_id_and_status(dtype, V, monkeypatch):
     monkeypatch.setenv("CIS_DIAG_SLOT_GROUPS", "64")
