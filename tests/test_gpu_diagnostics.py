@@ -268,6 +268,22 @@ def test_diagnostics_full_vocabulary_low_temperature_rows():
     assert torch.all(none["dvar"].double().abs() <= 2e-5)
 
 
+def test_diagnostics_full_workload_every_row():
+    """The benchmarked workload (T=16384, V=151936, GPU-generated): on every
+    row p in (0, 1], bias2 >= 0 and finite, dvar finite, and eps NaN-free
+    except where p = 1 (the closed-form and oracle tests fix the values)."""
+    b = synth.make_batch(6, device=DEV)
+    for mode in ("cis", "exact"):
+        out = binding.cis_mismatch_diagnostics(b.logits, b.extra["logits_infer"], b.ids,
+                                               binding.cis_default_params(mode))
+        torch.cuda.synchronize()
+        p = out["p"]
+        assert torch.all((p > 0) & (p <= 1)), mode
+        assert torch.isfinite(out["bias2"]).all() and torch.all(out["bias2"] >= -1e-6), mode
+        assert torch.isfinite(out["dvar"]).all() and torch.isfinite(out["logk"]).all(), mode
+        assert not torch.isnan(out["eps"][p < 1]).any(), mode
+
+
 @pytest.mark.parametrize("dtype,V", [(torch.float32, 64), (torch.bfloat16, 2056)])
 def test_diagnostics_bad_id_and_status(dtype, V, monkeypatch):
     monkeypatch.setenv("CIS_DIAG_SLOT_GROUPS", "64")

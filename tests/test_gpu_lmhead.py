@@ -208,6 +208,7 @@ def test_lmhead_full_size_sampled_tokens():
     # bf16 (2^-9) and fp32 accumulation over T tokens the sum is bounded by
     # sum_t |H[t, k]| sum_v |dz[t, v]| (2^-9 + T 2^-24), where
     # sum_v |dz[t, v]| = 2 |c_t| (1 - p_t) and c_t = w_t A_t / n (no l_old).
+    assert torch.isfinite(out["dhidden"]).all() and torch.isfinite(out["dweight"]).all()
     dw = out["dweight"].double()
     colsum = dw.sum(dim=0).abs()
     n = float(b.mask.sum())

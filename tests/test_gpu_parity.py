@@ -441,6 +441,13 @@ def _full_size_check(cfg, mode, dz_dtype, n_sample_rows=48):
     check_dz(out["dlogits"][torch.from_numpy(rows).to(DEV)], ref["dz"], ref["c"][rows])
     if nvalid < b.T:
         assert torch.count_nonzero(out["dlogits"][nvalid:]).item() == 0
+    # every valid row: finite, and sum_j dz_tj = c (sum_j softmax_j - 1) = 0 up
+    # to the bf16 rounding of each element (2^-9 relative, so 2^-8 of the
+    # row's L1 norm bounds the sum)
+    for r0 in range(0, nvalid, 2048):
+        dz = out["dlogits"][r0:min(nvalid, r0 + 2048)].float()
+        assert torch.isfinite(dz).all()
+        assert torch.all(dz.sum(dim=1).abs() <= 2.0 ** -8 * dz.abs().sum(dim=1) + 1e-30)
     st = binding.decode_stats(out["stats"])
     assert st["n_valid"] == nvalid and st["status"] == 0
     return n_band
