@@ -18,6 +18,7 @@ WsLayout ws_layout(int64_t T)
     WsLayout L;
     size_t o = 0;
     L.status = o;
+    L.ticket = o + 64;
     o += 256;
     L.scale = o;
     o = up(o + 4 * n);
@@ -29,6 +30,8 @@ WsLayout ws_layout(int64_t T)
     o = up(o + 4 * n);
     L.trunc = o;
     o = up(o + n);
+    L.parts = o;
+    o = up(o + (size_t)kRedPartBytes * ((n + kRedTokens - 1) / kRedTokens + (n == 0)));
     L.total = o;
     return L;
 }
@@ -294,9 +297,11 @@ CIS_API cis_status_t cis_loss_fwd_bwd(const void *logits, int32_t dtype, int64_t
     a.status = reinterpret_cast<int32_t *>(ws + L.status);
     a.P = make_dev_params(*params);
 
+    a.red_parts = ws + L.parts;
+    a.red_ticket = reinterpret_cast<uint32_t *>(ws + L.ticket);
     cudaError_t e = launch_scales(mask, T, cu_seqlens, B, params->agg,
-                                  reinterpret_cast<float *>(ws + L.scale), a.status, s,
-                                  params->global_counts);
+                                  reinterpret_cast<float *>(ws + L.scale), a.status,
+                                  a.red_ticket, s, params->global_counts);
     if (e != cudaSuccess)
         return cuda_status(e);
     if (T > 0 && is_seq_mode(params->mode)) {

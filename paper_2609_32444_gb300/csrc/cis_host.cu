@@ -185,7 +185,9 @@ CIS_API cis_status_t cis_loss_fwd_bwd_host(
     a.status = reinterpret_cast<int32_t *>(dptr(L.base.status));
     a.P = make_dev_params(*params);
     const int32_t *cu_dev = cu_seqlens ? reinterpret_cast<const int32_t *>(dptr(L.cu)) : nullptr;
-    CIS_TRY(launch_scales(a.mask, T, cu_dev, B, params->agg, scale, a.status, sc,
+    a.red_parts = dptr(L.base.parts);
+    a.red_ticket = reinterpret_cast<uint32_t *>(dptr(L.base.ticket));
+    CIS_TRY(launch_scales(a.mask, T, cu_dev, B, params->agg, scale, a.status, a.red_ticket, sc,
                           params->global_counts));
     if (T > 0 && is_seq_mode(params->mode)) {
         // the responses' weights from lp_old, read by every chunk's pass

@@ -37,6 +37,8 @@ struct PassArgs {
     const uint8_t *trunc_in;
     double *lp64_out;      // forward-only kernel: log p in fp64 (may be null)
     float *entropy_out;    // per-token entropy of the softmax (may be null)
+    void *red_parts;       // the reduction's per-CTA partial sums (workspace)
+    uint32_t *red_ticket;  // its completion counter (zeroed by the scales kernel)
 };
 
 // Host-side parameter checks and the kernels' copy of the parameters.
@@ -44,9 +46,13 @@ bool params_ok(const cis_params_t *p);
 DevParams make_dev_params(const cis_params_t &p);
 
 // Workspace layout (offsets in bytes from the 256-byte aligned base).
+// status: a 256-byte block (the status word at 0, the reduction's ticket at
+// 64); parts: one 64-byte partial sum per 256 tokens.
 struct WsLayout {
-    size_t status, scale, terms, logk, w, trunc, total;
+    size_t status, ticket, scale, terms, logk, w, trunc, parts, total;
 };
+constexpr int kRedTokens = 256;  // tokens per CTA of the reduction
+constexpr int kRedPartBytes = 64;
 WsLayout ws_layout(int64_t T);
 
 // Sequence operators: w[t], trunc[t] for the valid tokens of each response
@@ -77,8 +83,8 @@ bool cluster_path_applies(const PassArgs &a, int dtype, int out_dtype);
 cudaError_t launch_count_valid(const uint8_t *mask, int64_t T, const int32_t *cu_seqlens,
                                int64_t B, int64_t *counts, cudaStream_t s);
 cudaError_t launch_scales(const uint8_t *mask, int64_t T, const int32_t *cu_seqlens, int64_t B,
-                          int agg, float *scale, int32_t *status, cudaStream_t s,
-                          const int64_t *global_counts = nullptr);
+                          int agg, float *scale, int32_t *status, uint32_t *ticket,
+                          cudaStream_t s, const int64_t *global_counts = nullptr);
 
 // Elementwise weights (cis_weights).
 cudaError_t launch_weights(const float *lp_w, const float *lp_inf, const uint8_t *mask,

@@ -789,8 +789,10 @@ CIS_API cis_status_t cis_lmhead_fused(const void *hidden, const void *weight, in
                                           : reinterpret_cast<float *>(ws + L.dh);
 
     float *scale = reinterpret_cast<float *>(ws + L.base.scale);
-    cudaError_t e =
-        launch_scales(mask, T, cu_seqlens, B, P.agg, scale, a.status, s, P.global_counts);
+    a.red_parts = ws + L.base.parts;
+    a.red_ticket = reinterpret_cast<uint32_t *>(ws + L.base.ticket);
+    cudaError_t e = launch_scales(mask, T, cu_seqlens, B, P.agg, scale, a.status, a.red_ticket, s,
+                                  P.global_counts);
     if (e != cudaSuccess)
         return e == cudaErrorNotSupported ? CIS_ERR_UNSUPPORTED : CIS_ERR_CUDA;
     if (T > 0) {

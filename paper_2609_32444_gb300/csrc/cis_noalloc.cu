@@ -24,9 +24,11 @@ constexpr int64_t kMaxTokens = CIS_NOALLOC_MAX_TOKENS;
 
 // Bytes ws_layout() asks for at kMaxTokens: a 256-byte status block, then the
 // scale (4 B), term (8 B), log k (4 B), weight (4 B) and flag (1 B) arrays,
-// each rounded up to 256 bytes.
+// each rounded up to 256 bytes, and the reduction's partial sums (64 B per
+// 256 tokens).
 constexpr size_t kScratchBytes = 256 + 4 * kMaxTokens + 8 * kMaxTokens + 4 * kMaxTokens +
-                                 4 * kMaxTokens + 1 * kMaxTokens;
+                                 4 * kMaxTokens + 1 * kMaxTokens +
+                                 kRedPartBytes * ((kMaxTokens + kRedTokens - 1) / kRedTokens);
 
 // The scratch itself.  In host code this name is only a host-side stand-in:
 // its device address is looked up per device with cudaGetSymbolAddress.

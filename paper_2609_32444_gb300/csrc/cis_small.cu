@@ -4,7 +4,8 @@
 //                   (Algorithm 1) or 1/(G |y_i|) per response (Eq. 1); it
 //                   also clears the device status word of the call.
 //   cis_weights_kernel  cis_weights: Algorithm 1 / Table 8, one thread per token.
-//   cis_reduce_kernel   deterministic sums of the per-token loss terms and the
+//   cis_reduce_kernel   deterministic sums (one CTA per 256 tokens, then the
+//                   last CTA in index order) of the per-token loss terms and the
 //                   statistics the paper logs (App. D.1: share of tokens acted
 //                   on, largest |log k|; App. D.5: the truncated excess).
 #include "cis_kernels.h"
@@ -34,13 +35,15 @@ __device__ __forceinline__ T warp_sum(T v)
 // counts over every shard, used in place of this call's own.
 __global__ void __launch_bounds__(kSmallThreads)
     cis_scales_kernel(const uint8_t *mask, int64_t T, const int32_t *cu, int64_t B, int agg,
-                  float *scale, int32_t *status, const int64_t *global_counts)
+                  float *scale, int32_t *status, uint32_t *ticket, const int64_t *global_counts)
 {
     __shared__ long long part[kSmallThreads / 32];
     __shared__ int cnt[kMaxSeqInShared];
     const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
     if (threadIdx.x == 0 && status)
         *status = 0;
+    if (threadIdx.x == 0 && ticket)  // the reduction at the end of this call counts from 0
+        *ticket = 0;
     if (agg == CIS_AGG_SEQ_MEAN_TOKEN_MEAN && cu != nullptr) {
         // valid tokens of each response (one warp per response)
         for (int64_t i = wid; i < B; i += kSmallThreads / 32) {
@@ -237,48 +240,88 @@ __device__ __forceinline__ RedPart red_warp(RedPart v)
     return v;
 }
 
-// One CTA: thread i sums tokens i, i + 1024, ... in order, then a fixed tree
-// (within each warp, then over the 32 warps), so the sums are deterministic.
-__global__ void __launch_bounds__(kSmallThreads)
-    cis_reduce_kernel(const uint8_t *mask, int64_t T, const double *terms, const float *logk,
-                  const float *w, const uint8_t *trunc, const float *entropy,
-                  const int32_t *status, cis_stats_t *stats, double *loss_out)
+// Sums over the tokens in fp64, deterministic and spread over many SMs (fp64
+// arithmetic runs at a small fraction of the fp32 rate here, so one CTA
+// summing every token was bound by its SM's fp64 pipe).  CTA b takes tokens
+// [256 b, 256 b + 256), one per thread, and reduces them in a fixed tree
+// (within each warp, then over the warps in order) into parts[b]; the last
+// CTA to finish (a ticket, zeroed by the scales kernel at the start of the
+// call) adds the parts in index order the same way and writes the results.
+__device__ __forceinline__ RedPart block_red(RedPart p, RedPart *sh)
 {
-    __shared__ RedPart sh[kSmallThreads / 32];
-    RedPart p{0.0, 0.0, 0.0, 0, 0, 0.0f};
-    for (int64_t t = threadIdx.x; t < T; t += kSmallThreads) {
-        p.loss += terms[t];
-        if (!is_valid(mask, t))
-            continue;
-        p.nvalid += 1;
-        const float lk = logk[t];
-        p.maxlk = fmaxf(p.maxlk, fabsf(lk));
-        if (trunc[t]) {
-            p.ntrunc += 1;
-            p.excess += exp((double)lk) - (double)w[t];
-        }
-        if (entropy)
-            p.ent += (double)entropy[t];
-    }
+    constexpr int kWarps = kRedTokens / 32;
     p = red_warp(p);
     const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
     if (lane == 0)
         sh[wid] = p;
     __syncthreads();
+    RedPart r{0.0, 0.0, 0.0, 0, 0, 0.0f};
     if (wid == 0) {
-        p = red_warp(sh[lane]);
-        if (lane == 0) {
-            if (loss_out)
-                *loss_out = p.loss;
-            if (stats) {
-                stats->loss = p.loss;
-                stats->trunc_excess = p.excess;
-                stats->n_valid = p.nvalid;
-                stats->n_truncated = p.ntrunc;
-                stats->max_abs_logk = p.maxlk;
-                stats->status = status ? *status : 0;
-                stats->entropy_sum = p.ent;
+        r = lane < kWarps ? sh[lane] : r;
+        r = red_warp(r);
+    }
+    __syncthreads();
+    return r;  // valid in thread 0
+}
+
+__global__ void __launch_bounds__(kRedTokens)
+    cis_reduce_kernel(const uint8_t *mask, int64_t T, const double *terms, const float *logk,
+                  const float *w, const uint8_t *trunc, const float *entropy,
+                  const int32_t *status, RedPart *parts, uint32_t *ticket, cis_stats_t *stats,
+                  double *loss_out)
+{
+    __shared__ RedPart sh[kRedTokens / 32];
+    __shared__ bool last;
+    RedPart p{0.0, 0.0, 0.0, 0, 0, 0.0f};
+    const int64_t t = (int64_t)blockIdx.x * kRedTokens + threadIdx.x;
+    if (t < T) {
+        p.loss = terms[t];
+        if (is_valid(mask, t)) {
+            p.nvalid = 1;
+            const float lk = logk[t];
+            p.maxlk = fabsf(lk);
+            if (trunc[t]) {
+                p.ntrunc = 1;
+                p.excess = exp((double)lk) - (double)w[t];
             }
+            if (entropy)
+                p.ent = (double)entropy[t];
+        }
+    }
+    p = block_red(p, sh);
+    if (threadIdx.x == 0) {
+        parts[blockIdx.x] = p;
+        __threadfence();
+        last = atomicAdd(ticket, 1u) == gridDim.x - 1;
+    }
+    __syncthreads();
+    if (!last)
+        return;
+    __threadfence();
+    const volatile RedPart *vp = parts;
+    RedPart q{0.0, 0.0, 0.0, 0, 0, 0.0f};
+    for (unsigned b = threadIdx.x; b < gridDim.x; b += kRedTokens) {
+        RedPart x;
+        x.loss = vp[b].loss;
+        x.excess = vp[b].excess;
+        x.ent = vp[b].ent;
+        x.nvalid = vp[b].nvalid;
+        x.ntrunc = vp[b].ntrunc;
+        x.maxlk = vp[b].maxlk;
+        q = red_add(q, x);
+    }
+    q = block_red(q, sh);
+    if (threadIdx.x == 0) {
+        if (loss_out)
+            *loss_out = q.loss;
+        if (stats) {
+            stats->loss = q.loss;
+            stats->trunc_excess = q.excess;
+            stats->n_valid = q.nvalid;
+            stats->n_truncated = q.ntrunc;
+            stats->max_abs_logk = q.maxlk;
+            stats->status = status ? *status : 0;
+            stats->entropy_sum = q.ent;
         }
     }
 }
@@ -286,13 +329,13 @@ __global__ void __launch_bounds__(kSmallThreads)
 }  // namespace
 
 cudaError_t launch_scales(const uint8_t *mask, int64_t T, const int32_t *cu_seqlens, int64_t B,
-                          int agg, float *scale, int32_t *status, cudaStream_t s,
-                          const int64_t *global_counts)
+                          int agg, float *scale, int32_t *status, uint32_t *ticket,
+                          cudaStream_t s, const int64_t *global_counts)
 {
     if (agg == CIS_AGG_SEQ_MEAN_TOKEN_MEAN && B > kMaxSeqInShared)
         return cudaErrorNotSupported;
     cis_scales_kernel<<<1, kSmallThreads, 0, s>>>(mask, T, cu_seqlens, B, agg, scale, status,
-                                                  global_counts);
+                                                  ticket, global_counts);
     return cudaGetLastError();
 }
 
@@ -321,8 +364,13 @@ cudaError_t launch_weights(const float *lp_w, const float *lp_inf, const uint8_t
 
 cudaError_t launch_reduce(const PassArgs &a, cis_stats_t *stats, double *loss, cudaStream_t s)
 {
-    cis_reduce_kernel<<<1, kSmallThreads, 0, s>>>(a.mask, a.T, a.ws_terms, a.ws_logk, a.ws_w,
-                                               a.ws_trunc, a.entropy_out, a.status, stats, loss);
+    if (a.red_parts == nullptr || a.red_ticket == nullptr)
+        return cudaErrorInvalidValue;
+    static_assert(sizeof(RedPart) <= kRedPartBytes, "a partial sum must fit its slot");
+    const int64_t blocks = a.T > 0 ? (a.T + kRedTokens - 1) / kRedTokens : 1;
+    cis_reduce_kernel<<<(unsigned)blocks, kRedTokens, 0, s>>>(
+        a.mask, a.T, a.ws_terms, a.ws_logk, a.ws_w, a.ws_trunc, a.entropy_out, a.status,
+        static_cast<RedPart *>(a.red_parts), a.red_ticket, stats, loss);
     return cudaGetLastError();
 }
 
