@@ -415,8 +415,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                     // 64 bytes of the row in two full-sector stores (read back by
                     // the next two launches, DH and DW)
                     uint16_t *drow = g.dz + (int64_t)row * g.ld_dz + cl0 + c0;
-                    st_v8(drow, w);
-                    st_v8(drow + 16, w + 8);
+                    st_v8_cs(drow, w);
+                    st_v8_cs(drow + 16, w + 8);
                 }
             } else {
                 const int lr = m * kBM + r;  // row of the output block
