@@ -33,7 +33,9 @@
 // roles: warp 0 issues TMA loads, warp 1 issues tcgen05.mma (one thread) and
 // owns TMEM, warps 2..9 are the epilogue: two warps per TMEM lane quadrant
 // (one tile row per thread), each taking one 128-column half of the tile, so
-// that a tile's epilogue fits in the next tile's main loop.  All waits are bounded: a wait that runs out sets
+// that a tile's epilogue fits in the next tile's main loop.  Epilogue stores
+// are 32 bytes per thread (one whole sector of its row) where the output is
+// 32-byte aligned.  All waits are bounded: a wait that runs out sets
 // CIS_ERR_DEVICE_TIMEOUT, and the CTA drains its own loads and MMAs and runs
 // to its end, so that TMEM is always released.
 #include <cuda.h>
