@@ -39,6 +39,17 @@
  *   - T == 0 is a valid no-op (loss 0).
  *   - Non-finite logits: -inf is allowed anywhere except at the sampled
  *     token; NaN propagates into that row's outputs.
+ *   - Environment variables exist for tuning sweeps and tests only.  The
+ *     defaults are the measured best.  Other settings change summation
+ *     orders, never the tolerances.
+ *       CIS_SLICE_KB (8..200, default 80), CIS_CLUSTER (1..8) and
+ *       CIS_CLUSTER_THREADS (128, 256, 384 or 512; default 256) set the
+ *       fused pass's slice target, cluster size and CTA width.  They are read
+ *       once per process.
+ *       CIS_DIAG_WARPS (16 or 24; default 16) and CIS_DIAG_SLOT_GROUPS (>= 1)
+ *       set the diagnostics kernel's width and ring-slot size, and
+ *       CIS_DIAG_KERNEL=row selects its one-CTA kernel.  They are read at
+ *       each call.
  */
 #ifndef CIS_H
 #define CIS_H
