@@ -60,14 +60,14 @@ template <bool kEnt> struct ClusterShared {
     alignas(8) uint64_t xbar;          // arrival of the cluster's (m, s) pairs
     float2 part[kMaxCluster];
     MaxSum red[512 / 32];
-    float c, cs, B, lp;
+    float c, cs, B, dzy;
 };
 template <> struct ClusterShared<true> {
     alignas(8) uint64_t bar[kChunks];
     alignas(8) uint64_t xbar;          // arrival of the cluster's (m, s, u) triples
     float4 part[kMaxCluster];
     MaxSumU red[512 / 32];
-    float c, cs, B, lp;
+    float c, cs, B, dzy;
 };
 
 template <typename InT, typename OutT, int kThreads, bool kEnt>
@@ -214,38 +214,35 @@ __global__ void __launch_bounds__(kThreads) cis_fused_cluster_kernel(const PassA
     // for the others' word only at exit (so no CTA leaves while stores into
     // its shared memory may be in flight).
     cluster_arrive_relaxed();
-    MaxSum o{sh.part[0].x, sh.part[0].y};
-    MaxSumU ou{0.0f, 0.0f, 0.0f};
-    if constexpr (kEnt) {
-        ou = MaxSumU{sh.part[0].x, sh.part[0].y, sh.part[0].z};
-        for (unsigned r = 1; r < cs; ++r)
-            ou = msu_combine(ou, MaxSumU{sh.part[r].x, sh.part[r].y, sh.part[r].z});
-        o = MaxSum{ou.m, ou.s};
-    } else {
-        for (unsigned r = 1; r < cs; ++r)
-            o = ms_combine(o, MaxSum{sh.part[r].x, sh.part[r].y});
-    }
 
+    // Thread 0 forms the row's scalars: the serial part of every row, which
+    // the other threads wait for.  It combines the cluster's pairs (one
+    // rescaling step), and everything pass 2 does not need (the per-token
+    // outputs, the fp64 loss term, the entropy) is stored after the barrier,
+    // by rank 0 only.
+    MaxSumU ou{0.0f, 0.0f, 0.0f};
+    TokenWeight tw{0.0f, 0.0f, 0};
+    double term = 0.0;
+    float lp = 0.0f;
     if (threadIdx.x == 0) {
+        MaxSum o;
+        if constexpr (kEnt) {
+            ou = combine_flat(sh.part, cs);
+            o = MaxSum{ou.m, ou.s};
+        } else {
+            o = combine_flat(sh.part, cs);
+        }
         const RowScalars rs = row_scalars(o, zy);
-        if (kEnt && rank == 0)
-            a.entropy_out[t] = row_entropy(ou, zy, rs.lp);
         const bool has_old = a.lp_old != nullptr;
-        TokenWeight tw = token_weight(has_old ? (double)lold : rs.lp64, linf, a.P);
+        tw = token_weight(has_old ? lold : rs.lp, has_old ? 0.0f : rs.lp_lo, linf, a.P,
+                          has_old ? -1.0f : rs.omp);
         if (a.w_in) {  // a sequence operator: the response's weight
             tw.w = a.w_in[t];
             tw.trunc = a.trunc_in[t];
         }
-        const TokenLoss tl = token_loss(rs.lp64, has_old, lold, adv, sc, tw.w, a.P);
-        if (rank == 0) {
-            if (a.lp_out) a.lp_out[t] = rs.lp;
-            if (a.w_out) a.w_out[t] = tw.w;
-            if (a.trunc_out) a.trunc_out[t] = tw.trunc;
-            a.ws_w[t] = tw.w;
-            a.ws_trunc[t] = tw.trunc;
-            a.ws_logk[t] = tw.logk;
-            a.ws_terms[t] = tl.term;
-        }
+        const TokenLoss tl = token_loss(rs.lp, rs.lp_lo, has_old, lold, adv, sc, tw.w, a.P);
+        term = tl.term;
+        lp = rs.lp;
         // Pass 2 forms c softmax_j as cs 2^{z_j log2e - B}: with the power-of-two
         // scale K = clamp(ilogb(c) + 25, 0, 127) (below), B = fl(m log2e + bias
         // - K), and the rounding residual of B folded into cs.  The residual is
@@ -254,7 +251,10 @@ __global__ void __launch_bounds__(kThreads) cis_fused_cluster_kernel(const PassA
         const float c = tl.c;
         const int kexp = (int)((__float_as_uint(c) >> 23) & 0xff) - 127 + 25;
         const int K = kexp < 0 ? 0 : (kexp > 127 ? 127 : kexp);
-        float cs = ldexpf(c, -K);
+        // c 2^-K exactly: two power-of-two factors, each normal for K <= 127,
+        // and every product normal (c 2^-K has exponent -25 unless K is 0)
+        float cs = c * __int_as_float((127 - K / 2) << 23) *
+                   __int_as_float((127 - (K - K / 2)) << 23);
         float B = INFINITY;
         if (rs.bias_log2 != INFINITY) {
             const float p = rs.m * kLog2e, pe = fmaf(rs.m, kLog2e, -p);  // p + pe = m log2e
@@ -269,9 +269,20 @@ __global__ void __launch_bounds__(kThreads) cis_fused_cluster_kernel(const PassA
         sh.c = c;
         sh.cs = cs;
         sh.B = B;
-        sh.lp = rs.lp;
+        sh.dzy = c * (0.0f - rs.omp);  // c (p - 1); +0 when p = 1
     }
     __syncthreads();
+    if (threadIdx.x == 0 && rank == 0) {
+        if (a.lp_out) a.lp_out[t] = lp;
+        if (a.w_out) a.w_out[t] = tw.w;
+        if (a.trunc_out) a.trunc_out[t] = tw.trunc;
+        a.ws_w[t] = tw.w;
+        a.ws_trunc[t] = tw.trunc;
+        a.ws_logk[t] = tw.logk;
+        a.ws_terms[t] = term;
+        if (kEnt)
+            a.entropy_out[t] = row_entropy(ou, zy, lp);
+    }
 
     // Pass 2: dz = c (softmax - onehot) from the slice in shared memory.
     // c softmax_j is formed as (c 2^-K) 2^(x_j + K) with the flushing
@@ -279,8 +290,7 @@ __global__ void __launch_bounds__(kThreads) cis_fused_cluster_kernel(const PassA
     // 2^(x_j + K) would be subnormal, |c softmax_j| < 2^-150 rounds to zero in
     // fp32 and bf16 anyway; c 2^-K stays normal and 2^(x_j + K) finite.  The
     // final multiply keeps subnormal products.
-    const float c = sh.c, cs2 = sh.cs, B = sh.B;
-    const float dzy = c * expm1f(sh.lp);  // c (p - 1)
+    const float cs2 = sh.cs, B = sh.B, dzy = sh.dzy;
 #pragma unroll 2
     for (int g = threadIdx.x; g < ng; g += kThreads) {
         float z[8], v[8];

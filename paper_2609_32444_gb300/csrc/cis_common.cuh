@@ -10,10 +10,13 @@
 // Decisions (truncated or not, PPO clip active or not) are defined in fp64:
 // "log k > log cap" with log k = l_w - l_inf evaluated exactly.  The kernels
 // evaluate them in fp32 and keep that answer only when it is certain: the
-// fp32 operands carry relative errors of a few ulp (expm1f/log1pf/logf are
-// accurate to 1-2 ulp, the subtraction to 0.5 ulp), so a gap larger than
+// fp32 operands carry relative errors of a few ulp (expf/expm1f/log1pf/logf
+// are accurate to 1-2 ulp, a subtraction to 0.5 ulp), so a gap larger than
 // 4e-6 relative cannot change sign in exact arithmetic.  Inside that band the
 // comparison is redone in fp64.  The result equals the fp64 decision.
+// log p travels as an unevaluated fp32 pair (lp + lp_lo, better than fp32)
+// built with error-free sums: fp64 arithmetic is slow on this part (64 cycles
+// a dependent operation) and sits on each row's serial path.
 #pragma once
 
 #include <cuda_bf16.h>
@@ -97,6 +100,17 @@ __device__ __forceinline__ float max_nan(float a, float b)
     return r;
 }
 
+// Error-free sum (Knuth): a + b = s + e exactly, s = fl(a + b).  Where s is
+// not finite the error term is meaningless and is returned as 0.
+__device__ __forceinline__ float two_sum(float a, float b, float &e)
+{
+    const float s = __fadd_rn(a, b);
+    const float bv = __fsub_rn(s, a);
+    const float er = __fadd_rn(__fsub_rn(a, __fsub_rn(s, bv)), __fsub_rn(b, bv));
+    e = isfinite(s) ? er : 0.0f;
+    return s;
+}
+
 // +1: a > b for certain; -1: a < b for certain (a <= b in the fp64 sense);
 // 0: too close to call from fp32 values with relative errors below ~1e-6.
 __device__ __forceinline__ int certain_cmp(float a, float b)
@@ -116,47 +130,58 @@ struct TokenWeight {
     uint8_t trunc;
 };
 
-// Mismatch weight from log p (lw, training side, fp64 so that a log p carried
-// to better than fp32 keeps its accuracy) and log q (linf, inference side).
-// Algorithm 1: p = exp(lw), k = exp(lw - linf), phi = max(1-p, kappa),
-// w = min{k, 1 + lambda*phi}; Table 8 for the other modes.
-__device__ __forceinline__ TokenWeight token_weight(double lw, float linf, const DevParams &P)
+// Mismatch weight from log p (training side, the pair lw + lw_lo; lw_lo = 0
+// for an fp32 input) and log q (linf, inference side).  Algorithm 1:
+// p = exp(lw), k = exp(lw - linf), phi = max(1-p, kappa),
+// w = min{k, 1 + lambda*phi}; Table 8 for the other modes.  omp is 1 - p
+// where the caller already has it (row_scalars), else negative.
+__device__ __forceinline__ TokenWeight token_weight(float lw, float lw_lo, float linf,
+                                                    const DevParams &P, float omp = -1.0f)
 {
     TokenWeight r;
-    const double logk64 = lw - (double)linf;  // exact when lw is an fp32 value
-    const float logk = (float)logk64;
-    const float lwf = (float)lw;
+    float ke;
+    const float kh = two_sum(lw, -linf, ke);    // lw - linf = kh + ke exactly
+    const float logk = kh + (ke + lw_lo);       // log k, rounded about once
+    // the fp64 values, formed only where a decision is taken in fp64
+    auto lw64 = [&] { return (double)lw + (double)lw_lo; };
+    auto logk64 = [&] { return lw64() - (double)linf; };
     r.logk = logk;
     r.trunc = 0;
     r.w = 1.0f;
     switch (P.mode) {
     case CIS_MODE_CIS: {
-        const float lam_phi = P.lam_f * fmaxf(-expm1f(lwf), P.kappa_f);
-        const float lcap = log1pf(lam_phi);
-        const int s = certain_cmp(logk, lcap);
+        // k > cap compared directly: near the cap, k and cap lie in
+        // [1, 1 + lambda], where k's relative error is 2^-24 |log k| (the
+        // rounding of log k) plus expf's 2 ulp, at most 6e-6 for any finite
+        // fp32 lambda, inside certain_cmp's 4e-6 (k + cap)
+        const float om = omp >= 0.0f ? omp : -expm1f(lw);
+        const float lam_phi = P.lam_f * fmaxf(om, P.kappa_f);
+        const float cap = 1.0f + lam_phi;
+        const float k = expf(logk);
+        const int s = certain_cmp(k, cap);
         bool tr;
         if (s != 0) {
             tr = s > 0;
         } else {
-            const double phi = fmax(-expm1(lw), P.kappa);
-            tr = logk64 > log1p(P.lam * phi);
+            const double phi = fmax(-expm1(lw64()), P.kappa);
+            tr = logk64() > log1p(P.lam * phi);
         }
         r.trunc = tr;
-        r.w = tr ? 1.0f + lam_phi : expf(logk);
+        r.w = tr ? cap : k;
         break;
     }
     case CIS_MODE_TIS: {
         const int s = certain_cmp(logk, P.log_tis_cap_f);
-        const bool tr = s != 0 ? s > 0 : logk64 > P.log_tis_cap;
+        const bool tr = s != 0 ? s > 0 : logk64() > P.log_tis_cap;
         r.trunc = tr;
         r.w = tr ? P.tis_cap_f : expf(logk);
         break;
     }
     case CIS_MODE_EXACT: {
         const int sh = certain_cmp(logk, P.log_exact_hi_f);
-        const bool hi = sh != 0 ? sh > 0 : logk64 > P.log_exact_hi;
+        const bool hi = sh != 0 ? sh > 0 : logk64() > P.log_exact_hi;
         const int sl = certain_cmp(P.log_exact_lo_f, logk);
-        const bool lo = sl != 0 ? sl > 0 : logk64 < P.log_exact_lo;
+        const bool lo = sl != 0 ? sl > 0 : logk64() < P.log_exact_lo;
         r.trunc = hi || lo;
         r.w = hi ? P.exact_hi_f : (lo ? P.exact_lo_f : expf(logk));
         break;
@@ -164,17 +189,17 @@ __device__ __forceinline__ TokenWeight token_weight(double lw, float linf, const
     case CIS_MODE_BAND: {
         // Sec. 4.3: the CIS weight, lifted from below to (1 + p)/2 (the image
         // of e^eps = 1/2); both decisions in fp64
-        const double phi = fmax(-expm1(lw), P.kappa);
-        const double lo = 0.5 * (1.0 + exp(lw));
-        const bool up = logk64 > log1p(P.lam * phi);
-        const bool low = logk64 < log(lo);
+        const double phi = fmax(-expm1(lw64()), P.kappa);
+        const double lo = 0.5 * (1.0 + exp(lw64()));
+        const bool up = logk64() > log1p(P.lam * phi);
+        const bool low = logk64() < log(lo);
         r.trunc = up || low;
         r.w = up ? (float)(1.0 + P.lam * phi) : (low ? (float)lo : expf(logk));
         break;
     }
     case CIS_MODE_ICEPOP: {
         // Table 8: k on [lo, hi] (bounds included), else masked
-        const bool out = logk64 < P.log_icepop_lo || logk64 > P.log_icepop_hi;
+        const bool out = logk64() < P.log_icepop_lo || logk64() > P.log_icepop_hi;
         r.trunc = out;
         r.w = out ? 0.0f : expf(logk);
         break;
@@ -183,7 +208,7 @@ __device__ __forceinline__ TokenWeight token_weight(double lw, float linf, const
         // Table 8 / App. D.5: binary KL both ways in fp64 on probabilities
         // clamped to [1e-8, 1 - 1e-8]; masked when the larger exceeds phi
         const double lo = 1e-8, hi = 1.0 - 1e-8;
-        double p = exp(lw), q = exp((double)linf);
+        double p = exp(lw64()), q = exp((double)linf);
         p = p < lo ? lo : (p > hi ? hi : p);
         q = q < lo ? lo : (q > hi ? hi : q);
         const double kl_pq = p * log(p / q) + (1.0 - p) * log((1.0 - p) / (1.0 - q));
@@ -236,23 +261,25 @@ struct TokenLoss {
 
 // Eq. 1 for one token: rho = exp(lp - lp_old) (1 in value without lp_old),
 // objective w min(rho A, clip(rho) A); the min takes the unclipped branch on
-// ties, so g = 0 only where the clip is strictly active.  lp in fp64 (see
-// token_weight).
-__device__ __forceinline__ TokenLoss token_loss(double lp, bool has_old, float lp_old, float A,
-                                                float s, float w, const DevParams &P)
+// ties, so g = 0 only where the clip is strictly active.  log p as the pair
+// lp + lp_lo (see token_weight).
+__device__ __forceinline__ TokenLoss token_loss(float lp, float lp_lo, bool has_old, float lp_old,
+                                                float A, float s, float w, const DevParams &P)
 {
     float rho = 1.0f;
     bool g = true;
     if (has_old) {
-        const double lr64 = lp - (double)lp_old;
-        const float lr = (float)lr64;
+        float re;
+        const float rh = two_sum(lp, -lp_old, re);
+        const float lr = rh + (re + lp_lo);
+        auto lr64 = [&] { return ((double)lp + (double)lp_lo) - (double)lp_old; };
         rho = expf(lr);
         if (A > 0.0f) {
             const int c = certain_cmp(lr, P.log_rho_hi_f);
-            g = c != 0 ? c < 0 : !(lr64 > P.log_rho_hi);
+            g = c != 0 ? c < 0 : !(lr64() > P.log_rho_hi);
         } else if (A < 0.0f) {
             const int c = certain_cmp(lr, P.log_rho_lo_f);
-            g = c != 0 ? c > 0 : !(lr64 < P.log_rho_lo);
+            g = c != 0 ? c > 0 : !(lr64() < P.log_rho_lo);
         }
     }
     const float rho_c = fminf(fmaxf(rho, P.rho_lo_f), P.rho_hi_f);
@@ -335,6 +362,46 @@ __device__ __forceinline__ MaxSumU msu_combine(MaxSumU a, MaxSumU b)
     return {m, r.s, ua + ub};
 }
 
+// The pairs (triples) of n CTAs combined at once: the maximum first, then the
+// n rescaled sums added in rank order (independent exponentials, one
+// dependent step instead of n - 1).  Same empty-set and NaN rules as
+// ms_combine / msu_combine.
+__device__ __forceinline__ MaxSum combine_flat(const float2 *part, unsigned n)
+{
+    float M = part[0].x;
+    for (unsigned r = 1; r < n; ++r)
+        M = fmaxf(M, part[r].x);
+    float S = 0.0f;
+    for (unsigned r = 0; r < n; ++r) {
+        const float2 q = part[r];
+        S += (M == -INFINITY || q.x == -INFINITY) ? q.y * (M == -INFINITY ? 1.0f : 0.0f)
+                                                   : q.y * ex2_ftz((q.x - M) * kLog2e);
+    }
+    return {M, S};
+}
+__device__ __forceinline__ MaxSumU combine_flat(const float4 *part, unsigned n)
+{
+    float M = part[0].x;
+    for (unsigned r = 1; r < n; ++r)
+        M = fmaxf(M, part[r].x);
+    float S = 0.0f, U = 0.0f;
+    for (unsigned r = 0; r < n; ++r) {
+        const float4 q = part[r];
+        if (M == -INFINITY) {
+            S += q.y;
+            U += q.z;
+        } else if (q.x == -INFINITY) {
+            S += q.y * 0.0f;
+            U += q.z * 0.0f;
+        } else {
+            const float f = ex2_ftz((q.x - M) * kLog2e);
+            S += q.y * f;
+            U += fmaf(q.x - M, q.y, q.z) * f;
+        }
+    }
+    return {M, S, U};
+}
+
 __device__ __forceinline__ MaxSumU warp_msu(MaxSumU v)
 {
 #pragma unroll
@@ -369,15 +436,18 @@ __device__ __forceinline__ MaxSumU block_msu(MaxSumU v, MaxSumU *sh)
 //   d = z_y - log sum_{j != y} e^{z_j} = (z_y - m') - log s',
 // log p = -softplus(-d) is accurate for p near 0 and near 1 (Sec. 3.3 notes
 // that logit p stops being finite when p rounds to 1; d itself stays finite).
-// For d <= 0, log p = d - log1p(e^d) can be large in magnitude, so it is also
-// kept in fp64 (lp64, ~1e-6 absolute) for the weight; lse - m' is formed
-// without cancellation for pass 2.
+// For d <= 0, log p = d - log1p(e^d) can be large in magnitude, so its
+// rounding residual is kept too (lp_lo) for the weight; lse - m' is formed
+// without cancellation for pass 2.  z_y - m' and the sums with log s' and the
+// softplus are error-free fp32 sums (two_sum), not fp64.
 struct RowScalars {
     float lp;         // log p of the sampled token (fp32 output)
-    double lp64;      // the same, carried in fp64
+    float lp_lo;      // log p = lp + lp_lo to better than fp32 (0 for d > 0)
     float lse;        // logsumexp of the row
     float m;          // offset used for the exponent (m' or 0)
     float bias_log2;  // (lse - m) * log2(e), +inf when no other entry is finite
+    float omp;        // 1 - p, from the same exponential as the softplus
+    __device__ __forceinline__ double lp64() const { return (double)lp + (double)lp_lo; }
 };
 
 __device__ __forceinline__ RowScalars row_scalars(MaxSum o, float zy)
@@ -386,25 +456,39 @@ __device__ __forceinline__ RowScalars row_scalars(MaxSum o, float zy)
     if (o.m == -INFINITY && o.s == 0.0f) {
         // every other entry is -inf: p = 1
         r.lp = zy != zy ? zy : 0.0f;
-        r.lp64 = r.lp;
+        r.lp_lo = 0.0f;
+        r.omp = 0.0f;
         r.lse = zy;
         r.m = 0.0f;
         r.bias_log2 = INFINITY;
         return r;
     }
-    const double dz64 = (double)zy - (double)o.m;  // exact
+    float dl, ue;
+    const float dh = two_sum(zy, -o.m, dl);          // z_y - m' = dh + dl exactly
     const float ls = logf(o.s);
-    const float d = (float)(dz64 - (double)ls);      // logit p
+    const float u = two_sum(dh, -ls, ue);            // dh - ls = u + ue exactly
+    const float d = u + (ue + dl);                   // logit p
     float lse_m;                                     // lse - m'
+    // 1 - p = sigmoid(-d): e^{-d} / (1 + e^{-d}) for d > 0, 1 / (1 + e^d)
+    // otherwise, without the cancellation of 1 - e^{log p}
     if (d > 0.0f) {
-        const float t = log1pf(expf(-d));            // softplus(-d) = -log p
+        const float e = expf(-d);
+        const float t = log1pf(e);                   // softplus(-d) = -log p
+        r.omp = __fdividef(e, 1.0f + e);
         r.lp = -t;
-        r.lp64 = -(double)t;
-        lse_m = (float)(dz64 + (double)t);
+        r.lp_lo = 0.0f;
+        float ve;
+        const float v = two_sum(dh, t, ve);          // (z_y - m') + t
+        lse_m = v + (ve + dl);
     } else {
-        const float t = log1pf(expf(d));             // softplus(d)
-        r.lp64 = (dz64 - (double)ls) - (double)t;
-        r.lp = (float)r.lp64;
+        const float e = expf(d);
+        const float t = log1pf(e);                   // softplus(d)
+        r.omp = __fdividef(1.0f, 1.0f + e);
+        float xe;
+        const float x = two_sum(u, -t, xe);          // log p = x + xe + ue + dl
+        const float lo = xe + (ue + dl);
+        r.lp = x + lo;
+        r.lp_lo = isfinite(r.lp) ? lo - (r.lp - x) : 0.0f;
         lse_m = ls + t;
     }
     r.lse = o.m + lse_m;
@@ -425,7 +509,10 @@ __device__ __forceinline__ float row_entropy(MaxSumU o, float zy, float lp)
     if (o.m == -INFINITY && o.s == 0.0f)
         return zy != zy ? zy : 0.0f;  // every other entry is -inf: p = 1
     const float ls = logf(o.s);
-    const float d = (float)(((double)zy - (double)o.m) - (double)ls);
+    float dl, ue;
+    const float dh = two_sum(zy, -o.m, dl);
+    const float u = two_sum(dh, -ls, ue);
+    const float d = u + (ue + dl);  // logit p, as in row_scalars
     // log(1 - p) = -softplus(d)
     const float l1mp = d > 0.0f ? -(d + log1pf(expf(-d))) : -log1pf(expf(d));
     const float p = expf(lp), q = expf(l1mp);

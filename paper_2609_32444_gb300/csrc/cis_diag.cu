@@ -130,7 +130,7 @@ __global__ void __launch_bounds__(kDiagThreads)
         const double dp = ((double)zyt - (double)ot.m) - (double)logf(ot.s);
         const double dq = ((double)zyi - (double)oi.m) - (double)logf(oi.s);
         eps_out[t] = (float)(dp - dq);
-        if (logk_out) logk_out[t] = (float)(st.lp64 - si.lp64);
+        if (logk_out) logk_out[t] = (float)(st.lp64() - si.lp64());
         if (p_out) p_out[t] = expf(st.lp);
         sh.lse_p = st.lse;
         sh.lse_q = si.lse;
@@ -567,7 +567,7 @@ __global__ void __launch_bounds__(StreamCfg<NW>::kThreads, 1)
             }
             const RowScalars rs = row_scalars(o, zy);
             // lane 0 gets the inference row's values from lane 16
-            const double lp64_q = __shfl_sync(0xffffffffu, rs.lp64, 16);
+            const double lp64_q = __shfl_sync(0xffffffffu, rs.lp64(), 16);
             const float lse_q = __shfl_sync(0xffffffffu, rs.lse, 16);
             const float om_q = __shfl_sync(0xffffffffu, o.m, 16);
             const float os_q = __shfl_sync(0xffffffffu, o.s, 16);
@@ -578,7 +578,7 @@ __global__ void __launch_bounds__(StreamCfg<NW>::kThreads, 1)
                 const double dp = ((double)zy - (double)o.m) - (double)logf(o.s);
                 const double dq = ((double)zy_q - (double)om_q) - (double)logf(os_q);
                 a.eps[t] = (float)(dp - dq);
-                if (a.logk) a.logk[t] = (float)(rs.lp64 - lp64_q);
+                if (a.logk) a.logk[t] = (float)(rs.lp64() - lp64_q);
                 if (a.p) a.p[t] = expf(rs.lp);
                 sh.op = rs.lse * kLog2e;
                 sh.oq = lse_q * kLog2e;

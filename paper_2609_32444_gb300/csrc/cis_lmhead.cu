@@ -555,17 +555,19 @@ __global__ void cis_lmhead_token_kernel(const PassArgs a, const float2 *part, co
             // sequence operator, first sweep: log p only (the response's
             // weight needs every token of the response)
             if (a.lp64_out)
-                a.lp64_out[t] = rs.lp64;
+                a.lp64_out[t] = rs.lp64();
             return;
         }
         const bool has_old = a.lp_old != nullptr;
         const float lold = has_old ? a.lp_old[t] : 0.0f;
-        TokenWeight tw = token_weight(has_old ? (double)lold : rs.lp64, a.lp_inf[t], a.P);
+        TokenWeight tw = token_weight(has_old ? lold : rs.lp, has_old ? 0.0f : rs.lp_lo,
+                                      a.lp_inf[t], a.P, has_old ? -1.0f : rs.omp);
         if (a.w_in) {
             tw.w = a.w_in[t];
             tw.trunc = a.trunc_in[t];
         }
-        const TokenLoss tl = token_loss(rs.lp64, has_old, lold, a.adv[t], a.scale[t], tw.w, a.P);
+        const TokenLoss tl =
+            token_loss(rs.lp, rs.lp_lo, has_old, lold, a.adv[t], a.scale[t], tw.w, a.P);
         if (a.lp_out) a.lp_out[t] = rs.lp;
         if (a.w_out) a.w_out[t] = tw.w;
         if (a.trunc_out) a.trunc_out[t] = tw.trunc;

@@ -84,17 +84,19 @@ __global__ void __launch_bounds__(kRowThreads) cis_fused_row_kernel(const PassAr
             a.entropy_out[t] = row_entropy(ou, to_f32(row[y]), rs.lp);
         if (a.lp_out) a.lp_out[t] = rs.lp;
         if (a.lse_out) a.lse_out[t] = rs.lse;
-        if (!kBwd && a.lp64_out) a.lp64_out[t] = rs.lp64;
+        if (!kBwd && a.lp64_out) a.lp64_out[t] = rs.lp64();
         if (kBwd) {
             const bool has_old = a.lp_old != nullptr;
-            const double lw = has_old ? (double)a.lp_old[t] : rs.lp64;
-            TokenWeight tw = token_weight(lw, a.lp_inf[t], a.P);
+            TokenWeight tw = token_weight(has_old ? a.lp_old[t] : rs.lp,
+                                          has_old ? 0.0f : rs.lp_lo, a.lp_inf[t], a.P,
+                                          has_old ? -1.0f : rs.omp);
             if (a.w_in) {  // a sequence operator: the response's weight
                 tw.w = a.w_in[t];
                 tw.trunc = a.trunc_in[t];
             }
-            const TokenLoss tl = token_loss(rs.lp64, has_old, has_old ? a.lp_old[t] : 0.0f,
-                                            a.adv[t], a.scale[t], tw.w, a.P);
+            const TokenLoss tl = token_loss(rs.lp, rs.lp_lo, has_old,
+                                            has_old ? a.lp_old[t] : 0.0f, a.adv[t], a.scale[t],
+                                            tw.w, a.P);
             if (a.w_out) a.w_out[t] = tw.w;
             if (a.trunc_out) a.trunc_out[t] = tw.trunc;
             a.ws_w[t] = tw.w;

@@ -152,7 +152,7 @@ __global__ void cis_weights_kernel(const float *lp_w, const float *lp_inf, const
         uint8_t tr = 0;
         if (is_valid(mask, t)) {
             const float lw = lp_w[t], li = lp_inf[t];
-            const TokenWeight tw = token_weight((double)lw, li, P);
+            const TokenWeight tw = token_weight(lw, 0.0f, li, P);
             w = tw.w;
             tr = tw.trunc;
             if (eps_out)
