@@ -139,13 +139,14 @@ __global__ void __launch_bounds__(kThreads) cis_fused_cluster_kernel(const PassA
     cluster_arrive_relaxed();
 
     // Per-token inputs, fetched while the copy is in flight.
-    float zy = 0.0f, linf = 0.0f, lold = 0.0f, adv = 0.0f, sc = 0.0f;
+    float zy = 0.0f, linf = 0.0f, lold = 0.0f, adv = 0.0f, sc = 0.0f, qinv = 0.0f;
     if (threadIdx.x == 0) {
         zy = to_f32(reinterpret_cast<const InT *>(a.logits)[t * a.ld + y]);
         linf = a.lp_inf[t];
         lold = a.lp_old ? a.lp_old[t] : 0.0f;
         adv = a.adv[t];
         sc = a.scale[t];
+        qinv = expf(-linf);  // 1 / q, off the row's serial path
     }
     __syncthreads();  // barriers initialised before anyone polls them
 
@@ -216,14 +217,17 @@ __global__ void __launch_bounds__(kThreads) cis_fused_cluster_kernel(const PassA
     cluster_arrive_relaxed();
 
     // Thread 0 forms the row's scalars: the serial part of every row, which
-    // the other threads wait for.  It combines the cluster's pairs (one
-    // rescaling step), and everything pass 2 does not need (the per-token
-    // outputs, the fp64 loss term, the entropy) is stored after the barrier,
-    // by rank 0 only.
+    // the other threads wait for, and which shares the SM's issue slots with
+    // the other CTAs' streaming loops, so its instruction count sets its
+    // length.  In the common case (row_weight_direct) the weight comes from
+    // the row's statistics without logarithms, and log p, log k and the fp64
+    // loss term are formed after the barrier by rank 0 alone, which stores
+    // them.  Otherwise the log-domain path forms everything here.
     MaxSumU ou{0.0f, 0.0f, 0.0f};
     TokenWeight tw{0.0f, 0.0f, 0};
     double term = 0.0;
-    float lp = 0.0f;
+    float lp = 0.0f, tdir = 0.0f;
+    bool direct = false;
     if (threadIdx.x == 0) {
         MaxSum o;
         if constexpr (kEnt) {
@@ -232,23 +236,38 @@ __global__ void __launch_bounds__(kThreads) cis_fused_cluster_kernel(const PassA
         } else {
             o = combine_flat(sh.part, cs);
         }
-        const RowScalars rs = row_scalars(o, zy);
         const bool has_old = a.lp_old != nullptr;
-        tw = token_weight(has_old ? lold : rs.lp, has_old ? 0.0f : rs.lp_lo, linf, a.P,
-                          has_old ? -1.0f : rs.omp);
-        if (a.w_in) {  // a sequence operator: the response's weight
-            tw.w = a.w_in[t];
-            tw.trunc = a.trunc_in[t];
+        float c, omp, bias_log2;
+        DirectWeight dw;
+        direct = !has_old && a.w_in == nullptr && row_weight_direct(o, zy, linf, qinv, a.P, dw);
+        if (direct) {
+            tw.w = dw.w;
+            tw.trunc = dw.trunc;
+            omp = dw.omp;
+            tdir = dw.t;
+            c = sc * tw.w * adv;  // s w A rho with rho = 1, g = 1 (Eq. 1 without l_old)
+            // (lse - m') log2 e = log2(s' + e^{z_y - m'})
+            bias_log2 = log2f(o.s + __fdividef(1.0f, dw.E));
+        } else {
+            const RowScalars rs = row_scalars(o, zy);
+            tw = token_weight(has_old ? lold : rs.lp, has_old ? 0.0f : rs.lp_lo, linf, a.P,
+                              has_old ? -1.0f : rs.omp);
+            if (a.w_in) {  // a sequence operator: the response's weight
+                tw.w = a.w_in[t];
+                tw.trunc = a.trunc_in[t];
+            }
+            const TokenLoss tl = token_loss(rs.lp, rs.lp_lo, has_old, lold, adv, sc, tw.w, a.P);
+            term = tl.term;
+            lp = rs.lp;
+            c = tl.c;
+            omp = rs.omp;
+            bias_log2 = rs.bias_log2;
         }
-        const TokenLoss tl = token_loss(rs.lp, rs.lp_lo, has_old, lold, adv, sc, tw.w, a.P);
-        term = tl.term;
-        lp = rs.lp;
         // Pass 2 forms c softmax_j as cs 2^{z_j log2e - B}: with the power-of-two
         // scale K = clamp(ilogb(c) + 25, 0, 127) (below), B = fl(m log2e + bias
         // - K), and the rounding residual of B folded into cs.  The residual is
         // exact: the product's error from an FMA, the two sums' errors from
         // two-sums (fp32 throughout: fp64 operations take 64 cycles each here).
-        const float c = tl.c;
         const int kexp = (int)((__float_as_uint(c) >> 23) & 0xff) - 127 + 25;
         const int K = kexp < 0 ? 0 : (kexp > 127 ? 127 : kexp);
         // c 2^-K exactly: two power-of-two factors, each normal for K <= 127,
@@ -256,23 +275,26 @@ __global__ void __launch_bounds__(kThreads) cis_fused_cluster_kernel(const PassA
         float cs = c * __int_as_float((127 - K / 2) << 23) *
                    __int_as_float((127 - (K - K / 2)) << 23);
         float B = INFINITY;
-        if (rs.bias_log2 != INFINITY) {
-            const float p = rs.m * kLog2e, pe = fmaf(rs.m, kLog2e, -p);  // p + pe = m log2e
-            const float a = rs.bias_log2, k = -(float)K;
-            const float q = a + k, qv = q - a;
-            const float qe = (a - (q - qv)) + (k - qv);  // q + qe = bias - K
-            B = p + q;
-            const float bv = B - p;
-            const float se = (p - (B - bv)) + (q - bv);  // B + se = p + q
+        const float m = o.m == -INFINITY ? 0.0f : o.m;  // row_scalars' offset
+        if (bias_log2 != INFINITY) {
+            const float p = m * kLog2e, pe = fmaf(m, kLog2e, -p);  // p + pe = m log2e
+            float qe, se;
+            const float q = two_sum(bias_log2, -(float)K, qe);      // q + qe = bias - K
+            B = two_sum(p, q, se);                                   // B + se = p + q
             cs *= ex2_ftz(-(se + pe + qe));
         }
         sh.c = c;
         sh.cs = cs;
         sh.B = B;
-        sh.dzy = c * (0.0f - rs.omp);  // c (p - 1); +0 when p = 1
+        sh.dzy = c * (0.0f - omp);  // c (p - 1); +0 when p = 1
     }
     __syncthreads();
     if (threadIdx.x == 0 && rank == 0) {
+        if (direct) {  // log p, log k and the loss term, off the serial path
+            lp = -log1pf(tdir);  // p = 1 / (1 + t)
+            tw.logk = lp - linf;
+            term = -(double)sc * (double)tw.w * (double)adv;
+        }
         if (a.lp_out) a.lp_out[t] = lp;
         if (a.w_out) a.w_out[t] = tw.w;
         if (a.trunc_out) a.trunc_out[t] = tw.trunc;

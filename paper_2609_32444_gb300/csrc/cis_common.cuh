@@ -432,6 +432,74 @@ __device__ __forceinline__ MaxSumU block_msu(MaxSumU v, MaxSumU *sh)
     return r;
 }
 
+// The weight of the common case straight from a row's statistics, without
+// logarithms: the CIS, TIS, exact and no-correction operators with the
+// current log p as l_w (no l_old, no sequence weight).  From (m', s') over
+// j != y and z_y, with t = s' e^{m' - z_y} = (1 - p) / p:
+//   p = 1 / (1 + t),   1 - p = t p,   k = p / q = p e^{-l_inf},
+// each within ~8 ulp (expf, __fdividef: 2 ulp each), so k and the cap carry
+// relative errors near 2e-6, inside certain_cmp's 4e-6 (k + cap).  qinv is
+// e^{-l_inf}, formed by the caller ahead of time.  Returns false, deciding
+// nothing, where these forms would leave the normal fp32 range
+// (|m' - z_y| > 70, l_inf < -70, an empty or non-finite row) or the decision
+// is too close to call; the caller then takes the log-domain path
+// (row_scalars, token_weight), whose fp64 fallback settles it.
+struct DirectWeight {
+    float w;
+    float omp;  // 1 - p
+    float t;    // (1 - p) / p; log p = -log1p(t)
+    float E;    // e^{m' - z_y}
+    uint8_t trunc;
+};
+__device__ __forceinline__ bool row_weight_direct(MaxSum o, float zy, float linf, float qinv,
+                                                  const DevParams &P, DirectWeight &r)
+{
+    float dl;
+    const float dh = two_sum(o.m, -zy, dl);  // m' - z_y = dh + dl exactly
+    if (!(fabsf(dh) <= 70.0f) || !(linf >= -70.0f) || !(o.s >= 1.0f) || !(o.s <= 3.0e38f))
+        return false;
+    const float e = expf(dh);
+    r.E = fmaf(e, dl, e);
+    const float t = o.s * r.E;
+    const float p = __fdividef(1.0f, 1.0f + t);
+    const float k = p * qinv;
+    r.t = t;
+    r.omp = t * p;
+    r.trunc = 0;
+    r.w = 1.0f;
+    switch (P.mode) {
+    case CIS_MODE_CIS: {
+        const float cap = 1.0f + P.lam_f * fmaxf(r.omp, P.kappa_f);
+        const int s = certain_cmp(k, cap);
+        if (s == 0)
+            return false;
+        r.trunc = s > 0;
+        r.w = s > 0 ? cap : k;
+        return true;
+    }
+    case CIS_MODE_TIS: {
+        const int s = certain_cmp(k, P.tis_cap_f);
+        if (s == 0)
+            return false;
+        r.trunc = s > 0;
+        r.w = s > 0 ? P.tis_cap_f : k;
+        return true;
+    }
+    case CIS_MODE_EXACT: {
+        const int sh = certain_cmp(k, P.exact_hi_f), sl = certain_cmp(P.exact_lo_f, k);
+        if (sh == 0 || sl == 0)
+            return false;
+        r.trunc = sh > 0 || sl > 0;
+        r.w = sh > 0 ? P.exact_hi_f : (sl > 0 ? P.exact_lo_f : k);
+        return true;
+    }
+    case CIS_MODE_NONE:
+        return true;
+    default:
+        return false;
+    }
+}
+
 // Per-row scalars from (m', s') over j != y and z_y.  With the log-odds
 //   d = z_y - log sum_{j != y} e^{z_j} = (z_y - m') - log s',
 // log p = -softplus(-d) is accurate for p near 0 and near 1 (Sec. 3.3 notes
