@@ -58,16 +58,16 @@ __device__ __forceinline__ void store8<float>(float *dst, const float (&v)[8])
 template <bool kEnt> struct ClusterShared {
     alignas(8) uint64_t bar[kChunks];  // completion of each copy chunk
     alignas(8) uint64_t xbar;          // arrival of the cluster's (m, s) pairs
-    float2 part[kMaxCluster];
+    alignas(16) float2 part[kMaxCluster];
     MaxSum red[512 / 32];
-    float c, cs, B, dzy;
+    float4 row;  // pass 2's multiplier, exponent offset and c (p - 1): one load
 };
 template <> struct ClusterShared<true> {
     alignas(8) uint64_t bar[kChunks];
     alignas(8) uint64_t xbar;          // arrival of the cluster's (m, s, u) triples
     float4 part[kMaxCluster];
     MaxSumU red[512 / 32];
-    float c, cs, B, dzy;
+    float4 row;
 };
 
 template <typename InT, typename OutT, int kThreads, bool kEnt>
@@ -234,10 +234,10 @@ __global__ void __launch_bounds__(kThreads) cis_fused_cluster_kernel(const PassA
             ou = combine_flat(sh.part, cs);
             o = MaxSum{ou.m, ou.s};
         } else {
-            o = combine_flat(sh.part, cs);
+            o = cs == 4 ? combine4(sh.part) : combine_flat(sh.part, cs);
         }
         const bool has_old = a.lp_old != nullptr;
-        float c, omp, bias_log2;
+        float c, omp, bias_log2, scale = 1.0f;
         DirectWeight dw;
         direct = !has_old && a.w_in == nullptr && row_weight_direct(o, zy, linf, qinv, a.P, dw);
         if (direct) {
@@ -246,8 +246,15 @@ __global__ void __launch_bounds__(kThreads) cis_fused_cluster_kernel(const PassA
             omp = dw.omp;
             tdir = dw.t;
             c = sc * tw.w * adv;  // s w A rho with rho = 1, g = 1 (Eq. 1 without l_old)
-            // (lse - m') log2 e = log2(s' + e^{z_y - m'})
-            bias_log2 = log2f(o.s + __fdividef(1.0f, dw.E));
+            // The softmax's 1 / (s' + e^{z_y - m'}) = e^{m' - z_y} p, in
+            // [2^-102, 1] within the closed forms' range, replaces a logarithm:
+            // its binary exponent -J goes into the exponent offset (as the
+            // integer "bias" J) and its mantissa 2^J / (...) in [1, 2) into
+            // the multiplier, so that every product stays a normal number.
+            const float inv = dw.E * dw.p;
+            const int J = 127 - (int)((__float_as_uint(inv) >> 23) & 0xff);
+            bias_log2 = (float)J;
+            scale = inv * __int_as_float((127 + J) << 23);
         } else {
             const RowScalars rs = row_scalars(o, zy);
             tw = token_weight(has_old ? lold : rs.lp, has_old ? 0.0f : rs.lp_lo, linf, a.P,
@@ -265,9 +272,10 @@ __global__ void __launch_bounds__(kThreads) cis_fused_cluster_kernel(const PassA
         }
         // Pass 2 forms c softmax_j as cs 2^{z_j log2e - B}: with the power-of-two
         // scale K = clamp(ilogb(c) + 25, 0, 127) (below), B = fl(m log2e + bias
-        // - K), and the rounding residual of B folded into cs.  The residual is
-        // exact: the product's error from an FMA, the two sums' errors from
-        // two-sums (fp32 throughout: fp64 operations take 64 cycles each here).
+        // - K), and the rounding residual of B folded into cs (with the direct
+        // path's scale).  The residual is exact: the product's error from an
+        // FMA, the two sums' errors from two-sums (fp32 throughout: fp64
+        // operations take 64 cycles each here).
         const int kexp = (int)((__float_as_uint(c) >> 23) & 0xff) - 127 + 25;
         const int K = kexp < 0 ? 0 : (kexp > 127 ? 127 : kexp);
         // c 2^-K exactly: two power-of-two factors, each normal for K <= 127,
@@ -283,10 +291,7 @@ __global__ void __launch_bounds__(kThreads) cis_fused_cluster_kernel(const PassA
             B = two_sum(p, q, se);                                   // B + se = p + q
             cs *= ex2_ftz(-(se + pe + qe));
         }
-        sh.c = c;
-        sh.cs = cs;
-        sh.B = B;
-        sh.dzy = c * (0.0f - omp);  // c (p - 1); +0 when p = 1
+        sh.row = make_float4(cs * scale, B, c * (0.0f - omp), 0.0f);  // c (p - 1): +0 if p = 1
     }
     __syncthreads();
     if (threadIdx.x == 0 && rank == 0) {
@@ -312,7 +317,8 @@ __global__ void __launch_bounds__(kThreads) cis_fused_cluster_kernel(const PassA
     // 2^(x_j + K) would be subnormal, |c softmax_j| < 2^-150 rounds to zero in
     // fp32 and bf16 anyway; c 2^-K stays normal and 2^(x_j + K) finite.  The
     // final multiply keeps subnormal products.
-    const float cs2 = sh.cs, B = sh.B, dzy = sh.dzy;
+    const float4 row = sh.row;
+    const float cs2 = row.x, B = row.y, dzy = row.z;
 #pragma unroll 2
     for (int g = threadIdx.x; g < ng; g += kThreads) {
         float z[8], v[8];

@@ -379,6 +379,23 @@ __device__ __forceinline__ MaxSum combine_flat(const float2 *part, unsigned n)
     }
     return {M, S};
 }
+// Four pairs (the cluster of a 151,936-entry bf16 row), straight-line: two
+// 16-byte loads from a 16-byte aligned array, the maximum, then per pair one
+// rescaling exponential accumulated by an FMA, in rank order.
+__device__ __forceinline__ MaxSum combine4(const float2 *part)
+{
+    const float4 a = reinterpret_cast<const float4 *>(part)[0];
+    const float4 b = reinterpret_cast<const float4 *>(part)[1];
+    const float M = fmaxf(fmaxf(a.x, a.z), fmaxf(b.x, b.z));
+    if (M == -INFINITY)
+        return {M, ((a.y + a.w) + b.y) + b.w};
+    // an empty pair (m = -inf) gives ex2(-inf) = 0: s * 0, as in ms_combine
+    float S = a.y * ex2_ftz((a.x - M) * kLog2e);
+    S = fmaf(a.w, ex2_ftz((a.z - M) * kLog2e), S);
+    S = fmaf(b.y, ex2_ftz((b.x - M) * kLog2e), S);
+    S = fmaf(b.w, ex2_ftz((b.z - M) * kLog2e), S);
+    return {M, S};
+}
 __device__ __forceinline__ MaxSumU combine_flat(const float4 *part, unsigned n)
 {
     float M = part[0].x;
@@ -449,6 +466,7 @@ struct DirectWeight {
     float omp;  // 1 - p
     float t;    // (1 - p) / p; log p = -log1p(t)
     float E;    // e^{m' - z_y}
+    float p;
     uint8_t trunc;
 };
 __device__ __forceinline__ bool row_weight_direct(MaxSum o, float zy, float linf, float qinv,
@@ -464,6 +482,7 @@ __device__ __forceinline__ bool row_weight_direct(MaxSum o, float zy, float linf
     const float p = __fdividef(1.0f, 1.0f + t);
     const float k = p * qinv;
     r.t = t;
+    r.p = p;
     r.omp = t * p;
     r.trunc = 0;
     r.w = 1.0f;
