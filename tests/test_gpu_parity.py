@@ -462,3 +462,52 @@ def test_full_size_t16384_v151936(mode):
 
 def test_full_size_t65536_v151936_masked():
     _full_size_check(4, "cis", torch.bfloat16)
+
+
+@pytest.mark.parametrize("mode", ["cis", "tis", "exact", "none"])
+def test_direct_weight_boundaries_v151936(mode):
+    """The fused pass at V=151936 (4-CTA clusters) on rows built to sit at the
+    edges of its logarithm-free common case: inference log-probs that put
+    log k within 1e-7 .. 1e-3 of the operator's cap (either side, so that the
+    fp32 comparison is certain for some and hands over to the fp64 fallback
+    for others), z_y - m' near the +-70 range guard, and l_inf near -70.
+    Decisions outside the 4e-5 band, weights, loss and every dlogits entry are
+    checked against the oracle."""
+    T, lam = 64, 2.3
+    b = synth.make_batch(3, device=DEV, T=T)
+    z = b.logits.float()
+    ids = b.ids.long()
+    # rows 48..55: z_y - m' just inside / outside +-70 (m' = max over j != y)
+    zz = z.clone()
+    zz[torch.arange(T, device=DEV), ids] = -float("inf")
+    mprime = zz.max(dim=1).values
+    for i, off in enumerate([69.0, -69.0, 72.0, -72.0, 69.75, -69.75, 70.5, -70.5]):
+        t = 48 + i
+        z[t, ids[t]] = mprime[t] + off
+    b.logits = z.to(torch.bfloat16)
+    z_np = logits_for_oracle(b.logits)
+    ref_lp, _, _ = oracle.token_logprobs(z_np, b.ids.cpu().numpy())
+    deltas = np.array([0.0, 1e-7, -1e-7, 1e-6, -1e-6, 3e-6, -3e-6, 1e-5, -1e-5, 1e-4, -1e-4,
+                       1e-3, -1e-3, 5e-3, -5e-3, 2e-2])
+    lp_inf = ref_lp.copy()
+    for t in range(48):
+        d = deltas[t % len(deltas)]
+        if mode == "cis":
+            logcap = np.log1p(lam * max(-np.expm1(ref_lp[t]), 5e-3))
+        elif mode == "tis":
+            logcap = math.log(2.0)
+        elif mode == "exact":
+            logcap = math.log(1e6) if t % 2 else math.log(1e-6)
+        else:
+            logcap = 0.0
+        lp_inf[t] = ref_lp[t] - logcap - d  # log k = log cap + d
+    lp_inf[56:60] = [-69.0, -71.0, -69.9, -70.1]  # around the l_inf guard
+    b.lp_infer = torch.from_numpy(lp_inf.astype(np.float32))
+    b.adv = torch.from_numpy(np.where(np.arange(T) % 3 == 0, -1.0, 0.75).astype(np.float32))
+    g = to_dev(b)
+    for dz_dtype in (torch.float32, torch.bfloat16):
+        out = run_gpu(g, mode, lam, dz_dtype)
+        ref = run_oracle(b, mode, lam)
+        torch.cuda.synchronize()
+        check_token_outputs(out, ref, b, mode, lam)
+        check_dz(out["dlogits"], ref["dz"], ref["c"])
