@@ -336,6 +336,8 @@ struct StreamShared {
     float wsum[kMaxConsWarps][kNSums];
     double total[kNSums];
     float op, oq;
+    float2 rowstat[2];  // (m', s') of the training and the inference row
+    float zyv[2];       // their sampled entries
     int aborted;
 };
 
@@ -565,26 +567,46 @@ __global__ void __launch_bounds__(StreamCfg<NW>::kThreads, 1)
                 x.s = __shfl_xor_sync(0xffffffffu, o.s, off);
                 o = ms_combine(o, x);
             }
-            const RowScalars rs = row_scalars(o, zy);
-            // lane 0 gets the inference row's values from lane 16
+            // Pass 2 needs only the two rows' log-sum-exps; lanes 0 and 16
+            // form their own row's while the other warps wait, from the
+            // larger of m' and z_y so that no exponential overflows:
+            //   lse = z_y + log1p(s' e^{m' - z_y})   (z_y >= m', also p = 1)
+            //   lse = m' + log(s' + e^{z_y - m'})    (otherwise)
+            // The per-position outputs are formed after the barrier.
+            if ((lane & 15) == 0) {
+                const float lse = o.s == 0.0f ? zy  // no other finite entry: p = 1
+                                  : (zy >= o.m ? zy + log1pf(o.s * expf(o.m - zy))
+                                               : o.m + logf(o.s + expf(zy - o.m)));
+                if (r == 0)
+                    sh.op = lse * kLog2e;
+                else
+                    sh.oq = lse * kLog2e;
+                sh.rowstat[r] = make_float2(o.m, o.s);
+                sh.zyv[r] = zy;
+            }
+        }
+        cons_sync<kConsThreads>();
+        if (warp == (kConsWarps > 1 ? 1 : 0)) {
+            // eps, log k and p, off the serial path (warp 0 has the end-of-row
+            // sums to do); lane 16 forms the inference row's scalars
+            const int r = lane >> 4;
+            const MaxSum o = MaxSum{sh.rowstat[r].x, sh.rowstat[r].y};
+            const float zyr = sh.zyv[r];
+            const RowScalars rs = row_scalars(o, zyr);
             const double lp64_q = __shfl_sync(0xffffffffu, rs.lp64(), 16);
-            const float lse_q = __shfl_sync(0xffffffffu, rs.lse, 16);
             const float om_q = __shfl_sync(0xffffffffu, o.m, 16);
             const float os_q = __shfl_sync(0xffffffffu, o.s, 16);
-            const float zy_q = __shfl_sync(0xffffffffu, zy, 16);
+            const float zy_q = __shfl_sync(0xffffffffu, zyr, 16);
             if (lane == 0) {
                 // eps = logit p - logit q: Lemma 3.1's -delta_y + log sum_{j != y}
                 // w_j e^{delta_j} in the normalised gauge, from the log-odds
-                const double dp = ((double)zy - (double)o.m) - (double)logf(o.s);
+                const double dp = ((double)zyr - (double)o.m) - (double)logf(o.s);
                 const double dq = ((double)zy_q - (double)om_q) - (double)logf(os_q);
                 a.eps[t] = (float)(dp - dq);
                 if (a.logk) a.logk[t] = (float)(rs.lp64() - lp64_q);
                 if (a.p) a.p[t] = expf(rs.lp);
-                sh.op = rs.lse * kLog2e;
-                sh.oq = lse_q * kLog2e;
             }
         }
-        cons_sync<kConsThreads>();
 
         // pass 2
         float2 acc[kNSums];
