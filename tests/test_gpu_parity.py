@@ -5,7 +5,8 @@ need one):
   - log p of the sampled token: 2e-5 absolute, plus 4 fp32 ulps of |log p|
     (the output is fp32: the workloads' logits reach |z| ~ 650, so log p reaches
     ~ -1200, where one fp32 step is 1.2e-4; internally the weight uses log p
-    carried in fp64, so the weight tolerance below is not widened);
+    carried to better than fp32 (an fp32 pair, or p = 1/(1 + t) directly in the
+    fused pass's common case), so the weight tolerance below is not widened);
   - weights: 1e-5 relative;
   - truncation decisions: bit-exact when both sides get the same fp32 log-probs
     (cis_weights); end to end, bit-exact except for tokens whose fp64 log k lies
