@@ -112,7 +112,9 @@ __device__ __forceinline__ float two_sum(float a, float b, float &e)
 }
 
 // +1: a > b for certain; -1: a < b for certain (a <= b in the fp64 sense);
-// 0: too close to call from fp32 values with relative errors below ~1e-6.
+// 0: too close to call.  Near a == b the tolerance is 8e-6 relative, which
+// covers the operands' combined relative error (at most ~6e-6 where it is
+// used).
 __device__ __forceinline__ int certain_cmp(float a, float b)
 {
     float d = a - b;
