@@ -213,10 +213,11 @@ CIS_API cis_status_t cis_token_logprobs(const void *logits, int32_t dtype, int64
  *   eps_out   device float [T] or NULL: the log-odds displacement
  *             eps = logit p - logit q (Lemma 3.1); +-inf or NaN where p or q
  *             rounds to 1 (the weight itself stays finite).
- * Decisions are taken on log k = lp_train - lp_infer, evaluated exactly: CIS,
- * TIS and EXACT compare with log cap in fp32 where its error bound proves the
- * answer and in fp64 otherwise; the band, IcePop, KPop and the sequence
- * operators (log K summed in fp64) decide in fp64.  Errors:
+ * Decisions are taken on log k = lp_train - lp_infer, evaluated exactly.  CIS
+ * compares k with the cap, and TIS and EXACT compare log k with the log of the
+ * bound.  Each is settled in fp32 where its error bound proves the answer, else
+ * in fp64.  The band, IcePop, KPop and the sequence operators (log K summed in
+ * fp64) decide in fp64.  Errors:
  * CIS_ERR_INVALID_ARG for NULL required pointers, T < 0, parameters outside
  * the ranges of cis_params_t, or a sequence operator without cu_seqlens.
  */
