@@ -102,7 +102,7 @@ def _load():
         lib.oracle_loss_scales.restype = None
         lib.oracle_loss_fwd_bwd.argtypes = [
             P, i32, i64, i64, i64, P, P, P, P, P, P, i64, ctypes.POINTER(OracleParams), P,
-            P, i64, P, P, P, P, P, P, P, P, ctypes.c_int]
+            P, i64, P, P, P, P, P, P, P, P, P, P, ctypes.c_int]
         lib.oracle_loss_fwd_bwd.restype = ctypes.c_int
         lib.oracle_token_entropy.argtypes = [P, i32, i64, i64, i64, P, P, ctypes.c_int]
         lib.oracle_token_entropy.restype = None
@@ -240,8 +240,13 @@ def loss_fwd_bwd(logits, ids, lp_inf, adv, P: OracleParams, V=None, lp_old=None,
     """Weighted PPO-clipped token loss (Eq. 1, Algorithm 1) and d loss / d logits, fp64.
 
     ``rows``: indices of the rows whose dz is returned (None = all rows).
-    Returns a dict with loss, terms, lp, lse, w, trunc, c, dz ([len(rows), V] or
-    [T, V]) and rc (0, or -1 when a valid row has an out-of-range id).  The
+    Returns a dict with loss, terms, lp, lse, w, trunc, c, logk, dz
+    ([len(rows), V] or [T, V]), stats and rc (0, or -1 when a valid row has an
+    out-of-range id).  ``stats`` holds the batch statistics App. D logs and
+    Lemma B.2's truncated excess: n_valid, n_truncated (valid tokens whose
+    weight the operator changed), max_abs_logk (max over valid tokens of
+    |log k|, tokens whose log k is not a number left out) and trunc_excess
+    (sum over truncated tokens of k - w, k the token's own ratio).  The
     sequence operators need ``cu_seqlens``.
     """
     lib = _load()
@@ -259,17 +264,21 @@ def loss_fwd_bwd(logits, ids, lp_inf, adv, P: OracleParams, V=None, lp_old=None,
     rows_a = None if rows is None else np.ascontiguousarray(rows, dtype=np.int64)
     nrows = T if rows_a is None else rows_a.shape[0]
     dz = np.zeros((nrows, V), np.float64) if want_dz else None
-    out = {k: np.zeros(T, np.float64) for k in ("lp", "lse", "w", "terms", "c")}
+    out = {k: np.zeros(T, np.float64) for k in ("lp", "lse", "w", "terms", "c", "logk")}
     trunc = np.zeros(T, np.uint8)
     loss = ctypes.c_double(0.0)
+    stats = np.zeros(4, np.float64)
     rc = lib.oracle_loss_fwd_bwd(
         _ptr(a), dt, T, V, ld, _ptr(ids), _ptr(lp_inf), _ptr(lp_old), _ptr(adv), _ptr(mask),
         _ptr(cu), B, ctypes.byref(P), _ptr(w_fixed), _ptr(rows_a), nrows if rows_a is not None
         else 0, _ptr(dz), _ptr(out["lp"]), _ptr(out["lse"]), _ptr(out["w"]), _ptr(trunc),
-        _ptr(out["terms"]), _ptr(out["c"]), ctypes.byref(loss), nthreads)
+        _ptr(out["terms"]), _ptr(out["c"]), ctypes.byref(loss), _ptr(out["logk"]), _ptr(stats),
+        nthreads)
     if rc == -3:
         raise ValueError("a sequence operator needs cu_seqlens")
-    out.update(loss=loss.value, trunc=trunc, dz=dz, rc=rc)
+    out.update(loss=loss.value, trunc=trunc, dz=dz, rc=rc,
+               stats=dict(n_valid=int(stats[0]), n_truncated=int(stats[1]),
+                          max_abs_logk=float(stats[2]), trunc_excess=float(stats[3])))
     return out
 
 

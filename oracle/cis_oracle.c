@@ -474,7 +474,20 @@ void oracle_loss_scales(const uint8_t *mask, int64_t T, const int32_t *cu_seqlen
  * may be NULL.  w_fixed replaces the computed weights (used to freeze them for
  * finite differences).  dz is written for the rows listed in `rows` (nrows of
  * them, dz_out is [nrows, V]); rows == NULL means every row (dz_out [T, V]).
- * Per-token outputs (lp, lse, w, trunc, loss_terms, c) are for all T rows.
+ * Per-token outputs (lp, lse, w, trunc, loss_terms, c, logk) are for all T
+ * rows; logk_out and stats_out may be NULL.
+ *
+ * stats_out[0..3] are the batch statistics the paper logs while training
+ * (App. D: how many tokens the correction acted on, the largest |log k_t|)
+ * and the truncated excess of Lemma B.2 (k - f, the ratio mass a capped
+ * token loses):
+ *   [0] n_valid      number of valid tokens;
+ *   [1] n_truncated  valid tokens whose weight the operator changed;
+ *   [2] max_abs_logk max over valid tokens of |log k_t|, log k_t = l_w - l_inf
+ *                    (a token whose log k is not a number -- an out-of-range
+ *                    id, a NaN logit -- is left out; 0 when none is left);
+ *   [3] trunc_excess sum over truncated tokens of (k_t - w_t), k_t = exp(log
+ *                    k_t) the token's own ratio, in index order.
  * Returns 0, -1 if a valid row has an out-of-range id, -3 for a sequence
  * operator without cu_seqlens.
  */
@@ -484,7 +497,8 @@ int oracle_loss_fwd_bwd(const void *logits, int dtype, int64_t T, int64_t V, int
                         int64_t B, const oracle_params_t *P, const double *w_fixed,
                         const int64_t *rows, int64_t nrows, double *dz_out, double *lp_out,
                         double *lse_out, double *w_out, uint8_t *trunc_out,
-                        double *loss_terms, double *c_out, double *loss_out, int nthreads)
+                        double *loss_terms, double *c_out, double *loss_out, double *logk_out,
+                        double *stats_out, int nthreads)
 {
     size_t nT = (size_t)(T > 0 ? T : 1);
     double *s = (double *)malloc(sizeof(double) * nT);
@@ -504,7 +518,8 @@ int oracle_loss_fwd_bwd(const void *logits, int dtype, int64_t T, int64_t V, int
     double *wv = (double *)malloc(sizeof(double) * nT);
     uint8_t *trv = (uint8_t *)malloc(nT);
     uint8_t *badv = (uint8_t *)malloc(nT);
-    if (!lpv || !lwv || !wv || !trv || !badv) {
+    double *lkv = (double *)malloc(sizeof(double) * nT);
+    if (!lpv || !lwv || !wv || !trv || !badv || !lkv) {
         free(s);
         free(lse);
         free(cc);
@@ -514,6 +529,7 @@ int oracle_loss_fwd_bwd(const void *logits, int dtype, int64_t T, int64_t V, int
         free(wv);
         free(trv);
         free(badv);
+        free(lkv);
         return -2;
     }
     int bad = 0;
@@ -540,7 +556,7 @@ int oracle_loss_fwd_bwd(const void *logits, int dtype, int64_t T, int64_t V, int
         lwv[t] = lp_old ? lp_old[t] : lp;
     }
     /* 2. the weights (Algorithm 1 / Table 8), per token or per response */
-    int rc = weights_impl(lwv, lp_inf, mask, badv, T, cu_seqlens, B, P, wv, trv, NULL, NULL);
+    int rc = weights_impl(lwv, lp_inf, mask, badv, T, cu_seqlens, B, P, wv, trv, lkv, NULL);
     if (rc != 0) {
         free(s);
         free(lse);
@@ -551,6 +567,7 @@ int oracle_loss_fwd_bwd(const void *logits, int dtype, int64_t T, int64_t V, int
         free(wv);
         free(trv);
         free(badv);
+        free(lkv);
         return rc == -1 ? -3 : -2;
     }
     /* 3. the token terms of Eq. 1 and c_t */
@@ -587,12 +604,40 @@ int oracle_loss_fwd_bwd(const void *logits, int dtype, int64_t T, int64_t V, int
             w_out[t] = w;
         if (trunc_out)
             trunc_out[t] = (uint8_t)tr;
+        wv[t] = w;
+        trv[t] = (uint8_t)tr;
+    }
+    /* 4. the batch statistics (App. D training statistics; Lemma B.2's k - f),
+     * over the valid tokens in index order */
+    {
+        double n_valid = 0.0, n_trunc = 0.0, max_abs = 0.0, excess = 0.0;
+        for (int64_t t = 0; t < T; ++t) {
+            if (!row_valid(mask, t))
+                continue;
+            n_valid += 1.0;
+            if (!badv[t] && !isnan(lkv[t]) && fabs(lkv[t]) > max_abs)
+                max_abs = fabs(lkv[t]);
+            if (trv[t]) {
+                n_trunc += 1.0;
+                excess += exp(lkv[t]) - wv[t];
+            }
+        }
+        if (stats_out) {
+            stats_out[0] = n_valid;
+            stats_out[1] = n_trunc;
+            stats_out[2] = max_abs;
+            stats_out[3] = excess;
+        }
+        if (logk_out)
+            for (int64_t t = 0; t < T; ++t)
+                logk_out[t] = !row_valid(mask, t) ? 0.0 : (badv[t] ? NAN : lkv[t]);
     }
     free(lpv);
     free(lwv);
     free(wv);
     free(trv);
     free(badv);
+    free(lkv);
     /* loss = -sum_t s_t J_t, summed in index order. */
     double loss = 0.0;
     for (int64_t t = 0; t < T; ++t)

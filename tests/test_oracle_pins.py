@@ -317,6 +317,107 @@ def test_loss_closed_forms():
     assert out["loss"] == pytest.approx(2.0, rel=1e-13)  # A < 0: min picks rho*A = -2
 
 
+
+# ---------------------------------------------------------------- batch statistics
+def test_stats_lemma_b2_sum_and_displacement_count():
+    """The batch statistics of the pass (App. D logs how many tokens the
+    correction acts on and the largest |log k|; Lemma B.2 gives the ratio
+    mass a capped token loses).  With kappa = 0, Lemma B.2 gives
+    k - f = (1 - p)(e^eps - 1 - lambda)_+ per token, so the summed truncated
+    excess is that sum over the valid tokens, and a token is truncated exactly
+    when e^eps > 1 + lambda (Eq. 4's threshold).  p comes from a library
+    log-softmax of the logits, eps = logit p - logit q from the two
+    probabilities: neither the cap nor the truncation flag enters."""
+    from scipy.special import log_softmax
+    rng = _rng(70)
+    T, V, lam = 400, 40, 2.3
+    z = (rng.standard_normal((T, V)) * 2.5).astype(np.float32)
+    ids = rng.integers(0, V, T).astype(np.int32)
+    lp = log_softmax(z.astype(np.float64), axis=1)[np.arange(T), ids]
+    lq = np.minimum(lp + rng.standard_normal(T) * 1.2, -1e-6)
+    mask = (rng.random(T) > 0.15).astype(np.uint8)
+    out = oracle.loss_fwd_bwd(z, ids, lq, rng.standard_normal(T),
+                              oracle.params(lam=lam, kappa=0.0), mask=mask, want_dz=False)
+    st = out["stats"]
+    v = mask == 1
+    p, q = np.exp(lp), np.exp(lq)
+    eps = (lp - np.log1p(-p)) - (lq - np.log1p(-q))
+    excess = ((1 - p) * np.maximum(np.exp(eps) - 1 - lam, 0.0))[v].sum()
+    assert st["n_valid"] == int(v.sum())
+    assert st["n_truncated"] == int((np.exp(eps) > 1 + lam)[v].sum())
+    assert 20 < st["n_truncated"] < v.sum() - 20
+    assert st["trunc_excess"] == pytest.approx(excess, rel=1e-9)
+    assert st["max_abs_logk"] == pytest.approx(np.abs(lp - lq)[v].max(), rel=1e-12)
+    assert np.abs(np.abs(lp - lq)[~v]).max() > 0  # masked tokens would change nothing otherwise
+
+
+def _two_logit_batch(k_targets, x=0.0):
+    """Rows of two logits [0, x] with the sampled id 0 (p = 1/(1 + e^x)) and
+    an inference log-prob that puts the ratio k at each target."""
+    T = len(k_targets)
+    z = np.tile(np.array([0.0, x], np.float32), (T, 1))
+    lp = -math.log1p(math.exp(x))
+    lq = lp - np.log(np.asarray(k_targets, np.float64))
+    return z, np.zeros(T, np.int32), lq, lp
+
+
+@pytest.mark.parametrize("with_old", [False, True])
+@pytest.mark.parametrize("case", ["tis", "exact", "icepop", "band", "none"])
+def test_stats_hand_built_batches(case, with_old):
+    """Batches with known counts: which tokens an operator changes (Table 8,
+    Sec. 4.3), the excess k - w they lose (negative when the band lifts a
+    token or the exact ratio is clamped from below), masked tokens and a token
+    with an out-of-range id left out of everything but n_valid (with l_old
+    given, that token's log k is a finite number and must still be left
+    out)."""
+    if case == "tis":       # C = 2
+        ks, P = [3.0, 1.5, 5.0, 100.0, 0.25], oracle.params(mode=oracle.MODE_TIS)
+        want = dict(n_truncated=2, trunc_excess=(3 - 2) + (5 - 2), max_abs_logk=math.log(5.0))
+    elif case == "exact":   # clamp to [1e-6, 1e6]
+        ks, P = [1e7, 1e-7, 2.0, 100.0, 0.5], oracle.params(mode=oracle.MODE_EXACT)
+        want = dict(n_truncated=2, trunc_excess=(1e7 - 1e6) + (1e-7 - 1e-6),
+                    max_abs_logk=math.log(1e7))
+    elif case == "icepop":  # kept on [0.5, 5], else 0
+        ks, P = [0.25, 6.0, 1.0, 100.0, 5.0], oracle.params(mode=oracle.MODE_ICEPOP)
+        want = dict(n_truncated=2, trunc_excess=0.25 + 6.0, max_abs_logk=math.log(6.0))
+    elif case == "band":    # p = 1/2: cap 1 + 2.3/2 = 2.15, floor (1 + 1/2)/2 = 0.75
+        ks, P = [0.5, 3.0, 1.0, 100.0, 2.0], oracle.params(mode=oracle.MODE_BAND, lam=2.3)
+        want = dict(n_truncated=2, trunc_excess=(0.5 - 0.75) + (3.0 - 2.15),
+                    max_abs_logk=math.log(3.0))
+    else:
+        ks, P = [3.0, 0.1, 1.0, 100.0, 2.0], oracle.params(mode=oracle.MODE_NONE)
+        want = dict(n_truncated=0, trunc_excess=0.0, max_abs_logk=math.log(10.0))
+    ks = ks + [1e6]  # the last token's id is out of range
+    z, ids, lq, lp = _two_logit_batch(ks)
+    ids[-1] = 7
+    mask = np.array([1, 1, 1, 0, 1, 1], np.uint8)  # k = 100 is masked
+    lp_old = np.full(len(ks), lp) if with_old else None
+    out = oracle.loss_fwd_bwd(z, ids, lq, np.ones(len(ks)), P, mask=mask, lp_old=lp_old,
+                              want_dz=False)
+    assert out["rc"] == -1  # the out-of-range id is reported
+    st = out["stats"]
+    assert st["n_valid"] == 5
+    assert st["n_truncated"] == want["n_truncated"]
+    assert st["trunc_excess"] == pytest.approx(want["trunc_excess"], rel=1e-12, abs=1e-15)
+    assert st["max_abs_logk"] == pytest.approx(want["max_abs_logk"], rel=1e-12)
+
+
+def test_stats_sequence_operator_reading():
+    """Under Seq-TIS every valid token of a response whose K exceeds C is
+    flagged and carries w = C; the excess adds each such token's own ratio
+    minus C.  One response with k = 2, 1.5, 1 (K = 3 > 2) and one with
+    k = 1.2, 0.5 (K = 0.6)."""
+    z, ids, lq, _ = _two_logit_batch([2.0, 1.5, 1.0, 1.2, 0.5])
+    cu = np.array([0, 3, 5], np.int32)
+    out = oracle.loss_fwd_bwd(z, ids, lq, np.ones(5), oracle.params(mode=oracle.MODE_SEQ_TIS),
+                              cu_seqlens=cu, want_dz=False)
+    st = out["stats"]
+    assert out["trunc"].tolist() == [1, 1, 1, 0, 0]
+    assert st["n_truncated"] == 3
+    assert st["trunc_excess"] == pytest.approx((2 - 2) + (1.5 - 2) + (1 - 2), rel=1e-12)
+    assert st["max_abs_logk"] == pytest.approx(math.log(2.0), rel=1e-12)
+
+
 def _fd_setup(seed, T, V):
     rng = _rng(seed)
     z = (rng.integers(-128, 128, (T, V)) / 32).astype(np.float32)  # exact fp32 +- 2^-16
