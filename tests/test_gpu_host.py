@@ -46,3 +46,5 @@ def test_host_path_equals_device_path(cfg, T, V, chunk, agg):
     assert float(out["loss"][0]) == float(ref["loss"].cpu()[0])
     st = binding.decode_stats(out["stats"])
     assert st["status"] == 0 and st["n_valid"] == int(b.mask.sum())
+    # the batch statistics are reduced once over the whole batch, as on the device
+    assert st == binding.decode_stats(ref["stats"])

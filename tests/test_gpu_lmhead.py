@@ -20,6 +20,7 @@ import torch
 import oracle
 from _util import bf16_tensor_bits
 from paper_2609_32444_gb300 import binding, synth
+from test_gpu_parity import check_stats
 
 pytestmark = [pytest.mark.gpu,
               pytest.mark.skipif(not torch.cuda.is_available(), reason="needs a CUDA GPU")]
@@ -74,6 +75,7 @@ def _check_tokens(out, ref, rows, b, mode, full):
     if full:
         loss = float(out["loss"].cpu()[0])
         assert abs(loss - ref["loss"]) <= 1e-5 * np.abs(ref["terms"]).sum() + 1e-300
+        check_stats(out["stats"], ref, li, band=band, tr_gpu=tr)
 
 
 def _check_grad(got, want, want_abs, K, bf16_out):

@@ -22,7 +22,7 @@ import torch
 import oracle
 from _util import logits_for_oracle
 from paper_2609_32444_gb300 import binding, synth
-from test_gpu_parity import (DEV, TOL_LOSS, TOL_W, check_dz, lp_tol, to_dev)
+from test_gpu_parity import (DEV, TOL_LOSS, TOL_W, check_dz, check_stats, lp_tol, to_dev)
 
 pytestmark = [pytest.mark.gpu,
               pytest.mark.skipif(not torch.cuda.is_available(), reason="needs a CUDA GPU")]
@@ -174,6 +174,8 @@ def _check(out, ref, b, mode, lp_old=None, width=4e-5, rows_dz=None):
     if not band.any():
         loss = float(out["loss"].cpu()[0])
         assert abs(loss - ref["loss"]) <= TOL_LOSS * np.abs(ref["terms"]).sum() + 1e-300
+        check_stats(out["stats"], ref, li, lp_old=None if lp_old is None else
+                    lp_old.cpu().numpy(), band=band, tr_gpu=tr)
         if rows_dz is None:
             check_dz(out["dlogits"], ref["dz"], ref["c"])
         else:

@@ -16,7 +16,14 @@ need one):
     terms cancel; the bound is relative to the terms' scale);
   - fp32 dlogits: 1e-6 absolute for rows with |c_t| <= 1 and 1e-6 |c_t| above
     (dz_tj lies in [-|c_t|, |c_t|]); bf16 dlogits: at most 1 bf16 step from the
-    oracle's value rounded once to bf16 (nearest, ties to even).
+    oracle's value rounded once to bf16 (nearest, ties to even);
+  - batch statistics (App. D's logged counts, Lemma B.2's excess): n_valid
+    exact; n_truncated exact, or off by at most the number of tokens inside
+    the decision band; max |log k| within the largest per-token error of
+    log k = l_w - l_inf (the log p tolerance of l_w, plus an fp32 rounding of
+    the difference); the excess within the per-token error of k (that log
+    error, times k) and of w (1e-5 relative), summed over the tokens either
+    side flags, plus BAND k for each token whose decision differs.
 """
 import math
 
@@ -90,6 +97,44 @@ def decision_band(ref, lp_inf, mode, lam, kappa=5e-3, lp_old=None):
     return dist < BAND
 
 
+def check_stats(stats_dev, ref, lp_inf, lp_old=None, band=None, tr_gpu=None):
+    """The device cis_stats_t against the oracle's batch statistics.  `band`
+    marks tokens whose decision may legitimately differ; `tr_gpu` is the
+    GPU's per-token flag (needed when the band is not empty)."""
+    st = binding.decode_stats(stats_dev)
+    rs = ref["stats"]
+    assert st["n_valid"] == rs["n_valid"]
+    nb = 0 if band is None else int(band.sum())
+    assert abs(st["n_truncated"] - rs["n_truncated"]) <= nb
+    if nb == 0:
+        assert st["n_truncated"] == rs["n_truncated"]
+    li = np.asarray(lp_inf, np.float64)
+    lw = ref["lp"] if lp_old is None else np.asarray(lp_old, np.float64)
+    lk = ref["logk"]
+    num = np.isfinite(lk)
+    # log k error: l_w's (none when l_old is given) plus one rounding of l_w - l_inf
+    lw_err = np.zeros_like(lw) if lp_old is not None else \
+        TOL_LP + 2.0 ** -21 * np.abs(np.nan_to_num(lw))
+    lk_err = lw_err + 2.0 ** -23 * (np.abs(np.nan_to_num(lk)) + 1e-30)
+    tol_max = float(lk_err[num].max()) if num.any() else 0.0
+    assert abs(st["max_abs_logk"] - rs["max_abs_logk"]) <= tol_max + 1e-30
+    tr_ref = ref["trunc"].astype(bool)
+    flagged = tr_ref if tr_gpu is None else (tr_ref | np.asarray(tr_gpu).astype(bool))
+    flipped = np.zeros_like(tr_ref) if tr_gpu is None else \
+        (tr_ref != np.asarray(tr_gpu).astype(bool))
+    with np.errstate(over="ignore", invalid="ignore"):
+        k = np.exp(lk)
+        per = k * np.expm1(1.01 * lk_err) + TOL_W * np.abs(ref["w"]) + BAND * 1.01 * k * flipped
+    want = rs["trunc_excess"]
+    if not np.isfinite(want):
+        assert st["trunc_excess"] == want
+    else:
+        tol = float(per[flagged & num].sum())
+        assert abs(st["trunc_excess"] - want) <= tol + 1e-300, \
+            f"excess {st['trunc_excess']} vs {want} (tol {tol})"
+    return st
+
+
 def check_token_outputs(out, ref, b, mode, lam, lp_old=None, use_mask=True):
     mask = b.mask.cpu().numpy().astype(bool) if use_mask else np.ones(b.T, bool)
     lp = out["lp"].cpu().numpy().astype(np.float64)
@@ -106,6 +151,10 @@ def check_token_outputs(out, ref, b, mode, lam, lp_old=None, use_mask=True):
     mismatch = (tr != ref["trunc"]) & ~band
     assert not mismatch.any(), f"{mismatch.sum()} truncation decisions differ outside the band"
     assert not np.any(tr[~mask]) and np.all(w[~mask] == 0)
+    if "stats" in out:
+        check_stats(out["stats"], ref, b.lp_infer.cpu().numpy(),
+                    lp_old=None if lp_old is None else lp_old.cpu().numpy(), band=band,
+                    tr_gpu=tr)
     loss = float(out["loss"].cpu()[0])
     if np.isnan(ref["loss"]):
         assert np.isnan(loss)
