@@ -426,9 +426,11 @@ CIS_API cis_status_t cis_mismatch_diagnostics(const void *logits_train, const vo
  *     memory, sized for CIS_NOALLOC_MAX_TOKENS tokens; every GPU that loads the
  *     library keeps one until the process exits.  T > CIS_NOALLOC_MAX_TOKENS
  *     returns CIS_ERR_UNSUPPORTED before any GPU work.
- *   - The first call on a device looks the array's device address up
- *     (cudaGetSymbolAddress) with that device current; make that first call
- *     before any stream capture on that device.
+ *   - Every call looks the array's device address up (cudaGetSymbolAddress)
+ *     in the calling thread's current context, so a context that was reset or
+ *     replaced since the last call is never written through a stale address.
+ *     The first lookup on a device may load the library's device code there:
+ *     make the first call on each device before any stream capture on it.
  *   - No allocating routine is called.
  *   - All calls share the array.  Each call resets the status word and
  *     overwrites everything else it reads, so sequential calls are

@@ -8,33 +8,9 @@
 #include <stdlib.h>
 
 #include "cis_kernels.h"
+#include "cis_nvtx.h"
 
 namespace cis {
-
-WsLayout ws_layout(int64_t T)
-{
-    auto up = [](size_t x) { return (x + 255) / 256 * 256; };
-    const size_t n = (size_t)(T > 0 ? T : 0);
-    WsLayout L;
-    size_t o = 0;
-    L.status = o;
-    L.ticket = o + 64;
-    o += 256;
-    L.scale = o;
-    o = up(o + 4 * n);
-    L.terms = o;
-    o = up(o + 8 * n);
-    L.logk = o;
-    o = up(o + 4 * n);
-    L.w = o;
-    o = up(o + 4 * n);
-    L.trunc = o;
-    o = up(o + n);
-    L.parts = o;
-    o = up(o + (size_t)kRedPartBytes * ((n + kRedTokens - 1) / kRedTokens + (n == 0)));
-    L.total = o;
-    return L;
-}
 
 static bool finite_or_inf_nonneg(double x) { return x == x && x >= 0.0; }
 
@@ -157,6 +133,7 @@ CIS_API cis_status_t cis_default_params(cis_params_t *out)
 CIS_API cis_status_t cis_count_valid(const uint8_t *mask, int64_t T, const int32_t *cu_seqlens,
                                      int64_t B, int64_t *counts_out, void *stream)
 {
+    NvtxRange nvtx_range("cis_count_valid");
     if (T < 0 || B < 0 || counts_out == nullptr || (cu_seqlens == nullptr && B > 0))
         return CIS_ERR_INVALID_ARG;
     const cudaError_t e = launch_count_valid(mask, T, cu_seqlens, B, counts_out,
@@ -185,6 +162,7 @@ CIS_API cis_status_t cis_token_logprobs(const void *logits, int32_t dtype, int64
                                         float *lp_out, float *lse_out, float *entropy_out,
                                         int32_t *dev_status, void *stream)
 {
+    NvtxRange nvtx_range("cis_token_logprobs");
     if (!shape_ok(T, V, ld) || !dtype_ok(dtype))
         return CIS_ERR_INVALID_ARG;
     if (T == 0)
@@ -210,6 +188,7 @@ CIS_API cis_status_t cis_weights(const float *lp_train, const float *lp_infer,
                                  int64_t B, const cis_params_t *params, float *w_out,
                                  uint8_t *trunc_out, float *eps_out, void *stream)
 {
+    NvtxRange nvtx_range("cis_weights");
     if (T < 0 || !params_ok(params))
         return CIS_ERR_INVALID_ARG;
     const bool seq = is_seq_mode(params->mode);
@@ -249,6 +228,7 @@ CIS_API cis_status_t cis_loss_fwd_bwd(const void *logits, int32_t dtype, int64_t
                                       cis_stats_t *stats_out, double *loss_out, void *workspace,
                                       size_t workspace_bytes, void *stream)
 {
+    NvtxRange nvtx_range("cis_loss_fwd_bwd");
     if (!shape_ok(T, V, ld) || ld_out < V || !dtype_ok(dtype) || !dtype_ok(dlogits_dtype))
         return CIS_ERR_INVALID_ARG;
     if (!params_ok(params))

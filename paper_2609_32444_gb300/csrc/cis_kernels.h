@@ -53,7 +53,30 @@ struct WsLayout {
 };
 constexpr int kRedTokens = 256;  // tokens per CTA of the reduction
 constexpr int kRedPartBytes = 64;
-WsLayout ws_layout(int64_t T);
+constexpr size_t ws_round_up(size_t x) { return (x + 255) / 256 * 256; }
+constexpr WsLayout ws_layout(int64_t T)
+{
+    const size_t n = (size_t)(T > 0 ? T : 0);
+    WsLayout L{};
+    size_t o = 0;
+    L.status = o;
+    L.ticket = o + 64;
+    o += 256;
+    L.scale = o;
+    o = ws_round_up(o + 4 * n);
+    L.terms = o;
+    o = ws_round_up(o + 8 * n);
+    L.logk = o;
+    o = ws_round_up(o + 4 * n);
+    L.w = o;
+    o = ws_round_up(o + 4 * n);
+    L.trunc = o;
+    o = ws_round_up(o + n);
+    L.parts = o;
+    o = ws_round_up(o + (size_t)kRedPartBytes * ((n + kRedTokens - 1) / kRedTokens + (n == 0)));
+    L.total = o;
+    return L;
+}
 
 // Sequence operators: w[t], trunc[t] for the valid tokens of each response
 // from the fp64 sum of log k = lw - lp_inf over its valid tokens with an id

@@ -13,47 +13,33 @@
 // the library holds one copy until the process exits.  All calls share it:
 // the status word is reset at the start of every call and every other byte is
 // written before it is read, but two calls whose GPU work overlaps race.
-#include <mutex>
-
 #include "cis_kernels.h"
+#include "cis_nvtx.h"
 
 namespace cis {
 namespace {
 
 constexpr int64_t kMaxTokens = CIS_NOALLOC_MAX_TOKENS;
 
-// Bytes ws_layout() asks for at kMaxTokens: a 256-byte status block, then the
-// scale (4 B), term (8 B), log k (4 B), weight (4 B) and flag (1 B) arrays,
-// each rounded up to 256 bytes, and the reduction's partial sums (64 B per
-// 256 tokens).
-constexpr size_t kScratchBytes = 256 + 4 * kMaxTokens + 8 * kMaxTokens + 4 * kMaxTokens +
-                                 4 * kMaxTokens + 1 * kMaxTokens +
-                                 kRedPartBytes * ((kMaxTokens + kRedTokens - 1) / kRedTokens);
+// Exactly what cis_loss_fwd_bwd asks of a workspace for kMaxTokens tokens.
+constexpr size_t kScratchBytes = ws_layout(kMaxTokens).total;
+static_assert(kScratchBytes % 256 == 0, "the scratch is a whole number of 256-byte blocks");
 
 // The scratch itself.  In host code this name is only a host-side stand-in:
-// its device address is looked up per device with cudaGetSymbolAddress.
+// its device address is looked up with cudaGetSymbolAddress.
 static __device__ __align__(256) uint8_t g_scratch[kScratchBytes];
 
-constexpr int kMaxDevices = 64;
-std::mutex g_lock;
-void *g_scratch_addr[kMaxDevices] = {};
-
-// Device address of g_scratch on the current device (looked up once per device).
+// Device address of g_scratch in the current context.  Looked up on every
+// call, not cached: a cached address would outlive a context that a caller
+// tears down (cudaDeviceReset) or swaps for another on the same device, and
+// the next call would then write through a dangling pointer.  The lookup is a
+// host-side query; it allocates nothing.
 cis_status_t scratch_address(void **out)
 {
-    int dev = -1;
-    if (cudaGetDevice(&dev) != cudaSuccess)
+    void *p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_scratch) != cudaSuccess || p == nullptr)
         return CIS_ERR_CUDA;
-    if (dev < 0 || dev >= kMaxDevices)
-        return CIS_ERR_UNSUPPORTED;
-    std::lock_guard<std::mutex> guard(g_lock);
-    if (g_scratch_addr[dev] == nullptr) {
-        void *p = nullptr;
-        if (cudaGetSymbolAddress(&p, g_scratch) != cudaSuccess || p == nullptr)
-            return CIS_ERR_CUDA;
-        g_scratch_addr[dev] = p;
-    }
-    *out = g_scratch_addr[dev];
+    *out = p;
     return CIS_OK;
 }
 
@@ -69,9 +55,8 @@ extern "C" CIS_API cis_status_t cis_loss_fwd_bwd_noalloc(
     int32_t dlogits_dtype, int64_t ld_out, float *lp_out, float *w_out, uint8_t *trunc_out,
     float *entropy_out, cis_stats_t *stats_out, double *loss_out, void *stream)
 {
+    NvtxRange nvtx_range("cis_loss_fwd_bwd_noalloc");
     if (T > kMaxTokens)
-        return CIS_ERR_UNSUPPORTED;
-    if (ws_layout(T < 0 ? 0 : T).total > kScratchBytes)
         return CIS_ERR_UNSUPPORTED;
     void *scratch = nullptr;
     const cis_status_t st = scratch_address(&scratch);
