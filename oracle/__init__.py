@@ -323,3 +323,80 @@ def lmhead_fwd_bwd(hidden, weight, ids, lp_inf, adv, P: OracleParams, lp_old=Non
         out["dweight_abs"] = np.abs(out["dz"]).T @ np.abs(Hf)
     out["logits"] = Z
     return out
+
+
+def lmhead_token_groups(hidden, weight, ids, lp_inf, adv, P: OracleParams, lp_old=None,
+                        mask=None, dh_rows=None, dw_rows=None, group=1024, nthreads=0):
+    """The token pass through the LM head for batches whose logits do not fit
+    in host memory at once (fp64 [T, V] is 20 GB at T=16384, V=151936).
+
+    The same definitions as lmhead_fwd_bwd: z = H W^T in fp64 (Sec. 2.1), the
+    token pass on those logits (Eq. 1, Algorithm 1, Table 8), and the chain
+    rule through z = H W^T for the gradients.  Rows are independent, so the
+    tokens are taken ``group`` at a time only to bound memory: each row's
+    logits and results are those of the whole-batch computation; the token-mean
+    normaliser uses the whole batch's count (n_global).
+
+    Returns the per-token outputs of every token (lp, lse, w, trunc, c, terms,
+    logk), the loss (their exact sum), the batch statistics, dH and |dz||W| on
+    ``dh_rows`` (tokens) and dW and |dz|^T|H| on ``dw_rows`` (vocabulary
+    rows): dW[v] = sum_t c_t (softmax_tv - [y_t = v]) H_t over every token.
+    Token operators and the token-mean normaliser only (a group does not hold
+    whole responses)."""
+    import math
+    if P.mode in SEQ_MODES or P.agg != AGG_TOKEN_MEAN:
+        raise ValueError("token operators and the token-mean normaliser only")
+    Hf = bf16_bits_to_f64(hidden) if np.asarray(hidden).dtype == np.uint16 else \
+        np.asarray(hidden, np.float64)
+    Wf = bf16_bits_to_f64(weight) if np.asarray(weight).dtype == np.uint16 else \
+        np.asarray(weight, np.float64)
+    T = Hf.shape[0]
+    ids = np.asarray(ids, np.int32)
+    m = np.ones(T, np.uint8) if mask is None else np.asarray(mask, np.uint8)
+    n_valid = int(m.sum())
+    Pg = OracleParams.from_buffer_copy(P)
+    Pg.n_global = n_valid if P.n_global == 0 else P.n_global
+    keys = ("lp", "lse", "w", "c", "terms", "logk")
+    out = {k: np.zeros(T, np.float64) for k in keys}
+    out["trunc"] = np.zeros(T, np.uint8)
+    st = dict(n_valid=0, n_truncated=0, max_abs_logk=0.0, trunc_excess=0.0)
+    rc = 0
+    for g0 in range(0, T, group):
+        g1 = min(T, g0 + group)
+        Z = Hf[g0:g1] @ Wf.T
+        r = loss_fwd_bwd(Z, ids[g0:g1], np.asarray(lp_inf)[g0:g1], np.asarray(adv)[g0:g1], Pg,
+                         lp_old=None if lp_old is None else np.asarray(lp_old)[g0:g1],
+                         mask=m[g0:g1], want_dz=False, nthreads=nthreads)
+        del Z
+        for k in keys + ("trunc",):
+            out[k][g0:g1] = r[k]
+        rs = r["stats"]
+        st["n_valid"] += rs["n_valid"]
+        st["n_truncated"] += rs["n_truncated"]
+        st["max_abs_logk"] = max(st["max_abs_logk"], rs["max_abs_logk"])
+        st["trunc_excess"] += rs["trunc_excess"]
+        rc = rc or r["rc"]
+    out["loss"] = math.fsum(out["terms"])
+    out["stats"] = st
+    out["rc"] = rc
+
+    def dz_of(Zs, tok, cols):
+        """dz[t, v] = c_t (exp(z_tv - lse_t) - [y_t = v]) for tokens tok, columns cols."""
+        onehot = (ids[tok][:, None] == np.asarray(cols)[None, :]).astype(np.float64)
+        c = out["c"][tok][:, None]
+        live = (c != 0.0) & np.isfinite(out["lse"][tok])[:, None]  # masked rows: dz = 0
+        with np.errstate(over="ignore", invalid="ignore"):
+            d = c * (np.exp(Zs - out["lse"][tok][:, None]) - onehot)
+        return np.where(live, d, 0.0)
+
+    if dh_rows is not None:
+        rows = np.asarray(dh_rows, np.int64)
+        dz = dz_of(Hf[rows] @ Wf.T, rows, np.arange(Wf.shape[0]))
+        out["dhidden"] = dz @ Wf
+        out["dhidden_abs"] = np.abs(dz) @ np.abs(Wf)
+    if dw_rows is not None:
+        vs = np.asarray(dw_rows, np.int64)
+        dz = dz_of(Hf @ Wf[vs].T, np.arange(T), vs)
+        out["dweight"] = dz.T @ Hf
+        out["dweight_abs"] = np.abs(dz).T @ np.abs(Hf)
+    return out

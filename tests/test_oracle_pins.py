@@ -547,6 +547,46 @@ def test_lmhead_chain_rule_matches_finite_differences():
     np.testing.assert_allclose(base["dweight"], fdW, rtol=0, atol=1e-8 * scale)
 
 
+
+@pytest.mark.parametrize("mode", [oracle.MODE_CIS, oracle.MODE_TIS, oracle.MODE_EXACT])
+def test_lmhead_token_groups_is_the_whole_batch_computation(mode):
+    """The grouped LM-head oracle (tokens taken a few at a time, for batches
+    whose fp64 logits do not fit in memory) gives the per-token outputs, loss,
+    statistics, dH rows and dW rows of the finite-difference-pinned
+    whole-batch computation: grouping rows changes no row's arithmetic."""
+    rng = _rng(31)
+    T, Hd, V = 37, 16, 53
+    Hm = rng.standard_normal((T, Hd))
+    Wm = rng.standard_normal((V, Hd)) * 0.7
+    ids = rng.integers(0, V, T)
+    z0 = Hm @ Wm.T
+    lp0 = _log_softmax(z0)[np.arange(T), ids]
+    lp_inf = lp0 + rng.standard_normal(T) * 0.8
+    adv = rng.standard_normal(T)
+    mask = (rng.random(T) > 0.2).astype(np.uint8)
+    lp_old = lp0 - rng.normal(0.0, 0.2, T)
+    P = oracle.params(mode=mode)
+    for old in (None, lp_old):
+        whole = oracle.lmhead_fwd_bwd(Hm, Wm, ids, lp_inf, adv, P, lp_old=old, mask=mask)
+        dw_rows = np.array([0, 5, int(ids[3]), V - 1])
+        grp = oracle.lmhead_token_groups(Hm, Wm, ids, lp_inf, adv, P, lp_old=old, mask=mask,
+                                         dh_rows=np.arange(T), dw_rows=dw_rows, group=5)
+        for k in ("lp", "lse", "w", "c", "terms"):
+            np.testing.assert_allclose(grp[k], whole[k], rtol=1e-12, atol=1e-300)
+        assert np.array_equal(grp["trunc"], whole["trunc"])
+        assert grp["loss"] == pytest.approx(whole["loss"], rel=1e-12)
+        for k in ("n_valid", "n_truncated"):
+            assert grp["stats"][k] == whole["stats"][k]
+        for k in ("max_abs_logk", "trunc_excess"):
+            assert grp["stats"][k] == pytest.approx(whole["stats"][k], rel=1e-12, abs=1e-300)
+        sc = np.abs(whole["dweight"]).max()
+        np.testing.assert_allclose(grp["dhidden"], whole["dhidden"], rtol=0, atol=1e-12 * sc)
+        np.testing.assert_allclose(grp["dweight"], whole["dweight"][dw_rows], rtol=0,
+                                   atol=1e-12 * sc)
+        np.testing.assert_allclose(grp["dweight_abs"], whole["dweight_abs"][dw_rows],
+                                   rtol=1e-12)
+
+
 # ---------------------------------------------- the other operators of Table 8
 def _from_p_eps(p, eps):
     """log p and log q of tokens with training probability p and log-odds
