@@ -36,6 +36,7 @@
 #include "cis_dsmem.cuh"
 #include "cis_kernels.h"
 #include "cis_rowops.cuh"
+#include "cis_nvtx.h"
 
 namespace cis {
 namespace {
@@ -809,6 +810,7 @@ extern "C" CIS_API cis_status_t cis_mismatch_diagnostics(
     const cis_params_t *params, float *eps_out, float *logk_out, float *p_out, float *bias2_out,
     float *dvar_out, int32_t *dev_status, void *stream)
 {
+    NvtxRange nvtx_range("cis_mismatch_diagnostics");
     if (T < 0 || T > 0x7fffffffLL || V <= 0 || V > 0x7fffffffLL || ld_train < V ||
         ld_infer < V || (dtype != CIS_F32 && dtype != CIS_BF16))
         return CIS_ERR_INVALID_ARG;

@@ -14,6 +14,7 @@
 #include <vector>
 
 #include "cis_kernels.h"
+#include "cis_nvtx.h"
 
 namespace cis {
 namespace {
@@ -115,6 +116,7 @@ CIS_API cis_status_t cis_loss_fwd_bwd_host(
     cis_stats_t *stats_out, double *loss_out, int64_t chunk_tokens, void *workspace,
     size_t workspace_bytes, void *stream)
 {
+    NvtxRange nvtx_range("cis_loss_fwd_bwd_host");
     if (T < 0 || T > 0x7fffffffLL || V <= 0 || chunk_tokens <= 0 ||
         (dtype != CIS_F32 && dtype != CIS_BF16) ||
         (dlogits_dtype != CIS_F32 && dlogits_dtype != CIS_BF16))

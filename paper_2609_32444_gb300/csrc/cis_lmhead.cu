@@ -44,6 +44,7 @@
 
 #include "cis_kernels.h"
 #include "cis_tc.cuh"
+#include "cis_nvtx.h"
 
 namespace cis {
 namespace lm {
@@ -737,6 +738,7 @@ CIS_API cis_status_t cis_lmhead_fused(const void *hidden, const void *weight, in
                                       cis_stats_t *stats_out, double *loss_out, void *workspace,
                                       size_t workspace_bytes, void *stream)
 {
+    NvtxRange nvtx_range("cis_lmhead_fused");
     if (T < 0 || T > (1LL << 30) || V <= 0 || V > (1LL << 30) || H <= 0 || H > (1LL << 20))
         return CIS_ERR_INVALID_ARG;
     if (grad_dtype != CIS_F32 && grad_dtype != CIS_BF16)

@@ -6,6 +6,7 @@
 // caller-chosen poll limit, and reports the timeout the same way.
 #include "cis_dsmem.cuh"
 #include "cis_kernels.h"
+#include "cis_nvtx.h"
 
 namespace cis {
 namespace {
@@ -31,6 +32,7 @@ using namespace cis;
 extern "C" CIS_API cis_status_t cis_selftest_bounded_wait(uint32_t max_polls, int32_t cluster_scope,
                                                           int32_t *dev_status, void *stream)
 {
+    NvtxRange nvtx_range("cis_selftest_bounded_wait");
     if (dev_status == nullptr || max_polls == 0 || max_polls > kMaxPolls ||
         (cluster_scope != 0 && cluster_scope != 1))
         return CIS_ERR_INVALID_ARG;
