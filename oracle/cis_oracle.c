@@ -715,18 +715,20 @@ int oracle_mismatch_diagnostics(const void *z_train, const void *z_infer, int dt
             double *bvec = (double *)malloc(sizeof(double) * (size_t)V);
             double *fvec = (double *)malloc(sizeof(double) * (size_t)V);
             double *gvec = (double *)malloc(sizeof(double) * (size_t)V);
+            double *pv = (double *)malloc(sizeof(double) * (size_t)V);
             for (int64_t j = 0; j < V; ++j) {
                 lp[j] = logit_at(z_train, dtype, ld, t, j) - lse;
                 lq[j] = logit_at(z_infer, dtype, ld, t, j) - lsei;
+                pv[j] = exp(lp[j]); /* p_j, the training softmax */
             }
             /* eps by Lemma 3.1's definition, in the normalised gauge */
             double Sy = 0.0, acc = 0.0;
             for (int64_t j = 0; j < V; ++j)
                 if (j != y)
-                    Sy += exp(lp[j]);
+                    Sy += pv[j];
             for (int64_t j = 0; j < V; ++j)
                 if (j != y)
-                    acc += exp(lp[j]) / Sy * exp(lq[j] - lp[j]);
+                    acc += pv[j] / Sy * exp(lq[j] - lp[j]);
             eps = -(lq[y] - lp[y]) + log(acc);
             lk = lp[y] - lq[y];
             pt = exp(lp[y]);
@@ -744,7 +746,7 @@ int oracle_mismatch_diagnostics(const void *z_train, const void *z_infer, int dt
                 const double ky = exp(lp[yy] - lq[yy]);
                 double g2 = 0.0;
                 for (int64_t j = 0; j < V; ++j) {
-                    const double gj = (j == yy ? 1.0 : 0.0) - exp(lp[j]);
+                    const double gj = (j == yy ? 1.0 : 0.0) - pv[j];
                     bvec[j] += qy * (f - ky) * gj;
                     fvec[j] += qy * f * gj;
                     gvec[j] += qy * gj;
@@ -766,6 +768,7 @@ int oracle_mismatch_diagnostics(const void *z_train, const void *z_infer, int dt
             free(bvec);
             free(fvec);
             free(gvec);
+            free(pv);
         }
         eps_out[t] = eps;
         logk_out[t] = lk;
