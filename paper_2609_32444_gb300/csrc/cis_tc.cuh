@@ -47,10 +47,15 @@ __device__ __forceinline__ void bar_arrive(uint64_t *bar)
 {
     asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_addr(bar)) : "memory");
 }
-// Bounded wait for the phase with the given parity.  False if it never came
-// or, when `flag` is given, once the word it points to carries
-// kStatusTimeout: a wait elsewhere in the grid ran out, so this one stops
-// early.  The word is read every 256 polls only, off the fast path.
+// Bounded wait for the phase with the given parity: at most kMaxPolls polls.
+// False if it never came or, when `flag` is given, once the word it points to
+// carries kStatusTimeout: a wait elsewhere in the grid ran out, so this one
+// stops early.  The word is read every 256 polls only, off the fast path.
+// The polls carry no suspend-time hint (each returns within the hardware's
+// own limit): these GEMMs hand a stage or an accumulator from one warp to
+// another every few hundred cycles, and a thread suspended for up to 1 us
+// woke late enough to cost the full-size LM head 1.3-1.5%.  (Reading
+// %globaltimer in the loop, for a wall-clock limit, cost it 7%.)
 __device__ __forceinline__ bool bar_wait(uint64_t *bar, uint32_t parity,
                                          const volatile int32_t *flag = nullptr)
 {
@@ -59,10 +64,10 @@ __device__ __forceinline__ bool bar_wait(uint64_t *bar, uint32_t parity,
         uint32_t done;
         asm volatile(
             "{\n\t.reg .pred p;\n\t"
-            "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
+            "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
             "selp.u32 %0, 1, 0, p;\n\t}"
             : "=r"(done)
-            : "r"(a), "r"(parity), "r"(kPollSuspendNs)
+            : "r"(a), "r"(parity)
             : "memory");
         if (done)
             return true;
