@@ -572,7 +572,7 @@ def run_diag(args, rank, world, local):
                        "l2": "no flush: the 9.96 GB of logits per step exceed the L2"},
             "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                          "frac": achieved / peak, "traffic": profiled_traffic(6, args.tokens),
-                         "kernel": "cis_mismatch_stream_kernel<cis, 16 warps> (both rows "
+                         "kernel": "cis_mismatch_stream_kernel<cis, 16 warps, 1 CTA per SM> (both rows "
                                    "streamed through shared memory twice, HBM once)",
                          "algorithmic_bytes_per_launch": alg_bytes, "peak_source": peak_src},
             "cpu_baseline": cpu, "e2e": None, "gpu_launches": args.steps,

@@ -314,17 +314,19 @@ struct DiagArgs {
     int32_t *status;
 };
 
-// The layout for NW consumer warps (plus one producer warp): a ring slot
-// holds four groups per consumer thread of each row, as many slots as fit in
-// about 200 KB of shared memory (3 for 16 warps).  Each slot costs every warp
-// a wait, an arrive and the loop set-up; four groups a thread amortise that
-// (two, three, five and six measured slower).
-template <int NW> struct StreamCfg {
+// The layout for NW consumer warps (plus one producer warp) and CPS CTAs per
+// SM: a ring slot holds four groups per consumer thread of each row, as many
+// slots as fit in about 200 KB / CPS of shared memory (3 of 64 KB for 16
+// warps and one CTA).  Each slot costs every warp a wait, an arrive and the loop
+// set-up; four groups a thread amortise that (two, three, five and six
+// measured slower).
+template <int NW, int CPS = 1> struct StreamCfg {
     static constexpr int kConsThreads = NW * 32;
     static constexpr int kThreads = kConsThreads + 32;
     static constexpr int kSlotGroups = 4 * kConsThreads;  // 8-entry groups of each row per slot
     static constexpr int kSlotBytes = 2 * kSlotGroups * 16;
-    static constexpr int kRing = (200 * 1024) / kSlotBytes < 8 ? (200 * 1024) / kSlotBytes : 8;
+    static constexpr int kRingFit = (200 * 1024 / CPS) / kSlotBytes;
+    static constexpr int kRing = kRingFit < 8 ? kRingFit : 8;
     static constexpr size_t kSmem = (size_t)kRing * kSlotBytes + 128;
 };
 constexpr int kMaxRing = 8;
@@ -420,23 +422,24 @@ __device__ __forceinline__ void pass1_update(uint4 w, float &m, float &cm, float
     s = sum8_exp2_pk(w, make_float2(-cm, -cm), s);
 }
 
-// One CTA per SM walks rows t = blockIdx.x, blockIdx.x + gridDim.x, ...  Per
+// CPS CTAs per SM walk rows t = blockIdx.x, blockIdx.x + gridDim.x, ...  Per
 // row, a producer thread streams both rows through a ring of kRing shared-
 // memory slots twice (bulk copies of sg groups per row per slot): once for
 // pass 1 (from HBM) and once for pass 2 (the same bytes again, mostly from L2,
 // where pass 1 left them microseconds earlier; these copies mark the lines
-// evict-first).  The consumer warps:
+// evict-first).  Pass 2 takes the row's slots last-first, so that the bytes
+// pass 1 brought in last are read again first.  The consumer warps:
 //   pass 1: per thread a running (max, sum) of each row over its groups;
 //           warp, then CTA combination; lanes 0 and 16 of warp 0 form the two
 //           rows' scalars (log p, log q, lse; eps, log k, p for the output);
 //   pass 2: the nine sums, two candidates per packed instruction;
 //           warp sums in fp32, CTA sums in fp64 by warp 0, which also forms
 //           bias2 and dvar while the other warps start the next row.
-template <int MODE, int NW>
-__global__ void __launch_bounds__(StreamCfg<NW>::kThreads, 1)
+template <int MODE, int NW, int CPS>
+__global__ void __launch_bounds__(StreamCfg<NW, CPS>::kThreads, CPS)
     cis_mismatch_stream_kernel(const DiagArgs a, int sg)
 {
-    using C = StreamCfg<NW>;
+    using C = StreamCfg<NW, CPS>;
     constexpr int kConsWarps = NW, kConsThreads = C::kConsThreads, kRing = C::kRing;
     constexpr int kSlotGroups = C::kSlotGroups, kSlotBytes = C::kSlotBytes;
     extern __shared__ __align__(128) uint8_t dyn_smem[];
@@ -472,7 +475,7 @@ __global__ void __launch_bounds__(StreamCfg<NW>::kThreads, 1)
                         ab.wait(smem_u32(&sh.empty[s]), (u - 1) & 1);
                     if (ab.on())
                         break;
-                    const int g0 = st * sg, n = min(sg, ng - g0);
+                    const int g0 = (pass ? nst - 1 - st : st) * sg, n = min(sg, ng - g0);
                     const uint32_t bytes = (uint32_t)n * 16;
                     const uint32_t full = smem_u32(&sh.full[s]);
                     const uint32_t dst = smem_u32(ring + (size_t)s * kSlotBytes);
@@ -558,7 +561,7 @@ __global__ void __launch_bounds__(StreamCfg<NW>::kThreads, 1)
             // inference row's (lane l takes warps l, l + 16, ...), then a
             // fixed tree over the 16 lanes
             const int r = lane >> 4;
-            MaxSum o = sh.red[r][lane & 15];
+            MaxSum o = (lane & 15) < kConsWarps ? sh.red[r][lane & 15] : MaxSum{-INFINITY, 0.0f};
             for (int w = (lane & 15) + 16; w < kConsWarps; w += 16)
                 o = ms_combine(o, sh.red[r][w]);
 #pragma unroll
@@ -619,7 +622,7 @@ __global__ void __launch_bounds__(StreamCfg<NW>::kThreads, 1)
             const uint32_t s = k % kRing;
             ab.wait(smem_u32(&sh.full[s]), (k / kRing) & 1);
             const uint4 *slot = reinterpret_cast<const uint4 *>(ring + (size_t)s * kSlotBytes);
-            const int n = min(sg, ng - st * sg);
+            const int n = min(sg, ng - (nst - 1 - st) * sg);
 #pragma unroll 1
             for (int j = ct; j < n; j += kConsThreads) {
                 const uint4 u = slot[j], v = slot[kSlotGroups + j];
@@ -677,13 +680,21 @@ int diag_slot_groups(int max_groups)
     return v < 1 ? 1 : (v > max_groups ? max_groups : (int)v);
 }
 
-// Consumer warps (CIS_DIAG_WARPS, for tuning sweeps: 16 or 24; 16 measured
-// faster at V=151936 with four groups a thread per slot: 3 slots of 64 KB
-// against 2 of 96 KB for 24 warps).
+// Consumer warps per CTA (CIS_DIAG_WARPS, for tuning sweeps): 16 (the
+// default) or 24 with one CTA per SM, 8 with two, 4 with four; the ring
+// shrinks with the CTA.  At V=151936 (four groups a thread per slot) two CTAs
+// of 8 warps took 3.19 ms against 3.28 for one of 16: a CTA's warps meet
+// three times per row, and while one CTA waits at those barriers the SM's
+// other CTA issues.  But twice as many rows are then in flight (about 185 MB
+// between a row's two reads, more than the L2 holds), and pass 2 re-read a
+// third of its bytes from HBM: 13.2 GB of DRAM reads per call against 10.0.
+// One CTA of 16 warps keeps HBM at one read of each row.  24 warps in one CTA
+// (2 slots of 96 KB) were slower than 16 (3 of 64 KB).
 int diag_warps()
 {
     const char *e = getenv("CIS_DIAG_WARPS");
-    return (e && atoi(e) == 24) ? 24 : 16;
+    const int v = e ? atoi(e) : 16;
+    return (v == 24 || v == 8 || v == 4) ? v : 16;
 }
 
 bool diag_stream_applies(const void *zt, const void *zi, int dtype, int64_t V, int64_t ld_t,
@@ -698,11 +709,11 @@ bool diag_stream_applies(const void *zt, const void *zi, int dtype, int64_t V, i
     return !(e && e[0] == 'r');
 }
 
-template <int MODE, int NW>
+template <int MODE, int NW, int CPS>
 cudaError_t launch_stream_nw(const DiagArgs &a, cudaStream_t s)
 {
-    using C = StreamCfg<NW>;
-    auto kern = cis_mismatch_stream_kernel<MODE, NW>;
+    using C = StreamCfg<NW, CPS>;
+    auto kern = cis_mismatch_stream_kernel<MODE, NW, CPS>;
     cudaError_t e =
         cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)C::kSmem);
     if (e != cudaSuccess)
@@ -711,7 +722,8 @@ cudaError_t launch_stream_nw(const DiagArgs &a, cudaStream_t s)
     if ((e = cudaGetDevice(&dev)) != cudaSuccess ||
         (e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess)
         return e;
-    const int64_t grid = a.T < sms ? a.T : sms;
+    const int64_t slots = (int64_t)CPS * sms;
+    const int64_t grid = a.T < slots ? a.T : slots;
     kern<<<(unsigned)grid, C::kThreads, C::kSmem, s>>>(a, diag_slot_groups(C::kSlotGroups));
     return cudaGetLastError();
 }
@@ -719,7 +731,12 @@ cudaError_t launch_stream_nw(const DiagArgs &a, cudaStream_t s)
 template <int MODE>
 cudaError_t launch_stream_mode(const DiagArgs &a, cudaStream_t s)
 {
-    return diag_warps() == 24 ? launch_stream_nw<MODE, 24>(a, s) : launch_stream_nw<MODE, 16>(a, s);
+    switch (diag_warps()) {
+    case 24: return launch_stream_nw<MODE, 24, 1>(a, s);
+    case 8: return launch_stream_nw<MODE, 8, 2>(a, s);
+    case 4: return launch_stream_nw<MODE, 4, 4>(a, s);
+    default: return launch_stream_nw<MODE, 16, 1>(a, s);
+    }
 }
 
 // ---------------------------------------------------------------------------

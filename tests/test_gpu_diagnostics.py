@@ -63,8 +63,9 @@ U = 2.0 ** -24
 def n_thread(V, slot_groups=2048, threads=512):
     """Most candidates one thread sums in a row: the streaming kernel's ring
     slots of `slot_groups` groups of 8 (each of `threads` threads takes
-    ceil(slot_groups / threads) groups of a slot); this also bounds the one-CTA
-    kernel's 512 threads with 8-wide loads."""
+    ceil(slot_groups / threads) groups of a slot; the defaults are its layout
+    of 16 consumer warps); this also bounds the one-CTA kernel's 512 threads
+    with 8-wide loads."""
     groups = -(-V // 8)
     slots = -(-groups // slot_groups)
     return 8 * slots * max(1, -(-slot_groups // threads)) + 8
@@ -308,15 +309,19 @@ def test_diagnostics_stream_ragged_slots(mode, monkeypatch):
 
 def test_diagnostics_slot_sizes_agree(monkeypatch):
     """The same bf16 rows (V=24576: 3072 groups, so every consumer warp holds
-    groups in a full slot) through ring slots of 16 and 24 warps, of 64, 7
-    and 1 groups (the last wraps the ring hundreds of times per pass) and the
-    one-CTA kernel: results differ by summation order only."""
+    groups in a full slot) through ring slots of 16 and 24 warps, of 8 warps
+    in two CTAs per SM and 4 in four, of 64, 7 and 1 groups (the last wraps
+    the ring hundreds of times per pass) and the one-CTA kernel: results
+    differ by summation order only."""
     V, T = 24576, 16
     z, zi, ids = _rows(12, T, V, torch.bfloat16)
     P = binding.cis_default_params("cis")
     outs = []
-    configs = [("16", None), ("24", None), ("16", "64"), ("16", "7"), ("24", "1")]
-    n_ts = [n_thread(V, int(sg or 2048), 32 * int(w)) for w, sg in configs] + [n_thread(V)]
+    configs = [("16", None), ("24", None), ("8", None), ("4", None), ("16", "64"), ("16", "7"),
+               ("24", "1")]
+    # a full slot holds four groups per consumer thread
+    n_ts = [n_thread(V, int(sg or 128 * int(w)), 32 * int(w)) for w, sg in configs]
+    n_ts.append(n_thread(V))
     for warps, sg in configs:
         monkeypatch.setenv("CIS_DIAG_WARPS", warps)
         if sg is None:
