@@ -46,9 +46,13 @@
  *       CIS_CLUSTER_THREADS (128, 256, 384 or 512; default 256) set the
  *       fused pass's slice target, cluster size and CTA width.  They are read
  *       once per process.
- *       CIS_DIAG_WARPS (16 or 24; default 16) and CIS_DIAG_SLOT_GROUPS (>= 1)
- *       set the diagnostics kernel's width and ring-slot size, and
- *       CIS_DIAG_KERNEL=row selects its one-CTA kernel.  They are read at
+ *       CIS_DIAG_WARPS (16 or 24 with one CTA per SM, 8 with two, 4 with
+ *       four; default 16) and CIS_DIAG_SLOT_GROUPS (>= 1) set the diagnostics
+ *       kernel's width and ring-slot size, and CIS_DIAG_KERNEL=row selects its
+ *       one-CTA kernel.  They are read at each call.
+ *       CIS_LMHEAD_MC (a bit mask over the LM head's GEMMs: 1 logits, 2 dz,
+ *       4 dH, 8 dW; default 15) picks the GEMMs that run on 2-CTA clusters
+ *       sharing B tiles by multicast.  It changes no result bit.  Read at
  *       each call.
  */
 #ifndef CIS_H

@@ -186,7 +186,32 @@ __device__ __forceinline__ void tile_mn(const GemmArgs &g, int i, int &m, int &n
     }
 }
 
-template <int EPI, bool A_MN, bool B_MN>
+// Work unit u of a launch: a tile, or with MC (2-CTA clusters) a pair of
+// tiles in row tiles 2 mp and 2 mp + 1 of one column tile, CTA `rank` of the
+// cluster taking row tile 2 mp + rank.  The pair shares its B tile: each CTA
+// loads one half of it and multicasts it to both.  With an odd number of row
+// tiles the last pair's second tile lies past the rows (m == nMt): its CTA
+// still loads and multicasts its half of B, and its A reads as zeros, but its
+// epilogue writes nothing.
+template <bool MC> __device__ __forceinline__ int n_units(const GemmArgs &g)
+{
+    return MC ? ((g.nMt + 1) >> 1) * g.nNt : g.nMt * g.nNt;
+}
+template <bool MC>
+__device__ __forceinline__ void unit_mn(const GemmArgs &g, int u, int rank, int &m, int &n)
+{
+    if (!MC) {
+        tile_mn(g, u, m, n);
+        return;
+    }
+    GemmArgs gp = g;
+    gp.nMt = (g.nMt + 1) >> 1;  // the pairs' own grid of (row pair, column) units
+    int mp;
+    tile_mn(gp, u, mp, n);
+    m = 2 * mp + rank;
+}
+
+template <int EPI, bool A_MN, bool B_MN, bool MC>
 __global__ void __launch_bounds__(kThreads, 1)
     cis_lmhead_gemm_kernel(const __grid_constant__ CUtensorMap tmA,
                            const __grid_constant__ CUtensorMap tmB, const GemmArgs g)
@@ -198,13 +223,18 @@ __global__ void __launch_bounds__(kThreads, 1)
     __shared__ int aborted;
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int nTiles = g.nMt * g.nNt;
+    const int nUnits = n_units<MC>(g);
+    const int rank = MC ? (int)tc::cluster_ctarank() : 0;
+    const int unit0 = MC ? (int)(blockIdx.x >> 1) : (int)blockIdx.x;
+    const int ustep = MC ? (int)(gridDim.x >> 1) : (int)gridDim.x;
 
     if (threadIdx.x == 0) {
         aborted = 0;
         for (int s = 0; s < kStages; ++s) {
             tc::bar_init(&bars.full[s], 1);
-            tc::bar_init(&bars.empty[s], 1);
+            // with MC both CTAs' MMAs release a stage: the peer's multicast
+            // writes into this CTA's copy of it
+            tc::bar_init(&bars.empty[s], MC ? 2 : 1);
         }
         for (int b = 0; b < 2; ++b) {
             tc::bar_init(&bars.accfull[b], 1);
@@ -217,6 +247,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         tc::tmem_alloc(&tmem_base, kTmemCols);
     tc::fence_before_sync();
     __syncthreads();
+    if (MC)
+        tc::cluster_sync();  // the peer's barriers exist before anything signals them
     tc::fence_after_sync();
     const uint32_t tmem = tmem_base;
     const Abort ab{&aborted, g.status};
@@ -226,9 +258,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (lane == 0) {
             int stage = 0;
             uint32_t phase = 0, used = 0, last = 0;  // per stage: loaded, parity of its last load
-            for (int t = blockIdx.x; t < nTiles && !ab.on(); t += gridDim.x) {
+            for (int u = unit0; u < nUnits && !ab.on(); u += ustep) {
                 int m, n;
-                tile_mn(g, t, m, n);
+                unit_mn<MC>(g, u, rank, m, n);
                 for (int kb = 0; kb < g.nK; ++kb) {
                     ab.wait(&bars.empty[stage], phase ^ 1);
                     if (ab.on())
@@ -246,7 +278,19 @@ __global__ void __launch_bounds__(kThreads, 1)
                     } else {
                         tc::tma_load_2d(st, &tmA, ka, g.a_row0 + m * kBM, &bars.full[stage]);
                     }
-                    if (B_MN) {
+                    if (MC) {  // this CTA's half of B, to both CTAs
+                        if (B_MN) {
+#pragma unroll
+                            for (int i = 2 * rank; i < 2 * rank + 2; ++i)
+                                tc::tma_load_2d_mc(st + kStageA + i * kMnBox, &tmB,
+                                                   g.b_row0 + n * kBN + 64 * i, kbb,
+                                                   &bars.full[stage], 0x3);
+                        } else {
+                            tc::tma_load_2d_mc(st + kStageA + rank * (kStageB / 2), &tmB, kbb,
+                                               g.b_row0 + n * kBN + rank * (kBN / 2),
+                                               &bars.full[stage], 0x3);
+                        }
+                    } else if (B_MN) {
 #pragma unroll
                         for (int i = 0; i < kBN / 64; ++i)
                             tc::tma_load_2d(st + kStageA + i * kMnBox, &tmB,
@@ -277,7 +321,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             int stage = 0;
             uint32_t phase = 0;
             int i = 0;
-            for (int t = blockIdx.x; t < nTiles && !ab.on(); t += gridDim.x, ++i) {
+            for (int u = unit0; u < nUnits && !ab.on(); u += ustep, ++i) {
                 const int acc = i & 1;
                 ab.wait(&bars.accempty[acc], ((i >> 1) & 1) ^ 1);
                 tc::fence_after_sync();
@@ -297,7 +341,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                                                  : tc::desc_sw128(sb + kk * b_step);
                         tc::mma_bf16(d, da, db, kId, (kb | kk) != 0);
                     }
-                    tc::mma_commit(&bars.empty[stage]);
+                    if (MC)  // the stage is free in this CTA and in the peer
+                        tc::mma_commit_mc(&bars.empty[stage], 0x3);
+                    else
+                        tc::mma_commit(&bars.empty[stage]);
                     if (++stage == kStages) {
                         stage = 0;
                         phase ^= 1;
@@ -319,16 +366,18 @@ __global__ void __launch_bounds__(kThreads, 1)
         const uint32_t lane_off = (uint32_t)(lg * 32) << 16;
         const int cbeg = half * kHalf;
         int i = 0;
-        for (int t = blockIdx.x; t < nTiles; t += gridDim.x, ++i) {
+        for (int u = unit0; u < nUnits; u += ustep, ++i) {
             if (__syncthreads_or_epi(ab.on()))
                 break;
             int m, n;
-            tile_mn(g, t, m, n);
+            unit_mn<MC>(g, u, rank, m, n);
             const int acc = i & 1;
             ab.wait(&bars.accfull[acc], (i >> 1) & 1);
             tc::fence_after_sync();
             const uint32_t taddr = tmem + lane_off + acc * kBN;
-            if (EPI == kStats) {
+            if (MC && m >= g.nMt) {
+                // the padding tile of an odd row count: nothing to write
+            } else if (EPI == kStats) {
                 const int row = m * kBM + r;  // token
                 const int y_r = row < g.T ? g.ids[row] : -1;
                 const bool ent = g.part_u != nullptr;
@@ -490,6 +539,18 @@ __global__ void __launch_bounds__(kThreads, 1)
     __syncwarp();
     tc::fence_before_sync();
     __syncthreads();
+    if (MC) {
+        // neither CTA leaves while the other may still signal its barriers
+        tc::cluster_sync();
+        // after a wait ran out the peer may have issued one more multicast
+        // into a stage this CTA no longer waits for: give it time to land
+        if (aborted && threadIdx.x == 0) {
+            const long long t0 = clock64();
+            while (clock64() - t0 < (1ll << 20)) {
+            }
+        }
+        __syncthreads();
+    }
     if (warp == 1) {
         tc::fence_after_sync();
         tc::tmem_dealloc(tmem, kTmemCols);
@@ -623,7 +684,7 @@ cudaError_t launch_gemm(const CUtensorMap &a, const CUtensorMap &b, const GemmAr
     const int tiles = g.nMt * g.nNt;
     if (tiles <= 0 || g.nK <= 0)
         return cudaSuccess;
-    auto k = cis_lmhead_gemm_kernel<EPI, A_MN, B_MN>;
+    auto k = cis_lmhead_gemm_kernel<EPI, A_MN, B_MN, false>;
     const size_t smem = kSmemBytes;
     cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          (int)smem);
@@ -636,6 +697,53 @@ cudaError_t launch_gemm(const CUtensorMap &a, const CUtensorMap &b, const GemmAr
     const int grid = tiles < sms ? tiles : sms;
     k<<<grid, kThreads, smem, s>>>(a, b, g);
     return cudaGetLastError();
+}
+
+// The same GEMM on 2-CTA clusters that share each B tile (multicast).  `b`
+// must be a map whose box is half of B's tile: 128 rows for a K-major B, the
+// 64-wide boxes of an MN-major one.
+template <int EPI, bool A_MN = false, bool B_MN = false>
+cudaError_t launch_gemm_mc(const CUtensorMap &a, const CUtensorMap &b, const GemmArgs &g,
+                           cudaStream_t s)
+{
+    const int units = ((g.nMt + 1) / 2) * g.nNt;
+    if (units <= 0 || g.nK <= 0)
+        return cudaSuccess;
+    auto k = cis_lmhead_gemm_kernel<EPI, A_MN, B_MN, true>;
+    cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)kSmemBytes);
+    if (e != cudaSuccess)
+        return e;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = 2;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cudaLaunchConfig_t cfg = {};
+    cfg.blockDim = dim3(kThreads);
+    cfg.dynamicSmemBytes = kSmemBytes;
+    cfg.stream = s;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    cfg.gridDim = dim3(2);
+    int clusters = 0;
+    if ((e = cudaOccupancyMaxActiveClusters(&clusters, k, &cfg)) != cudaSuccess)
+        return e;
+    if (clusters <= 0)
+        return cudaErrorNotSupported;
+    cfg.gridDim = dim3((unsigned)(2 * (units < clusters ? units : clusters)));
+    e = cudaLaunchKernelEx(&cfg, k, a, b, g);
+    return e != cudaSuccess ? e : cudaGetLastError();
+}
+
+// Which GEMMs run on 2-CTA multicast clusters: a bit mask over FWD (1), DZ
+// (2), DH (4) and DW (8); all by default, CIS_LMHEAD_MC overrides it.  The
+// results are bit for bit the same either way: each tile's MMAs and epilogue
+// are unchanged, only where half of B comes from differs.
+static int mc_mask()
+{
+    const char *e = getenv("CIS_LMHEAD_MC");
+    return e && e[0] ? (int)strtol(e, nullptr, 0) & 15 : 15;
 }
 
 }  // namespace lm
@@ -808,9 +916,12 @@ CIS_API cis_status_t cis_lmhead_fused(const void *hidden, const void *weight, in
         const int nHt = (int)(H / lm::kBN);
         // K-major maps of H and W (FWD, DZ) and MN-major ones (boxes of 64
         // rows: W as DH's B operand, H as DW's)
-        CUtensorMap mH, mW, mWmn, mHmn;
+        // (mWh: W in boxes of half a B tile, for the multicast clusters)
+        const int mc = lm::mc_mask();
+        CUtensorMap mH, mW, mWh, mWmn, mHmn;
         if (!lm::make_map(&mH, hidden, H, T, H, lm::kBM) ||
             !lm::make_map(&mW, weight, H, V, H, lm::kBN) ||
+            !lm::make_map(&mWh, weight, H, V, H, lm::kBN / 2) ||
             !lm::make_map(&mWmn, weight, H, V, H, 64) ||
             !lm::make_map(&mHmn, hidden, H, T, H, 64))
             return CIS_ERR_UNSUPPORTED;
@@ -831,7 +942,8 @@ CIS_API cis_status_t cis_lmhead_fused(const void *hidden, const void *weight, in
         g.nNt = nVt;
         g.nK = (int)(H / lm::kBK);
         g.raster_n = 1;
-        if (lm::launch_gemm<lm::kStats>(mH, mW, g, s) != cudaSuccess)
+        if (((mc & 1) ? lm::launch_gemm_mc<lm::kStats>(mH, mWh, g, s)
+                      : lm::launch_gemm<lm::kStats>(mH, mW, g, s)) != cudaSuccess)
             return CIS_ERR_CUDA;
         // per-token scalars
         if (is_seq_mode(P.mode)) {
@@ -871,7 +983,8 @@ CIS_API cis_status_t cis_lmhead_fused(const void *hidden, const void *weight, in
             g.b_row0 = (int)v0;
             g.b_k0 = 0;
             g.col0 = (int)v0;
-            if (lm::launch_gemm<lm::kDz>(mH, mW, g, s) != cudaSuccess)
+            if (((mc & 2) ? lm::launch_gemm_mc<lm::kDz>(mH, mWh, g, s)
+                          : lm::launch_gemm<lm::kDz>(mH, mW, g, s)) != cudaSuccess)
                 return CIS_ERR_CUDA;
             // dz K-major (DH's A: rows are tokens) and MN-major (DW's A: its
             // M runs along dz's columns; rows past T read as zeros)
@@ -894,8 +1007,12 @@ CIS_API cis_status_t cis_lmhead_fused(const void *hidden, const void *weight, in
             g.out_v8 = (reinterpret_cast<uintptr_t>(dh_acc) & 31) == 0;
             g.rows_valid = (int)T;
             g.ld_out = H;
-            e = v0 == 0 ? lm::launch_gemm<lm::kStore, false, true>(mDz, mWmn, g, s)
-                        : lm::launch_gemm<lm::kAccum, false, true>(mDz, mWmn, g, s);
+            if (mc & 4)
+                e = v0 == 0 ? lm::launch_gemm_mc<lm::kStore, false, true>(mDz, mWmn, g, s)
+                            : lm::launch_gemm_mc<lm::kAccum, false, true>(mDz, mWmn, g, s);
+            else
+                e = v0 == 0 ? lm::launch_gemm<lm::kStore, false, true>(mDz, mWmn, g, s)
+                            : lm::launch_gemm<lm::kAccum, false, true>(mDz, mWmn, g, s);
             if (e != cudaSuccess)
                 return CIS_ERR_CUDA;
             // DW[chunk] = dz^T H: A = dz MN-major (M along the chunk's columns,
@@ -910,7 +1027,9 @@ CIS_API cis_status_t cis_lmhead_fused(const void *hidden, const void *weight, in
             g.out_bf16 = grad_dtype == CIS_BF16;
             g.out_v8 = (reinterpret_cast<uintptr_t>(g.out) & 31) == 0;
             g.rows_valid = (int)w;
-            if (lm::launch_gemm<lm::kStore, true, true>(mDzmn, mHmn, g, s) != cudaSuccess)
+            if (((mc & 8) ? lm::launch_gemm_mc<lm::kStore, true, true>(mDzmn, mHmn, g, s)
+                          : lm::launch_gemm<lm::kStore, true, true>(mDzmn, mHmn, g, s)) !=
+                cudaSuccess)
                 return CIS_ERR_CUDA;
         }
         if (grad_dtype == CIS_BF16) {

@@ -162,6 +162,39 @@ def test_lmhead_outputs_16_byte_aligned(grad):
                        ref["dweight"].view(torch.int16 if es == 2 else torch.int32))
 
 
+@pytest.mark.parametrize("T,V,H,chunk,grad", [(300, 1100, 256, 768, torch.float32),
+                                              (512, 4096, 2048, None, torch.float32),
+                                              (130, 1900, 512, 512, torch.bfloat16)])
+def test_lmhead_multicast_clusters_bit_identical(monkeypatch, T, V, H, chunk, grad):
+    """Every GEMM on 2-CTA clusters sharing each B tile (multicast, the
+    default) against every GEMM on one CTA (CIS_LMHEAD_MC=0): the same tiles
+    with the same MMAs and epilogues, so every output matches bit for bit.
+    T=300 gives an odd number of 128-row token tiles (FWD, DZ, DH), and the
+    last chunks of 332 and 364 columns odd numbers of 128-column vocabulary
+    tiles (DW), so the padding tile of the last pair is exercised; the first
+    case is also checked against the oracle."""
+    b = synth.make_batch(5, T=T, V=V, H=H)
+    outs = {}
+    for mc in ("15", "0"):
+        monkeypatch.setenv("CIS_LMHEAD_MC", mc)
+        outs[mc] = _run(b, grad_dtype=grad, chunk=chunk)
+    torch.cuda.synchronize()
+    a, r = outs["15"], outs["0"]
+    for k in ("lp", "w", "trunc", "dhidden", "dweight", "loss"):
+        x, y = a[k], r[k]
+        if x.dtype.is_floating_point:
+            x = x.view(torch.int16 if x.element_size() == 2 else
+                       (torch.int32 if x.element_size() == 4 else torch.int64))
+            y = y.view(x.dtype)
+        assert torch.equal(x, y), k
+    assert binding.decode_stats(a["stats"])["status"] == 0
+    if T == 300:
+        ref = _oracle(b)
+        _check_tokens(a, ref, np.arange(T), b, "cis", full=True)
+        _check_grad(a["dhidden"], ref["dhidden"], ref["dhidden_abs"], V, False)
+        _check_grad(a["dweight"], ref["dweight"], ref["dweight_abs"], T, False)
+
+
 def test_lmhead_workspace_too_small():
     """Less workspace than 256-column chunks need is refused on the host."""
     b = synth.make_batch(5, T=64, V=1024, H=256)
