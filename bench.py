@@ -428,8 +428,8 @@ def run_lmhead(args, rank, world, local):
     tp = -(-T // 128) * 128
     chunk = min(-(-V // 256) * 256, max(256, (1 << 30) // (2 * tp) // 256 * 256))
     n_chunks = -(-V // chunk)
-    # scales, FWD, token, (DZ, DH, DW) per chunk, reduce
-    launches_per_call = 3 + 3 * n_chunks + 1
+    # scales, FWD, token, (DZ, then DH and DW in one launch) per chunk, reduce
+    launches_per_call = 3 + 2 * n_chunks + 1
 
     def step():
         return binding.cis_lmhead_fused(b.hidden, b.weight, b.ids, b.lp_infer, b.adv, P,

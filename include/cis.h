@@ -52,8 +52,9 @@
  *       one-CTA kernel.  They are read at each call.
  *       CIS_LMHEAD_MC (a bit mask over the LM head's GEMMs: 1 logits, 2 dz,
  *       4 dH, 8 dW; default 15) picks the GEMMs that run on 2-CTA clusters
- *       sharing B tiles by multicast.  It changes no result bit.  Read at
- *       each call.
+ *       sharing B tiles by multicast, and CIS_LMHEAD_DUAL=0 runs a chunk's
+ *       dH and dW as two launches instead of one.  Neither changes a result
+ *       bit.  Read at each call.
  */
 #ifndef CIS_H
 #define CIS_H

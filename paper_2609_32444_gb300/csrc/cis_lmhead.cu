@@ -14,7 +14,8 @@
 //   DZ   recompute the chunk's z tiles, form dz = c (softmax - onehot) in bf16
 //        and write it as dz [Tp, w];
 //   DH   dH (+)= dz W[v0 : v0 + w]   (K = w, fp32 accumulator);
-//   DW   dW[v0 : v0 + w] = dz^T H    (K = T).
+//   DW   dW[v0 : v0 + w] = dz^T H    (K = T);
+//   DH and DW of a chunk run as one launch with a balanced schedule.
 //
 // dz exists one chunk at a time (the chunk width follows the workspace the
 // caller gives); z never exists outside TMEM.  Every operand is read where
@@ -40,7 +41,11 @@
 // to its end, so that TMEM is always released.
 #include <cuda.h>
 #include <cudaTypedefs.h>
+#include <array>
+#include <map>
+#include <memory>
 #include <mutex>
+#include <vector>
 
 #include "cis_kernels.h"
 #include "cis_tc.cuh"
@@ -185,7 +190,6 @@ __device__ __forceinline__ void tile_mn(const GemmArgs &g, int i, int &m, int &n
         n = i - m * g.nNt;
     }
 }
-
 // Work unit u of a launch: a tile, or with MC (2-CTA clusters) a pair of
 // tiles in row tiles 2 mp and 2 mp + 1 of one column tile, CTA `rank` of the
 // cluster taking row tile 2 mp + rank.  The pair shares its B tile: each CTA
@@ -193,7 +197,7 @@ __device__ __forceinline__ void tile_mn(const GemmArgs &g, int i, int &m, int &n
 // tiles the last pair's second tile lies past the rows (m == nMt): its CTA
 // still loads and multicasts its half of B, and its A reads as zeros, but its
 // epilogue writes nothing.
-template <bool MC> __device__ __forceinline__ int n_units(const GemmArgs &g)
+template <bool MC> __host__ __device__ __forceinline__ int n_units(const GemmArgs &g)
 {
     return MC ? ((g.nMt + 1) >> 1) * g.nNt : g.nMt * g.nNt;
 }
@@ -211,340 +215,328 @@ __device__ __forceinline__ void unit_mn(const GemmArgs &g, int u, int rank, int 
     m = 2 * mp + rank;
 }
 
-template <int EPI, bool A_MN, bool B_MN, bool MC>
-__global__ void __launch_bounds__(kThreads, 1)
-    cis_lmhead_gemm_kernel(const __grid_constant__ CUtensorMap tmA,
-                           const __grid_constant__ CUtensorMap tmB, const GemmArgs g)
+// Where the producer, or the MMA thread, is in the ring of stages.
+struct Ring {
+    int stage = 0;
+    uint32_t phase = 0;
+    __device__ __forceinline__ void next()
+    {
+        if (++stage == kStages) {
+            stage = 0;
+            phase ^= 1;
+        }
+    }
+};
+
+// The producer's loads for tile (m, n): nK stages.  `used` and `last` record
+// per stage whether it was ever loaded and the parity of its last load, for
+// the drain before the CTA leaves.  Returns early once the CTA aborted.
+template <bool A_MN, bool B_MN, bool MC>
+__device__ __forceinline__ void load_tile(const CUtensorMap &tmA, const CUtensorMap &tmB,
+                                          const GemmArgs &g, int m, int n, int rank,
+                                          uint8_t *ring, Barriers &bars, const Abort &ab,
+                                          Ring &p, uint32_t &used, uint32_t &last)
 {
-    extern __shared__ __align__(1024) uint8_t dsm[];
-    uint8_t *ring = dsm + ((1024 - (tc::smem_addr(dsm) & 1023)) & 1023);
-    __shared__ __align__(8) Barriers bars;
-    __shared__ uint32_t tmem_base;
-    __shared__ int aborted;
+    for (int kb = 0; kb < g.nK; ++kb) {
+        ab.wait(&bars.empty[p.stage], p.phase ^ 1);
+        if (ab.on())
+            return;
+        uint64_t *full = &bars.full[p.stage];
+        tc::bar_expect_tx(full, kStageBytes);
+        used |= 1u << p.stage;
+        last = (last & ~(1u << p.stage)) | (p.phase << p.stage);
+        uint8_t *st = ring + p.stage * kStageBytes;
+        const int ka = g.a_k0 + kb * kBK, kbb = g.b_k0 + kb * kBK;
+        if (A_MN) {  // MN-major: boxes of 64 rows of M along the inner dimension
+#pragma unroll
+            for (int i = 0; i < kBM / 64; ++i)
+                tc::tma_load_2d(st + i * kMnBox, &tmA, g.a_row0 + m * kBM + 64 * i, ka, full);
+        } else {
+            tc::tma_load_2d(st, &tmA, ka, g.a_row0 + m * kBM, full);
+        }
+        if (MC) {  // this CTA's half of B, to both CTAs
+            if (B_MN) {
+#pragma unroll
+                for (int i = 2 * rank; i < 2 * rank + 2; ++i)
+                    tc::tma_load_2d_mc(st + kStageA + i * kMnBox, &tmB,
+                                       g.b_row0 + n * kBN + 64 * i, kbb, full, 0x3);
+            } else {
+                tc::tma_load_2d_mc(st + kStageA + rank * (kStageB / 2), &tmB, kbb,
+                                   g.b_row0 + n * kBN + rank * (kBN / 2), full, 0x3);
+            }
+        } else if (B_MN) {
+#pragma unroll
+            for (int i = 0; i < kBN / 64; ++i)
+                tc::tma_load_2d(st + kStageA + i * kMnBox, &tmB, g.b_row0 + n * kBN + 64 * i,
+                                kbb, full);
+        } else {
+            tc::tma_load_2d(st + kStageA, &tmB, kbb, g.b_row0 + n * kBN, full);
+        }
+        p.next();
+    }
+}
 
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int nUnits = n_units<MC>(g);
-    const int rank = MC ? (int)tc::cluster_ctarank() : 0;
-    const int unit0 = MC ? (int)(blockIdx.x >> 1) : (int)blockIdx.x;
-    const int ustep = MC ? (int)(gridDim.x >> 1) : (int)gridDim.x;
+// The MMAs of one tile into the accumulator at TMEM column d: nK stages of
+// four K=16 steps.  Returns early once the CTA aborted.
+template <bool A_MN, bool B_MN, bool MC>
+__device__ __forceinline__ void mma_tile(const GemmArgs &g, uint32_t d, uint8_t *ring,
+                                         Barriers &bars, const Abort &ab, Ring &p)
+{
+    constexpr uint32_t kId =
+        tc::idesc_bf16(kBM, kBN) | ((uint32_t)A_MN << 15) | ((uint32_t)B_MN << 16);
+    // a K step of 16: 32 bytes along a K-major row, 16 rows (2 K groups) of an
+    // MN-major tile
+    constexpr uint32_t a_step = A_MN ? 16 * 128 : 32, b_step = B_MN ? 16 * 128 : 32;
+    for (int kb = 0; kb < g.nK; ++kb) {
+        ab.wait(&bars.full[p.stage], p.phase);
+        if (ab.on())
+            return;
+        tc::fence_after_sync();
+        const uint32_t sa = tc::smem_addr(ring + p.stage * kStageBytes);
+        const uint32_t sb = sa + kStageA;
+#pragma unroll
+        for (int kk = 0; kk < kBK / 16; ++kk) {
+            const uint64_t da = A_MN ? tc::desc_sw128_mn(sa + kk * a_step, kMnBox)
+                                     : tc::desc_sw128(sa + kk * a_step);
+            const uint64_t db = B_MN ? tc::desc_sw128_mn(sb + kk * b_step, kMnBox)
+                                     : tc::desc_sw128(sb + kk * b_step);
+            tc::mma_bf16(d, da, db, kId, (kb | kk) != 0);
+        }
+        if (MC)  // the stage is free in this CTA and in the peer
+            tc::mma_commit_mc(&bars.empty[p.stage], 0x3);
+        else
+            tc::mma_commit(&bars.empty[p.stage]);
+        p.next();
+    }
+}
 
+// The epilogue of one tile for one thread: TMEM lane r (tile row r of row
+// tile m), column half `half` of column tile n; taddr addresses the lane's
+// first column of the tile's accumulator.
+template <int EPI>
+__device__ __forceinline__ void epilogue_tile(const GemmArgs &g, uint32_t taddr, int m, int n,
+                                              int r, int half)
+{
+    const int cbeg = half * kHalf;
+    if (EPI == kStats) {
+        const int row = m * kBM + r;  // token
+        const int y_r = row < g.T ? g.ids[row] : -1;
+        const bool ent = g.part_u != nullptr;
+        float mx = -INFINITY, s = 0.0f, u = 0.0f, zyv = 0.0f;
+        bool got_y = false;
+        for (int c0 = cbeg; c0 < cbeg + kHalf; c0 += 32) {
+            float v[32];
+            tc::tmem_ld32(taddr + c0, v);
+            const int base = g.col0 + n * kBN + c0;
+            if (y_r >= base && y_r < base + 32) {
+#pragma unroll
+                for (int q = 0; q < 32; ++q)
+                    if (base + q == y_r)
+                        zyv = v[q];
+                got_y = true;
+            }
+            float cm = -INFINITY;
+#pragma unroll
+            for (int q = 0; q < 32; ++q) {
+                const int col = base + q;
+                v[q] = (col == y_r || col >= g.V) ? -INFINITY : v[q];
+                cm = fmaxf(cm, v[q]);
+            }
+            if (cm > mx) {
+                if (mx == -INFINITY) {
+                    s = 0.0f;
+                    u = 0.0f;
+                } else {
+                    const float d = mx - cm, f = ex2_ftz(d * kLog2e);
+                    u = fmaf(d, s, u) * f;
+                    s *= f;
+                }
+                mx = cm;
+            }
+            if (mx != -INFINITY) {
+                float a = 0.0f, au = 0.0f;
+                if (ent) {  // the entropy term, e (z - max)
+#pragma unroll
+                    for (int q = 0; q < 32; ++q) {
+                        const float d = v[q] - mx, e = ex2_ftz(d * kLog2e);
+                        a += e;
+                        au = fmaf(e, fmaxf(d, -1024.0f), au);
+                    }
+                } else {
+#pragma unroll
+                    for (int q = 0; q < 32; ++q)
+                        a += ex2_ftz((v[q] - mx) * kLog2e);
+                }
+                s += a;
+                u += au;
+            }
+        }
+        if (row < g.T) {  // one (max, sum) per 128-column half
+            const int64_t pi = (int64_t)(2 * n + half) * g.T + row;
+            g.part[pi] = make_float2(mx, s);
+            if (ent)
+                g.part_u[pi] = u;
+            if (got_y)
+                g.zy[row] = zyv;
+        }
+    } else if (EPI == kDz) {
+        const int row = m * kBM + r;  // token; rows up to Tp are allocated
+        const bool live = row < g.T;
+        // tokens with c = 0 (masked, clipped, past T) give 0 without
+        // touching the exponential (their lse is a placeholder)
+        const float c_r = live ? g.cvec[row] : 0.0f;
+        const float lse_r = live ? g.lse[row] : 0.0f;
+        const int y_r = live ? g.ids[row] : -1;
+        const int cl0 = n * kBN;  // chunk-local column of the tile
+        for (int c0 = cbeg; c0 < cbeg + kHalf; c0 += 32) {
+            float v[32];
+            tc::tmem_ld32(taddr + c0, v);
+            const int gc0 = g.col0 + cl0 + c0;  // vocabulary index of v[0]
+            uint32_t w[16];
+#pragma unroll
+            for (int q = 0; q < 32; q += 2) {
+                float d[2];
+#pragma unroll
+                for (int h = 0; h < 2; ++h) {
+                    const int gc = gc0 + q + h;
+                    d[h] = (gc < g.V && c_r != 0.0f)
+                               ? c_r * ex2_ftz((v[q + h] - lse_r) * kLog2e) -
+                                     (gc == y_r ? c_r : 0.0f)
+                               : 0.0f;
+                }
+                w[q >> 1] = pack_bf16x2(d[0], d[1]);
+            }
+            // 64 bytes of the row in two full-sector stores (read back by
+            // the next two launches, DH and DW)
+            uint16_t *drow = g.dz + (int64_t)row * g.ld_dz + cl0 + c0;
+            st_v8_cs(drow, w);
+            st_v8_cs(drow + 16, w + 8);
+        }
+    } else {
+        const int lr = m * kBM + r;  // row of the output block
+        const bool live = lr < g.rows_valid;
+        const int64_t o = (int64_t)lr * g.ld_out + (int64_t)n * kBN;
+        for (int c0 = cbeg; c0 < cbeg + kHalf; c0 += 32) {
+            float v[32];
+            tc::tmem_ld32(taddr + c0, v);
+            if (!live)
+                continue;
+            if (g.out_bf16) {
+                uint32_t w[16];
+#pragma unroll
+                for (int q = 0; q < 16; ++q)
+                    w[q] = pack_bf16x2(v[2 * q], v[2 * q + 1]);
+                uint16_t *dst = reinterpret_cast<uint16_t *>(g.out) + o + c0;
+                if (g.out_v8) {  // streaming: outputs are not re-read here
+                    st_v8_cs(dst, w);
+                    st_v8_cs(dst + 16, w + 8);
+                } else {
+                    uint4 *d4 = reinterpret_cast<uint4 *>(dst);
+#pragma unroll
+                    for (int q = 0; q < 4; ++q)
+                        __stcs(d4 + q, make_uint4(w[4 * q], w[4 * q + 1], w[4 * q + 2],
+                                                  w[4 * q + 3]));
+                }
+            } else if (g.out_v8) {
+                float *dst = reinterpret_cast<float *>(g.out) + o + c0;
+#pragma unroll
+                for (int q = 0; q < 4; ++q) {
+                    float x[8];
+#pragma unroll
+                    for (int e = 0; e < 8; ++e)
+                        x[e] = v[8 * q + e];
+                    if (EPI == kAccum) {
+                        float old[8];
+                        ld_v8(dst + 8 * q, old);
+#pragma unroll
+                        for (int e = 0; e < 8; ++e)
+                            x[e] += old[e];
+                    }
+                    st_v8_cs(dst + 8 * q, reinterpret_cast<const uint32_t *>(x));
+                }
+            } else {
+                float4 *dst = reinterpret_cast<float4 *>(
+                    reinterpret_cast<float *>(g.out) + o + c0);
+#pragma unroll
+                for (int q = 0; q < 8; ++q) {
+                    float4 x = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2],
+                                           v[4 * q + 3]);
+                    if (EPI == kAccum) {
+                        const float4 old = dst[q];
+                        x.x += old.x;
+                        x.y += old.y;
+                        x.z += old.z;
+                        x.w += old.w;
+                    }
+                    __stcs(dst + q, x);
+                }
+            }
+        }
+    }
+}
+
+// Shared memory of a GEMM CTA besides the ring.
+struct GemmShared {
+    Barriers bars;
+    uint32_t tmem_base;
+    int aborted;
+};
+
+// Barriers, TMEM and (MC) the cluster, before the roles start.
+template <bool MC> __device__ __forceinline__ void gemm_setup(GemmShared &sh, int warp)
+{
     if (threadIdx.x == 0) {
-        aborted = 0;
+        sh.aborted = 0;
         for (int s = 0; s < kStages; ++s) {
-            tc::bar_init(&bars.full[s], 1);
+            tc::bar_init(&sh.bars.full[s], 1);
             // with MC both CTAs' MMAs release a stage: the peer's multicast
             // writes into this CTA's copy of it
-            tc::bar_init(&bars.empty[s], MC ? 2 : 1);
+            tc::bar_init(&sh.bars.empty[s], MC ? 2 : 1);
         }
         for (int b = 0; b < 2; ++b) {
-            tc::bar_init(&bars.accfull[b], 1);
-            tc::bar_init(&bars.accempty[b], kEpiThreads);
+            tc::bar_init(&sh.bars.accfull[b], 1);
+            tc::bar_init(&sh.bars.accempty[b], kEpiThreads);
         }
-        tc::bar_init(&bars.done, 1);
+        tc::bar_init(&sh.bars.done, 1);
         tc::bar_init_fence();
     }
     if (warp == 1)
-        tc::tmem_alloc(&tmem_base, kTmemCols);
+        tc::tmem_alloc(&sh.tmem_base, kTmemCols);
     tc::fence_before_sync();
     __syncthreads();
     if (MC)
         tc::cluster_sync();  // the peer's barriers exist before anything signals them
     tc::fence_after_sync();
-    const uint32_t tmem = tmem_base;
-    const Abort ab{&aborted, g.status};
+}
 
-    if (warp == 0) {
-        // ---------------------------------------------------------- producer
-        if (lane == 0) {
-            int stage = 0;
-            uint32_t phase = 0, used = 0, last = 0;  // per stage: loaded, parity of its last load
-            for (int u = unit0; u < nUnits && !ab.on(); u += ustep) {
-                int m, n;
-                unit_mn<MC>(g, u, rank, m, n);
-                for (int kb = 0; kb < g.nK; ++kb) {
-                    ab.wait(&bars.empty[stage], phase ^ 1);
-                    if (ab.on())
-                        break;
-                    tc::bar_expect_tx(&bars.full[stage], kStageBytes);
-                    used |= 1u << stage;
-                    last = (last & ~(1u << stage)) | (phase << stage);
-                    uint8_t *st = ring + stage * kStageBytes;
-                    const int ka = g.a_k0 + kb * kBK, kbb = g.b_k0 + kb * kBK;
-                    if (A_MN) {  // MN-major: boxes of 64 rows of M along the inner dimension
-#pragma unroll
-                        for (int i = 0; i < kBM / 64; ++i)
-                            tc::tma_load_2d(st + i * kMnBox, &tmA, g.a_row0 + m * kBM + 64 * i, ka,
-                                            &bars.full[stage]);
-                    } else {
-                        tc::tma_load_2d(st, &tmA, ka, g.a_row0 + m * kBM, &bars.full[stage]);
-                    }
-                    if (MC) {  // this CTA's half of B, to both CTAs
-                        if (B_MN) {
-#pragma unroll
-                            for (int i = 2 * rank; i < 2 * rank + 2; ++i)
-                                tc::tma_load_2d_mc(st + kStageA + i * kMnBox, &tmB,
-                                                   g.b_row0 + n * kBN + 64 * i, kbb,
-                                                   &bars.full[stage], 0x3);
-                        } else {
-                            tc::tma_load_2d_mc(st + kStageA + rank * (kStageB / 2), &tmB, kbb,
-                                               g.b_row0 + n * kBN + rank * (kBN / 2),
-                                               &bars.full[stage], 0x3);
-                        }
-                    } else if (B_MN) {
-#pragma unroll
-                        for (int i = 0; i < kBN / 64; ++i)
-                            tc::tma_load_2d(st + kStageA + i * kMnBox, &tmB,
-                                            g.b_row0 + n * kBN + 64 * i, kbb, &bars.full[stage]);
-                    } else {
-                        tc::tma_load_2d(st + kStageA, &tmB, kbb, g.b_row0 + n * kBN,
-                                        &bars.full[stage]);
-                    }
-                    if (++stage == kStages) {
-                        stage = 0;
-                        phase ^= 1;
-                    }
-                }
-            }
-            // no load may still be landing when the CTA leaves
-            for (int s = 0; s < kStages; ++s)
-                if (used & (1u << s))
-                    tc::bar_wait(&bars.full[s], (last >> s) & 1);
-        }
-    } else if (warp == 1) {
-        // ---------------------------------------------------------- MMA issue
-        if (lane == 0) {
-            constexpr uint32_t kId = tc::idesc_bf16(kBM, kBN) | ((uint32_t)A_MN << 15) |
-                                     ((uint32_t)B_MN << 16);
-            // a K step of 16: 32 bytes along a K-major row, 16 rows (2 K
-            // groups) of an MN-major tile
-            constexpr uint32_t a_step = A_MN ? 16 * 128 : 32, b_step = B_MN ? 16 * 128 : 32;
-            int stage = 0;
-            uint32_t phase = 0;
-            int i = 0;
-            for (int u = unit0; u < nUnits && !ab.on(); u += ustep, ++i) {
-                const int acc = i & 1;
-                ab.wait(&bars.accempty[acc], ((i >> 1) & 1) ^ 1);
-                tc::fence_after_sync();
-                const uint32_t d = tmem + acc * kBN;
-                for (int kb = 0; kb < g.nK; ++kb) {
-                    ab.wait(&bars.full[stage], phase);
-                    if (ab.on())
-                        break;
-                    tc::fence_after_sync();
-                    const uint32_t sa = tc::smem_addr(ring + stage * kStageBytes);
-                    const uint32_t sb = sa + kStageA;
-#pragma unroll
-                    for (int kk = 0; kk < kBK / 16; ++kk) {
-                        const uint64_t da = A_MN ? tc::desc_sw128_mn(sa + kk * a_step, kMnBox)
-                                                 : tc::desc_sw128(sa + kk * a_step);
-                        const uint64_t db = B_MN ? tc::desc_sw128_mn(sb + kk * b_step, kMnBox)
-                                                 : tc::desc_sw128(sb + kk * b_step);
-                        tc::mma_bf16(d, da, db, kId, (kb | kk) != 0);
-                    }
-                    if (MC)  // the stage is free in this CTA and in the peer
-                        tc::mma_commit_mc(&bars.empty[stage], 0x3);
-                    else
-                        tc::mma_commit(&bars.empty[stage]);
-                    if (++stage == kStages) {
-                        stage = 0;
-                        phase ^= 1;
-                    }
-                }
-                tc::mma_commit(&bars.accfull[acc]);
-            }
-            // every MMA of this CTA is done before TMEM is released
-            tc::mma_commit(&bars.done);
-            tc::bar_wait(&bars.done, 0);
-        }
-    } else {
-        // ---------------------------------------------------------- epilogue
-        // warps 2..9: TMEM lane quadrant warp % 4 (one tile row per thread),
-        // column half (warp - 2) / 4 of the 256-column tile
-        const int lg = warp & 3;
-        const int half = (warp - 2) >> 2;
-        const int r = lg * 32 + lane;
-        const uint32_t lane_off = (uint32_t)(lg * 32) << 16;
-        const int cbeg = half * kHalf;
-        int i = 0;
-        for (int u = unit0; u < nUnits; u += ustep, ++i) {
-            if (__syncthreads_or_epi(ab.on()))
-                break;
-            int m, n;
-            unit_mn<MC>(g, u, rank, m, n);
-            const int acc = i & 1;
-            ab.wait(&bars.accfull[acc], (i >> 1) & 1);
-            tc::fence_after_sync();
-            const uint32_t taddr = tmem + lane_off + acc * kBN;
-            if (MC && m >= g.nMt) {
-                // the padding tile of an odd row count: nothing to write
-            } else if (EPI == kStats) {
-                const int row = m * kBM + r;  // token
-                const int y_r = row < g.T ? g.ids[row] : -1;
-                const bool ent = g.part_u != nullptr;
-                float mx = -INFINITY, s = 0.0f, u = 0.0f, zyv = 0.0f;
-                bool got_y = false;
-                for (int c0 = cbeg; c0 < cbeg + kHalf; c0 += 32) {
-                    float v[32];
-                    tc::tmem_ld32(taddr + c0, v);
-                    const int base = g.col0 + n * kBN + c0;
-                    if (y_r >= base && y_r < base + 32) {
-#pragma unroll
-                        for (int q = 0; q < 32; ++q)
-                            if (base + q == y_r)
-                                zyv = v[q];
-                        got_y = true;
-                    }
-                    float cm = -INFINITY;
-#pragma unroll
-                    for (int q = 0; q < 32; ++q) {
-                        const int col = base + q;
-                        v[q] = (col == y_r || col >= g.V) ? -INFINITY : v[q];
-                        cm = fmaxf(cm, v[q]);
-                    }
-                    if (cm > mx) {
-                        if (mx == -INFINITY) {
-                            s = 0.0f;
-                            u = 0.0f;
-                        } else {
-                            const float d = mx - cm, f = ex2_ftz(d * kLog2e);
-                            u = fmaf(d, s, u) * f;
-                            s *= f;
-                        }
-                        mx = cm;
-                    }
-                    if (mx != -INFINITY) {
-                        float a = 0.0f, au = 0.0f;
-                        if (ent) {  // the entropy term, e (z - max)
-#pragma unroll
-                            for (int q = 0; q < 32; ++q) {
-                                const float d = v[q] - mx, e = ex2_ftz(d * kLog2e);
-                                a += e;
-                                au = fmaf(e, fmaxf(d, -1024.0f), au);
-                            }
-                        } else {
-#pragma unroll
-                            for (int q = 0; q < 32; ++q)
-                                a += ex2_ftz((v[q] - mx) * kLog2e);
-                        }
-                        s += a;
-                        u += au;
-                    }
-                }
-                if (row < g.T) {  // one (max, sum) per 128-column half
-                    const int64_t pi = (int64_t)(2 * n + half) * g.T + row;
-                    g.part[pi] = make_float2(mx, s);
-                    if (ent)
-                        g.part_u[pi] = u;
-                    if (got_y)
-                        g.zy[row] = zyv;
-                }
-            } else if (EPI == kDz) {
-                const int row = m * kBM + r;  // token; rows up to Tp are allocated
-                const bool live = row < g.T;
-                // tokens with c = 0 (masked, clipped, past T) give 0 without
-                // touching the exponential (their lse is a placeholder)
-                const float c_r = live ? g.cvec[row] : 0.0f;
-                const float lse_r = live ? g.lse[row] : 0.0f;
-                const int y_r = live ? g.ids[row] : -1;
-                const int cl0 = n * kBN;  // chunk-local column of the tile
-                for (int c0 = cbeg; c0 < cbeg + kHalf; c0 += 32) {
-                    float v[32];
-                    tc::tmem_ld32(taddr + c0, v);
-                    const int gc0 = g.col0 + cl0 + c0;  // vocabulary index of v[0]
-                    uint32_t w[16];
-#pragma unroll
-                    for (int q = 0; q < 32; q += 2) {
-                        float d[2];
-#pragma unroll
-                        for (int h = 0; h < 2; ++h) {
-                            const int gc = gc0 + q + h;
-                            d[h] = (gc < g.V && c_r != 0.0f)
-                                       ? c_r * ex2_ftz((v[q + h] - lse_r) * kLog2e) -
-                                             (gc == y_r ? c_r : 0.0f)
-                                       : 0.0f;
-                        }
-                        w[q >> 1] = pack_bf16x2(d[0], d[1]);
-                    }
-                    // 64 bytes of the row in two full-sector stores (read back by
-                    // the next two launches, DH and DW)
-                    uint16_t *drow = g.dz + (int64_t)row * g.ld_dz + cl0 + c0;
-                    st_v8_cs(drow, w);
-                    st_v8_cs(drow + 16, w + 8);
-                }
-            } else {
-                const int lr = m * kBM + r;  // row of the output block
-                const bool live = lr < g.rows_valid;
-                const int64_t o = (int64_t)lr * g.ld_out + (int64_t)n * kBN;
-                for (int c0 = cbeg; c0 < cbeg + kHalf; c0 += 32) {
-                    float v[32];
-                    tc::tmem_ld32(taddr + c0, v);
-                    if (!live)
-                        continue;
-                    if (g.out_bf16) {
-                        uint32_t w[16];
-#pragma unroll
-                        for (int q = 0; q < 16; ++q)
-                            w[q] = pack_bf16x2(v[2 * q], v[2 * q + 1]);
-                        uint16_t *dst = reinterpret_cast<uint16_t *>(g.out) + o + c0;
-                        if (g.out_v8) {  // streaming: outputs are not re-read here
-                            st_v8_cs(dst, w);
-                            st_v8_cs(dst + 16, w + 8);
-                        } else {
-                            uint4 *d4 = reinterpret_cast<uint4 *>(dst);
-#pragma unroll
-                            for (int q = 0; q < 4; ++q)
-                                __stcs(d4 + q, make_uint4(w[4 * q], w[4 * q + 1], w[4 * q + 2],
-                                                          w[4 * q + 3]));
-                        }
-                    } else if (g.out_v8) {
-                        float *dst = reinterpret_cast<float *>(g.out) + o + c0;
-#pragma unroll
-                        for (int q = 0; q < 4; ++q) {
-                            float x[8];
-#pragma unroll
-                            for (int e = 0; e < 8; ++e)
-                                x[e] = v[8 * q + e];
-                            if (EPI == kAccum) {
-                                float old[8];
-                                ld_v8(dst + 8 * q, old);
-#pragma unroll
-                                for (int e = 0; e < 8; ++e)
-                                    x[e] += old[e];
-                            }
-                            st_v8_cs(dst + 8 * q, reinterpret_cast<const uint32_t *>(x));
-                        }
-                    } else {
-                        float4 *dst = reinterpret_cast<float4 *>(
-                            reinterpret_cast<float *>(g.out) + o + c0);
-#pragma unroll
-                        for (int q = 0; q < 8; ++q) {
-                            float4 x = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2],
-                                                   v[4 * q + 3]);
-                            if (EPI == kAccum) {
-                                const float4 old = dst[q];
-                                x.x += old.x;
-                                x.y += old.y;
-                                x.z += old.z;
-                                x.w += old.w;
-                            }
-                            __stcs(dst + q, x);
-                        }
-                    }
-                }
-            }
-            tc::fence_before_sync();
-            tc::bar_arrive(&bars.accempty[acc]);
-        }
-    }
+// The producer's last step: no load may still be landing when the CTA leaves.
+__device__ __forceinline__ void drain_loads(Barriers &bars, uint32_t used, uint32_t last)
+{
+    for (int s = 0; s < kStages; ++s)
+        if (used & (1u << s))
+            tc::bar_wait(&bars.full[s], (last >> s) & 1);
+}
+
+// The MMA thread's last step: every MMA of this CTA is done before TMEM is
+// released.
+__device__ __forceinline__ void drain_mmas(Barriers &bars)
+{
+    tc::mma_commit(&bars.done);
+    tc::bar_wait(&bars.done, 0);
+}
+
+// Every thread, after its role: TMEM freed once nothing uses it; with MC
+// neither CTA leaves while the other may still signal its barriers.
+template <bool MC> __device__ __forceinline__ void gemm_teardown(GemmShared &sh, int warp)
+{
     __syncwarp();
     tc::fence_before_sync();
     __syncthreads();
     if (MC) {
-        // neither CTA leaves while the other may still signal its barriers
         tc::cluster_sync();
         // after a wait ran out the peer may have issued one more multicast
         // into a stage this CTA no longer waits for: give it time to land
-        if (aborted && threadIdx.x == 0) {
+        if (sh.aborted && threadIdx.x == 0) {
             const long long t0 = clock64();
             while (clock64() - t0 < (1ll << 20)) {
             }
@@ -553,8 +545,181 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     if (warp == 1) {
         tc::fence_after_sync();
-        tc::tmem_dealloc(tmem, kTmemCols);
+        tc::tmem_dealloc(sh.tmem_base, kTmemCols);
     }
+}
+
+// The epilogue warps' part of one tile: wait for its accumulator, drain it,
+// hand it back.  Warps 2..9: TMEM lane quadrant warp % 4 (one tile row per
+// thread), column half (warp - 2) / 4 of the 256-column tile.
+template <int EPI, bool MC>
+__device__ __forceinline__ void epilogue_unit(const GemmArgs &g, int m, int n, int i,
+                                              uint32_t tmem, int warp, int lane, Barriers &bars,
+                                              const Abort &ab)
+{
+    const int lg = warp & 3;
+    const int half = (warp - 2) >> 2;
+    const uint32_t lane_off = (uint32_t)(lg * 32) << 16;
+    const int acc = i & 1;
+    ab.wait(&bars.accfull[acc], (i >> 1) & 1);
+    tc::fence_after_sync();
+    // with MC, the padding tile of an odd row count has nothing to write
+    if (!(MC && m >= g.nMt))
+        epilogue_tile<EPI>(g, tmem + lane_off + acc * kBN, m, n, lg * 32 + lane, half);
+    tc::fence_before_sync();
+    tc::bar_arrive(&bars.accempty[acc]);
+}
+
+// The MMA thread's part of one tile: a free accumulator, the tile's MMAs,
+// then the accumulator handed to the epilogue.
+template <bool A_MN, bool B_MN, bool MC>
+__device__ __forceinline__ void mma_unit(const GemmArgs &g, int i, uint32_t tmem, uint8_t *ring,
+                                         Barriers &bars, const Abort &ab, Ring &p)
+{
+    const int acc = i & 1;
+    ab.wait(&bars.accempty[acc], ((i >> 1) & 1) ^ 1);
+    tc::fence_after_sync();
+    mma_tile<A_MN, B_MN, MC>(g, tmem + acc * kBN, ring, bars, ab, p);
+    tc::mma_commit(&bars.accfull[acc]);
+}
+
+template <int EPI, bool A_MN, bool B_MN, bool MC>
+__global__ void __launch_bounds__(kThreads, 1)
+    cis_lmhead_gemm_kernel(const __grid_constant__ CUtensorMap tmA,
+                           const __grid_constant__ CUtensorMap tmB, const GemmArgs g)
+{
+    extern __shared__ __align__(1024) uint8_t dsm[];
+    uint8_t *ring = dsm + ((1024 - (tc::smem_addr(dsm) & 1023)) & 1023);
+    __shared__ __align__(8) GemmShared sh;
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int nUnits = n_units<MC>(g);
+    const int rank = MC ? (int)tc::cluster_ctarank() : 0;
+    const int unit0 = MC ? (int)(blockIdx.x >> 1) : (int)blockIdx.x;
+    const int ustep = MC ? (int)(gridDim.x >> 1) : (int)gridDim.x;
+
+    gemm_setup<MC>(sh, warp);
+    const uint32_t tmem = sh.tmem_base;
+    const Abort ab{&sh.aborted, g.status};
+
+    if (warp == 0) {
+        if (lane == 0) {  // producer
+            Ring p;
+            uint32_t used = 0, last = 0;
+            for (int u = unit0; u < nUnits && !ab.on(); u += ustep) {
+                int m, n;
+                unit_mn<MC>(g, u, rank, m, n);
+                load_tile<A_MN, B_MN, MC>(tmA, tmB, g, m, n, rank, ring, sh.bars, ab, p, used,
+                                          last);
+            }
+            drain_loads(sh.bars, used, last);
+        }
+    } else if (warp == 1) {
+        if (lane == 0) {  // MMA issue
+            Ring p;
+            int i = 0;
+            for (int u = unit0; u < nUnits && !ab.on(); u += ustep, ++i)
+                mma_unit<A_MN, B_MN, MC>(g, i, tmem, ring, sh.bars, ab, p);
+            drain_mmas(sh.bars);
+        }
+    } else {  // epilogue
+        int i = 0;
+        for (int u = unit0; u < nUnits; u += ustep, ++i) {
+            if (__syncthreads_or_epi(ab.on()))
+                break;
+            int m, n;
+            unit_mn<MC>(g, u, rank, m, n);
+            epilogue_unit<EPI, MC>(g, m, n, i, tmem, warp, lane, sh.bars, ab);
+        }
+    }
+    gemm_teardown<MC>(sh, warp);
+}
+
+// The dH and dW GEMMs of one vocabulary chunk in one launch.  Launched one
+// after the other, each ends in a partial wave: dH has 512 pair units of 512 K
+// blocks for 76 clusters (6.7 waves), dW 1024 of 256 (13.5 waves).  Here
+// every group (a cluster with MC, else a CTA) works through its own list of
+// units from both GEMMs: a greedy schedule made on the host, which hands the
+// units out in order (all of dH, then dW) to the group that frees up first, by
+// their K blocks.  The lists are kernel parameters.
+constexpr int kMaxSchedGroups = 160;
+constexpr int kMaxSchedUnits = 4096;
+constexpr uint16_t kSchedSecond = 0x8000;  // a unit of the second GEMM
+struct DualSched {
+    uint16_t off[kMaxSchedGroups + 1];  // group c takes unit[off[c]] .. unit[off[c + 1] - 1]
+    uint16_t unit[kMaxSchedUnits];      // unit index, | kSchedSecond for the second GEMM
+};
+
+// GEMM 0: dH (+)= dz W_c (A = dz K-major, B = W MN-major, EPI0 = kStore on
+// the first chunk, kAccum after); GEMM 1: dW_c = dz^T H (A = dz MN-major,
+// B = H MN-major, kStore).
+template <int EPI0, bool MC>
+__global__ void __launch_bounds__(kThreads, 1)
+    cis_lmhead_dual_kernel(const __grid_constant__ CUtensorMap tmA0,
+                           const __grid_constant__ CUtensorMap tmB0,
+                           const __grid_constant__ CUtensorMap tmA1,
+                           const __grid_constant__ CUtensorMap tmB1, const GemmArgs g0,
+                           const GemmArgs g1, const __grid_constant__ DualSched sc)
+{
+    extern __shared__ __align__(1024) uint8_t dsm[];
+    uint8_t *ring = dsm + ((1024 - (tc::smem_addr(dsm) & 1023)) & 1023);
+    __shared__ __align__(8) GemmShared sh;
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int rank = MC ? (int)tc::cluster_ctarank() : 0;
+    const int grp = MC ? (int)(blockIdx.x >> 1) : (int)blockIdx.x;
+    const int j0 = sc.off[grp], j1 = sc.off[grp + 1];
+
+    gemm_setup<MC>(sh, warp);
+    const uint32_t tmem = sh.tmem_base;
+    const Abort ab{&sh.aborted, g0.status};
+
+    if (warp == 0) {
+        if (lane == 0) {  // producer
+            Ring p;
+            uint32_t used = 0, last = 0;
+            for (int j = j0; j < j1 && !ab.on(); ++j) {
+                const int u = sc.unit[j];
+                int m, n;
+                if (u & kSchedSecond) {
+                    unit_mn<MC>(g1, u & ~kSchedSecond, rank, m, n);
+                    load_tile<true, true, MC>(tmA1, tmB1, g1, m, n, rank, ring, sh.bars, ab, p,
+                                              used, last);
+                } else {
+                    unit_mn<MC>(g0, u, rank, m, n);
+                    load_tile<false, true, MC>(tmA0, tmB0, g0, m, n, rank, ring, sh.bars, ab, p,
+                                               used, last);
+                }
+            }
+            drain_loads(sh.bars, used, last);
+        }
+    } else if (warp == 1) {
+        if (lane == 0) {  // MMA issue
+            Ring p;
+            for (int j = j0; j < j1 && !ab.on(); ++j) {
+                if (sc.unit[j] & kSchedSecond)
+                    mma_unit<true, true, MC>(g1, j - j0, tmem, ring, sh.bars, ab, p);
+                else
+                    mma_unit<false, true, MC>(g0, j - j0, tmem, ring, sh.bars, ab, p);
+            }
+            drain_mmas(sh.bars);
+        }
+    } else {  // epilogue
+        for (int j = j0; j < j1; ++j) {
+            if (__syncthreads_or_epi(ab.on()))
+                break;
+            const int u = sc.unit[j];
+            int m, n;
+            if (u & kSchedSecond) {
+                unit_mn<MC>(g1, u & ~kSchedSecond, rank, m, n);
+                epilogue_unit<kStore, MC>(g1, m, n, j - j0, tmem, warp, lane, sh.bars, ab);
+            } else {
+                unit_mn<MC>(g0, u, rank, m, n);
+                epilogue_unit<EPI0, MC>(g0, m, n, j - j0, tmem, warp, lane, sh.bars, ab);
+            }
+        }
+    }
+    gemm_teardown<MC>(sh, warp);
 }
 
 // dst[i] = bf16(src[i]) (round to nearest even)
@@ -734,6 +899,130 @@ cudaError_t launch_gemm_mc(const CUtensorMap &a, const CUtensorMap &b, const Gem
     cfg.gridDim = dim3((unsigned)(2 * (units < clusters ? units : clusters)));
     e = cudaLaunchKernelEx(&cfg, k, a, b, g);
     return e != cudaSuccess ? e : cudaGetLastError();
+}
+
+// The groups that run at once: co-resident 2-CTA clusters (MC), else SMs.
+template <typename K> cudaError_t resident_groups(K kern, bool mc, int *groups)
+{
+    int dev = 0, sms = 0;
+    cudaError_t e;
+    if ((e = cudaGetDevice(&dev)) != cudaSuccess ||
+        (e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess)
+        return e;
+    if (!mc) {
+        *groups = sms;
+        return cudaSuccess;
+    }
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = 2;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(2);
+    cfg.blockDim = dim3(kThreads);
+    cfg.dynamicSmemBytes = kSmemBytes;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    if ((e = cudaOccupancyMaxActiveClusters(groups, kern, &cfg)) != cudaSuccess)
+        return e;
+    return *groups > 0 ? cudaSuccess : cudaErrorNotSupported;
+}
+
+// The greedy schedule of a dual launch: units n0 of GEMM 0 (c0 K blocks
+// each), then n1 of GEMM 1 (c1 each), each to the group whose list ends
+// earliest (ties: the lowest group).  The units of one GEMM go out in order,
+// so the groups at work at any time hold neighbouring units, which share their
+// operands in L2.  False if it does not fit a DualSched.
+static bool make_dual_sched(int n0, int c0, int n1, int c1, int groups, DualSched *s)
+{
+    if (groups < 1 || groups > kMaxSchedGroups || n0 + n1 > kMaxSchedUnits || n0 < 0 ||
+        n1 < 0 || n0 >= kSchedSecond || n1 >= kSchedSecond)
+        return false;
+    std::vector<int64_t> end(groups, 0);
+    std::vector<std::vector<uint16_t>> lists(groups);
+    for (int j = 0; j < n0 + n1; ++j) {
+        int best = 0;
+        for (int c = 1; c < groups; ++c)
+            if (end[c] < end[best])
+                best = c;
+        const bool second = j >= n0;
+        end[best] += second ? c1 : c0;
+        lists[best].push_back(second ? (uint16_t)((j - n0) | kSchedSecond) : (uint16_t)j);
+    }
+    int k = 0;
+    for (int c = 0; c < groups; ++c) {
+        s->off[c] = (uint16_t)k;
+        for (uint16_t u : lists[c])
+            s->unit[k++] = u;
+    }
+    for (int c = groups; c <= kMaxSchedGroups; ++c)
+        s->off[c] = (uint16_t)k;
+    return true;
+}
+
+// One launch of cis_lmhead_dual_kernel over both GEMMs' units; false (and no
+// launch) if the schedule does not fit, so that the caller launches them one
+// after the other.  Schedules are kept per shape: a call makes two (full
+// chunks, the last chunk).
+template <int EPI0, bool MC>
+cudaError_t launch_dual(const CUtensorMap &a0, const CUtensorMap &b0, const GemmArgs &g0,
+                        const CUtensorMap &a1, const CUtensorMap &b1, const GemmArgs &g1,
+                        cudaStream_t s, bool *launched)
+{
+    *launched = false;
+    auto k = cis_lmhead_dual_kernel<EPI0, MC>;
+    cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)kSmemBytes);
+    if (e != cudaSuccess)
+        return e;
+    int groups = 0;
+    if ((e = resident_groups(k, MC, &groups)) != cudaSuccess)
+        return e;
+    const int n0 = MC ? n_units<true>(g0) : n_units<false>(g0);
+    const int n1 = MC ? n_units<true>(g1) : n_units<false>(g1);
+    if (g0.nK <= 0 || g1.nK <= 0 || n0 <= 0 || n1 <= 0)
+        return cudaSuccess;
+    static std::mutex mu;
+    static std::map<std::array<int, 5>, std::unique_ptr<DualSched>> cache;
+    const DualSched *sc = nullptr;
+    {
+        std::lock_guard<std::mutex> lock(mu);
+        const std::array<int, 5> key = {n0, g0.nK, n1, g1.nK, groups};
+        auto it = cache.find(key);
+        if (it == cache.end()) {
+            std::unique_ptr<DualSched> p(new DualSched());
+            if (!make_dual_sched(n0, g0.nK, n1, g1.nK, groups, p.get()))
+                return cudaSuccess;
+            it = cache.emplace(key, std::move(p)).first;
+        }
+        sc = it->second.get();
+    }
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = MC ? 2 : 1;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)(groups * (MC ? 2 : 1)));
+    cfg.blockDim = dim3(kThreads);
+    cfg.dynamicSmemBytes = kSmemBytes;
+    cfg.stream = s;
+    cfg.attrs = attr;
+    cfg.numAttrs = MC ? 1 : 0;
+    e = cudaLaunchKernelEx(&cfg, k, a0, b0, a1, b1, g0, g1, *sc);
+    if (e == cudaSuccess)
+        e = cudaGetLastError();
+    *launched = e == cudaSuccess;
+    return e;
+}
+
+// Whether a chunk's dH and dW run as one launch (CIS_LMHEAD_DUAL=0: one after
+// the other; the results are the same either way).
+static bool dual_on()
+{
+    const char *e = getenv("CIS_LMHEAD_DUAL");
+    return !(e && e[0] == '0');
 }
 
 // Which GEMMs run on 2-CTA multicast clusters: a bit mask over FWD (1), DZ
@@ -994,43 +1283,65 @@ CIS_API cis_status_t cis_lmhead_fused(const void *hidden, const void *weight, in
                 return CIS_ERR_UNSUPPORTED;
             // DH (+)= dz W[chunk]: A = dz [Tp, w] K-major, B = W rows v0 .. v0 + w
             // MN-major (N along Hd, K along the vocabulary)
-            g.nMt = nTt;
-            g.nNt = nHt;
-            g.nK = (int)((w + lm::kBK - 1) / lm::kBK);
-            g.raster_n = 0;
-            g.a_row0 = 0;
-            g.a_k0 = 0;
-            g.b_row0 = 0;
-            g.b_k0 = (int)v0;
-            g.out = dh_acc;
-            g.out_bf16 = 0;
-            g.out_v8 = (reinterpret_cast<uintptr_t>(dh_acc) & 31) == 0;
-            g.rows_valid = (int)T;
-            g.ld_out = H;
-            if (mc & 4)
-                e = v0 == 0 ? lm::launch_gemm_mc<lm::kStore, false, true>(mDz, mWmn, g, s)
-                            : lm::launch_gemm_mc<lm::kAccum, false, true>(mDz, mWmn, g, s);
-            else
-                e = v0 == 0 ? lm::launch_gemm<lm::kStore, false, true>(mDz, mWmn, g, s)
-                            : lm::launch_gemm<lm::kAccum, false, true>(mDz, mWmn, g, s);
-            if (e != cudaSuccess)
-                return CIS_ERR_CUDA;
+            lm::GemmArgs gdh = g;
+            gdh.nMt = nTt;
+            gdh.nNt = nHt;
+            gdh.nK = (int)((w + lm::kBK - 1) / lm::kBK);
+            gdh.raster_n = 0;
+            gdh.a_row0 = 0;
+            gdh.a_k0 = 0;
+            gdh.b_row0 = 0;
+            gdh.b_k0 = (int)v0;
+            gdh.out = dh_acc;
+            gdh.out_bf16 = 0;
+            gdh.out_v8 = (reinterpret_cast<uintptr_t>(dh_acc) & 31) == 0;
+            gdh.rows_valid = (int)T;
+            gdh.ld_out = H;
             // DW[chunk] = dz^T H: A = dz MN-major (M along the chunk's columns,
             // K along the tokens), B = H MN-major (N along Hd, K along tokens)
-            g.nMt = (int)((w + lm::kBM - 1) / lm::kBM);
-            g.nNt = nHt;
-            g.nK = (int)((T + lm::kBK - 1) / lm::kBK);
-            g.raster_n = 0;
-            g.b_k0 = 0;
-            g.out = static_cast<uint8_t *>(dweight) +
-                    (size_t)v0 * (size_t)H * (grad_dtype == CIS_BF16 ? 2 : 4);
-            g.out_bf16 = grad_dtype == CIS_BF16;
-            g.out_v8 = (reinterpret_cast<uintptr_t>(g.out) & 31) == 0;
-            g.rows_valid = (int)w;
-            if (((mc & 8) ? lm::launch_gemm_mc<lm::kStore, true, true>(mDzmn, mHmn, g, s)
-                          : lm::launch_gemm<lm::kStore, true, true>(mDzmn, mHmn, g, s)) !=
-                cudaSuccess)
-                return CIS_ERR_CUDA;
+            lm::GemmArgs gdw = gdh;
+            gdw.nMt = (int)((w + lm::kBM - 1) / lm::kBM);
+            gdw.nNt = nHt;
+            gdw.nK = (int)((T + lm::kBK - 1) / lm::kBK);
+            gdw.raster_n = 0;
+            gdw.b_k0 = 0;
+            gdw.out = static_cast<uint8_t *>(dweight) +
+                      (size_t)v0 * (size_t)H * (grad_dtype == CIS_BF16 ? 2 : 4);
+            gdw.out_bf16 = grad_dtype == CIS_BF16;
+            gdw.out_v8 = (reinterpret_cast<uintptr_t>(gdw.out) & 31) == 0;
+            gdw.rows_valid = (int)w;
+            // both in one launch where the schedule fits (and both take the
+            // same CTA grouping), else one after the other
+            bool done = false;
+            if (lm::dual_on() && ((mc & 12) == 12 || (mc & 12) == 0)) {
+                const bool pair = (mc & 12) == 12;
+                if (v0 == 0)
+                    e = pair ? lm::launch_dual<lm::kStore, true>(mDz, mWmn, gdh, mDzmn, mHmn, gdw,
+                                                                 s, &done)
+                             : lm::launch_dual<lm::kStore, false>(mDz, mWmn, gdh, mDzmn, mHmn,
+                                                                  gdw, s, &done);
+                else
+                    e = pair ? lm::launch_dual<lm::kAccum, true>(mDz, mWmn, gdh, mDzmn, mHmn, gdw,
+                                                                 s, &done)
+                             : lm::launch_dual<lm::kAccum, false>(mDz, mWmn, gdh, mDzmn, mHmn,
+                                                                  gdw, s, &done);
+                if (e != cudaSuccess)
+                    return CIS_ERR_CUDA;
+            }
+            if (!done) {
+                if (mc & 4)
+                    e = v0 == 0 ? lm::launch_gemm_mc<lm::kStore, false, true>(mDz, mWmn, gdh, s)
+                                : lm::launch_gemm_mc<lm::kAccum, false, true>(mDz, mWmn, gdh, s);
+                else
+                    e = v0 == 0 ? lm::launch_gemm<lm::kStore, false, true>(mDz, mWmn, gdh, s)
+                                : lm::launch_gemm<lm::kAccum, false, true>(mDz, mWmn, gdh, s);
+                if (e != cudaSuccess)
+                    return CIS_ERR_CUDA;
+                if (((mc & 8) ? lm::launch_gemm_mc<lm::kStore, true, true>(mDzmn, mHmn, gdw, s)
+                              : lm::launch_gemm<lm::kStore, true, true>(mDzmn, mHmn, gdw, s)) !=
+                    cudaSuccess)
+                    return CIS_ERR_CUDA;
+            }
         }
         if (grad_dtype == CIS_BF16) {
             lm::cis_lmhead_to_bf16_kernel<<<1184, 256, 0, s>>>(

@@ -167,27 +167,32 @@ def test_lmhead_outputs_16_byte_aligned(grad):
                                               (130, 1900, 512, 512, torch.bfloat16)])
 def test_lmhead_multicast_clusters_bit_identical(monkeypatch, T, V, H, chunk, grad):
     """Every GEMM on 2-CTA clusters sharing each B tile (multicast, the
-    default) against every GEMM on one CTA (CIS_LMHEAD_MC=0): the same tiles
-    with the same MMAs and epilogues, so every output matches bit for bit.
-    T=300 gives an odd number of 128-row token tiles (FWD, DZ, DH), and the
-    last chunks of 332 and 364 columns odd numbers of 128-column vocabulary
-    tiles (DW), so the padding tile of the last pair is exercised; the first
-    case is also checked against the oracle."""
+    default) against every GEMM on one CTA (CIS_LMHEAD_MC=0), each with a
+    chunk's dH and dW in one launch (the default) and in two
+    (CIS_LMHEAD_DUAL=0): the same tiles with the same MMAs and epilogues, so
+    every output matches bit for bit.  T=300 gives an odd number of 128-row
+    token tiles (FWD, DZ, DH), and the last chunks of 332 and 364 columns odd
+    numbers of 128-column vocabulary tiles (DW), so the padding tile of the
+    last pair is exercised; the first case is also checked against the
+    oracle."""
     b = synth.make_batch(5, T=T, V=V, H=H)
     outs = {}
     for mc in ("15", "0"):
-        monkeypatch.setenv("CIS_LMHEAD_MC", mc)
-        outs[mc] = _run(b, grad_dtype=grad, chunk=chunk)
+        for dual in ("1", "0"):
+            monkeypatch.setenv("CIS_LMHEAD_MC", mc)
+            monkeypatch.setenv("CIS_LMHEAD_DUAL", dual)
+            outs[mc, dual] = _run(b, grad_dtype=grad, chunk=chunk)
     torch.cuda.synchronize()
-    a, r = outs["15"], outs["0"]
-    for k in ("lp", "w", "trunc", "dhidden", "dweight", "loss"):
-        x, y = a[k], r[k]
-        if x.dtype.is_floating_point:
-            x = x.view(torch.int16 if x.element_size() == 2 else
-                       (torch.int32 if x.element_size() == 4 else torch.int64))
-            y = y.view(x.dtype)
-        assert torch.equal(x, y), k
-    assert binding.decode_stats(a["stats"])["status"] == 0
+    a = outs["15", "1"]
+    for key, r in outs.items():
+        for k in ("lp", "w", "trunc", "dhidden", "dweight", "loss"):
+            x, y = a[k], r[k]
+            if x.dtype.is_floating_point:
+                x = x.view(torch.int16 if x.element_size() == 2 else
+                           (torch.int32 if x.element_size() == 4 else torch.int64))
+                y = y.view(x.dtype)
+            assert torch.equal(x, y), (key, k)
+        assert binding.decode_stats(r["stats"])["status"] == 0, key
     if T == 300:
         ref = _oracle(b)
         _check_tokens(a, ref, np.arange(T), b, "cis", full=True)
