@@ -75,7 +75,7 @@ extern "C" {
 typedef enum {
     CIS_OK = 0,
     CIS_ERR_INVALID_ARG = 1,   /* host validation failed; nothing was queued   */
-    CIS_ERR_UNSUPPORTED = 2,   /* valid, but not supported by this build/GPU    */
+    CIS_ERR_UNSUPPORTED = 2,   /* valid, but not supported here (layout, GPU)   */
     CIS_ERR_CUDA = 3,          /* a CUDA runtime call or launch failed          */
     CIS_ERR_DEVICE_TIMEOUT = 4,/* device status bit: a bounded wait ran out     */
     CIS_ERR_BAD_TOKEN_ID = 8   /* device status bit: some valid y_t not in [0,V)*/

@@ -985,7 +985,7 @@ cudaError_t launch_dual(const CUtensorMap &a0, const CUtensorMap &b0, const Gemm
         return cudaSuccess;
     static std::mutex mu;
     static std::map<std::array<int, 5>, std::unique_ptr<DualSched>> cache;
-    const DualSched *sc = nullptr;
+    std::unique_ptr<DualSched> sc(new DualSched());  // this call's copy
     {
         std::lock_guard<std::mutex> lock(mu);
         const std::array<int, 5> key = {n0, g0.nK, n1, g1.nK, groups};
@@ -994,9 +994,11 @@ cudaError_t launch_dual(const CUtensorMap &a0, const CUtensorMap &b0, const Gemm
             std::unique_ptr<DualSched> p(new DualSched());
             if (!make_dual_sched(n0, g0.nK, n1, g1.nK, groups, p.get()))
                 return cudaSuccess;
+            if (cache.size() >= 64)  // a process that sees many shapes keeps the last few
+                cache.clear();
             it = cache.emplace(key, std::move(p)).first;
         }
-        sc = it->second.get();
+        *sc = *it->second;
     }
     cudaLaunchAttribute attr[1];
     attr[0].id = cudaLaunchAttributeClusterDimension;
