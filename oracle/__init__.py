@@ -110,6 +110,8 @@ def _load():
                                                     ctypes.POINTER(OracleParams), P, P, P, P, P,
                                                     ctypes.c_int]
         lib.oracle_mismatch_diagnostics.restype = ctypes.c_int
+        lib.oracle_binned_sums.argtypes = [P, P, i64, P, ctypes.c_int, P, ctypes.c_int, P, P]
+        lib.oracle_binned_sums.restype = None
         lib.oracle_max_threads.argtypes = []
         lib.oracle_max_threads.restype = ctypes.c_int
         _ = dbl
@@ -199,6 +201,28 @@ def mismatch_diagnostics(z_train, z_infer, ids, P: OracleParams, mask=None, nthr
     if rc != 0:
         raise ValueError("the diagnostics take a token operator")
     return out
+
+
+def binned_sums(key, edges, values=(), mask=None):
+    """Confidence-binned counts and fp64 sums (Sec. 4.3, Fig. 5b; App. A.5):
+    token t (mask 1) in bin b when edges[b] <= key[t] < edges[b + 1], the last
+    bin closed on the right; NaN or outside keys in no bin.  `key` and each
+    value array are float32 of length T.  Returns (counts [nbins] int64,
+    sums [len(values), nbins] float64)."""
+    lib = _load()
+    key = np.ascontiguousarray(key, dtype=np.float32)
+    T = key.shape[0]
+    edges = np.ascontiguousarray(edges, dtype=np.float64)
+    nbins = edges.shape[0] - 1
+    nv = len(values)
+    vals = (np.ascontiguousarray(np.stack([np.asarray(v, np.float32) for v in values]))
+            if nv else np.zeros((0, T), np.float32))
+    mask = _opt(mask, np.uint8)
+    counts = np.zeros(nbins, np.int64)
+    sums = np.zeros((nv, nbins), np.float64)
+    lib.oracle_binned_sums(_ptr(key), _ptr(mask), T, _ptr(edges), nbins, _ptr(vals), nv,
+                           _ptr(counts), _ptr(sums))
+    return counts, sums
 
 
 def weights(lp_w, lp_inf, P: OracleParams, mask=None, cu_seqlens=None):

@@ -778,3 +778,38 @@ int oracle_mismatch_diagnostics(const void *z_train, const void *z_infer, int dt
     }
     return 0;
 }
+
+/* Confidence-binned sums (Sec. 4.3, Fig. 5b: the sampled tokens binned by
+ * p_t, with E[k_t - f_t] in each bin; App. A.5: logarithmic bins of 1 - p_t).
+ * Token t with mask 1 falls in bin b when edges[b] <= key[t] < edges[b + 1],
+ * the last bin also taking key[t] == edges[nbins]; a NaN key or one outside
+ * [edges[0], edges[nbins]] falls in no bin.  For each bin: the count and, for
+ * each of the nv value arrays values[i * T .. i * T + T - 1], the fp64 sum over
+ * its tokens, added in token order.  Plain loops: the definition written out. */
+void oracle_binned_sums(const float *key, const uint8_t *mask, int64_t T, const double *edges,
+                        int nbins, const float *values, int nv, int64_t *counts, double *sums)
+{
+    for (int b = 0; b < nbins; ++b) {
+        counts[b] = 0;
+        for (int i = 0; i < nv; ++i)
+            sums[(int64_t)i * nbins + b] = 0.0;
+    }
+    for (int64_t t = 0; t < T; ++t) {
+        if (!row_valid(mask, t))
+            continue;
+        const double x = (double)key[t];
+        int bin = -1;
+        for (int b = 0; b < nbins; ++b) {
+            const int last = b == nbins - 1;
+            if (x >= edges[b] && (x < edges[b + 1] || (last && x == edges[b + 1]))) {
+                bin = b;
+                break;
+            }
+        }
+        if (bin < 0)
+            continue;
+        counts[bin] += 1;
+        for (int i = 0; i < nv; ++i)
+            sums[(int64_t)i * nbins + bin] += (double)values[(int64_t)i * T + t];
+    }
+}

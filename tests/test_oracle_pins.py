@@ -832,3 +832,59 @@ def test_diagnostics_closed_forms_for_no_correction_and_exact_ratio():
     # a truncating operator is biased and adds less variance than the exact ratio
     cis = oracle.mismatch_diagnostics(z, zi, ids, oracle.params(mode=oracle.MODE_CIS, lam=0.2))
     assert np.all(cis["bias2"] >= 0) and np.all(cis["dvar"] <= ex["dvar"] + 1e-15)
+
+
+# ---------------------------------------------------------------- confidence bins
+def test_binned_sums_match_numpy_histogram():
+    """Counts and per-bin sums (Sec. 4.3, Fig. 5b; App. A.5's logarithmic bins
+    of 1 - p) equal numpy's histogram with the same edges: half-open bins,
+    the last closed on the right, values outside the edges dropped; NaN keys
+    and masked tokens are in no bin."""
+    rng = _rng(71)
+    T = 5000
+    key = rng.uniform(-0.1, 1.1, T).astype(np.float32)
+    key[::97] = np.nan
+    # edges that float32 keys can equal exactly
+    edges = np.array([0.0, 0.05, 0.2, 0.3, 0.5, 0.565, 0.9, 0.99, 1.0], np.float32).astype(np.float64)
+    key[:8] = edges[:8]            # keys on interior edges go to the upper bin
+    key[8] = 1.0                   # the last edge closes the last bin
+    mask = (rng.random(T) < 0.8).astype(np.uint8)
+    v1 = rng.standard_normal(T).astype(np.float32)
+    v2 = rng.exponential(2.0, T).astype(np.float32)
+    counts, sums = oracle.binned_sums(key, edges, [v1, v2], mask=mask)
+    keep = (mask != 0) & ~np.isnan(key)
+    k64 = key[keep].astype(np.float64)
+    ref_c, _ = np.histogram(k64, bins=edges)
+    assert np.array_equal(counts, ref_c)
+    for i, v in enumerate((v1, v2)):
+        ref_s, _ = np.histogram(k64, bins=edges, weights=v[keep].astype(np.float64))
+        np.testing.assert_allclose(sums[i], ref_s, rtol=1e-12, atol=1e-12)
+    # brute force for the edge tokens themselves
+    for b in range(8):
+        if mask[b]:
+            assert edges[b] <= key[b] < edges[b + 1]
+
+
+def test_binned_sums_of_k_minus_f_on_the_token_pass():
+    """Fig. 5b's quantity: binning the sampled tokens by p and summing k - f
+    gives, for CIS, zero in every bin whose tokens are all under their caps
+    and the token pass's truncated excess (Lemma B.2's k - f) over all bins."""
+    rng = _rng(72)
+    T = 400
+    lp = np.log(rng.uniform(1e-4, 0.9999, T))
+    lp_inf = lp - rng.normal(0.0, 0.6, T)
+    P = oracle.params(mode=oracle.MODE_CIS, lam=2.3)
+    w, tr, lk, _ = oracle.weights(lp, lp_inf, P)
+    k = np.exp(lk)
+    edges = np.array([0.0, 0.1, 0.3, 0.565, 0.9, 0.99, 1.0])
+    counts, sums = oracle.binned_sums(np.exp(lp).astype(np.float32), edges,
+                                      [(k - w).astype(np.float32)])
+    assert counts.sum() == T
+    pbin = np.searchsorted(edges, np.exp(lp).astype(np.float32).astype(np.float64),
+                           side="right") - 1
+    for b in range(len(edges) - 1):
+        sel = pbin == b
+        if not tr[sel].any():
+            assert sums[0, b] == 0.0
+    excess = float(((k - w) * (tr != 0)).sum())
+    np.testing.assert_allclose(sums[0].sum(), excess, rtol=1e-6)
