@@ -416,6 +416,46 @@ CIS_API cis_status_t cis_mismatch_diagnostics(const void *logits_train, const vo
                                               void *stream);
 
 /*
+ * Confidence-binned counts and sums (Sec. 4.3, Fig. 5b: the sampled tokens
+ * binned by p_t, with E[k_t - f_t] in each bin; App. A.5: logarithmic bins of
+ * 1 - p_t).  The key is any per-token value (p, 1 - p, ...); the values are
+ * up to CIS_MAX_BIN_VALUES per-token arrays (k - f from the token pass, the
+ * diagnostics' bias2 and dvar, ...).  A bin's mean is its sum over its count.
+ *   key         device float [T].
+ *   mask        device uint8 [T] or NULL; masked tokens fall in no bin.
+ *   edges       host double [nbins + 1], strictly ascending, no NaN.  Token t
+ *               falls in bin b when edges[b] <= key[t] < edges[b + 1]; the
+ *               last bin also takes key[t] == edges[nbins].  A NaN key, or one
+ *               outside [edges[0], edges[nbins]], falls in no bin.
+ *   nbins       1 .. CIS_MAX_BINS.
+ *   values      host array of nvalues device float [T] pointers (NULL if
+ *               nvalues is 0).
+ *   nvalues     0 .. CIS_MAX_BIN_VALUES.
+ *   counts_out  device int64 [nbins].
+ *   sums_out    device double [nvalues, nbins] (value-major), fp64 sums; a
+ *               NaN value makes its bin's sum NaN.  NULL if nvalues is 0.
+ *   workspace   device, 256-byte aligned, at least
+ *               cis_binned_sums_workspace_size bytes.
+ * Deterministic: fixed-order fp64 sums, the same result on every call.
+ * Asynchronous on `stream`.  CIS_ERR_INVALID_ARG on a NULL required pointer,
+ * T < 0, nbins or nvalues out of range, edges not strictly ascending or a
+ * workspace that is too small or misaligned.
+ */
+#define CIS_MAX_BINS 64
+#define CIS_MAX_BIN_VALUES 4
+CIS_API cis_status_t cis_binned_sums(const float *key, const uint8_t *mask, int64_t T,
+                                     const double *edges, int32_t nbins,
+                                     const float *const *values, int32_t nvalues,
+                                     int64_t *counts_out, double *sums_out, void *workspace,
+                                     size_t workspace_bytes, void *stream);
+
+/* Bytes of device workspace cis_binned_sums needs.  Host only.
+ * CIS_ERR_INVALID_ARG if bytes is NULL, T < 0 or nbins / nvalues are out of
+ * range. */
+CIS_API cis_status_t cis_binned_sums_workspace_size(int64_t T, int32_t nbins, int32_t nvalues,
+                                                    size_t *bytes);
+
+/*
  * Largest T that cis_loss_fwd_bwd_noalloc accepts.
  */
 #define CIS_NOALLOC_MAX_TOKENS 65536

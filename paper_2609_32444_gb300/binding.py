@@ -121,6 +121,12 @@ def lib():
     L.cis_selftest_bounded_wait.restype = ctypes.c_int
     L.cis_profile_next_call.argtypes = [P, P]
     L.cis_profile_next_call.restype = ctypes.c_int
+    L.cis_binned_sums_workspace_size.argtypes = [i64, i32, i32, ctypes.POINTER(ctypes.c_size_t)]
+    L.cis_binned_sums_workspace_size.restype = ctypes.c_int
+    L.cis_binned_sums.argtypes = [P, P, i64, ctypes.POINTER(ctypes.c_double), i32,
+                                  ctypes.POINTER(ctypes.c_void_p), i32, P, P, P, ctypes.c_size_t,
+                                  P]
+    L.cis_binned_sums.restype = ctypes.c_int
     _lib = L
     return L
 
@@ -451,6 +457,35 @@ def cis_mismatch_diagnostics(logits_train: torch.Tensor, logits_infer: torch.Ten
         _ptr(out["p"]), _ptr(out["bias2"]), _ptr(out["dvar"]), _ptr(dev_status), _stream())
     _check(rc, "cis_mismatch_diagnostics")
     return out
+
+
+def cis_binned_sums(key: torch.Tensor, edges, values=(), mask=None):
+    """Confidence-binned counts and fp64 sums (Sec. 4.3, Fig. 5b; App. A.5):
+    `key` and each of `values` are device float [T] tensors, `edges` a
+    sequence of nbins + 1 strictly ascending floats.  Returns (counts int64
+    [nbins], sums float64 [len(values), nbins]) on the device."""
+    _need_cuda(key, mask, *values)
+    T = key.shape[0]
+    _vec(key, torch.float32, T, "key")
+    _vec(mask, torch.uint8, T, "mask")
+    for i, v in enumerate(values):
+        _vec(v, torch.float32, T, f"values[{i}]")
+    e = [float(x) for x in edges]
+    nb, nv = len(e) - 1, len(values)
+    need = ctypes.c_size_t(0)
+    _check(lib().cis_binned_sums_workspace_size(T, nb, nv, ctypes.byref(need)),
+           "cis_binned_sums_workspace_size")
+    wbuf = torch.empty(need.value + 256, dtype=torch.uint8, device=key.device)
+    ws = wbuf[(-wbuf.data_ptr()) % 256:][:need.value]
+    counts = torch.empty(nb, dtype=torch.int64, device=key.device)
+    sums = torch.empty((nv, nb), dtype=torch.float64, device=key.device)
+    earr = (ctypes.c_double * len(e))(*e)
+    varr = (ctypes.c_void_p * max(nv, 1))(*[v.data_ptr() for v in values])
+    rc = lib().cis_binned_sums(_ptr(key), _ptr(mask), T, earr, nb, varr if nv else None, nv,
+                               _ptr(counts), _ptr(sums) if nv else None, _ptr(ws), ws.numel(),
+                               _stream())
+    _check(rc, "cis_binned_sums")
+    return counts, sums
 
 
 def cis_selftest_bounded_wait(max_polls: int, cluster_scope: bool = False,

@@ -182,3 +182,40 @@ def test_selftest_bounded_wait_rejects_bad_arguments(binding):
     assert L.cis_selftest_bounded_wait(0, 0, dummy, None) == binding.CIS_ERR_INVALID_ARG
     assert L.cis_selftest_bounded_wait((1 << 21) + 1, 0, dummy, None) == binding.CIS_ERR_INVALID_ARG
     assert L.cis_selftest_bounded_wait(100, 2, dummy, None) == binding.CIS_ERR_INVALID_ARG
+
+
+def _bins_rc(binding, T=100, nbins=3, edges=(0.0, 0.25, 0.5, 1.0), nvalues=1, ws_bytes=1 << 20,
+             ws=0x20000, key=0x10000, counts=0x30000, sums=0x40000, values=(0x50000,)):
+    """cis_binned_sums with fake device pointers: every case here must fail
+    host validation before the GPU is touched."""
+    L = binding.lib()
+    e = (ctypes.c_double * len(edges))(*edges)
+    v = (ctypes.c_void_p * max(1, len(values)))(*values) if values is not None else None
+    return L.cis_binned_sums(ctypes.c_void_p(key) if key else None, None, T, e, nbins, v,
+                             nvalues, ctypes.c_void_p(counts) if counts else None,
+                             ctypes.c_void_p(sums) if sums else None,
+                             ctypes.c_void_p(ws) if ws else None, ws_bytes, None)
+
+
+@pytest.mark.parametrize("over", [
+    dict(T=-1), dict(nbins=0, edges=(0.0,)), dict(nbins=65, edges=tuple(range(66))),
+    dict(nvalues=5, values=(0x50000,) * 5), dict(nvalues=-1),
+    dict(edges=(0.0, 0.5, 0.5, 1.0)), dict(edges=(0.0, 0.7, 0.5, 1.0)),
+    dict(edges=(0.0, float("nan"), 0.5, 1.0)), dict(key=0), dict(counts=0), dict(sums=0),
+    dict(values=None), dict(ws=0), dict(ws=0x20010), dict(ws_bytes=64),
+])
+def test_binned_sums_host_validation(binding, over):
+    assert _bins_rc(binding, **over) == 1  # CIS_ERR_INVALID_ARG
+
+
+def test_binned_sums_workspace_size(binding):
+    """256-byte blocks of fp64 partials for up to 1024 CTAs of 256 tokens, plus
+    one block for the ticket."""
+    L = binding.lib()
+    n = ctypes.c_size_t()
+    assert L.cis_binned_sums_workspace_size(0, 1, 0, ctypes.byref(n)) == 0
+    assert n.value == 256 + 256
+    assert L.cis_binned_sums_workspace_size(1 << 30, 64, 4, ctypes.byref(n)) == 0
+    assert n.value == (1024 * 64 * 5 * 8 + 255) // 256 * 256 + 256
+    for bad in ((-1, 1, 0), (10, 0, 0), (10, 65, 0), (10, 4, 5)):
+        assert L.cis_binned_sums_workspace_size(*bad, ctypes.byref(n)) == 1
