@@ -217,6 +217,29 @@ def test_diagnostics_write_only_their_outputs(V):
         gb.check("diagnostics " + nm)
 
 
+@pytest.mark.parametrize("T,nbins,nv", [(1000, 18, 2), (300000, 64, 4), (0, 3, 1)])
+def test_binned_sums_write_only_their_outputs(T, nbins, nv):
+    """cis_binned_sums: counts, sums and the workspace (the CTAs' partials and
+    the ticket), one chunk a CTA and several."""
+    rng = np.random.default_rng(T + nbins)
+    key = torch.from_numpy(rng.random(T).astype(np.float32)).cuda()
+    vals = [torch.from_numpy(rng.standard_normal(T).astype(np.float32)).cuda() for _ in range(nv)]
+    L = binding.lib()
+    need = ctypes.c_size_t()
+    assert L.cis_binned_sums_workspace_size(T, nbins, nv, ctypes.byref(need)) == 0
+    ws = Guarded(need.value, seed=71)
+    counts = Guarded(8 * nbins, seed=72)
+    sums = Guarded(8 * nbins * nv, seed=73)
+    edges = np.linspace(0.0, 1.0, nbins + 1)
+    earr = (ctypes.c_double * (nbins + 1))(*edges)
+    varr = (ctypes.c_void_p * nv)(*[v.data_ptr() for v in vals])
+    rc = L.cis_binned_sums(_p(key) if T else None, None, T, earr, nbins, varr, nv, counts.ptr,
+                           sums.ptr, ws.ptr, need.value, _stream())
+    assert rc == 0
+    for nm, gb in dict(counts=counts, sums=sums, workspace=ws).items():
+        gb.check("binned sums " + nm)
+
+
 def test_noalloc_writes_only_its_outputs():
     """cis_loss_fwd_bwd_noalloc (scratch in the library's static array)."""
     b = _batch()
