@@ -159,14 +159,22 @@ struct Abort {
     volatile int *local;
     int32_t *status;
     __device__ __forceinline__ bool on() const { return *local != 0; }
-    __device__ __forceinline__ void wait(uint64_t *bar, uint32_t parity) const
+    // False once the CTA has aborted (now or earlier): the caller stops.  A
+    // phase that has already completed returns at the first poll, without
+    // reading the flag (the MMA thread waits once per stage, and every
+    // instruction of its loop counts).
+    __device__ __forceinline__ bool wait(uint64_t *bar, uint32_t parity) const
     {
+        if (tc::bar_try(bar, parity))
+            return true;
         if (*local)
-            return;
+            return false;
         if (!tc::bar_wait(bar, parity, status)) {
             *local = 1;
             set_status(status, kStatusTimeout);
+            return false;
         }
+        return true;
     }
 };
 
@@ -238,8 +246,7 @@ __device__ __forceinline__ void load_tile(const CUtensorMap &tmA, const CUtensor
                                           Ring &p, uint32_t &used, uint32_t &last)
 {
     for (int kb = 0; kb < g.nK; ++kb) {
-        ab.wait(&bars.empty[p.stage], p.phase ^ 1);
-        if (ab.on())
+        if (!ab.wait(&bars.empty[p.stage], p.phase ^ 1))
             return;
         uint64_t *full = &bars.full[p.stage];
         tc::bar_expect_tx(full, kStageBytes);
@@ -287,21 +294,23 @@ __device__ __forceinline__ void mma_tile(const GemmArgs &g, uint32_t d, uint8_t 
     // a K step of 16: 32 bytes along a K-major row, 16 rows (2 K groups) of an
     // MN-major tile
     constexpr uint32_t a_step = A_MN ? 16 * 128 : 32, b_step = B_MN ? 16 * 128 : 32;
+    // Descriptors of stage 0's A and B tiles; a stage, and a K step inside
+    // it, only move the start address, which sits in the low bits (address
+    // >> 4, below 2^14 for any shared-memory address), so they are added
+    // there.
+    const uint32_t s0 = tc::smem_addr(ring);
+    const uint64_t da0 = A_MN ? tc::desc_sw128_mn(s0, kMnBox) : tc::desc_sw128(s0);
+    const uint64_t db0 =
+        B_MN ? tc::desc_sw128_mn(s0 + kStageA, kMnBox) : tc::desc_sw128(s0 + kStageA);
     for (int kb = 0; kb < g.nK; ++kb) {
-        ab.wait(&bars.full[p.stage], p.phase);
-        if (ab.on())
+        if (!ab.wait(&bars.full[p.stage], p.phase))
             return;
         tc::fence_after_sync();
-        const uint32_t sa = tc::smem_addr(ring + p.stage * kStageBytes);
-        const uint32_t sb = sa + kStageA;
+        const uint64_t so = (uint64_t)((p.stage * kStageBytes) >> 4);
 #pragma unroll
-        for (int kk = 0; kk < kBK / 16; ++kk) {
-            const uint64_t da = A_MN ? tc::desc_sw128_mn(sa + kk * a_step, kMnBox)
-                                     : tc::desc_sw128(sa + kk * a_step);
-            const uint64_t db = B_MN ? tc::desc_sw128_mn(sb + kk * b_step, kMnBox)
-                                     : tc::desc_sw128(sb + kk * b_step);
-            tc::mma_bf16(d, da, db, kId, (kb | kk) != 0);
-        }
+        for (int kk = 0; kk < kBK / 16; ++kk)
+            tc::mma_bf16(d, da0 + so + (kk * a_step >> 4), db0 + so + (kk * b_step >> 4), kId,
+                         (kb | kk) != 0);
         if (MC)  // the stage is free in this CTA and in the peer
             tc::mma_commit_mc(&bars.empty[p.stage], 0x3);
         else
