@@ -370,13 +370,25 @@ __device__ __forceinline__ void bulk_g2s_evict_first(uint32_t dst, const void *s
 
 // A wait that runs out marks the CTA as aborted (and the status word): every
 // later wait then returns at once, so each role finishes its loops without
-// waiting again and the consumers still meet at every barrier.
+// waiting again and the consumers still meet at every barrier.  A slot that
+// has already landed costs one poll, without a read of the flag (every warp
+// waits once per slot: 3.28 -> 3.20 ms per call at V = 151936).
 struct StreamAbort {
     volatile int *flag;
     int32_t *status;
     __device__ __forceinline__ bool on() const { return *flag != 0; }
     __device__ __forceinline__ void wait(uint32_t bar, uint32_t parity) const
     {
+        uint32_t done;
+        asm volatile(
+            "{\n\t.reg .pred p;\n\t"
+            "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+            "selp.u32 %0, 1, 0, p;\n\t}"
+            : "=r"(done)
+            : "r"(bar), "r"(parity)
+            : "memory");
+        if (done)
+            return;
         if (*flag)
             return;
         if (!mbar_wait(bar, parity)) {
