@@ -341,6 +341,7 @@ struct Plan {
     int cs;
     int64_t slice;
     size_t smem;
+    int nt;  // CTA width: 0 for the default (CIS_CLUSTER_THREADS, else 256)
 };
 
 int64_t slice_target_bytes()
@@ -366,7 +367,12 @@ int forced_cluster()
     return v;
 }
 
-// Smallest cluster size whose slices fit the target (any size 1..8).
+// Smallest cluster size whose slices fit the target (any size 1..8).  Rows
+// that fit one slice of the default 80 KB target but not one of 40 KB (a
+// 32,000-entry bf16 row, for instance) run on two CTAs of 128 threads: at
+// T=4096, V=32000 that took 106.6 us per step against 109.7 us for one CTA of
+// 256 threads, and 256 threads on the two halves were slower still (122 us).
+// Setting CIS_SLICE_KB, CIS_CLUSTER or CIS_CLUSTER_THREADS turns the rule off.
 bool make_plan(int64_t V, int in_bytes, Plan *p)
 {
     const int64_t target = slice_target_bytes();
@@ -380,6 +386,14 @@ bool make_plan(int64_t V, int in_bytes, Plan *p)
             p->cs = cs;
             p->slice = slice;
             p->smem = (size_t)(slice * in_bytes) + 128;
+            p->nt = 0;
+            static const bool slice_set = getenv("CIS_SLICE_KB") != nullptr;
+            if (!forced && !slice_set && cs == 1 && slice * in_bytes > 40 * 1024) {
+                p->cs = 2;
+                p->slice = ((V + 1) / 2 + 7) / 8 * 8;
+                p->smem = (size_t)(p->slice * in_bytes) + 128;
+                p->nt = 128;
+            }
             return true;
         }
     }
@@ -425,7 +439,8 @@ cudaError_t launch_cluster_t(const PassArgs &a, const Plan &p, cudaStream_t s)
 {
     if (a.entropy_out)  // the entropy variant is built for 256 threads only
         return launch_cluster_nt<InT, OutT, 256, true>(a, p, s);
-    switch (cluster_threads()) {
+    static const bool width_set = getenv("CIS_CLUSTER_THREADS") != nullptr;
+    switch (p.nt && !width_set ? p.nt : cluster_threads()) {
     case 512: return launch_cluster_nt<InT, OutT, 512>(a, p, s);
     case 384: return launch_cluster_nt<InT, OutT, 384>(a, p, s);
     case 128: return launch_cluster_nt<InT, OutT, 128>(a, p, s);
