@@ -26,8 +26,10 @@
 //   - cis_mismatch_stream_kernel (bf16 rows, V a multiple of 8, 16-byte
 //     aligned rows): one CTA per SM walking its rows, a producer warp
 //     streaming both rows through a shared-memory ring with bulk copies, once
-//     per pass (HBM reads each row once: the second copy comes from L2); pass
-//     2 forms two candidates per instruction with the packed f32x2 FMA, add
+//     per pass (HBM reads each row once: the second copy comes from L2, and
+//     pass 1's bytes are prefetched into L2 two slots ahead), an epilogue warp
+//     forming each row's outputs while the consumer warps go on; pass 2
+//     forms two candidates per instruction with the packed f32x2 FMA, add
 //     and multiply;
 //   - cis_mismatch_kernel (any row): one CTA per position streaming both rows
 //     from global memory with vector loads, twice.
@@ -256,24 +258,25 @@ __device__ __forceinline__ float2 elem_weight2(float2 xp, float2 xq, float2 p, f
 // that need no negation:
 //   acc = [P2, R2, -RP, D = sum T1 p, -C2, -C3, -C4, -C5, QP]
 // with T2 = q (1 - f) = -q (f - 1), T1 = T2 (1 + f) = -q (f^2 - 1) and
-// r' = p - q f = -r; then C1 = sum q (f^2 - 1)(1 - 2p) = C2 + 2 D.
+// r' = p - q f = -r; then C1 = sum q (f^2 - 1)(1 - 2p) = C2 + 2 D.  T2, T1
+// and r' are each one FMA from -f, so each is rounded once, and two
+// instructions a pair fewer (3.15 -> 3.05 ms per call at T=16384, V=151936).
 template <int MODE>
 __device__ __forceinline__ void diag_pair(float2 zp, float2 zq, float2 nop, float2 noq,
                                           const DevParams &P, float2 (&acc)[kNSums])
 {
     const float2 l2e = make_float2(kLog2e, kLog2e);
-    const float2 one = make_float2(1.0f, 1.0f), m1 = make_float2(-1.0f, -1.0f);
+    const float2 m1 = make_float2(-1.0f, -1.0f);
     const float2 xp = __ffma2_rn(zp, l2e, nop), xq = __ffma2_rn(zq, l2e, noq);
     const float2 p = make_float2(ex2_ftz(xp.x), ex2_ftz(xp.y));
     const float2 q = make_float2(ex2_ftz(xq.x), ex2_ftz(xq.y));
     const float2 d = __ffma2_rn(xq, m1, xp);  // xp - xq, rounded once
     const float2 k = make_float2(ex2_ftz(d.x), ex2_ftz(d.y));
     const float2 f = elem_weight2<MODE>(xp, xq, p, q, k, P);
-    const float2 g = __ffma2_rn(f, m1, one);  // 1 - f (exact for f in [1/2, 2])
-    const float2 h = __fadd2_rn(f, one);      // 1 + f
-    const float2 T2 = __fmul2_rn(q, g);
-    const float2 T1 = __fmul2_rn(T2, h);
-    const float2 r = __ffma2_rn(__fmul2_rn(q, f), m1, p);  // p - q f
+    const float2 nf = __fmul2_rn(f, m1);
+    const float2 T2 = __ffma2_rn(q, nf, q);   // q (1 - f)
+    const float2 T1 = __ffma2_rn(T2, f, T2);  // T2 (1 + f)
+    const float2 r = __ffma2_rn(q, nf, p);    // p - q f
     acc[0] = __ffma2_rn(p, p, acc[0]);
     acc[1] = __ffma2_rn(r, r, acc[1]);
     acc[2] = __ffma2_rn(r, p, acc[2]);
@@ -322,7 +325,7 @@ struct DiagArgs {
 // measured slower).
 template <int NW, int CPS = 1> struct StreamCfg {
     static constexpr int kConsThreads = NW * 32;
-    static constexpr int kThreads = kConsThreads + 32;
+    static constexpr int kThreads = kConsThreads + 64;  // + the producer and epilogue warps
     static constexpr int kSlotGroups = 4 * kConsThreads;  // 8-entry groups of each row per slot
     static constexpr int kSlotBytes = 2 * kSlotGroups * 16;
     static constexpr int kRingFit = (200 * 1024 / CPS) / kSlotBytes;
@@ -330,17 +333,20 @@ template <int NW, int CPS = 1> struct StreamCfg {
     static constexpr size_t kSmem = (size_t)kRing * kSlotBytes + 128;
 };
 constexpr int kMaxRing = 8;
+constexpr int kPrefetchSlots = 2;  // L2 prefetch distance of pass 1, in slots
 constexpr int kMaxConsWarps = 32;
 
+// Per-row buffers are indexed [row parity]: the epilogue warp reads row i's
+// while the consumers fill row i + 1's.
 struct StreamShared {
     alignas(8) uint64_t full[kMaxRing];   // a slot's two copies have landed
     alignas(8) uint64_t empty[kMaxRing];  // every consumer warp is done with a slot
-    MaxSum red[2][kMaxConsWarps];
-    float wsum[kMaxConsWarps][kNSums];
-    double total[kNSums];
-    float op, oq;
-    float2 rowstat[2];  // (m', s') of the training and the inference row
-    float zyv[2];       // their sampled entries
+    alignas(8) uint64_t epi_full[2];      // every consumer warp has written its sums
+    alignas(8) uint64_t epi_empty[2];     // the epilogue warp is done with the buffer
+    MaxSum red[2][2][kMaxConsWarps];      // [parity][training, inference][warp] (m, s)
+    float wsum[2][kMaxConsWarps][kNSums]; // [parity][warp] the pass-2 sums
+    float2 rowstat[2][2];                 // [parity][engine] (m', s')
+    float zyv[2][2];                      // [parity][engine] the sampled entries
     int aborted;
 };
 
@@ -366,6 +372,12 @@ __device__ __forceinline__ void bulk_g2s_evict_first(uint32_t dst, const void *s
         " [%0], [%1], %2, [%3], pol;\n\t}" ::"r"(dst),
         "l"(src), "r"(bytes), "r"(bar)
         : "memory");
+}
+
+// An L2 prefetch of bytes at src (16-byte aligned, a multiple of 16 bytes).
+__device__ __forceinline__ void bulk_prefetch_l2(const void *src, uint32_t bytes)
+{
+    asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(src), "r"(bytes) : "memory");
 }
 
 // A wait that runs out marks the CTA as aborted (and the status word): every
@@ -434,6 +446,32 @@ __device__ __forceinline__ void pass1_update(uint4 w, float &m, float &cm, float
     s = sum8_exp2_pk(w, make_float2(-cm, -cm), s);
 }
 
+// The same over four groups (32 entries): one maximum for the four, so that
+// the compare and the rare rescale come once per 32 entries (3.20 -> 3.15 ms
+// per call at T=16384, V=151936).
+__device__ __forceinline__ void pass1_update4(const uint4 (&w)[4], float &m, float &cm, float2 &s)
+{
+    __nv_bfloat162 g[4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const __nv_bfloat162 *h = reinterpret_cast<const __nv_bfloat162 *>(&w[i]);
+        g[i] = __hmax2_nan(__hmax2_nan(h[0], h[1]), __hmax2_nan(h[2], h[3]));
+    }
+    const __nv_bfloat162 a = __hmax2_nan(__hmax2_nan(g[0], g[1]), __hmax2_nan(g[2], g[3]));
+    const float lm = max_nan(__low2float(a), __high2float(a));
+    if (lm > m || lm != lm) {  // as in pass1_update
+        const float ncm = lm * kLog2e;
+        const float f = ex2_ftz(fminf(cm - ncm, 0.0f));
+        s = __fmul2_rn(s, make_float2(f, f));
+        m = lm;
+        cm = ncm;
+    }
+    const float2 noff = make_float2(-cm, -cm);
+#pragma unroll
+    for (int i = 0; i < 4; ++i)
+        s = sum8_exp2_pk(w[i], noff, s);
+}
+
 // CPS CTAs per SM walk rows t = blockIdx.x, blockIdx.x + gridDim.x, ...  Per
 // row, a producer thread streams both rows through a ring of kRing shared-
 // memory slots twice (bulk copies of sg groups per row per slot): once for
@@ -441,12 +479,17 @@ __device__ __forceinline__ void pass1_update(uint4 w, float &m, float &cm, float
 // where pass 1 left them microseconds earlier; these copies mark the lines
 // evict-first).  Pass 2 takes the row's slots last-first, so that the bytes
 // pass 1 brought in last are read again first.  The consumer warps:
-//   pass 1: per thread a running (max, sum) of each row over its groups;
-//           warp, then CTA combination; lanes 0 and 16 of warp 0 form the two
-//           rows' scalars (log p, log q, lse; eps, log k, p for the output);
-//   pass 2: the nine sums, two candidates per packed instruction;
-//           warp sums in fp32, CTA sums in fp64 by warp 0, which also forms
-//           bias2 and dvar while the other warps start the next row.
+//   pass 1: per thread a running (max, sum) of each row over its groups,
+//           the maximum taken once per full slot (four groups); warp
+//           combination, then the row's one barrier, after which every warp
+//           combines the warps' pairs itself into both rows' lse;
+//   pass 2: the nine sums, two candidates per packed instruction; warp sums
+//           in fp32, handed to the epilogue warp through a buffer per row
+//           parity.
+// The epilogue warp adds the warps' sums in fp64 and forms eps, log k, p,
+// bias2 and dvar, while the consumers work on the next row: at T=16384,
+// V=151936 that took 3.05 -> 3.00 ms per call against warp 0 doing it between
+// two more barriers, with bit-identical outputs.
 template <int MODE, int NW, int CPS>
 __global__ void __launch_bounds__(StreamCfg<NW, CPS>::kThreads, CPS)
     cis_mismatch_stream_kernel(const DiagArgs a, int sg)
@@ -465,6 +508,10 @@ __global__ void __launch_bounds__(StreamCfg<NW, CPS>::kThreads, CPS)
             mbar_init(smem_u32(&sh.full[i]), 1);
             mbar_init(smem_u32(&sh.empty[i]), kConsWarps);
         }
+        for (int i = 0; i < 2; ++i) {
+            mbar_init(smem_u32(&sh.epi_full[i]), kConsWarps);
+            mbar_init(smem_u32(&sh.epi_empty[i]), 1);
+        }
         sh.aborted = 0;
     }
     __syncthreads();
@@ -480,6 +527,26 @@ __global__ void __launch_bounds__(StreamCfg<NW, CPS>::kThreads, CPS)
                 continue;
             const uint8_t *rp = reinterpret_cast<const uint8_t *>(a.zt + t * a.ld_t);
             const uint8_t *rq = reinterpret_cast<const uint8_t *>(a.zi + t * a.ld_i);
+            // Pass 1's bytes are prefetched into L2 kPrefetchSlots slots ahead
+            // of their copies: this row's slot st + kPrefetchSlots with
+            // pass-1 slot st, and the first slots of this CTA's next row with
+            // the last slots of pass 2.  Pass 1 then copies from L2 instead
+            // of waiting on HBM.  At T=16384, V=151936: 3.00 ms per call
+            // without, 2.80 ms with 2 slots ahead (10.20 GB read from HBM),
+            // 2.79 with 4 (10.32 GB) or 6 (10.97 GB), and 2.83 ms with the
+            // whole next row prefetched during pass 2 (15.47 GB: the L2 no
+            // longer holds both rows).  With several CTAs per SM more rows
+            // are in flight and the prefetch is left out.
+            int64_t tn = CPS == 1 ? t + gridDim.x : a.T;
+            for (; tn < a.T; tn += gridDim.x) {
+                const int64_t yn = a.ids[tn];
+                if ((a.mask == nullptr || a.mask[tn] != 0) && yn >= 0 && yn < a.V)
+                    break;
+            }
+            const uint8_t *np =
+                tn < a.T ? reinterpret_cast<const uint8_t *>(a.zt + tn * a.ld_t) : nullptr;
+            const uint8_t *nq =
+                tn < a.T ? reinterpret_cast<const uint8_t *>(a.zi + tn * a.ld_i) : nullptr;
             for (int pass = 0; pass < 2 && !ab.on(); ++pass)
                 for (int st = 0; st < nst; ++st, ++k) {
                     const uint32_t s = k % kRing, u = k / kRing;
@@ -495,10 +562,23 @@ __global__ void __launch_bounds__(StreamCfg<NW, CPS>::kThreads, CPS)
                     if (pass == 0) {
                         bulk_g2s(dst, rp + (int64_t)g0 * 16, bytes, full);
                         bulk_g2s(dst + kSlotGroups * 16, rq + (int64_t)g0 * 16, bytes, full);
+                        if (CPS == 1 && st + kPrefetchSlots < nst) {
+                            const int gn = (st + kPrefetchSlots) * sg;
+                            const uint32_t nb = (uint32_t)min(sg, ng - gn) * 16;
+                            bulk_prefetch_l2(rp + (int64_t)gn * 16, nb);
+                            bulk_prefetch_l2(rq + (int64_t)gn * 16, nb);
+                        }
                     } else {
                         bulk_g2s_evict_first(dst, rp + (int64_t)g0 * 16, bytes, full);
                         bulk_g2s_evict_first(dst + kSlotGroups * 16, rq + (int64_t)g0 * 16, bytes,
                                              full);
+                        const int pi = st - (nst - kPrefetchSlots);  // the next row's slot
+                        if (np != nullptr && pi >= 0 && pi < nst) {
+                            const int gn = pi * sg;
+                            const uint32_t nb = (uint32_t)min(sg, ng - gn) * 16;
+                            bulk_prefetch_l2(np + (int64_t)gn * 16, nb);
+                            bulk_prefetch_l2(nq + (int64_t)gn * 16, nb);
+                        }
                     }
                 }
         }
@@ -509,9 +589,63 @@ __global__ void __launch_bounds__(StreamCfg<NW, CPS>::kThreads, CPS)
         return;
     }
 
+    if (warp == kConsWarps + 1) {  // row epilogue
+        uint32_t rr = 0;  // valid rows so far
+        for (int64_t t = blockIdx.x; t < a.T && !ab.on(); t += gridDim.x) {
+            const int64_t y = a.ids[t];
+            if ((a.mask != nullptr && a.mask[t] == 0) || y < 0 || y >= a.V)
+                continue;
+            const int b = rr & 1;
+            ab.wait(smem_u32(&sh.epi_full[b]), (rr >> 1) & 1);
+            if (ab.on())
+                break;
+            // eps, log k and p; lane 16 forms the inference row's scalars
+            const int r = lane >> 4;
+            const MaxSum o = MaxSum{sh.rowstat[b][r].x, sh.rowstat[b][r].y};
+            const float zyr = sh.zyv[b][r];
+            const RowScalars rs = row_scalars(o, zyr);
+            const double lp64_q = __shfl_sync(0xffffffffu, rs.lp64(), 16);
+            const float om_q = __shfl_sync(0xffffffffu, o.m, 16);
+            const float os_q = __shfl_sync(0xffffffffu, o.s, 16);
+            const float zy_q = __shfl_sync(0xffffffffu, zyr, 16);
+            // the nine sums: the warps' fp32 sums added in fp64 in warp order
+            double v = 0.0;
+            if (lane < kNSums) {
+                v = sh.wsum[b][0][lane];
+                for (int w = 1; w < kConsWarps; ++w)
+                    v += sh.wsum[b][w][lane];
+            }
+            double S[kNSums];
+#pragma unroll
+            for (int i = 0; i < kNSums; ++i)
+                S[i] = __shfl_sync(0xffffffffu, v, i);
+            __syncwarp();
+            if (lane == 0) {
+                mbar_arrive(smem_u32(&sh.epi_empty[b]));  // the buffer is read
+                // eps = logit p - logit q: Lemma 3.1's -delta_y + log sum_{j != y}
+                // w_j e^{delta_j} in the normalised gauge, from the log-odds
+                const double dp = ((double)zyr - (double)o.m) - (double)logf(o.s);
+                const double dq = ((double)zy_q - (double)om_q) - (double)logf(os_q);
+                a.eps[t] = (float)(dp - dq);
+                if (a.logk) a.logk[t] = (float)(rs.lp64() - lp64_q);
+                if (a.p) a.p[t] = expf(rs.lp);
+                const double P2 = S[0], R2 = S[1], RP = -S[2], D = S[3], C2 = -S[4], C3 = -S[5],
+                             C4 = -S[6], C5 = -S[7], QP = S[8];
+                const double C1 = C2 + 2.0 * D, C6 = C5 + 2.0 * QP;
+                const double bias2 = R2 - 2.0 * C3 * RP + C3 * C3 * P2;
+                const double dvar =
+                    C1 + P2 * C2 - (C4 - (2.0 + C3) * C5 - C3 * C6 + C3 * (2.0 + C3) * P2);
+                if (a.bias2) a.bias2[t] = (float)bias2;
+                if (a.dvar) a.dvar[t] = (float)dvar;
+            }
+            ++rr;
+        }
+        return;
+    }
+
     // consumers
     const int ct = threadIdx.x;
-    uint32_t k = 0;
+    uint32_t k = 0, rr = 0;  // ring slots used; valid rows so far
     for (int64_t t = blockIdx.x; t < a.T; t += gridDim.x) {
         const bool valid = a.mask == nullptr || a.mask[t] != 0;
         const int64_t y = a.ids[t];
@@ -528,9 +662,11 @@ __global__ void __launch_bounds__(StreamCfg<NW, CPS>::kThreads, CPS)
             }
             continue;
         }
-        // the sampled entries, read early (used after pass 1)
+        const int b = rr & 1;
+        // the sampled entries, read early (used after pass 1): lane 0 the
+        // training row's, lane 16 the inference row's
         float zy = 0.0f;
-        if (warp == 0 && (lane == 0 || lane == 16))
+        if ((lane & 15) == 0)
             zy = to_f32(lane == 0 ? a.zt[t * a.ld_t + y] : a.zi[t * a.ld_i + y]);
         const int gy = (int)(y >> 3), iy = (int)(y & 7);
 
@@ -542,6 +678,25 @@ __global__ void __launch_bounds__(StreamCfg<NW, CPS>::kThreads, CPS)
             ab.wait(smem_u32(&sh.full[s]), (k / kRing) & 1);
             const uint4 *slot = reinterpret_cast<const uint4 *>(ring + (size_t)s * kSlotBytes);
             const int g0 = st * sg, n = min(sg, ng - g0);
+            if (n == 4 * kConsThreads) {  // a full slot: four groups a thread
+                uint4 u[4], v[4];
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                    u[i] = slot[ct + i * kConsThreads];
+                    v[i] = slot[kSlotGroups + ct + i * kConsThreads];
+                }
+                const int rel = gy - g0 - ct;  // the sampled entry's group, if this thread's
+                if (rel >= 0 && rel < 4 * kConsThreads && rel % kConsThreads == 0) {
+#pragma unroll
+                    for (int i = 0; i < 4; ++i)
+                        if (rel == i * kConsThreads) {
+                            u[i] = drop_entry(u[i], iy);
+                            v[i] = drop_entry(v[i], iy);
+                        }
+                }
+                pass1_update4(u, m_p, cm_p, s_p);
+                pass1_update4(v, m_q, cm_q, s_q);
+            } else
 #pragma unroll 1
             for (int j = ct; j < n; j += kConsThreads) {
                 uint4 u = slot[j], v = slot[kSlotGroups + j];
@@ -564,63 +719,48 @@ __global__ void __launch_bounds__(StreamCfg<NW, CPS>::kThreads, CPS)
         rp = warp_ms(rp);
         rq = warp_ms(rq);
         if (lane == 0) {
-            sh.red[0][warp] = rp;
-            sh.red[1][warp] = rq;
+            sh.red[b][0][warp] = rp;
+            sh.red[b][1][warp] = rq;
         }
         cons_sync<kConsThreads>();
-        if (warp == 0) {
-            // lanes 0-15 combine the training row's warp pairs, 16-31 the
-            // inference row's (lane l takes warps l, l + 16, ...), then a
-            // fixed tree over the 16 lanes
-            const int r = lane >> 4;
-            MaxSum o = (lane & 15) < kConsWarps ? sh.red[r][lane & 15] : MaxSum{-INFINITY, 0.0f};
-            for (int w = (lane & 15) + 16; w < kConsWarps; w += 16)
-                o = ms_combine(o, sh.red[r][w]);
+        // Every warp combines the warps' pairs in the same fixed order (lanes
+        // 0-15 the training row's, lane l taking warps l, l + 16, ..., 16-31
+        // the inference row's, then a tree over the 16 lanes), so that pass 2
+        // starts without a second barrier.  sh.red is double-buffered by row
+        // parity: a warp rewrites this row's buffer two rows later, after the
+        // next row's barrier, which every warp reaches only once it has read
+        // this one.
+        const int r = lane >> 4;
+        MaxSum o = (lane & 15) < kConsWarps ? sh.red[b][r][lane & 15] : MaxSum{-INFINITY, 0.0f};
+        for (int w = (lane & 15) + 16; w < kConsWarps; w += 16)
+            o = ms_combine(o, sh.red[b][r][w]);
 #pragma unroll
-            for (int off = 8; off > 0; off >>= 1) {
-                MaxSum x;
-                x.m = __shfl_xor_sync(0xffffffffu, o.m, off);
-                x.s = __shfl_xor_sync(0xffffffffu, o.s, off);
-                o = ms_combine(o, x);
-            }
-            // Pass 2 needs only the two rows' log-sum-exps; lanes 0 and 16
-            // form their own row's while the other warps wait, from the
-            // larger of m' and z_y so that no exponential overflows:
-            //   lse = z_y + log1p(s' e^{m' - z_y})   (z_y >= m', also p = 1)
-            //   lse = m' + log(s' + e^{z_y - m'})    (otherwise)
-            // The per-position outputs are formed after the barrier.
-            if ((lane & 15) == 0) {
-                const float lse = o.s == 0.0f ? zy  // no other finite entry: p = 1
-                                  : (zy >= o.m ? zy + log1pf(o.s * expf(o.m - zy))
-                                               : o.m + logf(o.s + expf(zy - o.m)));
-                if (r == 0)
-                    sh.op = lse * kLog2e;
-                else
-                    sh.oq = lse * kLog2e;
-                sh.rowstat[r] = make_float2(o.m, o.s);
-                sh.zyv[r] = zy;
-            }
+        for (int off = 8; off > 0; off >>= 1) {
+            MaxSum x;
+            x.m = __shfl_xor_sync(0xffffffffu, o.m, off);
+            x.s = __shfl_xor_sync(0xffffffffu, o.s, off);
+            o = ms_combine(o, x);
         }
-        cons_sync<kConsThreads>();
-        if (warp == (kConsWarps > 1 ? 1 : 0)) {
-            // eps, log k and p, off the serial path (warp 0 has the end-of-row
-            // sums to do); lane 16 forms the inference row's scalars
-            const int r = lane >> 4;
-            const MaxSum o = MaxSum{sh.rowstat[r].x, sh.rowstat[r].y};
-            const float zyr = sh.zyv[r];
-            const RowScalars rs = row_scalars(o, zyr);
-            const double lp64_q = __shfl_sync(0xffffffffu, rs.lp64(), 16);
-            const float om_q = __shfl_sync(0xffffffffu, o.m, 16);
-            const float os_q = __shfl_sync(0xffffffffu, o.s, 16);
-            const float zy_q = __shfl_sync(0xffffffffu, zyr, 16);
-            if (lane == 0) {
-                // eps = logit p - logit q: Lemma 3.1's -delta_y + log sum_{j != y}
-                // w_j e^{delta_j} in the normalised gauge, from the log-odds
-                const double dp = ((double)zyr - (double)o.m) - (double)logf(o.s);
-                const double dq = ((double)zy_q - (double)om_q) - (double)logf(os_q);
-                a.eps[t] = (float)(dp - dq);
-                if (a.logk) a.logk[t] = (float)(rs.lp64() - lp64_q);
-                if (a.p) a.p[t] = expf(rs.lp);
+        // Pass 2 needs only the two rows' log-sum-exps, from the larger of m'
+        // and z_y so that no exponential overflows:
+        //   lse = z_y + log1p(s' e^{m' - z_y})   (z_y >= m', also p = 1)
+        //   lse = m' + log(s' + e^{z_y - m'})    (otherwise)
+        float lse = 0.0f;
+        if ((lane & 15) == 0)
+            lse = o.s == 0.0f ? zy  // no other finite entry: p = 1
+                  : (zy >= o.m ? zy + log1pf(o.s * expf(o.m - zy))
+                               : o.m + logf(o.s + expf(zy - o.m)));
+        const float op = __shfl_sync(0xffffffffu, lse, 0) * kLog2e;
+        const float oq = __shfl_sync(0xffffffffu, lse, 16) * kLog2e;
+        if (warp == 0) {
+            // the row statistics for the epilogue warp, once it is done with
+            // this buffer (two rows ago)
+            if (lane == 0)
+                ab.wait(smem_u32(&sh.epi_empty[b]), ((rr >> 1) & 1) ^ 1);
+            __syncwarp();
+            if ((lane & 15) == 0) {
+                sh.rowstat[b][r] = make_float2(o.m, o.s);
+                sh.zyv[b][r] = zy;
             }
         }
 
@@ -629,7 +769,7 @@ __global__ void __launch_bounds__(StreamCfg<NW, CPS>::kThreads, CPS)
 #pragma unroll
         for (int i = 0; i < kNSums; ++i)
             acc[i] = make_float2(0.0f, 0.0f);
-        const float2 nop = make_float2(-sh.op, -sh.op), noq = make_float2(-sh.oq, -sh.oq);
+        const float2 nop = make_float2(-op, -op), noq = make_float2(-oq, -oq);
         for (int st = 0; st < nst; ++st, ++k) {
             const uint32_t s = k % kRing;
             ab.wait(smem_u32(&sh.full[s]), (k / kRing) & 1);
@@ -647,38 +787,26 @@ __global__ void __launch_bounds__(StreamCfg<NW, CPS>::kThreads, CPS)
             if (lane == 0)
                 mbar_arrive(smem_u32(&sh.empty[s]));
         }
-        // warp sums in fp32 (fp64 arithmetic is scarce on this part), the
-        // CTA's in fp64 by lanes 0-8 of warp 0, in warp order
+        // warp sums in fp32 (fp64 arithmetic is scarce on this part); the
+        // epilogue warp adds the warps' in fp64 and forms the outputs while
+        // this warp goes on to the next row
+        float ws[kNSums];
 #pragma unroll
         for (int i = 0; i < kNSums; ++i) {
             float v = acc[i].x + acc[i].y;
 #pragma unroll
             for (int o = 16; o > 0; o >>= 1)
                 v += __shfl_xor_sync(0xffffffffu, v, o);
-            if (lane == 0)
-                sh.wsum[warp][i] = v;
+            ws[i] = v;
         }
-        cons_sync<kConsThreads>();
-        if (warp == 0) {
-            if (lane < kNSums) {
-                double v = sh.wsum[0][lane];
-                for (int w = 1; w < kConsWarps; ++w)
-                    v += sh.wsum[w][lane];
-                sh.total[lane] = v;
-            }
-            __syncwarp();
-            if (lane == 0) {
-                const double *S = sh.total;
-                const double P2 = S[0], R2 = S[1], RP = -S[2], D = S[3], C2 = -S[4], C3 = -S[5],
-                             C4 = -S[6], C5 = -S[7], QP = S[8];
-                const double C1 = C2 + 2.0 * D, C6 = C5 + 2.0 * QP;
-                const double bias2 = R2 - 2.0 * C3 * RP + C3 * C3 * P2;
-                const double dvar =
-                    C1 + P2 * C2 - (C4 - (2.0 + C3) * C5 - C3 * C6 + C3 * (2.0 + C3) * P2);
-                if (a.bias2) a.bias2[t] = (float)bias2;
-                if (a.dvar) a.dvar[t] = (float)dvar;
-            }
+        if (lane == 0) {
+            ab.wait(smem_u32(&sh.epi_empty[b]), ((rr >> 1) & 1) ^ 1);
+#pragma unroll
+            for (int i = 0; i < kNSums; ++i)
+                sh.wsum[b][warp][i] = ws[i];
+            mbar_arrive(smem_u32(&sh.epi_full[b]));
         }
+        ++rr;
     }
 }
 
