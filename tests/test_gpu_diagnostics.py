@@ -444,10 +444,17 @@ def test_diagnostics_full_vocabulary_low_temperature_rows():
 
 
 def test_diagnostics_full_workload_every_row():
-    """The benchmarked workload (T=16384, V=151936, GPU-generated): on every
-    row p in (0, 1], bias2 >= 0 and finite, dvar finite, and eps NaN-free
-    except where p = 1 (the closed-form and oracle tests fix the values)."""
+    """The benchmarked workload (T=16384, V=151936, GPU-generated) in the
+    launch the benchmark times: on every row p in (0, 1], bias2 >= 0 and
+    finite, dvar finite, and eps NaN-free except where p = 1; and eight
+    sampled rows against the O(V^2) oracle (one host thread each, about 40 s).
+    With one CTA per SM a CTA walks rows c, c + grid, ..., so the samples
+    take each CTA's first and second row (both parities of the per-row
+    buffers), rows deep into a CTA's sequence (the ring, the L2 prefetch of
+    the next row and the epilogue warp long in steady state) and the last row
+    of the batch."""
     b = synth.make_batch(6, device=DEV)
+    outs = {}
     for mode in ("cis", "exact"):
         out = binding.cis_mismatch_diagnostics(b.logits, b.extra["logits_infer"], b.ids,
                                                binding.cis_default_params(mode))
@@ -457,6 +464,16 @@ def test_diagnostics_full_workload_every_row():
         assert torch.isfinite(out["bias2"]).all() and torch.all(out["bias2"] >= -1e-6), mode
         assert torch.isfinite(out["dvar"]).all() and torch.isfinite(out["logk"]).all(), mode
         assert not torch.isnan(out["eps"][p < 1]).any(), mode
+        outs[mode] = out
+    grid = min(b.T, torch.cuda.get_device_properties(DEV).multi_processor_count)
+    picks = [0, grid, 75 + 53 * grid, 75 + 54 * grid, 5000, 12345, b.T - 1 - grid, b.T - 1]
+    rows = torch.tensor(sorted({t for t in picks if 0 <= t < b.T}), device=DEV)
+    z = b.logits[rows].cpu()
+    zi = b.extra["logits_infer"][rows].cpu()
+    ids = b.ids[rows].cpu().numpy()
+    ref = _oracle_rows_parallel(z, zi, ids, ["cis"])["cis"]
+    got = {k: v[rows] for k, v in outs["cis"].items()}
+    _compare(got, ref, z, zi, "cis", n_thread(b.V))
 
 
 @pytest.mark.parametrize("dtype,V", [(torch.float32, 64), (torch.bfloat16, 2056)])
