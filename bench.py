@@ -61,7 +61,7 @@ def parse_args():
     ap.add_argument("--workload", type=int, default=3, choices=[2, 3, 4, 5, 6])
     ap.add_argument("--dlogits", choices=["bf16", "f32"], default="bf16")
     ap.add_argument("--e2e-steps", type=int, default=10)
-    ap.add_argument("--e2e-chunk", type=int, default=2048)
+    ap.add_argument("--e2e-chunk", type=int, default=512)
     ap.add_argument("--cpu-seconds", type=float, default=10.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--tokens", type=int, default=None,

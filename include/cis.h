@@ -309,7 +309,10 @@ CIS_API cis_status_t cis_loss_host_workspace_size(int64_t T, int64_t V, int32_t 
  * The rows stream through the GPU in chunks of chunk_tokens: while the fused
  * kernel runs on chunk k (on `stream`), the next chunks are copied in and the
  * previous ones copied out on copy streams the library creates once per
- * device (one per staging buffer and direction).  The
+ * device (one per staging buffer and direction).  The first chunk's copy in
+ * and the last one's copy out run alone, so small chunks overlap more: at
+ * T=16384, V=151936 (bf16), chunks of 512 rows (150 MB) took 30-32 ms per call
+ * against 35-42 ms for chunks of 2048.  The
  * normaliser and the loss cover the whole batch, so every output equals that
  * of cis_loss_fwd_bwd.  Asynchronous on `stream`: the host outputs are valid
  * once `stream` has completed the call's work.  Errors: as cis_loss_fwd_bwd,

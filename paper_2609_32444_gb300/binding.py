@@ -324,7 +324,7 @@ def cis_loss_host_workspace_size(T, V, dtype, dlogits_dtype, chunk_tokens, B=0) 
 
 def cis_loss_fwd_bwd_host(logits: torch.Tensor, ids: torch.Tensor, lp_infer: torch.Tensor,
                           adv: torch.Tensor, params: cis_params_t, dlogits: torch.Tensor,
-                          lp_old=None, mask=None, cu_seqlens=None, chunk_tokens=2048,
+                          lp_old=None, mask=None, cu_seqlens=None, chunk_tokens=512,
                           workspace=None, outputs=None, want_entropy=False):
     """The fused pass with every tensor in HOST memory (pinned for overlap);
     rows stream through the GPU in chunks.  ``outputs``: optional dict of host
