@@ -364,6 +364,40 @@ def test_diagnostics_many_rows_per_cta():
     _compare(out, ref, z, zi, "cis", n_thread(V), m.numpy())
 
 
+def test_diagnostics_several_rows_per_cta_with_short_slots(monkeypatch):
+    """T=400 rows of V=2056 through 64-group slots (five slots a pass), so
+    that every CTA walks two or three rows, with every third row masked and
+    two bad ids: the producer's L2 prefetch of a CTA's next valid row skips
+    the masked ones, and the epilogue warp's per-row buffers alternate
+    between the rows that remain.  Every row matches the oracle."""
+    monkeypatch.setenv("CIS_DIAG_SLOT_GROUPS", "64")
+    V, T = 2056, 400
+    z, zi, ids = _rows(21, T, V, torch.bfloat16)
+    m = torch.ones(T, dtype=torch.uint8)
+    m[::3] = 0
+    bad = [155, 307]  # valid rows (not multiples of 3) with ids out of range
+    ids[bad[0]] = V
+    ids[bad[1]] = -1
+    st = torch.zeros(1, dtype=torch.int32, device=DEV)
+    out = binding.cis_mismatch_diagnostics(z.to(DEV), zi.to(DEV), ids.to(DEV),
+                                           binding.cis_default_params("cis"), mask=m.to(DEV),
+                                           dev_status=st)
+    torch.cuda.synchronize()
+    assert int(st.item()) == binding.CIS_ERR_BAD_TOKEN_ID
+    for k, v in out.items():
+        assert torch.isnan(v[bad]).all(), k
+    keep = m.numpy().astype(bool)
+    keep[bad] = False  # compared as masked below: the oracle takes in-range ids only
+    ids_ok = ids.clone()
+    ids_ok[bad] = 0
+    ref = oracle.mismatch_diagnostics(logits_for_oracle(z), logits_for_oracle(zi), ids_ok.numpy(),
+                                      oracle.params(mode=oracle.MODE_CIS), mask=keep.astype(np.uint8))
+    got = {k: v.clone() for k, v in out.items()}
+    for k in got:
+        got[k][bad] = 0.0
+    _compare(got, ref, z, zi, "cis", n_thread(V, 64), keep.astype(np.uint8))
+
+
 def test_diagnostics_all_other_entries_neg_inf(monkeypatch):
     """A row whose entries other than y are -inf for the training engine
     (p = 1, every other candidate has k = f = 0).  logit p is infinite there:
