@@ -822,14 +822,14 @@ int diag_slot_groups(int max_groups)
 
 // Consumer warps per CTA (CIS_DIAG_WARPS, for tuning sweeps): 16 (the
 // default) or 24 with one CTA per SM, 8 with two, 4 with four; the ring
-// shrinks with the CTA.  At V=151936 (four groups a thread per slot) two CTAs
-// of 8 warps took 3.19 ms against 3.28 for one of 16: a CTA's warps meet
-// three times per row, and while one CTA waits at those barriers the SM's
-// other CTA issues.  But twice as many rows are then in flight (about 185 MB
-// between a row's two reads, more than the L2 holds), and pass 2 re-read a
-// third of its bytes from HBM: 13.2 GB of DRAM reads per call against 10.0.
-// One CTA of 16 warps keeps HBM at one read of each row.  24 warps in one CTA
-// (2 slots of 96 KB) were slower than 16 (3 of 64 KB).
+// shrinks with the CTA.  At V=151936, two CTAs of 8 warps took 2.84 ms and
+// four of 4 2.83 ms (without the L2 prefetch, which they leave out) against
+// 2.81 for one of 16.  They keep two or four rows in flight per SM (about 185
+// MB between a row's two reads at two, more than the L2 holds), and pass 2
+// then re-read a third of its bytes from HBM: 13.2 GB of DRAM reads per call
+// against 10.0 (an earlier build).  One CTA of 16 warps keeps HBM at one read
+// of each row.  24 warps in one CTA (2 slots of 96 KB) were slower than 16 (3
+// of 64 KB).
 int diag_warps()
 {
     const char *e = getenv("CIS_DIAG_WARPS");
