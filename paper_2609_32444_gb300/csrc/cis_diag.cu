@@ -317,12 +317,12 @@ struct DiagArgs {
     int32_t *status;
 };
 
-// The layout for NW consumer warps (plus one producer warp) and CPS CTAs per
-// SM: a ring slot holds four groups per consumer thread of each row, as many
-// slots as fit in about 200 KB / CPS of shared memory (3 of 64 KB for 16
-// warps and one CTA).  Each slot costs every warp a wait, an arrive and the loop
-// set-up; four groups a thread amortise that (two, three, five and six
-// measured slower).
+// The layout for NW consumer warps (plus a producer and an epilogue warp)
+// and CPS CTAs per SM: a ring slot holds four groups per consumer thread of
+// each row, as many slots as fit in about 200 KB / CPS of shared memory (3 of
+// 64 KB for 16 warps and one CTA).  Each slot costs every warp a wait, an
+// arrive and the loop set-up; four groups a thread amortise that (two, three,
+// five and six measured slower).
 template <int NW, int CPS = 1> struct StreamCfg {
     static constexpr int kConsThreads = NW * 32;
     static constexpr int kThreads = kConsThreads + 64;  // + the producer and epilogue warps
