@@ -367,9 +367,15 @@ def run_ours(args, rank, world, local):
     peak, peak_src = measured_peaks()
     achieved = alg_bytes / (kernel_ms / 1e3) / 1e9
     traffic = profiled_traffic(args.workload, args.tokens)
+    # the library's layout: rows of 40-80 KB on two CTAs of 128 threads, the
+    # rest on clusters of CTAs of 256 threads
+    in_t = "bf16" if isz == 2 else "f32"
+    out_t = "bf16" if osz == 2 else "f32"
+    width = 128 if 40 * 1024 < V * isz <= 80 * 1024 else 256
     roof = {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
             "frac": achieved / peak, "traffic": traffic,
-            "kernel": "cis_fused_cluster_kernel<bf16,bf16,256> (fused fwd+bwd vocabulary pass)",
+            "kernel": f"cis_fused_cluster_kernel<{in_t},{out_t},{width}> "
+                      "(fused fwd+bwd vocabulary pass)",
             "kernel_ms": kernel_ms, "algorithmic_bytes_per_launch": alg_bytes,
             "peak_source": peak_src, "frac_of_nominal_8000": achieved / NOMINAL_HBM_GBS,
             "step_frac": alg_bytes / (ms_per_step / 1e3) / 1e9 / peak}
