@@ -45,8 +45,8 @@
  *       CIS_SLICE_KB (8..200, default 80), CIS_CLUSTER (1..8) and
  *       CIS_CLUSTER_THREADS (128, 256, 384 or 512; default 256) set the
  *       fused pass's slice target, cluster size and CTA width.  By default a
- *       row of 40 to 80 KB runs on two CTAs of 128 threads.  They are read
- *       once per process.
+ *       row of 40 to 80 KB runs on two CTAs of 128 threads (CIS_SLICE_KB or
+ *       CIS_CLUSTER turns that off).  They are read once per process.
  *       CIS_DIAG_WARPS (16 or 24 with one CTA per SM, 8 with two, 4 with
  *       four; default 16) and CIS_DIAG_SLOT_GROUPS (>= 1) set the diagnostics
  *       kernel's width and ring-slot size, and CIS_DIAG_KERNEL=row selects its

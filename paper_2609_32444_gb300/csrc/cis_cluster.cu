@@ -372,7 +372,8 @@ int forced_cluster()
 // 32,000-entry bf16 row, for instance) run on two CTAs of 128 threads: at
 // T=4096, V=32000 that took 106.6 us per step against 109.7 us for one CTA of
 // 256 threads, and 256 threads on the two halves were slower still (122 us).
-// Setting CIS_SLICE_KB, CIS_CLUSTER or CIS_CLUSTER_THREADS turns the rule off.
+// Setting CIS_SLICE_KB or CIS_CLUSTER turns the rule off; CIS_CLUSTER_THREADS
+// sets the width of its two CTAs.
 bool make_plan(int64_t V, int in_bytes, Plan *p)
 {
     const int64_t target = slice_target_bytes();
